@@ -1,0 +1,393 @@
+"""Throughput of the DAMP decode-step state update on GB300.
+
+Workload (one "step" = one decode step of one linear-attention layer over the
+whole batch: operand staging, reconstruction, decay, delta read, rank-1
+correction, output, requantization and write-back):
+    KDA decode, B = 256 request slots, H = 32 heads, d_k = d_v = 128,
+    K_hi = 10 FP16 key channels per head, the rest UINT8 + H_32 (G = 32),
+    BF16 q/k/v, FP32 gates/beta/o.
+Metric: microseconds per step and achieved HBM bandwidth, counted from the
+algorithmic bytes of a step (state read + write, q/k/v/beta/gates, o), against
+the measured GB300 copy bandwidth.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Under torchrun every rank runs its own batch (weak scaling, no data exchange);
+the step time is the maximum over ranks.  `--impl reference` times the CPU
+oracle on a bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import workloads as wl  # noqa: E402
+
+METRIC = "mixed-precision state-update µs/step & achieved HBM TB/s (B=256, vs 8 TB/s peak)"
+WORKLOAD = wl.KDA_B256
+N_INPUT_SETS = 8
+POOLS = 2
+
+
+def algorithmic_bytes(w: wl.Workload, packed: bool = True) -> int:
+    """Bytes a step must move: every state read and written once, operands read once, o written."""
+    B, H, Hq, dk, dv, K = w.batch, w.heads, w.qk_heads, w.d_k, w.d_v, w.k_hi
+    if packed:
+        state = 2 * K * dv + (dk - K) * dv + 4 * (dk - K) * (dv // 32)
+    else:
+        state = 4 * dk * dv
+    esz = 2 if w.in_dtype == "bf16" else 4
+    ops = 2 * B * Hq * dk * esz + B * H * dv * esz + B * H * 4 + B * H * (dk if w.kind == "kda" else 1) * 4
+    ops += (H * dk) if packed else 0  # the permutation
+    return 2 * B * H * state + ops + B * H * dv * 4
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_27513_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(f.encode() + fh.read())
+    return h.hexdigest()[:16]
+
+
+def measured_peaks() -> dict:
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f)
+    except OSError:
+        return {}
+
+
+def ncu_traffic(name: str):
+    """DRAM bytes per launch from the committed ncu summary, if taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", f"{name}.txt")
+    try:
+        kv = {}
+        with open(path) as f:
+            for line in f:
+                if "=" in line and not line.lstrip().startswith("#"):
+                    k, v = line.split("=", 1)
+                    kv[k.strip()] = v.strip()
+        if kv.get("source_hash") == kernel_source_hash():
+            return float(kv["dram_bytes_per_launch"])
+    except (OSError, KeyError, ValueError):
+        pass
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while the timed region runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self) -> dict:
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in (self.out or "").splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ GPU arm ---
+
+def gpu_arm(args, rank: int, world: int):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2608_27513_gb300 as damp
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    from paper_2608_27513_gb300 import build
+    if rank == 0:
+        build.build()
+    if world > 1:
+        dist.barrier()
+    w = WORKLOAD
+    L = damp.Layout(w.heads, w.qk_heads, w.d_k, w.d_v, w.k_hi, w.lo_format)
+    stream = torch.cuda.current_stream()
+
+    # ---- state: FP32 prefix on the GPU, then the prefill hand-off into the packed cache ----
+    prefix_in = wl.torch_step_inputs(w, 16, dev, seed_offset=1000 + rank)
+    S = damp.new_fp32_state(L, w.batch, dev)
+    o = torch.empty((w.batch, w.heads, w.d_v), device=dev)
+    for t in range(w.prefix):
+        d = prefix_in[t % len(prefix_in)]
+        damp.fp32_kda_decode_step(L, S, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o)
+    perm = torch.from_numpy(wl.random_perm(w)).to(dev)
+    pools = [damp.new_state(L, w.batch, dev) for _ in range(POOLS)]
+    for p in pools:
+        damp.quantize_state(L, S, perm, p)
+    fp32_pools = [S] + [S.clone() for _ in range(POOLS - 1)]
+    inputs = wl.torch_step_inputs(w, N_INPUT_SETS, dev, seed_offset=rank)
+    torch.cuda.synchronize()
+
+    def run_packed(i, o_buf):
+        d = inputs[i % N_INPUT_SETS]
+        damp.kda_decode_step(L, pools[i % POOLS], perm, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o_buf)
+
+    def run_fp32(i, o_buf):
+        d = inputs[i % N_INPUT_SETS]
+        damp.fp32_kda_decode_step(L, fp32_pools[i % POOLS], d["q"], d["k"], d["v"], d["g"], d["beta"], o=o_buf)
+
+    def timed(fn, steps, warmup, per_launch=True):
+        for i in range(warmup):
+            fn(i, o)
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)] \
+            if per_launch else []
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for i in range(steps):
+            if per_launch:
+                ev[i][0].record(stream)
+            fn(i, o)
+            if per_launch:
+                ev[i][1].record(stream)
+        t1.record(stream)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        total_ms = t0.elapsed_time(t1)
+        launch_ms = statistics.mean(a.elapsed_time(b) for a, b in ev) if per_launch else total_ms / steps
+        return total_ms, launch_ms
+
+    def max_over_ranks(x):
+        if world == 1:
+            return x
+        t = torch.tensor([x], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    with ClockSampler(dev.index) as clk:
+        total_ms, launch_ms = timed(run_packed, args.steps, args.warmup)
+    total_ms = max_over_ranks(total_ms)
+    launch_ms = max_over_ranks(launch_ms)
+    if damp.device_status() != 0:
+        raise RuntimeError("device status word set during the timed region")
+
+    # ---- the in-house FP32-state kernel on the same inputs (speedup reference) ----
+    fp_steps = max(args.steps // 4, 10)
+    fp_total, fp_launch = timed(run_fp32, fp_steps, max(args.warmup, 3))
+    fp_launch = max_over_ranks(fp_launch)
+
+    # ---- end to end through the C ABI from pinned host buffers ----
+    host_in = [{k: v.cpu().pin_memory() for k, v in d.items()} for d in inputs[:2]]
+    dev_in = [{k: torch.empty_like(v) for k, v in d.items()} for d in inputs[:2]]
+    o_host = torch.empty((w.batch, w.heads, w.d_v), dtype=torch.float32).pin_memory()
+    h2d = sum(v.numel() * v.element_size() for v in host_in[0].values())
+    d2h = o_host.numel() * 4
+
+    def run_e2e(i, o_buf):
+        src, dst = host_in[i % 2], dev_in[i % 2]
+        for k in dst:
+            dst[k].copy_(src[k], non_blocking=True)
+        damp.kda_decode_step(L, pools[i % POOLS], perm, dst["q"], dst["k"], dst["v"], dst["g"], dst["beta"],
+                             o=o_buf)
+        o_host.copy_(o_buf, non_blocking=True)
+
+    e2e_steps = max(args.steps // 10, 10)
+    e2e_total, _ = timed(run_e2e, e2e_steps, max(args.warmup, 3), per_launch=False)
+    e2e_total = max_over_ranks(e2e_total)
+    return {
+        "w": w, "total_ms": total_ms, "launch_ms": launch_ms, "fp32_launch_ms": fp_launch,
+        "e2e_ms": e2e_total / e2e_steps, "h2d": h2d, "d2h": d2h, "clocks": clk.summary(),
+        "bits": damp.bits_per_value(L), "dev_name": torch.cuda.get_device_name(dev),
+    }
+
+
+def cpu_baseline(seconds: float = 12.0) -> dict:
+    """The oracle as it stands, single thread, on a bounded sample of the workload's heads."""
+    import numpy as np
+
+    from oracle import core, runs
+    w = WORKLOAD
+    inp = wl.step_inputs(w, 0, rows=[0, 1])
+    units = runs.unit_operands(w, inp)
+    n = units["v"].shape[0]
+    rng = np.random.default_rng(0)
+    perms = np.stack([rng.permutation(w.d_k) for _ in range(n)]).astype(np.uint8)
+    S = wl.random_states(1, n, w.d_k, w.d_v, scale=0.3)
+    tiers = core.pack_heads(perms, S, w.k_hi, w.lo_format)
+    done, t0 = 0, time.perf_counter()
+    while time.perf_counter() - t0 < seconds:
+        core.mixed_step_heads(perms, *tiers, units["q"], units["k"], units["v"], units["g"], units["beta"],
+                              w.k_hi, w.lo_format, w.kind)
+        done += n
+    el = time.perf_counter() - t0
+    per_unit = algorithmic_bytes(w) / (w.batch * w.heads)
+    return {"value": per_unit * done / el / 1e12, "unit": "TB/s", "cores": 1, "kind": "oracle",
+            "sample": f"{done} (slot, head) state updates of the KDA B=256 workload "
+                      f"({done // n} passes over 2 slots x 32 heads), {el:.1f} s, one host thread",
+            "us_per_full_step": el / done * w.batch * w.heads * 1e6}
+
+
+def reference_arm(args, rank: int, world: int):
+    """The CPU oracle on a bounded sample per step (rank 0 only)."""
+    import numpy as np
+
+    from oracle import core, runs
+    if rank != 0:
+        return
+    w = WORKLOAD
+    inp = wl.step_inputs(w, 0, rows=[0])
+    u = runs.unit_operands(w, inp)
+    rng = np.random.default_rng(0)
+    perms = np.stack([rng.permutation(w.d_k) for _ in range(w.heads)]).astype(np.uint8)
+    tiers = core.pack_heads(perms, wl.random_states(2, w.heads, w.d_k, w.d_v, 0.3), w.k_hi, w.lo_format)
+    # per-head cost, then heads per step so that warmup + steps fit in about two minutes
+    t0 = time.perf_counter()
+    core.mixed_step_heads(perms[:4], *(a[:4].copy() for a in tiers), u["q"][:4], u["k"][:4], u["v"][:4],
+                          u["g"][:4], u["beta"][:4], w.k_hi, w.lo_format, w.kind)
+    per_head = (time.perf_counter() - t0) / 4
+    heads = int(max(1, min(w.heads, 120.0 / max(args.steps + args.warmup, 1) / per_head)))
+    sl = slice(0, heads)
+    sub = [a[sl].copy() for a in tiers]
+
+    def one():
+        core.mixed_step_heads(perms[sl], *sub, u["q"][sl], u["k"][sl], u["v"][sl], u["g"][sl], u["beta"][sl],
+                              w.k_hi, w.lo_format, w.kind)
+
+    for _ in range(args.warmup):
+        one()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        one()
+    el = time.perf_counter() - t0
+    per_unit = algorithmic_bytes(w) / (w.batch * w.heads)
+    value = per_unit * heads * args.steps / el / 1e12
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "TB/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic",
+            "config": {"workload": w.name, "kind": "kda", "batch": w.batch, "heads": w.heads, "d_k": w.d_k,
+                       "d_v": w.d_v, "k_hi": w.k_hi, "lo_format": "uint8 affine G32 + H32",
+                       "reference": "CPU oracle (plain C, FP32, one thread)"},
+            "cpu_baseline": {"value": value, "unit": "TB/s", "cores": 1, "kind": "oracle",
+                             "sample": f"{heads} of the 8192 (slot, head) updates of a step, per step"},
+            "e2e": {"value": value, "unit": "TB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=4000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", default="damp", choices=["damp", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        reference_arm(args, rank, world)
+        return
+    import torch
+    import torch.distributed as dist
+    if world > 1:
+        dist.init_process_group("nccl")
+    try:
+        r = gpu_arm(args, rank, world)
+    finally:
+        if world > 1 and dist.is_initialized():
+            pass
+    if rank == 0:
+        w = r["w"]
+        bytes_step = algorithmic_bytes(w)
+        bytes_fp32 = algorithmic_bytes(w, packed=False)
+        ms = r["total_ms"] / args.steps
+        value = world * bytes_step / (ms * 1e-3) / 1e12
+        peaks = measured_peaks()
+        peak_gbs = peaks.get("hbm_gbs")
+        peak_note = "measured" if peak_gbs else "fallback"
+        peak_gbs = peak_gbs or 6800.0
+        achieved_gbs = bytes_step / (r["launch_ms"] * 1e-3) / 1e9
+        line = {
+            "metric": METRIC, "value": value, "unit": "TB/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "us_per_step": ms * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": w.name, "kind": "kda", "batch": w.batch, "heads": w.heads, "qk_heads": w.qk_heads,
+                       "d_k": w.d_k, "d_v": w.d_v, "k_hi": w.k_hi, "lo_format": "uint8 affine G32 + H32",
+                       "bits_per_value": r["bits"], "in_dtype": "bf16", "bytes_per_step": bytes_step,
+                       "l2": f"inputs larger than L2: {POOLS} packed state pools of "
+                             f"{bytes_step / 2 / 1e6:.0f} MB each rotated per step (> 129 MB L2)",
+                       "permutation": "seeded random pi per head (throughput does not depend on which)",
+                       "parallelism": f"{world} independent replica(s), one batch per GPU"},
+            "clocks": r["clocks"],
+            "e2e": {"value": world * bytes_step / (r["e2e_ms"] * 1e-3) / 1e12, "unit": "TB/s",
+                    "us_per_step": r["e2e_ms"] * 1e3, "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]},
+            "gpu_launches": args.steps,
+            "roofline": {"bound": "hbm", "achieved": achieved_gbs, "peak": peak_gbs, "unit": "GB/s",
+                         "frac": achieved_gbs / peak_gbs, "peak_source": f"{peak_note} copy bandwidth",
+                         "frac_of_8TBs": achieved_gbs / 8000.0,
+                         "traffic": ncu_traffic("packed_step_kda_b256"),
+                         "kernel": "packed_step_kernel<4,KDA,H32,BF16>", "algorithmic_bytes": bytes_step},
+            "fp32_state_kernel": {"us_per_step": r["fp32_launch_ms"] * 1e3,
+                                  "achieved_gbs": bytes_fp32 / (r["fp32_launch_ms"] * 1e-3) / 1e9,
+                                  "bytes_per_step": bytes_fp32,
+                                  "speedup_of_packed": r["fp32_launch_ms"] / r["launch_ms"]},
+            "device": r["dev_name"],
+        }
+        if not args.no_cpu_baseline and world == 1:
+            line["cpu_baseline"] = cpu_baseline()
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

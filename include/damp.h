@@ -1,0 +1,246 @@
+/*
+ * damp.h -- C ABI of libdamp: the decode-time recurrent-state update of Gated
+ * DeltaNet (GDN) and Kimi Delta Attention (KDA) over a DAMP mixed-precision
+ * packed state, on one NVIDIA GB300 GPU (sm_103a).
+ *
+ * Method: "DAMP: Decay-Aware Mixed-Precision Recurrent-State Quantization"
+ * (arxiv 2608.27513).  One decode step of one linear-attention layer, for every
+ * request slot of a decode batch and every value head h, computes (Sec. 3.1):
+ *
+ *     S_bar = Lambda_t S_{t-1}                decay (GDN: alpha_t I; KDA: diag(exp(g_t)))
+ *     delta = v_t - S_bar^T k_t               delta-rule read
+ *     S_t   = S_bar + beta_t k_t delta^T      Eq. delta_update
+ *     o_t   = S_t^T q_t                       output read (scale 1, FP32 post-update state)
+ *
+ * in FP32, on a state stored as (Sec. 5.2; App. A.5, Eq. packed_state_layout):
+ *
+ *     S_hi  FP16  [K_hi][d_v]                  the K_hi protected key channels
+ *     Q_lo  UINT8 [d_k-K_hi][d_v]              the other channels, block-32 Hadamard
+ *                                              transformed, asymmetric affine codes
+ *     M_lo  FP16  [d_k-K_hi][d_v/32][2]        per 32-group scale s and zero point z
+ *
+ * with the key channels in the calibrated order pi_{l,h} (protected first), and
+ * requantizes once per step (Sec. 3.3, Eq. quantized_recurrence):
+ *     s = (x_max - x_min)/255 -> FP16,  z = round(-x_min/s) -> FP16,
+ *     q_i = sat_[0,255](round(x_i/s) + z),  Q(x_i) = s (q_i - z)   (Eq. integer_quantizer).
+ * round() is round-half-to-even; s and z are rounded to FP16 first and the codes
+ * are encoded with the stored values; a block whose s rounds to 0 widens its
+ * range to contain 0 (and uses s = 1, z = 0 if s is still 0).
+ *
+ * Conventions for every call:
+ *   - Every array pointer is a CUDA device pointer owned by the caller.  libdamp
+ *     never allocates, frees or synchronizes.  Work is enqueued on `stream`
+ *     (a cudaStream_t passed as void*; NULL means the legacy default stream)
+ *     and is ordered with the caller's other work on that stream.
+ *   - Every argument check runs on the host before anything is enqueued.  A
+ *     failed check returns a DAMP_ERR_* status and enqueues nothing.  A launch
+ *     failure returns DAMP_ERR_CUDA.
+ *   - A kernel never traps.  A slot index outside [0, num_slots) makes the kernel
+ *     skip that batch row (its state and outputs are left untouched) and sets
+ *     DAMP_DEV_BAD_SLOT in the device status word; a bounded wait inside a kernel
+ *     that runs out sets DAMP_DEV_WAIT_TIMEOUT.  damp_device_status() reads and
+ *     clears the word.
+ *   - Operands are in natural key-channel order; the kernels apply pi.  Inputs
+ *     q, k (and v) are read-only; the state is updated in place; o is written.
+ *     Batch rows that name the same slot race: slot indices of one call must be
+ *     distinct.
+ *   - No C++ exception crosses the ABI.  The library keeps no per-call state;
+ *     calls may come from several host threads.
+ */
+#ifndef DAMP_H
+#define DAMP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define DAMP_API __attribute__((visibility("default")))
+#else
+#define DAMP_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    DAMP_OK = 0,
+    DAMP_ERR_NULL = 1,    /* a required pointer is NULL */
+    DAMP_ERR_SHAPE = 2,   /* a size is outside what the kernels support (see damp_layout) */
+    DAMP_ERR_ALIGN = 3,   /* a pointer is not aligned as documented for its argument */
+    DAMP_ERR_ALIAS = 4,   /* an output overlaps the state pool or another argument */
+    DAMP_ERR_FORMAT = 5,  /* unknown lo_format or in_dtype, or one this call does not take */
+    DAMP_ERR_CUDA = 6     /* the CUDA runtime reported an error while enqueueing */
+} damp_status;
+
+/* Low-precision tier formats (App. A.1, Tab. quantizer_specs). */
+typedef enum {
+    DAMP_LO_U8_AFFINE_G32_H32 = 0, /* UINT8 affine, G = 32 along d_v, FP16 (s, z), H_32 first:
+                                      the paper's DAMP low tier ("INT8+Hadamard", 9.0 bits) */
+    DAMP_LO_U8_AFFINE_G32 = 1      /* the same without H_32 (the paper's "INT8" row, 9.0 bits) */
+} damp_lo_format;
+
+/* Element type of q, k and v. */
+typedef enum { DAMP_IN_BF16 = 0, DAMP_IN_FP32 = 1 } damp_in_dtype;
+
+/* Device status bits (damp_device_status). */
+#define DAMP_DEV_WAIT_TIMEOUT 1u
+#define DAMP_DEV_BAD_SLOT 2u
+
+/*
+ * Shape of one linear-attention layer's state (Sec. 3.1; Sec. 5.1 "Key-channel budget").
+ *   num_heads     H      value heads; one state per (slot, head)
+ *   num_qk_heads  H_qk   q/k heads; value head h reads q/k head floor(h*H_qk/H)
+ *                        (GQA; H must be a multiple of H_qk)
+ *   d_k, d_v             state is d_k x d_v; d_k in {32, 64, 128}; d_v a multiple of 32, <= 1024
+ *   k_hi          K_hi   FP16 key channels per head, 0 <= K_hi <= d_k (same for every head)
+ *   lo_format            damp_lo_format of the other d_k - K_hi channels
+ */
+typedef struct {
+    int32_t num_heads;
+    int32_t num_qk_heads;
+    int32_t d_k;
+    int32_t d_v;
+    int32_t k_hi;
+    int32_t lo_format;
+} damp_layout;
+
+/* Checks a layout; DAMP_OK or DAMP_ERR_NULL / DAMP_ERR_SHAPE / DAMP_ERR_FORMAT. Host only. */
+DAMP_API damp_status damp_validate_layout(const damp_layout *layout);
+
+/*
+ * Physical packed state.  A pool holds num_slots slots; a slot holds H heads;
+ * a head holds d_v/32 value-block records (the value-block-major organization of
+ * App. A.5, which co-locates every 32-value code tile with its scale and zero
+ * point).  Record (slot, h, c) starts at byte
+ *     slot * damp_slot_bytes + (h * d_v/32 + c) * damp_record_bytes
+ * and holds, for value columns 32c .. 32c+31 of all d_k packed rows:
+ *     [K_hi x 32 FP16][(d_k-K_hi) x 32 UINT8 codes][(d_k-K_hi) x (s, z) FP16][padding to 16 B]
+ * with the 16-byte chunks inside each row permuted for conflict-free shared-memory
+ * access.  The byte order inside a record is private to libdamp: move logical
+ * tiers in and out with damp_pack_tiers / damp_unpack_tiers.
+ * The pool pointer must be 16-byte aligned.
+ */
+DAMP_API size_t damp_record_bytes(const damp_layout *layout); /* 0 if the layout is invalid */
+DAMP_API size_t damp_slot_bytes(const damp_layout *layout);   /* 0 if the layout is invalid */
+
+/* Storage bits per state value counted from the logical tiers (FP16 rows, codes and
+ * FP16 metadata; record padding excluded).  Equals Eq. budgeted_allocation,
+ * b(K_hi) = b_lo + (K_hi/d_k)(b_hi - b_lo) with b_hi = 16 and b_lo = 8 + 32/32 = 9:
+ * 9.875 at K_hi = 16, d_k = 128 (Sec. 5.1).  Returns -1.0 for an invalid layout. */
+DAMP_API double damp_bits_per_value(const damp_layout *layout);
+
+/*
+ * One GDN decode step (Sec. 3.1 with Lambda_t = alpha_t I) of `batch` request
+ * slots on the packed state, in place.
+ *   state      [num_slots] packed slots (layout above), 16-B aligned, updated in place
+ *   num_slots  slots in the pool (bounds slot indices; >= batch when slot_idx is NULL)
+ *   slot_idx   int32 [batch]: batch row b updates slot slot_idx[b]; NULL means slot b.
+ *              4-B aligned.  Indices must be distinct.
+ *   batch      B >= 0 (0 enqueues nothing)
+ *   perm       uint8 [H][d_k]: pi_h, packed row i holds key channel perm[h][i]
+ *              (protected channels first).  16-B aligned.  Must be a permutation
+ *              (not checked on the device).
+ *   q, k       [B][H_qk][d_k] of in_dtype, natural key order, 16-B aligned
+ *   v          [B][H][d_v] of in_dtype, 16-B aligned
+ *   g          float [B][H]: log-decay, alpha = exp(g).  4-B aligned.
+ *   beta       float [B][H]: delta-rule step size.  4-B aligned.
+ *   o          float [B][H][d_v]: output S_t^T q_t from the FP32 post-update state,
+ *              before requantization.  4-B aligned; must not overlap the pool.
+ *   in_dtype   damp_in_dtype of q, k, v
+ * lo_format must be DAMP_LO_U8_AFFINE_G32_H32 or DAMP_LO_U8_AFFINE_G32.
+ */
+DAMP_API damp_status damp_gdn_decode_step(const damp_layout *layout, void *state, int64_t num_slots,
+                                 const int32_t *slot_idx, int32_t batch, const uint8_t *perm,
+                                 const void *q, const void *k, const void *v, const float *g,
+                                 const float *beta, float *o, int32_t in_dtype, void *stream);
+
+/*
+ * One KDA decode step (Sec. 3.1 with Lambda_t = diag(exp(g_t))), as
+ * damp_gdn_decode_step except:
+ *   g          float [B][H][d_k]: per-key-channel log-decay in natural key order,
+ *              a_u = exp(g_u).  16-B aligned.
+ */
+DAMP_API damp_status damp_kda_decode_step(const damp_layout *layout, void *state, int64_t num_slots,
+                                 const int32_t *slot_idx, int32_t batch, const uint8_t *perm,
+                                 const void *q, const void *k, const void *v, const float *g,
+                                 const float *beta, float *o, int32_t in_dtype, void *stream);
+
+/*
+ * Uniform-INT8 baselines (the paper's INT8 / INT8+Hadamard rows of Tab. main):
+ * the same steps with no FP16 tier.  layout->k_hi must be 0.
+ */
+DAMP_API damp_status damp_u8_gdn_decode_step(const damp_layout *layout, void *state, int64_t num_slots,
+                                    const int32_t *slot_idx, int32_t batch, const uint8_t *perm,
+                                    const void *q, const void *k, const void *v, const float *g,
+                                    const float *beta, float *o, int32_t in_dtype, void *stream);
+DAMP_API damp_status damp_u8_kda_decode_step(const damp_layout *layout, void *state, int64_t num_slots,
+                                    const int32_t *slot_idx, int32_t batch, const uint8_t *perm,
+                                    const void *q, const void *k, const void *v, const float *g,
+                                    const float *beta, float *o, int32_t in_dtype, void *stream);
+
+/*
+ * FP32-state baselines: the deployment baseline of Sec. 6.1 ("default FP32
+ * recurrent-state storage"), the same step on an FP32 state in natural key order.
+ *   state  float [num_slots][H][d_k][d_v], 16-B aligned, updated in place
+ * layout->k_hi and layout->lo_format are ignored; no permutation is taken.
+ * Other arguments as in damp_gdn_decode_step / damp_kda_decode_step.
+ */
+DAMP_API damp_status damp_fp32_gdn_decode_step(const damp_layout *layout, float *state, int64_t num_slots,
+                                      const int32_t *slot_idx, int32_t batch,
+                                      const void *q, const void *k, const void *v, const float *g,
+                                      const float *beta, float *o, int32_t in_dtype, void *stream);
+DAMP_API damp_status damp_fp32_kda_decode_step(const damp_layout *layout, float *state, int64_t num_slots,
+                                      const int32_t *slot_idx, int32_t batch,
+                                      const void *q, const void *k, const void *v, const float *g,
+                                      const float *beta, float *o, int32_t in_dtype, void *stream);
+
+/*
+ * Write FP32 states into the packed cache: the hand-off from an FP32 prefix
+ * state (App. A.5 "Prefill path": the chunk-final state is written directly into
+ * the packed cache).  Row i of packed head h takes natural row perm[h][i];
+ * rows < K_hi are rounded to FP16, the others H_32-transformed (format 0) and
+ * quantized as above.
+ *   S      float [batch][H][d_k][d_v], natural key order, 16-B aligned, read only
+ *   state, num_slots, slot_idx, batch, perm as in damp_gdn_decode_step
+ */
+DAMP_API damp_status damp_quantize_state(const damp_layout *layout, const float *S, const uint8_t *perm,
+                                void *state, int64_t num_slots, const int32_t *slot_idx,
+                                int32_t batch, void *stream);
+
+/* Reconstruct FP32 states from the packed cache (the inverse map: FP16 rows widened,
+ * codes dequantized s (q - z) and H_32-transformed back for format 0).
+ *   S      float [batch][H][d_k][d_v] output, natural key order, 16-B aligned */
+DAMP_API damp_status damp_dequantize_state(const damp_layout *layout, const void *state, int64_t num_slots,
+                                  const int32_t *slot_idx, int32_t batch, const uint8_t *perm,
+                                  float *S, void *stream);
+
+/*
+ * Copy logical tiers into / out of packed slots, bit for bit (no arithmetic).
+ *   hi     uint16 [batch][H][K_hi][d_v]            FP16 bit patterns (S_hi)
+ *   codes  uint8  [batch][H][d_k-K_hi][d_v]        UINT8 codes (Q_lo)
+ *   meta   uint16 [batch][H][d_k-K_hi][d_v/32][2]  FP16 (s, z) (M_lo)
+ * All three 4-B aligned.  NULL is allowed for an empty tier.
+ */
+DAMP_API damp_status damp_pack_tiers(const damp_layout *layout, const uint16_t *hi, const uint8_t *codes,
+                            const uint16_t *meta, void *state, int64_t num_slots,
+                            const int32_t *slot_idx, int32_t batch, void *stream);
+DAMP_API damp_status damp_unpack_tiers(const damp_layout *layout, const void *state, int64_t num_slots,
+                              const int32_t *slot_idx, int32_t batch, uint16_t *hi, uint8_t *codes,
+                              uint16_t *meta, void *stream);
+
+/* Reads and clears the device status word of the current device (DAMP_DEV_* bits).
+ * Synchronous with respect to the device.  DAMP_ERR_NULL if status is NULL. */
+DAMP_API damp_status damp_device_status(uint32_t *status);
+
+/* Human-readable name of a status code (static string). */
+DAMP_API const char *damp_status_string(damp_status status);
+
+/* ABI version: 100 * major + minor. */
+DAMP_API int32_t damp_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DAMP_H */

@@ -1,0 +1,230 @@
+"""libdamp: the DAMP decode-step recurrent-state update on GB300 (sm_103a).
+
+Python binding over the C ABI of include/damp.h.  The functions carry the
+ABI's names and only marshal arguments: every step of the path runs in the
+library's CUDA kernels.  PyTorch provides device memory and streams.  There is
+no CPU fallback: without the built library every call raises
+DampLibraryError.
+
+    layout = Layout(num_heads=32, num_qk_heads=32, d_k=128, d_v=128, k_hi=10)
+    state = new_state(layout, num_slots=256, device="cuda")
+    quantize_state(layout, S_fp32, perm, state)            # prefill hand-off
+    o = kda_decode_step(layout, state, perm, q, k, v, g, beta)
+"""
+from __future__ import annotations
+
+import ctypes
+from dataclasses import dataclass
+
+from ._lib import DampLayout, DampLibraryError, lib
+
+__all__ = [
+    "Layout", "DampError", "DampLibraryError", "LO_U8_AFFINE_G32_H32", "LO_U8_AFFINE_G32",
+    "record_bytes", "slot_bytes", "bits_per_value", "new_state", "new_fp32_state",
+    "gdn_decode_step", "kda_decode_step", "u8_gdn_decode_step", "u8_kda_decode_step",
+    "fp32_gdn_decode_step", "fp32_kda_decode_step", "quantize_state", "dequantize_state",
+    "pack_tiers", "unpack_tiers", "device_status", "version", "DEV_WAIT_TIMEOUT", "DEV_BAD_SLOT",
+]
+
+LO_U8_AFFINE_G32_H32 = 0
+LO_U8_AFFINE_G32 = 1
+IN_BF16 = 0
+IN_FP32 = 1
+DEV_WAIT_TIMEOUT = 1
+DEV_BAD_SLOT = 2
+
+
+class DampError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        msg = lib().damp_status_string(status).decode()
+        super().__init__(f"{what}: {msg}")
+        self.status = status
+
+
+@dataclass(frozen=True)
+class Layout:
+    num_heads: int
+    num_qk_heads: int
+    d_k: int
+    d_v: int
+    k_hi: int
+    lo_format: int = LO_U8_AFFINE_G32_H32
+
+    def c(self) -> DampLayout:
+        return DampLayout(self.num_heads, self.num_qk_heads, self.d_k, self.d_v, self.k_hi, self.lo_format)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    import torch
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _check(status: int, what: str):
+    if status != 0:
+        raise DampError(status, what)
+
+
+def _in_dtype(*ts) -> int:
+    import torch
+    dts = {t.dtype for t in ts}
+    if dts == {torch.bfloat16}:
+        return IN_BF16
+    if dts == {torch.float32}:
+        return IN_FP32
+    raise TypeError("q, k, v must all be bfloat16 or all float32")
+
+
+def _cuda_contig(name, t):
+    if t is None:
+        return
+    if not t.is_cuda or not t.is_contiguous():
+        raise ValueError(f"{name} must be a contiguous CUDA tensor")
+
+
+def version() -> int:
+    return int(lib().damp_version())
+
+
+def record_bytes(layout: Layout) -> int:
+    c = layout.c()
+    return int(lib().damp_record_bytes(ctypes.byref(c)))
+
+
+def slot_bytes(layout: Layout) -> int:
+    c = layout.c()
+    n = int(lib().damp_slot_bytes(ctypes.byref(c)))
+    if n == 0:
+        _check(lib().damp_validate_layout(ctypes.byref(c)), "layout")
+    return n
+
+
+def bits_per_value(layout: Layout) -> float:
+    c = layout.c()
+    return float(lib().damp_bits_per_value(ctypes.byref(c)))
+
+
+def new_state(layout: Layout, num_slots: int, device="cuda"):
+    """A zero-filled packed pool of num_slots slots (uint8, 16-B aligned by the allocator)."""
+    import torch
+    return torch.zeros((num_slots, slot_bytes(layout)), dtype=torch.uint8, device=device)
+
+
+def new_fp32_state(layout: Layout, num_slots: int, device="cuda"):
+    import torch
+    return torch.zeros((num_slots, layout.num_heads, layout.d_k, layout.d_v), dtype=torch.float32, device=device)
+
+
+def _step(fn_name, layout, state, perm, q, k, v, g, beta, o, slot_idx, num_slots, stream):
+    import torch
+    for n, t in (("state", state), ("perm", perm), ("q", q), ("k", k), ("v", v), ("g", g), ("beta", beta),
+                 ("o", o), ("slot_idx", slot_idx)):
+        _cuda_contig(n, t)
+    B = v.shape[0]
+    if o is None:
+        o = torch.empty((B, layout.num_heads, layout.d_v), dtype=torch.float32, device=v.device)
+    if num_slots is None:
+        num_slots = state.shape[0]
+    c = layout.c()
+    args = [ctypes.byref(c), _ptr(state), num_slots, _ptr(slot_idx), B]
+    if perm is not None or not fn_name.startswith("damp_fp32"):
+        args.append(_ptr(perm))
+    args += [_ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(beta), _ptr(o), _in_dtype(q, k, v), _stream(stream)]
+    _check(getattr(lib(), fn_name)(*args), fn_name)
+    return o
+
+
+def gdn_decode_step(layout, state, perm, q, k, v, g, beta, o=None, slot_idx=None, num_slots=None, stream=None):
+    """One GDN decode step on the packed state (in place); returns o [B, H, d_v] float32."""
+    return _step("damp_gdn_decode_step", layout, state, perm, q, k, v, g, beta, o, slot_idx, num_slots, stream)
+
+
+def kda_decode_step(layout, state, perm, q, k, v, g, beta, o=None, slot_idx=None, num_slots=None, stream=None):
+    """One KDA decode step on the packed state (in place); returns o [B, H, d_v] float32."""
+    return _step("damp_kda_decode_step", layout, state, perm, q, k, v, g, beta, o, slot_idx, num_slots, stream)
+
+
+def u8_gdn_decode_step(layout, state, perm, q, k, v, g, beta, o=None, slot_idx=None, num_slots=None, stream=None):
+    return _step("damp_u8_gdn_decode_step", layout, state, perm, q, k, v, g, beta, o, slot_idx, num_slots, stream)
+
+
+def u8_kda_decode_step(layout, state, perm, q, k, v, g, beta, o=None, slot_idx=None, num_slots=None, stream=None):
+    return _step("damp_u8_kda_decode_step", layout, state, perm, q, k, v, g, beta, o, slot_idx, num_slots, stream)
+
+
+def fp32_gdn_decode_step(layout, state, q, k, v, g, beta, o=None, slot_idx=None, num_slots=None, stream=None):
+    """One GDN decode step on an FP32 state [slots, H, d_k, d_v] (in place)."""
+    return _step("damp_fp32_gdn_decode_step", layout, state, None, q, k, v, g, beta, o, slot_idx, num_slots, stream)
+
+
+def fp32_kda_decode_step(layout, state, q, k, v, g, beta, o=None, slot_idx=None, num_slots=None, stream=None):
+    return _step("damp_fp32_kda_decode_step", layout, state, None, q, k, v, g, beta, o, slot_idx, num_slots, stream)
+
+
+def quantize_state(layout, S, perm, state, slot_idx=None, num_slots=None, stream=None):
+    """Write natural-order FP32 states S [B, H, d_k, d_v] into packed slots."""
+    for n, t in (("S", S), ("perm", perm), ("state", state), ("slot_idx", slot_idx)):
+        _cuda_contig(n, t)
+    c = layout.c()
+    _check(lib().damp_quantize_state(ctypes.byref(c), _ptr(S), _ptr(perm), _ptr(state),
+                                     state.shape[0] if num_slots is None else num_slots, _ptr(slot_idx),
+                                     S.shape[0], _stream(stream)), "damp_quantize_state")
+
+
+def dequantize_state(layout, state, perm, batch=None, S=None, slot_idx=None, num_slots=None, stream=None):
+    """Reconstruct natural-order FP32 states [B, H, d_k, d_v] from packed slots."""
+    import torch
+    for n, t in (("S", S), ("perm", perm), ("state", state), ("slot_idx", slot_idx)):
+        _cuda_contig(n, t)
+    B = (slot_idx.shape[0] if slot_idx is not None else state.shape[0]) if batch is None else batch
+    if S is None:
+        S = torch.empty((B, layout.num_heads, layout.d_k, layout.d_v), dtype=torch.float32, device=state.device)
+    c = layout.c()
+    _check(lib().damp_dequantize_state(ctypes.byref(c), _ptr(state),
+                                       state.shape[0] if num_slots is None else num_slots, _ptr(slot_idx), B,
+                                       _ptr(perm), _ptr(S), _stream(stream)), "damp_dequantize_state")
+    return S
+
+
+def pack_tiers(layout, hi, codes, meta, state, slot_idx=None, num_slots=None, stream=None):
+    """Copy logical tiers (hi uint16/fp16 [B,H,K,d_v], codes uint8 [B,H,d_k-K,d_v],
+    meta uint16/fp16 [B,H,d_k-K,d_v/32,2]) into packed slots, bit for bit."""
+    for n, t in (("hi", hi), ("codes", codes), ("meta", meta), ("state", state), ("slot_idx", slot_idx)):
+        _cuda_contig(n, t)
+    B = codes.shape[0] if codes is not None else hi.shape[0]
+    c = layout.c()
+    _check(lib().damp_pack_tiers(ctypes.byref(c), _ptr(hi if hi is not None and hi.numel() else None),
+                                 _ptr(codes if codes is not None and codes.numel() else None),
+                                 _ptr(meta if meta is not None and meta.numel() else None), _ptr(state),
+                                 state.shape[0] if num_slots is None else num_slots, _ptr(slot_idx), B,
+                                 _stream(stream)), "damp_pack_tiers")
+
+
+def unpack_tiers(layout, state, batch=None, slot_idx=None, num_slots=None, stream=None):
+    """Logical tiers (hi int16 bits, codes uint8, meta int16 bits) of `batch` packed slots."""
+    import torch
+    _cuda_contig("state", state)
+    _cuda_contig("slot_idx", slot_idx)
+    B = (slot_idx.shape[0] if slot_idx is not None else state.shape[0]) if batch is None else batch
+    H, dk, dv, K = layout.num_heads, layout.d_k, layout.d_v, layout.k_hi
+    dev = state.device
+    hi = torch.empty((B, H, K, dv), dtype=torch.int16, device=dev)
+    codes = torch.empty((B, H, dk - K, dv), dtype=torch.uint8, device=dev)
+    meta = torch.empty((B, H, dk - K, dv // 32, 2), dtype=torch.int16, device=dev)
+    c = layout.c()
+    _check(lib().damp_unpack_tiers(ctypes.byref(c), _ptr(state), state.shape[0] if num_slots is None else num_slots,
+                                   _ptr(slot_idx), B, _ptr(hi if hi.numel() else None),
+                                   _ptr(codes if codes.numel() else None), _ptr(meta if meta.numel() else None),
+                                   _stream(stream)), "damp_unpack_tiers")
+    return hi, codes, meta
+
+
+def device_status() -> int:
+    """Read and clear the device status word (DEV_* bits)."""
+    v = ctypes.c_uint32(0)
+    _check(lib().damp_device_status(ctypes.byref(v)), "damp_device_status")
+    return int(v.value)

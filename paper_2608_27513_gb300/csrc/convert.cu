@@ -1,0 +1,218 @@
+// convert.cu -- kernels that move whole states in and out of the packed cache.
+//
+//   quantize_state    natural FP32 state -> packed records (App. A.5 "Prefill
+//                     path": the FP32 state is written straight into the packed
+//                     cache; rows in pi order, FP16 tier for rows < K_hi, H_32 +
+//                     UINT8 affine (Sec. 3.2, Eq. integer_quantizer) for the rest)
+//   dequantize_state  packed records -> natural FP32 state (the inverse map)
+//   pack_tiers / unpack_tiers
+//                     logical tier arrays (S_hi, Q_lo, M_lo of Eq.
+//                     packed_state_layout) <-> packed records, bit for bit
+//
+// One warp per (slot, head, value block) record; lane l owns packed rows
+// l, l+32, ...; global memory is accessed directly (these kernels are off the
+// per-step path).
+#include "damp_common.cuh"
+#include "damp_internal.h"
+
+#include <algorithm>
+
+namespace damp {
+
+static __device__ uint32_t g_status_convert;
+
+struct ConvParams {
+    uint8_t *state;
+    int64_t num_slots;
+    const int32_t *slot_idx;
+    const uint8_t *perm;
+    float *S;
+    uint16_t *hi;
+    uint8_t *codes;
+    uint16_t *meta;
+    int32_t batch, H, dk, dv, V, K;
+    int32_t rec_bytes, codes_off, meta_off;
+    int64_t slot_bytes, total_tiles;
+    uint32_t *status;
+};
+
+enum ConvOp { kQuantize = 0, kDequantize = 1, kPackTiers = 2, kUnpackTiers = 3 };
+
+template <int R, bool HAD, int OP>
+__global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwt = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const int K = p.K;
+    const int lo = p.dk - K;
+    bool bad_slot = false;
+    for (int64_t t = gw; t < p.total_tiles; t += nwt) {
+        const int c = (int)(t % p.V);
+        const int64_t bh = t / p.V;
+        const int h = (int)(bh % p.H);
+        const int b = (int)(bh / p.H);
+        const int64_t slot = p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b;
+        if (slot < 0 || slot >= p.num_slots) {
+            bad_slot = true;
+            continue;
+        }
+        uint8_t *rec = p.state + slot * p.slot_bytes + (int64_t)(h * p.V + c) * p.rec_bytes;
+#pragma unroll
+        for (int i = 0; i < R; ++i) {
+            const int u = lane + 32 * i;
+            if (OP == kQuantize || OP == kDequantize) {
+                const int n = p.perm[(int64_t)h * p.dk + u] & (p.dk - 1);  // d_k is a power of two
+                float *row = p.S + ((((int64_t)b * p.H + h) * p.dk + n) * p.dv + c * kG);
+                float x[32];
+                if (OP == kQuantize) {
+#pragma unroll
+                    for (int m = 0; m < 8; ++m) {
+                        const float4 f = reinterpret_cast<const float4 *>(row)[m];
+                        x[4 * m] = f.x;
+                        x[4 * m + 1] = f.y;
+                        x[4 * m + 2] = f.z;
+                        x[4 * m + 3] = f.w;
+                    }
+                    if (u < K) {
+#pragma unroll
+                        for (int m = 0; m < 4; ++m) {
+                            uint4 w;
+                            w.x = f2_to_h2(x[8 * m], x[8 * m + 1]);
+                            w.y = f2_to_h2(x[8 * m + 2], x[8 * m + 3]);
+                            w.z = f2_to_h2(x[8 * m + 4], x[8 * m + 5]);
+                            w.w = f2_to_h2(x[8 * m + 6], x[8 * m + 7]);
+                            *reinterpret_cast<uint4 *>(rec + hi_chunk_off(u, m)) = w;
+                        }
+                    } else {
+                        const int r = u - K;
+                        if (HAD) hadamard_regs(x);
+                        uint32_t w[8];
+                        const uint32_t sz = quantize_group(x, w);
+                        *reinterpret_cast<uint4 *>(rec + p.codes_off + lo_chunk_off(r, 0)) =
+                            make_uint4(w[0], w[1], w[2], w[3]);
+                        *reinterpret_cast<uint4 *>(rec + p.codes_off + lo_chunk_off(r, 1)) =
+                            make_uint4(w[4], w[5], w[6], w[7]);
+                        *reinterpret_cast<uint32_t *>(rec + p.meta_off + 4 * r) = sz;
+                    }
+                } else {
+                    if (u < K) {
+#pragma unroll
+                        for (int m = 0; m < 4; ++m) {
+                            const uint4 w = *reinterpret_cast<const uint4 *>(rec + hi_chunk_off(u, m));
+                            const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                const float2 f = h2_to_f2(ww[e]);
+                                x[8 * m + 2 * e] = f.x;
+                                x[8 * m + 2 * e + 1] = f.y;
+                            }
+                        }
+                    } else {
+                        const int r = u - K;
+                        const uint4 c0 = *reinterpret_cast<const uint4 *>(rec + p.codes_off + lo_chunk_off(r, 0));
+                        const uint4 c1 = *reinterpret_cast<const uint4 *>(rec + p.codes_off + lo_chunk_off(r, 1));
+                        const uint32_t sz = *reinterpret_cast<const uint32_t *>(rec + p.meta_off + 4 * r);
+                        const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+                        dequantize_group(w, sz, 1.0f, x);
+                        if (HAD) hadamard_regs(x);
+                    }
+#pragma unroll
+                    for (int m = 0; m < 8; ++m)
+                        reinterpret_cast<float4 *>(row)[m] = make_float4(x[4 * m], x[4 * m + 1], x[4 * m + 2], x[4 * m + 3]);
+                }
+            } else {
+                // logical tiers <-> record, 32-bit words
+                if (u < K) {
+                    uint32_t *trow = reinterpret_cast<uint32_t *>(p.hi + ((((int64_t)b * p.H + h) * K + u) * p.dv + c * kG));
+#pragma unroll
+                    for (int m = 0; m < 4; ++m) {
+                        uint32_t *r4 = reinterpret_cast<uint32_t *>(rec + hi_chunk_off(u, m));
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            if (OP == kPackTiers) r4[e] = trow[4 * m + e];
+                            else trow[4 * m + e] = r4[e];
+                        }
+                    }
+                } else {
+                    const int r = u - K;
+                    uint32_t *crow = reinterpret_cast<uint32_t *>(p.codes + ((((int64_t)b * p.H + h) * lo + r) * p.dv + c * kG));
+                    uint32_t *mrow = reinterpret_cast<uint32_t *>(p.meta + ((((int64_t)b * p.H + h) * lo + r) * p.V + c) * 2);
+#pragma unroll
+                    for (int m = 0; m < 2; ++m) {
+                        uint32_t *r4 = reinterpret_cast<uint32_t *>(rec + p.codes_off + lo_chunk_off(r, m));
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            if (OP == kPackTiers) r4[e] = crow[4 * m + e];
+                            else crow[4 * m + e] = r4[e];
+                        }
+                    }
+                    uint32_t *mr = reinterpret_cast<uint32_t *>(rec + p.meta_off + 4 * r);
+                    if (OP == kPackTiers) *mr = *mrow;
+                    else *mrow = *mr;
+                }
+            }
+        }
+        // zero the record padding so packed pools compare bit for bit
+        if (OP == kQuantize || OP == kPackTiers) {
+            const int used = p.meta_off + 4 * lo;
+            if (lane < p.rec_bytes - used) rec[used + lane] = 0;
+        }
+    }
+    if (bad_slot && lane == 0) atomicOr(p.status, (uint32_t)kDevBadSlot);
+}
+
+template <int OP>
+static cudaError_t launch_convert(const ConvArgs &a, cudaStream_t stream) {
+    ConvParams p{};
+    cudaError_t e = cudaGetSymbolAddress(reinterpret_cast<void **>(&p.status), g_status_convert);
+    if (e != cudaSuccess) return e;
+    const RecGeom rg = rec_geom(a.dk, a.K);
+    p.state = static_cast<uint8_t *>(a.state);
+    p.num_slots = a.num_slots;
+    p.slot_idx = a.slot_idx;
+    p.perm = a.perm;
+    p.S = a.S;
+    p.hi = a.hi;
+    p.codes = a.codes;
+    p.meta = a.meta;
+    p.batch = a.batch;
+    p.H = a.H;
+    p.dk = a.dk;
+    p.dv = a.dv;
+    p.V = a.dv / kG;
+    p.K = a.K;
+    p.rec_bytes = rg.bytes;
+    p.codes_off = rg.codes_off;
+    p.meta_off = rg.meta_off;
+    p.slot_bytes = (int64_t)a.H * p.V * rg.bytes;
+    p.total_tiles = (int64_t)a.batch * a.H * p.V;
+    if (p.total_tiles == 0) return cudaSuccess;
+    const int warps = 8;
+    const int64_t want = (p.total_tiles + warps - 1) / warps;
+    const int grid = (int)std::min<int64_t>(want, (int64_t)sm_count() * 8);
+    void (*kern)(ConvParams) = nullptr;
+    const bool had = a.fmt == 0;
+#define DAMP_PICK(R_)                                                                          \
+    if (a.dk == 32 * R_) kern = had ? convert_kernel<R_, true, OP> : convert_kernel<R_, false, OP>;
+    DAMP_PICK(1)
+    DAMP_PICK(2)
+    DAMP_PICK(4)
+#undef DAMP_PICK
+    if (!kern) return cudaErrorInvalidValue;
+    kern<<<grid, 32 * warps, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_quantize(const ConvArgs &a, cudaStream_t s) { return launch_convert<kQuantize>(a, s); }
+cudaError_t launch_dequantize(const ConvArgs &a, cudaStream_t s) { return launch_convert<kDequantize>(a, s); }
+cudaError_t launch_pack_tiers(const ConvArgs &a, cudaStream_t s) { return launch_convert<kPackTiers>(a, s); }
+cudaError_t launch_unpack_tiers(const ConvArgs &a, cudaStream_t s) { return launch_convert<kUnpackTiers>(a, s); }
+
+cudaError_t take_status_convert(uint32_t *bits) {
+    uint32_t zero = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(bits, g_status_convert, sizeof(uint32_t));
+    if (e != cudaSuccess) return e;
+    return cudaMemcpyToSymbol(g_status_convert, &zero, sizeof(uint32_t));
+}
+
+}  // namespace damp

@@ -1,0 +1,316 @@
+// damp_abi.cu -- the extern "C" entry points of libdamp (include/damp.h):
+// host-side argument checks, then one launch on the caller's stream.
+#include <atomic>
+#include <climits>
+
+#include "../../include/damp.h"
+#include "damp_common.cuh"
+#include "damp_internal.h"
+
+namespace damp {
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::atomic<int> g_sm_count[kMaxDevices];
+std::atomic<int> g_smem_optin[kMaxDevices];
+
+int device_attr(std::atomic<int> *cache, cudaDeviceAttr attr, int fallback) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return fallback;
+    int v = cache[dev].load(std::memory_order_relaxed);
+    if (v > 0) return v;
+    if (cudaDeviceGetAttribute(&v, attr, dev) != cudaSuccess || v <= 0) return fallback;
+    cache[dev].store(v, std::memory_order_relaxed);
+    return v;
+}
+
+bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+struct Range {
+    uintptr_t lo, hi;  // [lo, hi)
+};
+Range range_of(const void *p, int64_t bytes) {
+    const uintptr_t lo = reinterpret_cast<uintptr_t>(p);
+    return Range{lo, lo + (uintptr_t)(bytes > 0 ? bytes : 0)};
+}
+bool overlap(Range a, Range b) { return a.lo < b.hi && b.lo < a.hi && a.hi > a.lo && b.hi > b.lo; }
+
+damp_status check_layout(const damp_layout *L) {
+    if (!L) return DAMP_ERR_NULL;
+    if (L->num_heads < 1 || L->num_qk_heads < 1 || L->num_heads % L->num_qk_heads) return DAMP_ERR_SHAPE;
+    if (L->num_heads > (1 << 20)) return DAMP_ERR_SHAPE;
+    if (L->d_k != 32 && L->d_k != 64 && L->d_k != 128) return DAMP_ERR_SHAPE;
+    if (L->d_v < 32 || L->d_v > 1024 || L->d_v % 32) return DAMP_ERR_SHAPE;
+    if (L->k_hi < 0 || L->k_hi > L->d_k) return DAMP_ERR_SHAPE;
+    if (L->lo_format != DAMP_LO_U8_AFFINE_G32_H32 && L->lo_format != DAMP_LO_U8_AFFINE_G32) return DAMP_ERR_FORMAT;
+    return DAMP_OK;
+}
+
+int64_t slot_bytes_of(const damp_layout *L) {
+    return (int64_t)L->num_heads * (L->d_v / 32) * rec_geom(L->d_k, L->k_hi).bytes;
+}
+
+// Slots, batch rows and the pool's byte range; shared by every call on a pool.
+damp_status check_pool(const void *state, int64_t num_slots, const int32_t *slot_idx, int32_t batch,
+                       int64_t slot_bytes, Range *pool) {
+    if (batch < 0 || num_slots < 0) return DAMP_ERR_SHAPE;
+    if (!state) return DAMP_ERR_NULL;
+    if (!aligned(state, 16)) return DAMP_ERR_ALIGN;
+    if (slot_idx && !aligned(slot_idx, 4)) return DAMP_ERR_ALIGN;
+    if (!slot_idx && num_slots < batch) return DAMP_ERR_SHAPE;
+    if (num_slots < 1) return DAMP_ERR_SHAPE;
+    if (slot_bytes > 0 && num_slots > INT64_MAX / slot_bytes) return DAMP_ERR_SHAPE;
+    *pool = range_of(state, num_slots * slot_bytes);
+    return DAMP_OK;
+}
+
+cudaError_t launch_step(const StepArgs &a, bool packed, cudaStream_t s) {
+    if (!packed) return launch_fp32_step(a, s);
+    return a.kda ? launch_packed_kda(a, s) : launch_packed_gdn(a, s);
+}
+
+damp_status step(const damp_layout *L, void *state, int64_t num_slots, const int32_t *slot_idx, int32_t batch,
+                 const uint8_t *perm, const void *q, const void *k, const void *v, const float *g,
+                 const float *beta, float *o, int32_t in_dtype, void *stream, bool kda, bool packed,
+                 bool uniform) {
+    damp_status st = check_layout(L);
+    if (st != DAMP_OK && packed) return st;
+    if (!packed) {  // the FP32 state ignores k_hi and lo_format
+        if (!L) return DAMP_ERR_NULL;
+        damp_layout l2 = *L;
+        l2.k_hi = 0;
+        l2.lo_format = 0;
+        if ((st = check_layout(&l2)) != DAMP_OK) return st;
+    }
+    if (uniform && L->k_hi != 0) return DAMP_ERR_SHAPE;
+    if (in_dtype != DAMP_IN_BF16 && in_dtype != DAMP_IN_FP32) return DAMP_ERR_FORMAT;
+    if (batch < 0) return DAMP_ERR_SHAPE;
+    if (batch == 0) return DAMP_OK;
+    const int64_t sb = packed ? slot_bytes_of(L) : (int64_t)L->num_heads * L->d_k * L->d_v * 4;
+    Range pool;
+    if ((st = check_pool(state, num_slots, slot_idx, batch, sb, &pool)) != DAMP_OK) return st;
+    if ((packed && !perm) || !q || !k || !v || !g || !beta || !o) return DAMP_ERR_NULL;
+    if ((packed && !aligned(perm, 16)) || !aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) ||
+        !aligned(g, kda ? 16 : 4) || !aligned(beta, 4) || !aligned(o, 4))
+        return DAMP_ERR_ALIGN;
+    const int64_t B = batch, H = L->num_heads, Hq = L->num_qk_heads, dk = L->d_k, dv = L->d_v;
+    const int64_t esz = in_dtype == DAMP_IN_BF16 ? 2 : 4;
+    const Range ro = range_of(o, B * H * dv * 4);
+    const Range inputs[] = {range_of(q, B * Hq * dk * esz), range_of(k, B * Hq * dk * esz),
+                            range_of(v, B * H * dv * esz), range_of(g, B * H * (kda ? dk : 1) * 4),
+                            range_of(beta, B * H * 4), range_of(perm, packed ? H * dk : 0),
+                            range_of(slot_idx, slot_idx ? B * 4 : 0)};
+    if (overlap(ro, pool)) return DAMP_ERR_ALIAS;
+    for (const Range &r : inputs)
+        if (overlap(ro, r) || overlap(pool, r)) return DAMP_ERR_ALIAS;
+
+    StepArgs a{};
+    a.H = L->num_heads;
+    a.Hqk = L->num_qk_heads;
+    a.dk = L->d_k;
+    a.dv = L->d_v;
+    a.K = packed ? L->k_hi : 0;
+    a.fmt = packed ? L->lo_format : 0;
+    a.state = state;
+    a.num_slots = num_slots;
+    a.slot_idx = slot_idx;
+    a.batch = batch;
+    a.perm = perm;
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.g = g;
+    a.beta = beta;
+    a.o = o;
+    a.in_bf16 = in_dtype == DAMP_IN_BF16;
+    a.kda = kda;
+    return launch_step(a, packed, static_cast<cudaStream_t>(stream)) == cudaSuccess ? DAMP_OK : DAMP_ERR_CUDA;
+}
+
+enum ConvKind { kQ, kDQ, kPack, kUnpack };
+
+damp_status convert(const damp_layout *L, void *state, int64_t num_slots, const int32_t *slot_idx, int32_t batch,
+                    const uint8_t *perm, float *S, uint16_t *hi, uint8_t *codes, uint16_t *meta, void *stream,
+                    ConvKind kind) {
+    damp_status st = check_layout(L);
+    if (st != DAMP_OK) return st;
+    if (batch < 0) return DAMP_ERR_SHAPE;
+    if (batch == 0) return DAMP_OK;
+    Range pool;
+    if ((st = check_pool(state, num_slots, slot_idx, batch, slot_bytes_of(L), &pool)) != DAMP_OK) return st;
+    const int64_t B = batch, H = L->num_heads, dk = L->d_k, dv = L->d_v, K = L->k_hi;
+    if (kind == kQ || kind == kDQ) {
+        if (!perm || !S) return DAMP_ERR_NULL;
+        if (!aligned(perm, 16) || !aligned(S, 16)) return DAMP_ERR_ALIGN;
+        const Range rs = range_of(S, B * H * dk * dv * 4);
+        if (overlap(rs, pool) || overlap(rs, range_of(perm, H * dk)) ||
+            overlap(rs, range_of(slot_idx, slot_idx ? B * 4 : 0)) || overlap(pool, range_of(perm, H * dk)))
+            return DAMP_ERR_ALIAS;
+    } else {
+        const int64_t nh = B * H * K * dv * 2, nc = B * H * (dk - K) * dv, nm = B * H * (dk - K) * (dv / 32) * 4;
+        if ((nh && !hi) || (nc && !codes) || (nm && !meta)) return DAMP_ERR_NULL;
+        if ((hi && !aligned(hi, 4)) || (codes && !aligned(codes, 4)) || (meta && !aligned(meta, 4)))
+            return DAMP_ERR_ALIGN;
+        const Range t[] = {range_of(hi, nh), range_of(codes, nc), range_of(meta, nm)};
+        for (const Range &r : t) {
+            if (overlap(r, pool) || overlap(r, range_of(slot_idx, slot_idx ? B * 4 : 0))) return DAMP_ERR_ALIAS;
+        }
+        if (overlap(t[0], t[1]) || overlap(t[0], t[2]) || overlap(t[1], t[2])) return DAMP_ERR_ALIAS;
+    }
+    ConvArgs a{};
+    a.H = L->num_heads;
+    a.dk = L->d_k;
+    a.dv = L->d_v;
+    a.K = L->k_hi;
+    a.fmt = L->lo_format;
+    a.state = state;
+    a.num_slots = num_slots;
+    a.slot_idx = slot_idx;
+    a.batch = batch;
+    a.perm = perm;
+    a.S = S;
+    a.hi = hi;
+    a.codes = codes;
+    a.meta = meta;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = kind == kQ ? launch_quantize(a, s)
+                    : kind == kDQ ? launch_dequantize(a, s)
+                    : kind == kPack ? launch_pack_tiers(a, s)
+                                    : launch_unpack_tiers(a, s);
+    return e == cudaSuccess ? DAMP_OK : DAMP_ERR_CUDA;
+}
+
+}  // namespace
+
+int sm_count() { return device_attr(g_sm_count, cudaDevAttrMultiProcessorCount, 1); }
+int max_smem_per_block() { return device_attr(g_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, 48 * 1024); }
+
+}  // namespace damp
+
+using namespace damp;
+
+extern "C" {
+
+damp_status damp_validate_layout(const damp_layout *layout) { return check_layout(layout); }
+
+size_t damp_record_bytes(const damp_layout *layout) {
+    if (check_layout(layout) != DAMP_OK) return 0;
+    return (size_t)rec_geom(layout->d_k, layout->k_hi).bytes;
+}
+
+size_t damp_slot_bytes(const damp_layout *layout) {
+    if (check_layout(layout) != DAMP_OK) return 0;
+    return (size_t)slot_bytes_of(layout);
+}
+
+double damp_bits_per_value(const damp_layout *L) {
+    if (check_layout(L) != DAMP_OK) return -1.0;
+    const double hi = 16.0 * L->k_hi * L->d_v;
+    const double lo = (8.0 + 32.0 / 32.0) * (double)(L->d_k - L->k_hi) * L->d_v;  // UINT8 + FP16 (s,z) per 32
+    return (hi + lo) / ((double)L->d_k * L->d_v);
+}
+
+damp_status damp_gdn_decode_step(const damp_layout *layout, void *state, int64_t num_slots, const int32_t *slot_idx,
+                                 int32_t batch, const uint8_t *perm, const void *q, const void *k, const void *v,
+                                 const float *g, const float *beta, float *o, int32_t in_dtype, void *stream) {
+    return step(layout, state, num_slots, slot_idx, batch, perm, q, k, v, g, beta, o, in_dtype, stream, false, true,
+                false);
+}
+
+damp_status damp_kda_decode_step(const damp_layout *layout, void *state, int64_t num_slots, const int32_t *slot_idx,
+                                 int32_t batch, const uint8_t *perm, const void *q, const void *k, const void *v,
+                                 const float *g, const float *beta, float *o, int32_t in_dtype, void *stream) {
+    return step(layout, state, num_slots, slot_idx, batch, perm, q, k, v, g, beta, o, in_dtype, stream, true, true,
+                false);
+}
+
+damp_status damp_u8_gdn_decode_step(const damp_layout *layout, void *state, int64_t num_slots,
+                                    const int32_t *slot_idx, int32_t batch, const uint8_t *perm, const void *q,
+                                    const void *k, const void *v, const float *g, const float *beta, float *o,
+                                    int32_t in_dtype, void *stream) {
+    return step(layout, state, num_slots, slot_idx, batch, perm, q, k, v, g, beta, o, in_dtype, stream, false, true,
+                true);
+}
+
+damp_status damp_u8_kda_decode_step(const damp_layout *layout, void *state, int64_t num_slots,
+                                    const int32_t *slot_idx, int32_t batch, const uint8_t *perm, const void *q,
+                                    const void *k, const void *v, const float *g, const float *beta, float *o,
+                                    int32_t in_dtype, void *stream) {
+    return step(layout, state, num_slots, slot_idx, batch, perm, q, k, v, g, beta, o, in_dtype, stream, true, true,
+                true);
+}
+
+damp_status damp_fp32_gdn_decode_step(const damp_layout *layout, float *state, int64_t num_slots,
+                                      const int32_t *slot_idx, int32_t batch, const void *q, const void *k,
+                                      const void *v, const float *g, const float *beta, float *o, int32_t in_dtype,
+                                      void *stream) {
+    return step(layout, state, num_slots, slot_idx, batch, nullptr, q, k, v, g, beta, o, in_dtype, stream, false,
+                false, false);
+}
+
+damp_status damp_fp32_kda_decode_step(const damp_layout *layout, float *state, int64_t num_slots,
+                                      const int32_t *slot_idx, int32_t batch, const void *q, const void *k,
+                                      const void *v, const float *g, const float *beta, float *o, int32_t in_dtype,
+                                      void *stream) {
+    return step(layout, state, num_slots, slot_idx, batch, nullptr, q, k, v, g, beta, o, in_dtype, stream, true,
+                false, false);
+}
+
+damp_status damp_quantize_state(const damp_layout *layout, const float *S, const uint8_t *perm, void *state,
+                                int64_t num_slots, const int32_t *slot_idx, int32_t batch, void *stream) {
+    return convert(layout, state, num_slots, slot_idx, batch, perm, const_cast<float *>(S), nullptr, nullptr,
+                   nullptr, stream, kQ);
+}
+
+damp_status damp_dequantize_state(const damp_layout *layout, const void *state, int64_t num_slots,
+                                  const int32_t *slot_idx, int32_t batch, const uint8_t *perm, float *S,
+                                  void *stream) {
+    return convert(layout, const_cast<void *>(state), num_slots, slot_idx, batch, perm, S, nullptr, nullptr, nullptr,
+                   stream, kDQ);
+}
+
+damp_status damp_pack_tiers(const damp_layout *layout, const uint16_t *hi, const uint8_t *codes, const uint16_t *meta,
+                            void *state, int64_t num_slots, const int32_t *slot_idx, int32_t batch, void *stream) {
+    return convert(layout, state, num_slots, slot_idx, batch, nullptr, nullptr, const_cast<uint16_t *>(hi),
+                   const_cast<uint8_t *>(codes), const_cast<uint16_t *>(meta), stream, kPack);
+}
+
+damp_status damp_unpack_tiers(const damp_layout *layout, const void *state, int64_t num_slots,
+                              const int32_t *slot_idx, int32_t batch, uint16_t *hi, uint8_t *codes, uint16_t *meta,
+                              void *stream) {
+    return convert(layout, const_cast<void *>(state), num_slots, slot_idx, batch, nullptr, nullptr, hi, codes, meta,
+                   stream, kUnpack);
+}
+
+damp_status damp_device_status(uint32_t *status) {
+    if (!status) return DAMP_ERR_NULL;
+    uint32_t all = 0, bits = 0;
+    if (take_status_packed_gdn(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_packed_kda(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_fp32(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_convert(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    *status = all;
+    return DAMP_OK;
+}
+
+const char *damp_status_string(damp_status s) {
+    switch (s) {
+        case DAMP_OK: return "DAMP_OK";
+        case DAMP_ERR_NULL: return "DAMP_ERR_NULL: a required pointer is NULL";
+        case DAMP_ERR_SHAPE: return "DAMP_ERR_SHAPE: a size is outside what the kernels support";
+        case DAMP_ERR_ALIGN: return "DAMP_ERR_ALIGN: a pointer is not aligned as documented";
+        case DAMP_ERR_ALIAS: return "DAMP_ERR_ALIAS: an output overlaps the state pool or another argument";
+        case DAMP_ERR_FORMAT: return "DAMP_ERR_FORMAT: unknown or unsupported lo_format / in_dtype";
+        case DAMP_ERR_CUDA: return "DAMP_ERR_CUDA: the CUDA runtime reported an error while enqueueing";
+    }
+    return "unknown damp_status";
+}
+
+int32_t damp_version(void) { return 100; }
+
+}  // extern "C"

@@ -1,0 +1,291 @@
+// damp_common.cuh -- device helpers shared by libdamp's kernels (sm_103a).
+//
+// Inline PTX for the mbarrier / bulk-copy (TMA engine) pipeline, the packed
+// record geometry, the block-32 Hadamard butterflies and the UINT8 affine
+// requantizer of Sec. 3.2 (Eq. integer_quantizer).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace damp {
+
+constexpr int kG = 32;                        // quantization group = value block (App. A.1)
+constexpr float kInvSqrt32 = 0.17677669529663687f;  // fp32(1/sqrt(32)), H_32 normalization
+constexpr unsigned kFull = 0xffffffffu;
+
+enum : uint32_t { kDevWaitTimeout = 1u, kDevBadSlot = 2u };
+
+// ---------------------------------------------------------------------------
+// Packed record geometry (one (slot, head, value block) record).
+//   hi rows:   K x 64 B   at 0;   16-B chunk m of row u at 16 * (m ^ ((u >> 1) & 3))
+//   codes:     (d_k-K) x 32 B;    16-B chunk m of lo row r at 16 * (m ^ ((r >> 2) & 1))
+//   meta:      (d_k-K) x 4 B      (s, z) as two binary16
+// The chunk permutations make 8 consecutive rows read by a quarter warp hit
+// distinct shared-memory banks.
+// ---------------------------------------------------------------------------
+struct RecGeom {
+    int codes_off, meta_off, bytes;
+};
+
+__host__ __device__ inline RecGeom rec_geom(int d_k, int k_hi) {
+    RecGeom g;
+    g.codes_off = 64 * k_hi;
+    g.meta_off = g.codes_off + 32 * (d_k - k_hi);
+    g.bytes = (g.meta_off + 4 * (d_k - k_hi) + 15) & ~15;
+    return g;
+}
+
+__host__ __device__ inline int hi_chunk_off(int u, int m) { return 64 * u + 16 * (m ^ ((u >> 1) & 3)); }
+__host__ __device__ inline int lo_chunk_off(int r, int m) { return 32 * r + 16 * (m ^ ((r >> 2) & 1)); }
+
+// ---------------------------------------------------------------------------
+// PTX wrappers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+__device__ __forceinline__ uint64_t global_timer_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Bounded wait on an mbarrier phase: gives up after ~2 s (or 2^26 polls) and
+// returns false, so a lost copy ends the kernel with an error flag, not a hang.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 0; it < (1u << 26); ++it) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((it & 255u) == 255u && global_timer_ns() - t0 > 2000000000ull) break;
+    }
+    return false;
+}
+
+// 1-D bulk copy global -> shared (TMA engine), completion on an mbarrier.
+// Addresses 16-B aligned, size a multiple of 16.
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+        "l"(src), "r"(bytes), "r"(bar)
+        : "memory");
+}
+
+// 1-D bulk copy shared -> global, tracked by bulk groups.
+__device__ __forceinline__ void bulk_s2g(void *dst, uint32_t src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(src), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_all() {
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+// Generic-proxy writes to shared memory become visible to the async proxy (bulk store).
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ uint4 lds128(uint32_t a) {
+    uint4 v;
+    asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ void sts128(uint32_t a, uint4 v) {
+    asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(a), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+__device__ __forceinline__ uint32_t lds32(uint32_t a) {
+    uint32_t v;
+    asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ void sts32(uint32_t a, uint32_t v) {
+    asm volatile("st.shared.b32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
+    uint32_t d;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
+    return d;
+}
+
+// per-lane clamp of two signed 16-bit lanes to [0, 255]
+__device__ __forceinline__ uint32_t clamp_u8x2(uint32_t v) {
+    uint32_t d;
+    asm("min.relu.s16x2 %0, %1, %2;" : "=r"(d) : "r"(v), "r"(0x00FF00FFu));
+    return d;
+}
+
+__device__ __forceinline__ float fmin3(float a, float b, float c) {
+    float d;
+    asm("min.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
+// ---------------------------------------------------------------------------
+// Block-32 Hadamard (Sylvester order, normalized by fp32(1/sqrt 32)).
+// ---------------------------------------------------------------------------
+
+// Across the 32 lanes of a warp: lane j holds x_j, returns (H_32 x)_j.
+__device__ __forceinline__ float hadamard_lanes(float x, int lane) {
+#pragma unroll
+    for (int m = 1; m < 32; m <<= 1) {
+        const float y = __shfl_xor_sync(kFull, x, m);
+        x = (lane & m) ? (y - x) : (x + y);
+    }
+    return x * kInvSqrt32;
+}
+
+// Inside one thread: x[0..31] -> H_32 x.
+__device__ __forceinline__ void hadamard_regs(float (&x)[32]) {
+#pragma unroll
+    for (int m = 1; m < 32; m <<= 1) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            if ((j & m) == 0) {
+                const float a = x[j], b = x[j + m];
+                x[j] = a + b;
+                x[j + m] = a - b;
+            }
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < 32; ++j) x[j] *= kInvSqrt32;
+}
+
+// ---------------------------------------------------------------------------
+// UINT8 affine codec of one 32-group held in registers (Sec. 3.2; App. A.1).
+// ---------------------------------------------------------------------------
+
+// Byte b of the word placed in the low mantissa of 2^23: exact float 2^23 + byte.
+__device__ __forceinline__ float u8_biased(uint32_t word, int b) {
+    return __uint_as_float(prmt(word, 0x4B000000u, 0x7650u + b) );
+}
+
+// Scale and zero point of a group from its extrema:
+//   s = fp16((max - min)/255), z = fp16(round_even(-min / s)); a block whose s
+//   rounds to 0 widens [min, max] to contain 0, and s = 1, z = 0 if s is still 0.
+// Returns the packed (s, z) binary16 pair; s_out / inv_out / z_out as float.
+__device__ __forceinline__ uint32_t affine_params(float mn, float mx, float &inv_out, float &z_out) {
+    float s = __half2float(__float2half_rn((mx - mn) * (1.0f / 255.0f)));
+    if (s == 0.0f) {
+        mn = fminf(mn, 0.0f);
+        mx = fmaxf(mx, 0.0f);
+        s = __half2float(__float2half_rn((mx - mn) * (1.0f / 255.0f)));
+        if (s == 0.0f) s = 1.0f;
+    }
+    const float inv = __frcp_rn(s);
+    const __half zh = __float2half_rn(rintf(-mn * inv));
+    const __half sh = __float2half_rn(s);
+    z_out = __half2float(zh);
+    inv_out = inv;
+    return (uint32_t)__half_as_ushort(sh) | ((uint32_t)__half_as_ushort(zh) << 16);
+}
+
+// Codes of 4 values: q = sat_[0,255](round_even(x / s) + z), packed little-endian.
+// fma(x, 1/s, 1.5*2^23 + z) rounds to the integer grid; its low 16 bits are the
+// signed integer; min.relu.s16x2 saturates two lanes at a time.
+__device__ __forceinline__ uint32_t encode4(float x0, float x1, float x2, float x3, float inv, float magic_z) {
+    const uint32_t a = __float_as_uint(fmaf(x0, inv, magic_z));
+    const uint32_t b = __float_as_uint(fmaf(x1, inv, magic_z));
+    const uint32_t c = __float_as_uint(fmaf(x2, inv, magic_z));
+    const uint32_t d = __float_as_uint(fmaf(x3, inv, magic_z));
+    const uint32_t ab = clamp_u8x2(prmt(a, b, 0x5410u));
+    const uint32_t cd = clamp_u8x2(prmt(c, d, 0x5410u));
+    return prmt(ab, cd, 0x6420u);
+}
+
+__device__ __forceinline__ void minmax32(const float (&y)[32], float &mn, float &mx) {
+    float a[11], b[11];
+#pragma unroll
+    for (int i = 0; i < 10; ++i) {
+        a[i] = fmin3(y[3 * i], y[3 * i + 1], y[3 * i + 2]);
+        b[i] = fmax3(y[3 * i], y[3 * i + 1], y[3 * i + 2]);
+    }
+    a[10] = fminf(y[30], y[31]);
+    b[10] = fmaxf(y[30], y[31]);
+    const float a0 = fmin3(a[0], a[1], a[2]), a1 = fmin3(a[3], a[4], a[5]), a2 = fmin3(a[6], a[7], a[8]);
+    const float b0 = fmax3(b[0], b[1], b[2]), b1 = fmax3(b[3], b[4], b[5]), b2 = fmax3(b[6], b[7], b[8]);
+    mn = fmin3(fmin3(a0, a1, a2), a[9], a[10]);
+    mx = fmax3(fmax3(b0, b1, b2), b[9], b[10]);
+}
+
+// Quantize y[0..31] (one lo row, one value block) into 8 code words + packed (s, z).
+__device__ __forceinline__ uint32_t quantize_group(const float (&y)[32], uint32_t (&w)[8]) {
+    float mn, mx, inv, z;
+    minmax32(y, mn, mx);
+    const uint32_t sz = affine_params(mn, mx, inv, z);
+    const float magic_z = 12582912.0f + z;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) w[i] = encode4(y[4 * i], y[4 * i + 1], y[4 * i + 2], y[4 * i + 3], inv, magic_z);
+    return sz;
+}
+
+// Dequantize 8 code words with (s, z): x_j = (q_j - z) * s * scale (scale folds a decay).
+__device__ __forceinline__ void dequantize_group(const uint32_t (&w)[8], uint32_t sz, float scale, float (&x)[32]) {
+    const float s = __half2float(__ushort_as_half((unsigned short)(sz & 0xffffu)));
+    const float z = __half2float(__ushort_as_half((unsigned short)(sz >> 16)));
+    const float zb = 8388608.0f + z;  // 2^23 + z, exact for |z| <= 2^23
+    const float sa = s * scale;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+#pragma unroll
+        for (int b = 0; b < 4; ++b) x[4 * i + b] = (u8_biased(w[i], b) - zb) * sa;
+    }
+}
+
+__device__ __forceinline__ float2 h2_to_f2(uint32_t w) {
+    __half2 h;
+    memcpy(&h, &w, 4);
+    return __half22float2(h);
+}
+
+// two floats -> packed binary16 pair, round to nearest even (low half = a)
+__device__ __forceinline__ uint32_t f2_to_h2(float a, float b) {
+    const __half2 h = __floats2half2_rn(a, b);
+    uint32_t w;
+    memcpy(&w, &h, 4);
+    return w;
+}
+
+__device__ __forceinline__ float load_in(const void *p, int64_t i, bool bf16) {
+    if (bf16) return __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(p)[i]);
+    return reinterpret_cast<const float *>(p)[i];
+}
+
+}  // namespace damp

@@ -1,0 +1,58 @@
+// damp_internal.h -- host-side parameter blocks and launcher declarations shared
+// by libdamp's translation units (not part of the public ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace damp {
+
+struct StepArgs {
+    // layout
+    int32_t H, Hqk, dk, dv, K, fmt;
+    // buffers
+    void *state;  // packed pool or FP32 state
+    int64_t num_slots;
+    const int32_t *slot_idx;
+    int32_t batch;
+    const uint8_t *perm;
+    const void *q, *k, *v;
+    const float *g, *beta;
+    float *o;
+    int32_t in_bf16;  // 1: q/k/v are bf16, 0: fp32
+    int32_t kda;      // 1: per-channel decay g[B][H][d_k], 0: scalar g[B][H]
+};
+
+struct ConvArgs {
+    int32_t H, dk, dv, K, fmt;
+    void *state;
+    int64_t num_slots;
+    const int32_t *slot_idx;
+    int32_t batch;
+    const uint8_t *perm;
+    float *S;  // natural FP32 states [batch][H][d_k][d_v]
+    uint16_t *hi;
+    uint8_t *codes;
+    uint16_t *meta;
+};
+
+// Launchers (return the CUDA error of the launch; they perform no host-side argument checks).
+cudaError_t launch_packed_gdn(const StepArgs &a, cudaStream_t s);
+cudaError_t launch_packed_kda(const StepArgs &a, cudaStream_t s);
+cudaError_t launch_fp32_step(const StepArgs &a, cudaStream_t s);
+cudaError_t launch_quantize(const ConvArgs &a, cudaStream_t s);
+cudaError_t launch_dequantize(const ConvArgs &a, cudaStream_t s);
+cudaError_t launch_pack_tiers(const ConvArgs &a, cudaStream_t s);
+cudaError_t launch_unpack_tiers(const ConvArgs &a, cudaStream_t s);
+
+// Read-and-clear of each translation unit's device status word.
+cudaError_t take_status_packed_gdn(uint32_t *bits);
+cudaError_t take_status_packed_kda(uint32_t *bits);
+cudaError_t take_status_fp32(uint32_t *bits);
+cudaError_t take_status_convert(uint32_t *bits);
+
+// Streaming multiprocessors / opt-in shared memory per block of the current device (cached per device).
+int sm_count();
+int max_smem_per_block();
+
+}  // namespace damp

@@ -1,0 +1,23 @@
+// decode_packed_kda.cu -- instantiations of the fused packed decode step for
+// KDA (per-key-channel decay, Lambda_t = diag(exp(g_t))).
+#include "launch_packed.cuh"
+
+namespace damp {
+
+static __device__ uint32_t g_status_packed_kda;
+
+cudaError_t launch_packed_kda(const StepArgs &a, cudaStream_t s) {
+    uint32_t *status = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(reinterpret_cast<void **>(&status), g_status_packed_kda);
+    if (e != cudaSuccess) return e;
+    return launch_packed_impl<true>(a, s, status);
+}
+
+cudaError_t take_status_packed_kda(uint32_t *bits) {
+    uint32_t zero = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(bits, g_status_packed_kda, sizeof(uint32_t));
+    if (e != cudaSuccess) return e;
+    return cudaMemcpyToSymbol(g_status_packed_kda, &zero, sizeof(uint32_t));
+}
+
+}  // namespace damp

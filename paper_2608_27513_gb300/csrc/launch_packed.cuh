@@ -1,0 +1,102 @@
+// launch_packed.cuh -- host-side launcher of the fused packed decode step.
+// Included once per decay kind (GDN / KDA) so the two sets of template
+// instantiations compile in parallel translation units.
+#pragma once
+
+#include <algorithm>
+
+#include "damp_internal.h"
+#include "decode_packed.cuh"
+
+namespace damp {
+
+// Launch shape: one CTA per SM with kPackedWarps warps; every warp owns a
+// contiguous range of tiles and keeps kPackedStages-1 tile loads in flight.
+constexpr int kPackedWarps = 8;
+constexpr int kPackedStages = 3;
+
+template <bool KDA>
+static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, uint32_t *status) {
+    const int V = a.dv / kG;
+    const RecGeom rg = rec_geom(a.dk, a.K);
+    const int esz = a.in_bf16 ? 2 : 4;
+    PackedParams p{};
+    p.state = static_cast<uint8_t *>(a.state);
+    p.num_slots = a.num_slots;
+    p.slot_idx = a.slot_idx;
+    p.perm = a.perm;
+    p.q = a.q;
+    p.k = a.k;
+    p.v = a.v;
+    p.g = a.g;
+    p.beta = a.beta;
+    p.o = a.o;
+    p.batch = a.batch;
+    p.H = a.H;
+    p.Hqk = a.Hqk;
+    p.dk = a.dk;
+    p.dv = a.dv;
+    p.V = V;
+    p.K = a.K;
+    p.rec_bytes = rg.bytes;
+    p.codes_off = rg.codes_off;
+    p.meta_off = rg.meta_off;
+    p.slot_bytes = (int64_t)a.H * V * rg.bytes;
+    p.bytes_v = kG * esz;
+    p.bytes_qk = a.dk * esz;
+    p.bytes_g = KDA ? a.dk * 4 : 0;
+    p.bytes_perm = a.dk;
+    // stage: [record][v][q][k][g][perm], each 16-B aligned
+    int off = rg.bytes;
+    p.off_v = off;
+    off += p.bytes_v;
+    p.off_q = off;
+    off += p.bytes_qk;
+    p.off_k = off;
+    off += p.bytes_qk;
+    p.off_g = off;
+    off += p.bytes_g;
+    p.off_perm = off;
+    off += p.bytes_perm;
+    p.stage_bytes = (off + 127) & ~127;
+    p.nstage = kPackedStages;
+    p.stage0_off = (kScratchBytes + 127) & ~127;
+    p.warp_smem = p.stage0_off + p.nstage * p.stage_bytes;
+    p.total_tiles = (int64_t)a.batch * a.H * V;
+    p.status = status;
+    if (p.total_tiles == 0) return cudaSuccess;
+
+    // shrink the warp count (then the ring) until the per-CTA shared memory fits
+    const int smem_cap = max_smem_per_block();
+    int warps = kPackedWarps;
+    while (warps > 1 && warps * p.warp_smem > smem_cap) --warps;
+    if (warps * p.warp_smem > smem_cap) {
+        p.nstage = 2;
+        p.warp_smem = p.stage0_off + p.nstage * p.stage_bytes;
+    }
+    if (warps * p.warp_smem > smem_cap) return cudaErrorInvalidConfiguration;
+    const int64_t want = (p.total_tiles + warps - 1) / warps;
+    const int grid = (int)std::min<int64_t>(want, (int64_t)sm_count());
+    const int smem = p.warp_smem * warps;
+
+    void (*kern)(PackedParams) = nullptr;
+    const bool had = a.fmt == 0;
+#define DAMP_PICK(R_)                                                                          \
+    if (a.dk == 32 * R_) {                                                                     \
+        if (had) kern = a.in_bf16 ? packed_step_kernel<R_, KDA, true, true>                    \
+                                  : packed_step_kernel<R_, KDA, true, false>;                  \
+        else kern = a.in_bf16 ? packed_step_kernel<R_, KDA, false, true>                       \
+                              : packed_step_kernel<R_, KDA, false, false>;                     \
+    }
+    DAMP_PICK(1)
+    DAMP_PICK(2)
+    DAMP_PICK(4)
+#undef DAMP_PICK
+    if (!kern) return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, 32 * warps, smem, stream>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace damp

@@ -1,0 +1,157 @@
+"""Parity helpers: run the CUDA path and the oracle on the same seeded inputs and
+compare them element by element.
+
+Tolerances (the decode-step contract):
+  * o and the FP16 tier: |gpu - ref| <= 1e-5 + 1e-3 |ref| per element;
+  * UINT8 codes: at most 0.1% of codes differ (aggregated over a test), and
+    every difference is a float-ordering tie of the oracle's own values:
+      - in a group whose (s, z) agree, a code differs by at most 1 and only
+        where the oracle's x/s + z lies within TIE of a half-integer;
+      - a group's (s, z) may differ only where the oracle's scale
+        s32 = (x_max - x_min)/255 lies within TIE_REL of a binary16 rounding
+        midpoint or -x_min/s within TIE of a half-integer; then s is within
+        one binary16 ulp, z within 1, and every reconstructed level s (q - z)
+        within one quantization step (raw codes shift with z).
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import paper_2608_27513_gb300 as damp
+import workloads as wl
+from oracle import core, runs
+
+RTOL, ATOL = 1e-3, 1e-5
+CODE_FRAC = 1e-3
+TIE = 2e-3        # code units
+TIE_REL = 2e-5    # relative distance of s32 to a binary16 rounding boundary
+
+
+def layout_of(w: wl.Workload) -> damp.Layout:
+    return damp.Layout(w.heads, w.qk_heads, w.d_k, w.d_v, w.k_hi, w.lo_format)
+
+
+def to_dev(a: np.ndarray, dev, dtype=None):
+    t = torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    return t.to(dtype) if dtype is not None else t
+
+
+def inputs_to_dev(w: wl.Workload, inp: dict, dev) -> dict:
+    dt = torch.bfloat16 if w.in_dtype == "bf16" else torch.float32
+    return {"q": to_dev(inp["q"], dev, dt), "k": to_dev(inp["k"], dev, dt), "v": to_dev(inp["v"], dev, dt),
+            "g": to_dev(inp["g"], dev), "beta": to_dev(inp["beta"], dev)}
+
+
+def tiers_to_dev(w: wl.Workload, tiers, rows: int, dev):
+    hi, codes, meta = tiers
+    H, dk, dv, K = w.heads, w.d_k, w.d_v, w.k_hi
+    return (to_dev(hi.view(np.int16).reshape(rows, H, K, dv), dev),
+            to_dev(codes.reshape(rows, H, dk - K, dv), dev),
+            to_dev(meta.view(np.int16).reshape(rows, H, dk - K, dv // 32, 2), dev))
+
+
+def tiers_from_dev(w: wl.Workload, dev_tiers, units: int):
+    hi, codes, meta = (t.cpu().numpy() for t in dev_tiers)
+    H, dk, dv, K = w.heads, w.d_k, w.d_v, w.k_hi
+    return (hi.view(np.uint16).reshape(units, K, dv), codes.reshape(units, dk - K, dv),
+            meta.view(np.uint16).reshape(units, dk - K, dv // 32, 2))
+
+
+def oracle_step(w: wl.Workload, perm_units, tiers, u: dict):
+    """One oracle step from packed tiers: returns (o, new tiers, lo pre-quantization values).
+
+    The pre-quantization values x (FP32, in the low tier's domain) are what the
+    codes round; they serve to recognise rounding ties.
+    """
+    n = perm_units.shape[0]
+    S = core.unpack_heads(perm_units, *tiers, w.k_hi, w.lo_format, w.d_k, w.d_v)
+    o = core.delta_step_heads(S, u["q"], u["k"], u["v"], u["g"], u["beta"], w.kind)
+    new = core.pack_heads(perm_units, S, w.k_hi, w.lo_format)
+    lo_rows = np.stack([S[i][perm_units[i][w.k_hi:]] for i in range(n)])  # [n, d_k-K, d_v] natural
+    if w.lo_format == core.FMT_U8_H32 and lo_rows.size:
+        lo_rows = core.hadamard32(lo_rows.reshape(-1, 32)).reshape(lo_rows.shape)
+    return o, new, lo_rows
+
+
+class CodeStats:
+    def __init__(self):
+        self.codes = 0
+        self.mismatched = 0
+        self.groups = 0
+        self.meta_mismatched = 0
+
+    def check_fraction(self):
+        if self.codes:
+            assert self.mismatched <= CODE_FRAC * self.codes, \
+                f"{self.mismatched} of {self.codes} codes differ (> {CODE_FRAC:.1%})"
+
+
+def _f16(bits):
+    return core.f16_to_f32(bits.astype(np.uint16)).astype(np.float64)
+
+
+def compare_tiers(w: wl.Workload, ref, gpu, lo_pre, stats: CodeStats, what=""):
+    """Compare packed tiers; lo_pre = oracle pre-quantization values [n, d_k-K, d_v]."""
+    hi_r, codes_r, meta_r = ref
+    hi_g, codes_g, meta_g = gpu
+    if hi_r.size:
+        a, b = _f16(hi_g), _f16(hi_r)
+        bad = np.abs(a - b) > ATOL + RTOL * np.abs(b)
+        assert not bad.any(), f"{what}: FP16 tier differs at {np.argwhere(bad)[:5].tolist()}"
+    if not codes_r.size:
+        return
+    n, lo, dv = codes_r.shape
+    G = dv // 32
+    cr = codes_r.reshape(n, lo, G, 32).astype(np.int64)
+    cg = codes_g.reshape(n, lo, G, 32).astype(np.int64)
+    d = np.abs(cr - cg)
+    s_r, z_r = _f16(meta_r[..., 0]), _f16(meta_r[..., 1])
+    s_g, z_g = _f16(meta_g[..., 0]), _f16(meta_g[..., 1])
+    meta_diff = (meta_r != meta_g).any(axis=-1)  # [n, lo, G]
+    x = lo_pre.reshape(n, lo, G, 32).astype(np.float64)
+    # groups with equal (s, z): codes within 1 LSB, and differing only at ties of x/s + z
+    same = ~meta_diff[..., None]
+    assert np.all(d[np.broadcast_to(same, d.shape)] <= 1), f"{what}: a code differs by more than 1 LSB"
+    t = x / s_r[..., None] + z_r[..., None]
+    near = np.abs(np.abs(t - np.floor(t)) - 0.5) < TIE
+    code_bad = (d > 0) & ~near & same
+    assert not code_bad.any(), f"{what}: codes differ away from a rounding tie at {np.argwhere(code_bad)[:5].tolist()}"
+    if meta_diff.any():
+        # (s, z) may move only because the oracle's own group sits at a rounding tie:
+        # s32 = (x_max - x_min)/255 at a binary16 midpoint, or -x_min/s at a half-integer.
+        assert np.all(np.abs(s_g - s_r)[meta_diff] <= np.abs(s_r)[meta_diff] * 2.0 ** -10 + 1e-30), \
+            f"{what}: scale differs by more than one binary16 ulp"
+        assert np.all(np.abs(z_g - z_r)[meta_diff] <= 1), f"{what}: zero point differs by more than 1"
+        xmin, xmax = x.min(axis=-1), x.max(axis=-1)
+        s32 = (xmax - xmin) / 255.0
+        sp = np.spacing(s32.astype(np.float16)).astype(np.float64)
+        frac_s = np.abs((s32 / sp) - np.floor(s32 / sp) - 0.5)   # 0 at a binary16 rounding midpoint
+        frac_z = np.abs((-xmin / s_r) - np.floor(-xmin / s_r) - 0.5)
+        tie = (frac_s * sp < TIE_REL * np.abs(s32) + 1e-30) | (frac_z < TIE)
+        bad = meta_diff & ~tie
+        assert not bad.any(), f"{what}: (s, z) differ away from a rounding tie at {np.argwhere(bad)[:5].tolist()}"
+        # in such a group the reconstructed level s (q - z) moves by at most one step
+        rec_r = s_r[..., None] * (cr - z_r[..., None])
+        rec_g = s_g[..., None] * (cg - z_g[..., None])
+        step = np.maximum(s_r, s_g)[..., None] * 1.01
+        far = (np.abs(rec_g - rec_r) > step) & meta_diff[..., None]
+        assert not far.any(), f"{what}: a reconstructed value moves by more than one step at {np.argwhere(far)[:5].tolist()}"
+    stats.codes += d.size
+    stats.mismatched += int((d > 0).sum())
+    stats.groups += meta_diff.size
+    stats.meta_mismatched += int(meta_diff.sum())
+
+
+def compare_o(o_gpu, o_ref, what=""):
+    bad = np.abs(o_gpu - o_ref) > ATOL + RTOL * np.abs(o_ref)
+    assert not bad.any(), (f"{what}: o differs at {np.argwhere(bad)[:5].tolist()} "
+                           f"max {np.abs(o_gpu - o_ref).max():g}")
+
+
+def initial_tiers(w: wl.Workload, rows, perms, prefix=None):
+    """Oracle FP32 prefix for the given batch rows, packed with the per-head perms."""
+    rows = list(rows)
+    S0 = runs.prefix_states(w, rows, steps=prefix).reshape(len(rows) * w.heads, w.d_k, w.d_v)
+    perm_units = np.tile(perms, (len(rows), 1))
+    return perm_units, core.pack_heads(perm_units, S0, w.k_hi, w.lo_format)

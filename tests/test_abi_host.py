@@ -1,0 +1,140 @@
+"""The C-ABI library on the host: it loads, exports every symbol include/damp.h
+declares, sizes its records as documented, and rejects bad arguments before
+enqueueing anything (no call here reaches the GPU)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2608_27513_gb300 as damp
+from paper_2608_27513_gb300 import _lib, build
+from tests.golden.load import paper_values
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    build.build()
+    return _lib.lib()
+
+
+def declared_functions():
+    src = open(os.path.join(ROOT, "include", "damp.h")).read()
+    return sorted(set(re.findall(r"DAMP_API\s+[\w\s\*]+?\b(damp_\w+)\s*\(", src)))
+
+
+def test_header_declares_the_expected_entry_points():
+    names = declared_functions()
+    for n in ("damp_gdn_decode_step", "damp_kda_decode_step", "damp_quantize_state", "damp_dequantize_state",
+              "damp_fp32_gdn_decode_step", "damp_fp32_kda_decode_step", "damp_u8_gdn_decode_step",
+              "damp_u8_kda_decode_step", "damp_pack_tiers", "damp_unpack_tiers"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(L):
+    for name in declared_functions():
+        assert hasattr(L, name), name
+    assert set(declared_functions()) == set(_lib.SIGNATURES)
+
+
+def test_library_has_no_cpu_fallback_symbols(L):
+    # the product library is CUDA only: it does not link the oracle
+    out = os.popen(f"nm -D {_lib.LIB_PATH}").read()
+    assert "dor_" not in out
+
+
+def _layout(**kw):
+    base = dict(num_heads=32, num_qk_heads=32, d_k=128, d_v=128, k_hi=16, lo_format=0)
+    base.update(kw)
+    return damp.Layout(**base)
+
+
+def test_record_geometry_and_bits(L):
+    pv = paper_values()
+    for K in (0, 4, 8, 10, 16, 32, 128):
+        lay = _layout(k_hi=K)
+        logical = 64 * K + 32 * (128 - K) + 4 * (128 - K)  # per value block: FP16 rows, codes, (s, z)
+        assert damp.record_bytes(lay) == (logical + 15) // 16 * 16
+        assert damp.slot_bytes(lay) == 32 * 4 * damp.record_bytes(lay)
+        assert damp.bits_per_value(lay) == 8.0 * logical / (128 * 32)
+    assert damp.bits_per_value(_layout(k_hi=16)) == pv["damp_bits_k16_dk128"]
+    assert damp.bits_per_value(_layout(k_hi=0)) == pv["bits_int8_hadamard"]
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(d_k=96), 2), (dict(d_k=256), 2), (dict(d_v=48), 2), (dict(d_v=2048), 2), (dict(k_hi=129), 2),
+    (dict(k_hi=-1), 2), (dict(num_qk_heads=5), 2), (dict(num_heads=0), 2), (dict(lo_format=2), 5)])
+def test_layout_validation(L, kw, status):
+    c = _layout(**kw).c()
+    assert L.damp_validate_layout(ctypes.byref(c)) == status
+    assert L.damp_record_bytes(ctypes.byref(c)) == 0
+    assert L.damp_bits_per_value(ctypes.byref(c)) == -1.0
+
+
+class FakeBuffers:
+    """Distinct, aligned host addresses standing in for device buffers (never dereferenced)."""
+
+    def __init__(self, n=16, size=1 << 24):
+        self.bufs = [ctypes.create_string_buffer(size + 256) for _ in range(n)]
+        self.ptrs = [(ctypes.addressof(b) + 255) // 256 * 256 for b in self.bufs]
+
+    def __getitem__(self, i):
+        return ctypes.c_void_p(self.ptrs[i])
+
+
+def _call_step(L, lay, fb, **over):
+    c = lay.c()
+    args = dict(layout=ctypes.byref(c), state=fb[0], num_slots=4, slot_idx=None, batch=4, perm=fb[1], q=fb[2],
+                k=fb[3], v=fb[4], g=fb[5], beta=fb[6], o=fb[7], in_dtype=0, stream=None)
+    args.update(over)
+    return L.damp_kda_decode_step(*args.values())
+
+
+def test_step_rejects_bad_arguments_before_launch(L):
+    fb = FakeBuffers()
+    lay = _layout()
+    off = lambda i, d: ctypes.c_void_p(fb.ptrs[i] + d)
+    assert _call_step(L, lay, fb, batch=0) == 0                      # empty batch: nothing enqueued
+    assert _call_step(L, lay, fb, batch=-1) == 2
+    assert _call_step(L, lay, fb, state=None) == 1
+    assert _call_step(L, lay, fb, perm=None) == 1
+    assert _call_step(L, lay, fb, o=None) == 1
+    assert _call_step(L, lay, fb, num_slots=3) == 2                   # fewer slots than rows, no slot_idx
+    assert _call_step(L, lay, fb, state=off(0, 8)) == 3
+    assert _call_step(L, lay, fb, q=off(2, 4)) == 3
+    assert _call_step(L, lay, fb, g=off(5, 4)) == 3                   # KDA gates are bulk-copied: 16 B
+    assert _call_step(L, lay, fb, o=off(7, 2)) == 3
+    assert _call_step(L, lay, fb, in_dtype=7) == 5
+    assert _call_step(L, lay, fb, o=off(0, 4096)) == 4                # o inside the pool
+    assert _call_step(L, lay, fb, q=off(0, 1 << 12)) == 4             # an input inside the pool
+    assert _call_step(L, lay, fb, o=fb[2]) == 4                       # o over q
+    assert _call_step(L, _layout(lo_format=3), fb) == 5
+    c = _layout(k_hi=8).c()
+    assert L.damp_u8_kda_decode_step(ctypes.byref(c), *[fb[0], 4, None, 4, fb[1], fb[2], fb[3], fb[4], fb[5],
+                                                        fb[6], fb[7], 0, None]) == 2
+
+
+def test_gdn_gate_alignment_is_4_bytes(L):
+    fb = FakeBuffers()
+    c = _layout().c()
+    args = [ctypes.byref(c), fb[0], 4, None, 4, fb[1], fb[2], fb[3], fb[4], ctypes.c_void_p(fb.ptrs[5] + 5),
+            fb[6], fb[7], 0, None]
+    assert L.damp_gdn_decode_step(*args) == 3
+
+
+def test_conversions_reject_bad_arguments(L):
+    fb = FakeBuffers()
+    c = _layout().c()
+    assert L.damp_quantize_state(ctypes.byref(c), None, fb[1], fb[0], 4, None, 4, None) == 1
+    assert L.damp_quantize_state(ctypes.byref(c), fb[2], fb[1], fb[0], 4, None, 8, None) == 2
+    assert L.damp_dequantize_state(ctypes.byref(c), fb[0], 4, None, 4, fb[1], fb[0], None) == 4
+    assert L.damp_pack_tiers(ctypes.byref(c), fb[2], None, fb[4], fb[0], 4, None, 4, None) == 1
+    assert L.damp_unpack_tiers(ctypes.byref(c), fb[0], 4, None, 4, fb[2], fb[2], fb[4], None) == 4
+    assert L.damp_device_status(None) == 1
+
+
+def test_status_strings(L):
+    for s in range(7):
+        assert L.damp_status_string(s).decode().startswith("DAMP_")

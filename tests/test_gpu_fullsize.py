@@ -1,0 +1,61 @@
+"""Parity at the full decode-batch sizes, in the launch configuration the bench
+times: the GPU steps the whole batch; the oracle computes sampled batch rows
+(every head of each sampled row) from the full 256-step FP32 prefix."""
+import numpy as np
+import pytest
+import torch
+
+import paper_2608_27513_gb300 as damp
+import workloads as wl
+from oracle import runs
+from tests import parity as P
+
+pytestmark = pytest.mark.gpu
+DEV = torch.device("cuda:0")
+
+
+def _fullsize(w, sample_rows, steps):
+    perms, _ = runs.calibrate_layout(w, n_docs=4, n_tokens=64)
+    perm_units, tiers = P.initial_tiers(w, sample_rows, perms)
+    L = P.layout_of(w)
+    state = damp.new_state(L, w.batch, DEV)
+    dperm = P.to_dev(perms, DEV)
+    # every other slot holds a packed random state of the same magnitude
+    gen = torch.Generator(device=DEV)
+    gen.manual_seed(w.seed)
+    S = 0.3 * torch.randn((w.batch, w.heads, w.d_k, w.d_v), generator=gen, device=DEV)
+    damp.quantize_state(L, S, dperm, state)
+    del S
+    sidx = torch.tensor(sample_rows, dtype=torch.int32, device=DEV)
+    stats = P.CodeStats()
+    step = damp.kda_decode_step if w.kind == "kda" else damp.gdn_decode_step
+    for t in range(steps):
+        inp = wl.step_inputs(w, t)  # all rows
+        sub = {k: v[sample_rows] for k, v in inp.items()}
+        u = runs.unit_operands(w, sub)
+        o_ref, new_ref, lo_pre = P.oracle_step(w, perm_units, tiers, u)
+        damp.pack_tiers(L, *P.tiers_to_dev(w, tiers, len(sample_rows), DEV), state, slot_idx=sidx)
+        d = P.inputs_to_dev(w, inp, DEV)
+        o = step(L, state, dperm, d["q"], d["k"], d["v"], d["g"], d["beta"])
+        got = P.tiers_from_dev(w, damp.unpack_tiers(L, state, batch=len(sample_rows), slot_idx=sidx),
+                               len(sample_rows) * w.heads)
+        P.compare_o(o.cpu().numpy()[sample_rows].reshape(-1, w.d_v), o_ref, f"{w.name} step {t}")
+        P.compare_tiers(w, new_ref, got, lo_pre, stats, f"{w.name} step {t}")
+        tiers = new_ref
+    stats.check_fraction()
+    assert damp.device_status() == 0
+
+
+def test_kda_b256_full_batch_sampled_rows():
+    """KDA B=256, H=32, d=128, K_hi=10, BF16: rows 0, 77, 255 against the oracle."""
+    _fullsize(wl.KDA_B256, [0, 77, 255], 2)
+
+
+def test_gdn_b64_gqa_full_batch_sampled_rows():
+    """GDN B=64, 32 value heads / 16 q-k heads, d=128, K_hi=8, BF16: rows 0, 31, 63."""
+    _fullsize(wl.GDN_B64_GQA, [0, 31, 63], 2)
+
+
+@pytest.mark.parametrize("kind", ["gdn", "kda"])
+def test_sweep_k16_full_batch_sampled_rows(kind):
+    _fullsize(wl.sweep(kind, 16), [5, 200], 1)
