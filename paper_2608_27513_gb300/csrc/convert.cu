@@ -63,29 +63,27 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
             if (OP == kQuantize || OP == kDequantize) {
                 const int n = p.perm[(int64_t)h * p.dk + u] & (p.dk - 1);  // d_k is a power of two
                 float *row = p.S + ((((int64_t)b * p.H + h) * p.dk + n) * p.dv + c * kG);
-                float x[32];
+                float2 x[16];
                 if (OP == kQuantize) {
 #pragma unroll
                     for (int m = 0; m < 8; ++m) {
                         const float4 f = reinterpret_cast<const float4 *>(row)[m];
-                        x[4 * m] = f.x;
-                        x[4 * m + 1] = f.y;
-                        x[4 * m + 2] = f.z;
-                        x[4 * m + 3] = f.w;
+                        x[2 * m] = make_float2(f.x, f.y);
+                        x[2 * m + 1] = make_float2(f.z, f.w);
                     }
                     if (u < K) {
 #pragma unroll
                         for (int m = 0; m < 4; ++m) {
                             uint4 w;
-                            w.x = f2_to_h2(x[8 * m], x[8 * m + 1]);
-                            w.y = f2_to_h2(x[8 * m + 2], x[8 * m + 3]);
-                            w.z = f2_to_h2(x[8 * m + 4], x[8 * m + 5]);
-                            w.w = f2_to_h2(x[8 * m + 6], x[8 * m + 7]);
+                            w.x = f2_to_h2(x[4 * m].x, x[4 * m].y);
+                            w.y = f2_to_h2(x[4 * m + 1].x, x[4 * m + 1].y);
+                            w.z = f2_to_h2(x[4 * m + 2].x, x[4 * m + 2].y);
+                            w.w = f2_to_h2(x[4 * m + 3].x, x[4 * m + 3].y);
                             *reinterpret_cast<uint4 *>(rec + hi_chunk_off(u, m)) = w;
                         }
                     } else {
                         const int r = u - K;
-                        if (HAD) hadamard_regs(x);
+                        if (HAD) hadamard_pairs(x);
                         uint32_t w[8];
                         const uint32_t sz = quantize_group(x, w);
                         *reinterpret_cast<uint4 *>(rec + p.codes_off + lo_chunk_off(r, 0)) =
@@ -99,13 +97,10 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
 #pragma unroll
                         for (int m = 0; m < 4; ++m) {
                             const uint4 w = *reinterpret_cast<const uint4 *>(rec + hi_chunk_off(u, m));
-                            const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-                            for (int e = 0; e < 4; ++e) {
-                                const float2 f = h2_to_f2(ww[e]);
-                                x[8 * m + 2 * e] = f.x;
-                                x[8 * m + 2 * e + 1] = f.y;
-                            }
+                            x[4 * m] = h2_to_f2(w.x);
+                            x[4 * m + 1] = h2_to_f2(w.y);
+                            x[4 * m + 2] = h2_to_f2(w.z);
+                            x[4 * m + 3] = h2_to_f2(w.w);
                         }
                     } else {
                         const int r = u - K;
@@ -114,11 +109,11 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
                         const uint32_t sz = *reinterpret_cast<const uint32_t *>(rec + p.meta_off + 4 * r);
                         const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
                         dequantize_group(w, sz, 1.0f, x);
-                        if (HAD) hadamard_regs(x);
+                        if (HAD) hadamard_pairs(x);
                     }
 #pragma unroll
                     for (int m = 0; m < 8; ++m)
-                        reinterpret_cast<float4 *>(row)[m] = make_float4(x[4 * m], x[4 * m + 1], x[4 * m + 2], x[4 * m + 3]);
+                        reinterpret_cast<float4 *>(row)[m] = make_float4(x[2 * m].x, x[2 * m].y, x[2 * m + 1].x, x[2 * m + 1].y);
                 }
             } else {
                 // logical tiers <-> record, 32-bit words
@@ -164,7 +159,8 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
 template <int OP>
 static cudaError_t launch_convert(const ConvArgs &a, cudaStream_t stream) {
     ConvParams p{};
-    cudaError_t e = cudaGetSymbolAddress(reinterpret_cast<void **>(&p.status), g_status_convert);
+    static uint32_t *cache[64];
+    cudaError_t e = symbol_address_cached(&g_status_convert, cache, &p.status);
     if (e != cudaSuccess) return e;
     const RecGeom rg = rec_geom(a.dk, a.K);
     p.state = static_cast<uint8_t *>(a.state);

@@ -184,6 +184,61 @@ damp_status convert(const damp_layout *L, void *state, int64_t num_slots, const 
 }  // namespace
 
 int sm_count() { return device_attr(g_sm_count, cudaDevAttrMultiProcessorCount, 1); }
+
+namespace {
+struct SmemEntry {
+    std::atomic<const void *> kernel{nullptr};
+    std::atomic<int> bytes{0};
+};
+constexpr int kSmemEntries = 256;
+SmemEntry g_smem_set[kMaxDevices][kSmemEntries];
+}  // namespace
+
+cudaError_t ensure_smem_limit(const void *kernel, int bytes) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    SmemEntry *slot = nullptr;
+    if (dev >= 0 && dev < kMaxDevices) {
+        const size_t h = (reinterpret_cast<uintptr_t>(kernel) >> 4) % kSmemEntries;
+        for (size_t i = 0; i < kSmemEntries; ++i) {
+            SmemEntry &en = g_smem_set[dev][(h + i) % kSmemEntries];
+            const void *k = en.kernel.load(std::memory_order_acquire);
+            if (k == kernel) {
+                if (en.bytes.load(std::memory_order_acquire) >= bytes) return cudaSuccess;
+                slot = &en;
+                break;
+            }
+            if (k == nullptr) {
+                const void *expected = nullptr;
+                if (en.kernel.compare_exchange_strong(expected, kernel) || expected == kernel) {
+                    slot = &en;
+                    break;
+                }
+            }
+        }
+    }
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess && slot) {
+        int cur = slot->bytes.load(std::memory_order_relaxed);
+        while (cur < bytes && !slot->bytes.compare_exchange_weak(cur, bytes)) {
+        }
+    }
+    return e;
+}
+
+cudaError_t symbol_address_cached(const void *symbol, uint32_t **cache, uint32_t **out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < kMaxDevices && cache[dev]) {
+        *out = cache[dev];
+        return cudaSuccess;
+    }
+    e = cudaGetSymbolAddress(reinterpret_cast<void **>(out), symbol);
+    if (e == cudaSuccess && dev >= 0 && dev < kMaxDevices) cache[dev] = *out;
+    return e;
+}
 int max_smem_per_block() { return device_attr(g_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, 48 * 1024); }
 
 }  // namespace damp

@@ -20,11 +20,11 @@ enum : uint32_t { kDevWaitTimeout = 1u, kDevBadSlot = 2u };
 
 // ---------------------------------------------------------------------------
 // Packed record geometry (one (slot, head, value block) record).
-//   hi rows:   K x 64 B   at 0;   16-B chunk m of row u at 16 * (m ^ ((u >> 1) & 3))
+//   hi rows:   K x 64 B   at 0;   row-major binary16 (lanes read one column each)
 //   codes:     (d_k-K) x 32 B;    16-B chunk m of lo row r at 16 * (m ^ ((r >> 2) & 1))
 //   meta:      (d_k-K) x 4 B      (s, z) as two binary16
-// The chunk permutations make 8 consecutive rows read by a quarter warp hit
-// distinct shared-memory banks.
+// The chunk permutation of the codes makes the 8 consecutive rows that a
+// quarter warp reads with 128-bit loads hit distinct shared-memory banks.
 // ---------------------------------------------------------------------------
 struct RecGeom {
     int codes_off, meta_off, bytes;
@@ -38,7 +38,7 @@ __host__ __device__ inline RecGeom rec_geom(int d_k, int k_hi) {
     return g;
 }
 
-__host__ __device__ inline int hi_chunk_off(int u, int m) { return 64 * u + 16 * (m ^ ((u >> 1) & 3)); }
+__host__ __device__ inline int hi_chunk_off(int u, int m) { return 64 * u + 16 * m; }
 __host__ __device__ inline int lo_chunk_off(int r, int m) { return 32 * r + 16 * (m ^ ((r >> 2) & 1)); }
 
 // ---------------------------------------------------------------------------
@@ -197,10 +197,27 @@ __device__ __forceinline__ float u8_biased(uint32_t word, int b) {
     return __uint_as_float(prmt(word, 0x4B000000u, 0x7650u + b) );
 }
 
+// ---------------------------------------------------------------------------
+// Packed FP32 pairs (FFMA2 / FADD2 / FMUL2 on sm_100+): two lanes of FP32
+// arithmetic per issue slot, each component rounded exactly like the scalar op.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float2 splat2(float a) { return make_float2(a, a); }
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
+__device__ __forceinline__ float2 add2(float2 a, float2 b) { return __fadd2_rn(a, b); }
+__device__ __forceinline__ float2 mul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
+
+__device__ __forceinline__ float rcp_approx(float x) {
+    float r;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+    return r;
+}
+
 // Scale and zero point of a group from its extrema:
 //   s = fp16((max - min)/255), z = fp16(round_even(-min / s)); a block whose s
 //   rounds to 0 widens [min, max] to contain 0, and s = 1, z = 0 if s is still 0.
-// Returns the packed (s, z) binary16 pair; s_out / inv_out / z_out as float.
+// Returns the packed (s, z) binary16 pair; inv_out ~ 1/s and z_out as float.
+// The reciprocal is the hardware approximation (within one ulp): a code can only
+// move where x/s + z sits at a rounding tie.
 __device__ __forceinline__ uint32_t affine_params(float mn, float mx, float &inv_out, float &z_out) {
     float s = __half2float(__float2half_rn((mx - mn) * (1.0f / 255.0f)));
     if (s == 0.0f) {
@@ -209,7 +226,7 @@ __device__ __forceinline__ uint32_t affine_params(float mn, float mx, float &inv
         s = __half2float(__float2half_rn((mx - mn) * (1.0f / 255.0f)));
         if (s == 0.0f) s = 1.0f;
     }
-    const float inv = __frcp_rn(s);
+    const float inv = rcp_approx(s);
     const __half zh = __float2half_rn(rintf(-mn * inv));
     const __half sh = __float2half_rn(s);
     z_out = __half2float(zh);
@@ -220,53 +237,63 @@ __device__ __forceinline__ uint32_t affine_params(float mn, float mx, float &inv
 // Codes of 4 values: q = sat_[0,255](round_even(x / s) + z), packed little-endian.
 // fma(x, 1/s, 1.5*2^23 + z) rounds to the integer grid; its low 16 bits are the
 // signed integer; min.relu.s16x2 saturates two lanes at a time.
-__device__ __forceinline__ uint32_t encode4(float x0, float x1, float x2, float x3, float inv, float magic_z) {
-    const uint32_t a = __float_as_uint(fmaf(x0, inv, magic_z));
-    const uint32_t b = __float_as_uint(fmaf(x1, inv, magic_z));
-    const uint32_t c = __float_as_uint(fmaf(x2, inv, magic_z));
-    const uint32_t d = __float_as_uint(fmaf(x3, inv, magic_z));
-    const uint32_t ab = clamp_u8x2(prmt(a, b, 0x5410u));
-    const uint32_t cd = clamp_u8x2(prmt(c, d, 0x5410u));
+__device__ __forceinline__ uint32_t encode4(float2 x01, float2 x23, float2 inv2, float2 magic2) {
+    const float2 a = fma2(x01, inv2, magic2);
+    const float2 b = fma2(x23, inv2, magic2);
+    const uint32_t ab = clamp_u8x2(prmt(__float_as_uint(a.x), __float_as_uint(a.y), 0x5410u));
+    const uint32_t cd = clamp_u8x2(prmt(__float_as_uint(b.x), __float_as_uint(b.y), 0x5410u));
     return prmt(ab, cd, 0x6420u);
 }
 
-__device__ __forceinline__ void minmax32(const float (&y)[32], float &mn, float &mx) {
-    float a[11], b[11];
+__device__ __forceinline__ void minmax32(const float2 (&y)[16], float &mn, float &mx) {
+    float a[6], b[6];
 #pragma unroll
-    for (int i = 0; i < 10; ++i) {
-        a[i] = fmin3(y[3 * i], y[3 * i + 1], y[3 * i + 2]);
-        b[i] = fmax3(y[3 * i], y[3 * i + 1], y[3 * i + 2]);
+    for (int i = 0; i < 5; ++i) {  // pairs 3i .. 3i+2 hold six values
+        a[i] = fmin3(fmin3(y[3 * i].x, y[3 * i].y, y[3 * i + 1].x), y[3 * i + 1].y, fminf(y[3 * i + 2].x, y[3 * i + 2].y));
+        b[i] = fmax3(fmax3(y[3 * i].x, y[3 * i].y, y[3 * i + 1].x), y[3 * i + 1].y, fmaxf(y[3 * i + 2].x, y[3 * i + 2].y));
     }
-    a[10] = fminf(y[30], y[31]);
-    b[10] = fmaxf(y[30], y[31]);
-    const float a0 = fmin3(a[0], a[1], a[2]), a1 = fmin3(a[3], a[4], a[5]), a2 = fmin3(a[6], a[7], a[8]);
-    const float b0 = fmax3(b[0], b[1], b[2]), b1 = fmax3(b[3], b[4], b[5]), b2 = fmax3(b[6], b[7], b[8]);
-    mn = fmin3(fmin3(a0, a1, a2), a[9], a[10]);
-    mx = fmax3(fmax3(b0, b1, b2), b[9], b[10]);
+    a[5] = fminf(y[15].x, y[15].y);
+    b[5] = fmaxf(y[15].x, y[15].y);
+    mn = fmin3(fmin3(a[0], a[1], a[2]), fmin3(a[3], a[4], a[5]), a[5]);
+    mx = fmax3(fmax3(b[0], b[1], b[2]), fmax3(b[3], b[4], b[5]), b[5]);
 }
 
-// Quantize y[0..31] (one lo row, one value block) into 8 code words + packed (s, z).
-__device__ __forceinline__ uint32_t quantize_group(const float (&y)[32], uint32_t (&w)[8]) {
+// Quantize y (one lo row, one value block, 16 pairs) into 8 code words + packed (s, z).
+__device__ __forceinline__ uint32_t quantize_group(const float2 (&y)[16], uint32_t (&w)[8]) {
     float mn, mx, inv, z;
     minmax32(y, mn, mx);
     const uint32_t sz = affine_params(mn, mx, inv, z);
-    const float magic_z = 12582912.0f + z;
+    const float2 inv2 = splat2(inv), magic2 = splat2(12582912.0f + z);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) w[i] = encode4(y[4 * i], y[4 * i + 1], y[4 * i + 2], y[4 * i + 3], inv, magic_z);
+    for (int i = 0; i < 8; ++i) w[i] = encode4(y[2 * i], y[2 * i + 1], inv2, magic2);
     return sz;
 }
 
-// Dequantize 8 code words with (s, z): x_j = (q_j - z) * s * scale (scale folds a decay).
-__device__ __forceinline__ void dequantize_group(const uint32_t (&w)[8], uint32_t sz, float scale, float (&x)[32]) {
+// Dequantize 8 code words with (s, z): x_j = (q_j - z) * (s * scale) (scale folds a decay).
+// 2^23 + q comes straight from a byte permute; subtracting 2^23 + z is exact.
+__device__ __forceinline__ void dequantize_group(const uint32_t (&w)[8], uint32_t sz, float scale, float2 (&x)[16]) {
     const float s = __half2float(__ushort_as_half((unsigned short)(sz & 0xffffu)));
     const float z = __half2float(__ushort_as_half((unsigned short)(sz >> 16)));
-    const float zb = 8388608.0f + z;  // 2^23 + z, exact for |z| <= 2^23
-    const float sa = s * scale;
+    const float2 nzb = splat2(-(8388608.0f + z));  // -(2^23 + z), exact for |z| <= 2^23
+    const float2 sa = splat2(s * scale);
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-#pragma unroll
-        for (int b = 0; b < 4; ++b) x[4 * i + b] = (u8_biased(w[i], b) - zb) * sa;
+        x[2 * i] = mul2(add2(make_float2(u8_biased(w[i], 0), u8_biased(w[i], 1)), nzb), sa);
+        x[2 * i + 1] = mul2(add2(make_float2(u8_biased(w[i], 2), u8_biased(w[i], 3)), nzb), sa);
     }
+}
+
+// In-thread H_32 on 16 pairs (component j of the group is y[j/2].x or .y).
+__device__ __forceinline__ void hadamard_pairs(float2 (&y)[16]) {
+    float x[32];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+        x[2 * j] = y[j].x;
+        x[2 * j + 1] = y[j].y;
+    }
+    hadamard_regs(x);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) y[j] = make_float2(x[2 * j], x[2 * j + 1]);
 }
 
 __device__ __forceinline__ float2 h2_to_f2(uint32_t w) {

@@ -55,4 +55,11 @@ cudaError_t take_status_convert(uint32_t *bits);
 int sm_count();
 int max_smem_per_block();
 
+// Raises a kernel's dynamic shared-memory limit to at least `bytes` on the current
+// device (the attribute call is made once per kernel, device and larger size).
+cudaError_t ensure_smem_limit(const void *kernel, int bytes);
+
+// Device address of a __device__ status word, looked up once per device.
+cudaError_t symbol_address_cached(const void *symbol, uint32_t **cache_per_device, uint32_t **out);
+
 }  // namespace damp

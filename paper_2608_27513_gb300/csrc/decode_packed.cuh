@@ -8,19 +8,22 @@
 // the update, and a quantization group is 32 columns of one row, so a tile is
 // (slot, head, value block c): all d_k packed rows x 32 columns.  A tile is one
 // contiguous record (value-block-major, App. A.5) and is self-contained: no
-// cross-tile reduction.  One warp owns one tile at a time; lane l owns packed
-// rows l, l+32, ... with all 32 columns in registers, so min/max and the
-// requantizer of a group are thread-local.  The two column reductions
-// r = S_bar^T k and o = S^T q go through shared memory.
+// cross-tile reduction.  One warp owns one tile at a time:
+//   * UINT8 rows: lane l owns low-tier rows l, l+32, ... with all 32 columns in
+//     registers, so min/max and requantization of a group are thread-local; the
+//     column reductions r = S_bar^T k and o = S^T q go through shared memory.
+//     The code is branch-free: lanes past the last row process a clamped row
+//     with zero weights and skip its store.
+//   * FP16 rows: lane j owns column j of all K_hi rows, so their part of both
+//     reductions stays in the lane.
 //
-// Domains: the low tier stores codes of H_32-transformed rows (App. A.5).  Since
-// H_32 acts on the value axis only and is symmetric and orthonormal, the update
-// can be carried out in the transformed domain: with S~ = S H,
-//     r~ = H r,  S~_t = Lambda S~ + beta k (H v - r~)^T,  o = H (S~^T q).
-// Low-tier rows therefore never pass through a butterfly; only the 32-vectors
-// v, r_hi, d and o do (a 5-step butterfly across the warp's lanes).  FP16 rows
-// stay in the natural domain: their partial sums are reduced separately and
-// transformed once per tile.
+// Domains: the low tier stores codes of H_32-transformed rows (App. A.5).  H_32
+// acts on the value axis only and is symmetric and orthonormal, so with
+// S~ = S H the low-tier rows are updated in the transformed domain:
+//     r = H r~_lo + r_hi,  d = v - r,  S~_t = Lambda S~ + beta k (H d)^T,
+//     o = H o~_lo + o_hi.
+// Low-tier rows never pass through a butterfly; only the 32-vectors r~_lo, d and
+// o~_lo do (a 5-step butterfly across the warp's lanes).
 //
 // Pipeline: a persistent grid; every warp walks a contiguous range of tiles.
 // Lane 0 keeps NSTAGE-1 tiles in flight with 1-D bulk copies (TMA engine) into a
@@ -50,59 +53,75 @@ struct PackedParams {
     uint32_t *status;
 };
 
-constexpr int kPartOff = 64;                        // after NSTAGE (<= 8) mbarriers
-constexpr int kPartStride = 36;                     // floats per row of the partial-sum buffer
-constexpr int kDvecOff = kPartOff + 32 * kPartStride * 4;
-constexpr int kScratchBytes = kDvecOff + 64 * 4;    // bytes before the first stage (rounded up by the host)
+// per-warp scratch before the stage ring
+constexpr int kPartOff = 64;                              // after NSTAGE (<= 8) mbarriers
+constexpr int kPartStride = 36;                           // floats per row of the partial-sum buffer
+constexpr int kDvecOff = kPartOff + 32 * kPartStride * 4; // 32 floats: H d for the low tier
+constexpr int kHopsOff = kDvecOff + 32 * 4;               // FP16-row operands, 32 B per row pair
+__host__ __device__ constexpr int scratch_bytes(int k_hi) { return kHopsOff + 32 * ((k_hi + 1) / 2); }
 
 __device__ __forceinline__ float ldsf(uint32_t a) { return __uint_as_float(lds32(a)); }
 
-// Column sum over the lanes' 32-vectors: lane j returns sum_l v_l[j].
-// Uses part[32][36]; the caller brackets it with __syncwarp.
-__device__ __forceinline__ float column_sum(const float (&v)[32], uint32_t part, int lane) {
+// Column sum over the lanes' 32-vectors (16 pairs): lane j returns sum_l v_l[j].
+__device__ __forceinline__ float column_sum(const float2 (&v)[16], uint32_t part, int lane) {
 #pragma unroll
     for (int jj = 0; jj < 8; ++jj) {
-        uint4 w;
-        w.x = __float_as_uint(v[4 * jj]);
-        w.y = __float_as_uint(v[4 * jj + 1]);
-        w.z = __float_as_uint(v[4 * jj + 2]);
-        w.w = __float_as_uint(v[4 * jj + 3]);
-        sts128(part + (lane * kPartStride + 4 * jj) * 4, w);
+        sts128(part + (lane * kPartStride + 4 * jj) * 4,
+               make_uint4(__float_as_uint(v[2 * jj].x), __float_as_uint(v[2 * jj].y), __float_as_uint(v[2 * jj + 1].x),
+                          __float_as_uint(v[2 * jj + 1].y)));
     }
     __syncwarp();
-    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+    float2 s0 = make_float2(0.f, 0.f), s1 = s0;
 #pragma unroll
     for (int l = 0; l < 32; l += 4) {
-        s0 += ldsf(part + ((l + 0) * kPartStride + lane) * 4);
-        s1 += ldsf(part + ((l + 1) * kPartStride + lane) * 4);
-        s2 += ldsf(part + ((l + 2) * kPartStride + lane) * 4);
-        s3 += ldsf(part + ((l + 3) * kPartStride + lane) * 4);
+        s0 = add2(s0, make_float2(ldsf(part + ((l + 0) * kPartStride + lane) * 4),
+                                  ldsf(part + ((l + 1) * kPartStride + lane) * 4)));
+        s1 = add2(s1, make_float2(ldsf(part + ((l + 2) * kPartStride + lane) * 4),
+                                  ldsf(part + ((l + 3) * kPartStride + lane) * 4)));
     }
     __syncwarp();
-    return (s0 + s1) + (s2 + s3);
+    const float2 t = add2(s0, s1);
+    return t.x + t.y;
 }
 
-// Sum of the first n rows of part[][] at column `lane`.
-__device__ __forceinline__ float partial_rows_sum(uint32_t part, int n, int lane) {
-    float s = 0.f;
-    for (int l = 0; l < n; ++l) s += ldsf(part + (l * kPartStride + lane) * 4);
-    return s;
+__device__ __forceinline__ float bf16_at(uint32_t base, int i) {
+    const uint32_t w = lds32(base + 2 * (i & ~1));
+    return __uint_as_float((i & 1) ? (w & 0xffff0000u) : (w << 16));
 }
 
-__device__ __forceinline__ void store_row_scaled(uint32_t part, int lane, const float (&x)[32], float c) {
-#pragma unroll
-    for (int jj = 0; jj < 8; ++jj) {
-        uint4 w;
-        w.x = __float_as_uint(x[4 * jj] * c);
-        w.y = __float_as_uint(x[4 * jj + 1] * c);
-        w.z = __float_as_uint(x[4 * jj + 2] * c);
-        w.w = __float_as_uint(x[4 * jj + 3] * c);
-        sts128(part + (lane * kPartStride + 4 * jj) * 4, w);
+__device__ __forceinline__ float h16_to_f32(uint32_t h) { return __half2float(__ushort_as_half((unsigned short)h)); }
+
+__device__ __forceinline__ void sts16(uint32_t a, unsigned short v) {
+    asm volatile("st.shared.b16 [%0], %1;" ::"r"(a), "h"(v) : "memory");
+}
+
+// (batch row, head, value block) of a tile index, advanced without divisions.
+struct Cursor {
+    int b, h, c;
+};
+__device__ __forceinline__ Cursor cursor_at(int64_t t, int H, int V) {
+    Cursor k;
+    const int64_t bh = t / V;
+    k.c = (int)(t - bh * V);
+    k.b = (int)(bh / H);
+    k.h = (int)(bh - (int64_t)k.b * H);
+    return k;
+}
+__device__ __forceinline__ void advance(Cursor &k, int H, int V) {
+    if (++k.c == V) {
+        k.c = 0;
+        if (++k.h == H) {
+            k.h = 0;
+            ++k.b;
+        }
     }
 }
 
-template <int R, bool KDA, bool HAD, bool BF16>
+// RL = ceil((d_k - K_hi) / 32): low-tier row slots per lane, fixed at compile time
+// so that the row loops unroll into one basic block.
+template <int RL, bool KDA, bool HAD, bool BF16>
 __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams p) {
+    constexpr int R = RL > 0 ? RL : 1;
     extern __shared__ __align__(128) uint8_t smem[];
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
@@ -111,9 +130,12 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
     const uint32_t bar0 = ws;
     const uint32_t part = ws + kPartOff;
     const uint32_t dvec = ws + kDvecOff;
+    const uint32_t hops = ws + kHopsOff;
     const uint32_t stage0 = ws + p.stage0_off;
     const int esz = BF16 ? 2 : 4;
     const int K = p.K;
+    const int lo = p.dk - K;  // low-tier rows
+    const int H = p.H, V = p.V;
 
     const int64_t gw = (int64_t)blockIdx.x * nw + warp;
     const int64_t nwt = (int64_t)gridDim.x * nw;
@@ -127,216 +149,227 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
     }
     __syncwarp();
 
-    // ---- producer (lane 0): bulk copies of tile t into stage s ----
-    auto issue = [&](int64_t t, int s) {
-        const int c = (int)(t % p.V);
-        const int64_t bh = t / p.V;
-        const int h = (int)(bh % p.H);
-        const int b = (int)(bh / p.H);
-        const int64_t slot = p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b;
+    auto slot_of = [&](int b) -> int64_t { return p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b; };
+
+    // ---- producer (lane 0): bulk copies of tile t (cursor k) into stage s ----
+    auto issue = [&](int64_t t, const Cursor &k, int s) {
+        const int64_t slot = slot_of(k.b);
         const bool ok = slot >= 0 && slot < p.num_slots;
-        const bool ops = (t == t0) || (c == 0);
+        const bool ops = (t == t0) || (k.c == 0);
         const uint32_t st = stage0 + (uint32_t)(s * p.stage_bytes);
         const uint32_t bar = bar0 + 8 * s;
         uint32_t bytes = (uint32_t)p.bytes_v;
         if (ok) bytes += (uint32_t)p.rec_bytes;
         if (ops) bytes += 2u * p.bytes_qk + p.bytes_g + p.bytes_perm;
         mbar_arrive_expect_tx(bar, bytes);
-        if (ok) bulk_g2s(st, p.state + slot * p.slot_bytes + (int64_t)(h * p.V + c) * p.rec_bytes, p.rec_bytes, bar);
-        bulk_g2s(st + p.off_v, (const uint8_t *)p.v + (((int64_t)b * p.H + h) * p.dv + c * kG) * esz, p.bytes_v, bar);
+        const int64_t bh = (int64_t)k.b * H + k.h;
+        if (ok) bulk_g2s(st, p.state + slot * p.slot_bytes + (int64_t)(k.h * V + k.c) * p.rec_bytes, p.rec_bytes, bar);
+        bulk_g2s(st + p.off_v, (const uint8_t *)p.v + (bh * p.dv + k.c * kG) * esz, p.bytes_v, bar);
         if (ops) {
-            const int hq = (h * p.Hqk) / p.H;
-            const int64_t qoff = ((int64_t)b * p.Hqk + hq) * p.dk * esz;
+            const int hq = (k.h * p.Hqk) / H;
+            const int64_t qoff = ((int64_t)k.b * p.Hqk + hq) * p.dk * esz;
             bulk_g2s(st + p.off_q, (const uint8_t *)p.q + qoff, p.bytes_qk, bar);
             bulk_g2s(st + p.off_k, (const uint8_t *)p.k + qoff, p.bytes_qk, bar);
-            if (KDA) bulk_g2s(st + p.off_g, p.g + ((int64_t)b * p.H + h) * p.dk, p.bytes_g, bar);
-            bulk_g2s(st + p.off_perm, p.perm + (int64_t)h * p.dk, p.bytes_perm, bar);
+            if (KDA) bulk_g2s(st + p.off_g, p.g + bh * p.dk, p.bytes_g, bar);
+            bulk_g2s(st + p.off_perm, p.perm + (int64_t)k.h * p.dk, p.bytes_perm, bar);
         }
     };
 
+    Cursor cur = cursor_at(t0, H, V);
+    Cursor pre = cur;  // next tile to load (lane 0)
+    int64_t t_pre = t0;
     if (lane == 0) {
-        for (int j = 0; j < p.nstage - 1 && t0 + j < t1; ++j) issue(t0 + j, j);
+        for (int j = 0; j < p.nstage - 1 && t_pre < t1; ++j) {
+            issue(t_pre, pre, j);
+            ++t_pre;
+            advance(pre, H, V);
+        }
     }
 
-    float kk[R], qq[R], bk[R], aa[R];
+    // low-tier row operands of this lane (zero weights for lanes past the last row)
+    float2 kk[R], qq[R], bk[R];
+    float aa[R];
     int s = 0;
     uint32_t parity = 0;
     bool timed_out = false, bad_slot = false;
     int64_t t_fail = t1;
 
-    for (int64_t t = t0; t < t1; ++t) {
+    for (int64_t t = t0; t < t1; ++t, advance(cur, H, V)) {
         const uint32_t st = stage0 + (uint32_t)(s * p.stage_bytes);
         if (!__all_sync(kFull, mbar_wait_bounded(bar0 + 8 * s, parity))) {
             timed_out = true;
             t_fail = t;
             break;
         }
-        const int c = (int)(t % p.V);
-        const int64_t bh = t / p.V;
-        const int h = (int)(bh % p.H);
-        const int b = (int)(bh / p.H);
-        const int64_t slot = p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b;
+        const int b = cur.b, h = cur.h, c = cur.c;
+        const int64_t slot = slot_of(b);
         const bool ok = slot >= 0 && slot < p.num_slots;
         bad_slot |= !ok;
 
         // ---- per-(slot, head) operands, gathered into calibrated key order ----
         if (t == t0 || c == 0) {
-            const float beta = p.beta[(int64_t)b * p.H + h];
-            const float alpha = KDA ? 0.f : expf(p.g[(int64_t)b * p.H + h]);
+            const float beta = p.beta[(int64_t)b * H + h];
+            const float alpha = KDA ? 0.f : expf(p.g[(int64_t)b * H + h]);
+            // d_k is a power of two: masking keeps a malformed permutation in bounds
+            auto chan = [&](int u) { return (int)(lds32(st + p.off_perm + (u & ~3)) >> (8 * (u & 3))) & (p.dk - 1); };
+            auto kv_at = [&](int ch) { return BF16 ? bf16_at(st + p.off_k, ch) : ldsf(st + p.off_k + 4 * ch); };
+            auto qv_at = [&](int ch) { return BF16 ? bf16_at(st + p.off_q, ch) : ldsf(st + p.off_q + 4 * ch); };
+            auto av_at = [&](int ch) { return KDA ? expf(ldsf(st + p.off_g + 4 * ch)) : alpha; };
 #pragma unroll
             for (int i = 0; i < R; ++i) {
-                const int u = lane + 32 * i;
-                // d_k is a power of two: masking keeps a malformed permutation in bounds
-                const int ch = (int)(lds32(st + p.off_perm + (u & ~3)) >> (8 * (u & 3))) & (p.dk - 1);
-                float kv, qv;
-                if (BF16) {
-                    const uint32_t kw = lds32(st + p.off_k + 2 * (ch & ~1));
-                    const uint32_t qw = lds32(st + p.off_q + 2 * (ch & ~1));
-                    kv = __uint_as_float((ch & 1) ? (kw & 0xffff0000u) : (kw << 16));
-                    qv = __uint_as_float((ch & 1) ? (qw & 0xffff0000u) : (qw << 16));
-                } else {
-                    kv = ldsf(st + p.off_k + 4 * ch);
-                    qv = ldsf(st + p.off_q + 4 * ch);
-                }
-                kk[i] = kv;
-                qq[i] = qv;
-                bk[i] = beta * kv;
-                aa[i] = KDA ? expf(ldsf(st + p.off_g + 4 * ch)) : alpha;
+                const int r = lane + 32 * i;
+                const bool live = r < lo;
+                const int ch = chan(live ? K + r : (lo > 0 ? K + lo - 1 : 0));  // stays inside perm
+                const float kv = live ? kv_at(ch) : 0.f;
+                kk[i] = splat2(kv);
+                qq[i] = splat2(live ? qv_at(ch) : 0.f);
+                bk[i] = splat2(beta * kv);
+                aa[i] = av_at(ch);
             }
-        }
-
-        // ---- v block -> transformed domain ----
-        float vj;
-        if (BF16) {
-            const uint32_t w = lds32(st + p.off_v + 2 * (lane & ~1));
-            vj = __uint_as_float((lane & 1) ? (w & 0xffff0000u) : (w << 16));
-        } else {
-            vj = ldsf(st + p.off_v + 4 * lane);
-        }
-        const float vt = HAD ? hadamard_lanes(vj, lane) : vj;
-
-        float x[R][32];
-        float acc[32];
-        float rhi = 0.f;
-
-        if (ok) {
-            // ---- phase 1: reconstruct, decay, partial r = S_bar^T k ----
-#pragma unroll
-            for (int j = 0; j < 32; ++j) acc[j] = 0.f;
-#pragma unroll
-            for (int i = 0; i < R; ++i) {
-                const int u = lane + 32 * i;
-                if (u < K) {
-#pragma unroll
-                    for (int m = 0; m < 4; ++m) {
-                        const uint4 w = lds128(st + hi_chunk_off(u, m));
-                        const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const float2 f = h2_to_f2(ww[e]);
-                            x[i][8 * m + 2 * e] = f.x * aa[i];
-                            x[i][8 * m + 2 * e + 1] = f.y * aa[i];
-                        }
-                    }
-                    store_row_scaled(part, lane, x[i], kk[i]);
-                } else {
-                    const int r = u - K;
-                    const uint4 c0 = lds128(st + p.codes_off + lo_chunk_off(r, 0));
-                    const uint4 c1 = lds128(st + p.codes_off + lo_chunk_off(r, 1));
-                    const uint32_t sz = lds32(st + p.meta_off + 4 * r);
-                    const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-                    dequantize_group(w, sz, aa[i], x[i]);
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) acc[j] = fmaf(x[i][j], kk[i], acc[j]);
-                }
-                if (32 * i < K) {  // warp-uniform: this slot holds FP16 rows
-                    __syncwarp();
-                    rhi += partial_rows_sum(part, min(32, K - 32 * i), lane);
-                    __syncwarp();
-                }
+            // FP16 rows in pairs: {a_u, a_u+1, k_u, k_u+1} {q_u, q_u+1, bk_u, bk_u+1}
+            for (int u = 2 * lane; u < K; u += 64) {
+                const int c0 = chan(u);
+                const bool two = u + 1 < K;
+                const int c1 = two ? chan(u + 1) : c0;
+                const float k0 = kv_at(c0), k1 = two ? kv_at(c1) : 0.f;
+                sts128(hops + 16 * u, make_uint4(__float_as_uint(av_at(c0)), __float_as_uint(two ? av_at(c1) : 0.f),
+                                                 __float_as_uint(k0), __float_as_uint(k1)));
+                sts128(hops + 16 * u + 16,
+                       make_uint4(__float_as_uint(qv_at(c0)), __float_as_uint(two ? qv_at(c1) : 0.f),
+                                  __float_as_uint(beta * k0), __float_as_uint(beta * k1)));
             }
-            const float rlo = column_sum(acc, part, lane);
-            const float rt = rlo + ((HAD && K > 0) ? hadamard_lanes(rhi, lane) : rhi);
-            const float dt = vt - rt;                                        // d~ = H(v - r)
-            const float dn = (HAD && K > 0) ? hadamard_lanes(dt, lane) : dt;  // natural d
-            sts32(dvec + 4 * lane, __float_as_uint(dt));
-            sts32(dvec + 128 + 4 * lane, __float_as_uint(dn));
-        }
-
-        // ---- keep the ring full: next load goes into the stage of tile t-1 ----
-        if (lane == 0 && t + p.nstage - 1 < t1) {
-            bulk_wait_read_all();
-            const int sn = (s + p.nstage - 1) % p.nstage;
-            issue(t + p.nstage - 1, sn);
-        }
-
-        if (ok) {
             __syncwarp();
-            float d[32];
+        }
+
+        const float vj = BF16 ? bf16_at(st + p.off_v, lane) : ldsf(st + p.off_v + 4 * lane);
+
+        if (ok) {
+            const float vt = HAD ? hadamard_lanes(vj, lane) : vj;  // H v
+            float2 x[R][16];
+            float2 acc[16];
+            // ---- phase 1, low tier: reconstruct, decay, partial r~ = S~_bar^T k ----
+#pragma unroll
+            for (int i = 0; i < RL; ++i) {
+                const int r = min(lane + 32 * i, lo - 1);
+                const uint4 c0 = lds128(st + p.codes_off + lo_chunk_off(r, 0));
+                const uint4 c1 = lds128(st + p.codes_off + lo_chunk_off(r, 1));
+                const uint32_t sz = lds32(st + p.meta_off + 4 * r);
+                const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+                dequantize_group(w, sz, aa[i], x[i]);
+#pragma unroll
+                for (int j = 0; j < 16; ++j) acc[j] = (i == 0) ? mul2(x[i][j], kk[i]) : fma2(x[i][j], kk[i], acc[j]);
+            }
+            if (RL == 0) {
+#pragma unroll
+                for (int j = 0; j < 16; ++j) acc[j] = make_float2(0.f, 0.f);
+            }
+
+            // ---- phase 1, FP16 tier (lane = column), two rows per step ----
+            const uint32_t col = st + 2 * lane;
+            float2 rh = make_float2(0.f, 0.f);
+            for (int u = 0; u < K; u += 2) {
+                const uint4 op = lds128(hops + 16 * u);
+                uint16_t h0, h1 = 0;
+                asm volatile("ld.shared.u16 %0, [%1];" : "=h"(h0) : "r"(col + 64 * u));
+                if (u + 1 < K) asm volatile("ld.shared.u16 %0, [%1];" : "=h"(h1) : "r"(col + 64 * u + 64));
+                const float2 xh = mul2(make_float2(h16_to_f32(h0), h16_to_f32(h1)),
+                                       make_float2(__uint_as_float(op.x), __uint_as_float(op.y)));
+                rh = fma2(xh, make_float2(__uint_as_float(op.z), __uint_as_float(op.w)), rh);
+            }
+            const float rhi = rh.x + rh.y;
+            const float rlo = column_sum(acc, part, lane);  // r~_lo (transformed domain when HAD)
+
+            // r = H r~_lo + r_hi;  d = v - r (natural, FP16 rows);  H d = H v - r~_lo - H r_hi (low tier)
+            float dj, dt;
+            if (HAD) {
+                if (K > 0) {
+                    const float hr_lo = hadamard_lanes(rlo, lane);
+                    const float hr_hi = hadamard_lanes(rhi, lane);
+                    dj = vj - (hr_lo + rhi);
+                    dt = vt - (rlo + hr_hi);
+                } else {
+                    dj = 0.f;
+                    dt = vt - rlo;
+                }
+            } else {
+                dj = vj - (rlo + rhi);
+                dt = dj;
+            }
+            sts32(dvec + 4 * lane, __float_as_uint(dt));
+
+            // ---- keep the ring full: next load goes into the stage of tile t-1 ----
+            if (lane == 0 && t_pre < t1) {
+                bulk_wait_read_all();
+                issue(t_pre, pre, (s + p.nstage - 1) % p.nstage);
+                ++t_pre;
+                advance(pre, H, V);
+            }
+            __syncwarp();
+
+            // ---- phase 2, low tier: rank-1 correction, partial o~, requantize in place ----
+            float2 d[16];
 #pragma unroll
             for (int jj = 0; jj < 8; ++jj) {
                 const uint4 w = lds128(dvec + 16 * jj);
-                d[4 * jj] = __uint_as_float(w.x);
-                d[4 * jj + 1] = __uint_as_float(w.y);
-                d[4 * jj + 2] = __uint_as_float(w.z);
-                d[4 * jj + 3] = __uint_as_float(w.w);
+                d[2 * jj] = make_float2(__uint_as_float(w.x), __uint_as_float(w.y));
+                d[2 * jj + 1] = make_float2(__uint_as_float(w.z), __uint_as_float(w.w));
             }
-            // ---- phase 2: rank-1 correction, partial o, requantize in place ----
-            float ohi = 0.f;
 #pragma unroll
-            for (int j = 0; j < 32; ++j) acc[j] = 0.f;
+            for (int i = 0; i < RL; ++i) {
+                const int r = lane + 32 * i;
 #pragma unroll
-            for (int i = 0; i < R; ++i) {
-                const int u = lane + 32 * i;
-                if (u < K) {
-#pragma unroll
-                    for (int jj = 0; jj < 8; ++jj) {
-                        const uint4 w = lds128(dvec + 128 + 16 * jj);
-                        x[i][4 * jj] = fmaf(bk[i], __uint_as_float(w.x), x[i][4 * jj]);
-                        x[i][4 * jj + 1] = fmaf(bk[i], __uint_as_float(w.y), x[i][4 * jj + 1]);
-                        x[i][4 * jj + 2] = fmaf(bk[i], __uint_as_float(w.z), x[i][4 * jj + 2]);
-                        x[i][4 * jj + 3] = fmaf(bk[i], __uint_as_float(w.w), x[i][4 * jj + 3]);
-                    }
-                    store_row_scaled(part, lane, x[i], qq[i]);
-#pragma unroll
-                    for (int m = 0; m < 4; ++m) {
-                        uint32_t hw[4];
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            hw[e] = f2_to_h2(x[i][8 * m + 2 * e], x[i][8 * m + 2 * e + 1]);
-                        }
-                        sts128(st + hi_chunk_off(u, m), make_uint4(hw[0], hw[1], hw[2], hw[3]));
-                    }
-                } else {
-                    const int r = u - K;
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        x[i][j] = fmaf(bk[i], d[j], x[i][j]);
-                        acc[j] = fmaf(x[i][j], qq[i], acc[j]);
-                    }
-                    uint32_t w[8];
-                    const uint32_t sz = quantize_group(x[i], w);
-                    sts128(st + p.codes_off + lo_chunk_off(r, 0), make_uint4(w[0], w[1], w[2], w[3]));
-                    sts128(st + p.codes_off + lo_chunk_off(r, 1), make_uint4(w[4], w[5], w[6], w[7]));
-                    sts32(st + p.meta_off + 4 * r, sz);
+                for (int j = 0; j < 16; ++j) {
+                    x[i][j] = fma2(bk[i], d[j], x[i][j]);
+                    acc[j] = (i == 0) ? mul2(x[i][j], qq[i]) : fma2(x[i][j], qq[i], acc[j]);
                 }
-                if (32 * i < K) {
-                    __syncwarp();
-                    ohi += partial_rows_sum(part, min(32, K - 32 * i), lane);
-                    __syncwarp();
-                }
+                uint32_t w[8];
+                const uint32_t sz = quantize_group(x[i], w);
+                // a lane past the last row writes into its own slice of the (idle)
+                // partial-sum buffer instead of branching around the stores
+                const bool live = r < lo;
+                const uint32_t trash = part + lane * kPartStride * 4;
+                sts128(live ? st + p.codes_off + lo_chunk_off(r, 0) : trash, make_uint4(w[0], w[1], w[2], w[3]));
+                sts128(live ? st + p.codes_off + lo_chunk_off(r, 1) : trash + 16, make_uint4(w[4], w[5], w[6], w[7]));
+                sts32(live ? st + p.meta_off + 4 * r : trash + 32, sz);
+            }
+            if (RL == 0) {
+#pragma unroll
+                for (int j = 0; j < 16; ++j) acc[j] = make_float2(0.f, 0.f);
+            }
+            __syncwarp();
+
+            // ---- phase 2, FP16 tier: S = S_bar + beta k d, o_hi, FP16 store ----
+            float2 oh = make_float2(0.f, 0.f);
+            for (int u = 0; u < K; u += 2) {
+                const uint4 op0 = lds128(hops + 16 * u);
+                const uint4 op1 = lds128(hops + 16 * u + 16);
+                uint16_t h0, h1 = 0;
+                asm volatile("ld.shared.u16 %0, [%1];" : "=h"(h0) : "r"(col + 64 * u));
+                if (u + 1 < K) asm volatile("ld.shared.u16 %0, [%1];" : "=h"(h1) : "r"(col + 64 * u + 64));
+                const float2 xh = mul2(make_float2(h16_to_f32(h0), h16_to_f32(h1)),
+                                       make_float2(__uint_as_float(op0.x), __uint_as_float(op0.y)));
+                const float2 y = fma2(make_float2(__uint_as_float(op1.z), __uint_as_float(op1.w)), splat2(dj), xh);
+                oh = fma2(y, make_float2(__uint_as_float(op1.x), __uint_as_float(op1.y)), oh);
+                const uint32_t hy = f2_to_h2(y.x, y.y);
+                sts16(col + 64 * u, (unsigned short)(hy & 0xffffu));
+                if (u + 1 < K) sts16(col + 64 * u + 64, (unsigned short)(hy >> 16));
             }
             const float olo = column_sum(acc, part, lane);
-            const float oj = ((HAD) ? hadamard_lanes(olo, lane) : olo) + ohi;
-            p.o[((int64_t)b * p.H + h) * p.dv + c * kG + lane] = oj;
+            const float oj = (HAD ? hadamard_lanes(olo, lane) : olo) + (oh.x + oh.y);
+            p.o[((int64_t)b * H + h) * p.dv + c * kG + lane] = oj;
 
             // ---- write the updated record back ----
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) {
-                bulk_s2g(p.state + slot * p.slot_bytes + (int64_t)(h * p.V + c) * p.rec_bytes, st, p.rec_bytes);
+                bulk_s2g(p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * p.rec_bytes, st, p.rec_bytes);
                 bulk_commit();
             }
+        } else if (lane == 0 && t_pre < t1) {
+            bulk_wait_read_all();
+            issue(t_pre, pre, (s + p.nstage - 1) % p.nstage);
+            ++t_pre;
+            advance(pre, H, V);
         }
         __syncwarp();
         if (++s == p.nstage) {

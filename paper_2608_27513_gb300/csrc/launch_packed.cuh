@@ -60,7 +60,7 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
     off += p.bytes_perm;
     p.stage_bytes = (off + 127) & ~127;
     p.nstage = kPackedStages;
-    p.stage0_off = (kScratchBytes + 127) & ~127;
+    p.stage0_off = (scratch_bytes(a.K) + 127) & ~127;
     p.warp_smem = p.stage0_off + p.nstage * p.stage_bytes;
     p.total_tiles = (int64_t)a.batch * a.H * V;
     p.status = status;
@@ -81,19 +81,22 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
 
     void (*kern)(PackedParams) = nullptr;
     const bool had = a.fmt == 0;
-#define DAMP_PICK(R_)                                                                          \
-    if (a.dk == 32 * R_) {                                                                     \
-        if (had) kern = a.in_bf16 ? packed_step_kernel<R_, KDA, true, true>                    \
-                                  : packed_step_kernel<R_, KDA, true, false>;                  \
-        else kern = a.in_bf16 ? packed_step_kernel<R_, KDA, false, true>                       \
-                              : packed_step_kernel<R_, KDA, false, false>;                     \
+#define DAMP_PICK(RL_)                                                                         \
+    if (rl == RL_) {                                                                           \
+        if (had) kern = a.in_bf16 ? packed_step_kernel<RL_, KDA, true, true>                   \
+                                  : packed_step_kernel<RL_, KDA, true, false>;                 \
+        else kern = a.in_bf16 ? packed_step_kernel<RL_, KDA, false, true>                      \
+                              : packed_step_kernel<RL_, KDA, false, false>;                    \
     }
+    const int rl = (a.dk - a.K + 31) / 32;
+    DAMP_PICK(0)
     DAMP_PICK(1)
     DAMP_PICK(2)
+    DAMP_PICK(3)
     DAMP_PICK(4)
 #undef DAMP_PICK
     if (!kern) return cudaErrorInvalidValue;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e = ensure_smem_limit(reinterpret_cast<const void *>(kern), smem);
     if (e != cudaSuccess) return e;
     kern<<<grid, 32 * warps, smem, stream>>>(p);
     return cudaGetLastError();
