@@ -84,6 +84,8 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
                     } else {
                         const int r = u - K;
                         if (HAD) hadamard_pairs(x);
+#pragma unroll
+                        for (int m = 0; m < 16; ++m) x[m] = mul2(x[m], splat2(kDown));  // working scale
                         uint32_t w[8];
                         const uint32_t sz = quantize_group(x, w);
                         *reinterpret_cast<uint4 *>(rec + p.codes_off + lo_chunk_off(r, 0)) =

@@ -3,7 +3,7 @@
 #include <atomic>
 #include <climits>
 
-#include "../../include/damp.h"
+#include "damp.h"
 #include "damp_common.cuh"
 #include "damp_internal.h"
 

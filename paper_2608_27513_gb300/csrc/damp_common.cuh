@@ -108,6 +108,9 @@ __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.comm
 __device__ __forceinline__ void bulk_wait_read_all() {
     asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
+__device__ __forceinline__ void bulk_wait_read_all_but_newest() {
+    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 // Generic-proxy writes to shared memory become visible to the async proxy (bulk store).
@@ -212,37 +215,53 @@ __device__ __forceinline__ float rcp_approx(float x) {
     return r;
 }
 
-// Scale and zero point of a group from its extrema:
+// ---------------------------------------------------------------------------
+// Scaled working domain.  Low-tier values are kept multiplied by 2^-39 while a
+// tile is in registers (exact power-of-two scaling: every FP32 rounding is the
+// same as in the unscaled domain for |x| >= 2^-87).  This lets the requantizer
+// land each code directly on the binary32 denormal grid (below).
+// ---------------------------------------------------------------------------
+constexpr float kDown = 0x1p-39f;
+constexpr float kUp = 0x1p39f;
+
+// Scale and zero point of a group from its scaled extrema mn', mx':
 //   s = fp16((max - min)/255), z = fp16(round_even(-min / s)); a block whose s
 //   rounds to 0 widens [min, max] to contain 0, and s = 1, z = 0 if s is still 0.
-// Returns the packed (s, z) binary16 pair; inv_out ~ 1/s and z_out as float.
-// The reciprocal is the hardware approximation (within one ulp): a code can only
-// move where x/s + z sits at a rounding tie.
-__device__ __forceinline__ uint32_t affine_params(float mn, float mx, float &inv_out, float &z_out) {
-    float s = __half2float(__float2half_rn((mx - mn) * (1.0f / 255.0f)));
-    if (s == 0.0f) {
-        mn = fminf(mn, 0.0f);
-        mx = fmaxf(mx, 0.0f);
-        s = __half2float(__float2half_rn((mx - mn) * (1.0f / 255.0f)));
-        if (s == 0.0f) s = 1.0f;
-    }
+// Returns the packed (s, z) binary16 pair, inv ~ 1/s (hardware reciprocal,
+// within one ulp: a code can only move where x/s + z sits at a rounding tie)
+// and z as float.
+__device__ __forceinline__ uint32_t affine_params_scaled(float mn, float mx, float &inv_out, float &z_out) {
+    // branch-free so that the chains of several rows interleave
+    const float s0 = __half2float(__float2half_rn((mx - mn) * (kUp / 255.0f)));
+    const float mn0 = fminf(mn, 0.0f), mx0 = fmaxf(mx, 0.0f);
+    float s1 = __half2float(__float2half_rn((mx0 - mn0) * (kUp / 255.0f)));
+    s1 = (s1 == 0.0f) ? 1.0f : s1;
+    const bool degenerate = s0 == 0.0f;
+    const float s = degenerate ? s1 : s0;
+    const float m = degenerate ? mn0 : mn;
     const float inv = rcp_approx(s);
-    const __half zh = __float2half_rn(rintf(-mn * inv));
-    const __half sh = __float2half_rn(s);
+    const __half zh = __float2half_rn(rintf(-m * (inv * kUp)));
+    const __half sh = __float2half_rn(s);  // exact: s is already a binary16 value
     z_out = __half2float(zh);
     inv_out = inv;
     return (uint32_t)__half_as_ushort(sh) | ((uint32_t)__half_as_ushort(zh) << 16);
 }
 
-// Codes of 4 values: q = sat_[0,255](round_even(x / s) + z), packed little-endian.
-// fma(x, 1/s, 1.5*2^23 + z) rounds to the integer grid; its low 16 bits are the
-// signed integer; min.relu.s16x2 saturates two lanes at a time.
-__device__ __forceinline__ uint32_t encode4(float2 x01, float2 x23, float2 inv2, float2 magic2) {
-    const float2 a = fma2(x01, inv2, magic2);
-    const float2 b = fma2(x23, inv2, magic2);
-    const uint32_t ab = clamp_u8x2(prmt(__float_as_uint(a.x), __float_as_uint(a.y), 0x5410u));
-    const uint32_t cd = clamp_u8x2(prmt(__float_as_uint(b.x), __float_as_uint(b.y), 0x5410u));
-    return prmt(ab, cd, 0x6420u);
+// Codes of 4 scaled values: q = sat_[0,255](round_even(x / s) + z), packed
+// little-endian.  fma(x', inv * 2^-110, z * 2^-149) computes x/s + z scaled by
+// 2^-149 and rounds it once onto the denormal grid, so its bit pattern is the
+// integer round_even(x/s + z) (with the sign bit set when negative);
+// cvt.pack.sat saturates two such integers to [0, 255] and packs them.
+__device__ __forceinline__ uint32_t pack_sat_u8(uint32_t hi_byte, uint32_t lo_byte, uint32_t upper) {
+    uint32_t d;
+    asm("cvt.pack.sat.u8.s32.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(hi_byte), "r"(lo_byte), "r"(upper));
+    return d;
+}
+__device__ __forceinline__ uint32_t encode4(float2 x01, float2 x23, float2 inv2, float2 zc2) {
+    const float2 a = fma2(x01, inv2, zc2);
+    const float2 b = fma2(x23, inv2, zc2);
+    const uint32_t upper = pack_sat_u8(__float_as_uint(b.y), __float_as_uint(b.x), 0u);
+    return pack_sat_u8(__float_as_uint(a.y), __float_as_uint(a.x), upper);
 }
 
 __device__ __forceinline__ void minmax32(const float2 (&y)[16], float &mn, float &mx) {
@@ -258,18 +277,20 @@ __device__ __forceinline__ void minmax32(const float2 (&y)[16], float &mn, float
     mx = fmax3(fmax3(b[0], b[1], b[2]), fmax3(b[3], b[4], b[5]), b[5]);
 }
 
-// Quantize y (one lo row, one value block, 16 pairs) into 8 code words + packed (s, z).
+// Quantize y' (one lo row, one value block, 16 pairs, scaled by 2^-39) into
+// 8 code words + packed (s, z).
 __device__ __forceinline__ uint32_t quantize_group(const float2 (&y)[16], uint32_t (&w)[8]) {
     float mn, mx, inv, z;
     minmax32(y, mn, mx);
-    const uint32_t sz = affine_params(mn, mx, inv, z);
-    const float2 inv2 = splat2(inv), magic2 = splat2(12582912.0f + z);
+    const uint32_t sz = affine_params_scaled(mn, mx, inv, z);
+    const float2 inv2 = splat2(inv * 0x1p-110f), zc2 = splat2(z * 0x1p-149f);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) w[i] = encode4(y[2 * i], y[2 * i + 1], inv2, magic2);
+    for (int i = 0; i < 8; ++i) w[i] = encode4(y[2 * i], y[2 * i + 1], inv2, zc2);
     return sz;
 }
 
-// Dequantize 8 code words with (s, z): x_j = (q_j - z) * (s * scale) (scale folds a decay).
+// Dequantize 8 code words with (s, z): x_j = (q_j - z) * (s * scale); scale folds
+// the decay and, on the hot path, the 2^-39 working scale.
 // 2^23 + q comes straight from a byte permute; subtracting 2^23 + z is exact.
 __device__ __forceinline__ void dequantize_group(const uint32_t (&w)[8], uint32_t sz, float scale, float2 (&x)[16]) {
     const float s = __half2float(__ushort_as_half((unsigned short)(sz & 0xffffu)));

@@ -55,33 +55,39 @@ struct PackedParams {
 
 // per-warp scratch before the stage ring
 constexpr int kPartOff = 64;                              // after NSTAGE (<= 8) mbarriers
-constexpr int kPartStride = 36;                           // floats per row of the partial-sum buffer
+constexpr int kPartStride = 68;                           // floats per lane row: 32 (r, p) pairs + padding
 constexpr int kDvecOff = kPartOff + 32 * kPartStride * 4; // 32 floats: H d for the low tier
 constexpr int kHopsOff = kDvecOff + 32 * 4;               // FP16-row operands, 32 B per row pair
-__host__ __device__ constexpr int scratch_bytes(int k_hi) { return kHopsOff + 32 * ((k_hi + 1) / 2); }
+__host__ __device__ constexpr int scratch_bytes(int k_hi) { return kHopsOff + 16 * ((k_hi + 3) & ~3); }
 
 __device__ __forceinline__ float ldsf(uint32_t a) { return __uint_as_float(lds32(a)); }
 
-// Column sum over the lanes' 32-vectors (16 pairs): lane j returns sum_l v_l[j].
-__device__ __forceinline__ float column_sum(const float2 (&v)[16], uint32_t part, int lane) {
+// Column sums of two per-lane 32-vectors at once: lane j returns
+// (sum_l a_l[j], sum_l b_l[j]) over the 32 lanes l.
+__device__ __forceinline__ float2 column_sum2(const float2 (&a)[16], const float2 (&b)[16], uint32_t part, int lane) {
 #pragma unroll
-    for (int jj = 0; jj < 8; ++jj) {
-        sts128(part + (lane * kPartStride + 4 * jj) * 4,
-               make_uint4(__float_as_uint(v[2 * jj].x), __float_as_uint(v[2 * jj].y), __float_as_uint(v[2 * jj + 1].x),
-                          __float_as_uint(v[2 * jj + 1].y)));
+    for (int m = 0; m < 16; ++m) {  // row of lane l: (a_j, b_j) pairs in column order
+        sts128(part + (lane * kPartStride + 4 * m) * 4,
+               make_uint4(__float_as_uint(a[m].x), __float_as_uint(b[m].x), __float_as_uint(a[m].y),
+                          __float_as_uint(b[m].y)));
     }
     __syncwarp();
-    float2 s0 = make_float2(0.f, 0.f), s1 = s0;
+    float2 s0 = make_float2(0.f, 0.f), s1 = s0, s2 = s0, s3 = s0;
 #pragma unroll
     for (int l = 0; l < 32; l += 4) {
-        s0 = add2(s0, make_float2(ldsf(part + ((l + 0) * kPartStride + lane) * 4),
-                                  ldsf(part + ((l + 1) * kPartStride + lane) * 4)));
-        s1 = add2(s1, make_float2(ldsf(part + ((l + 2) * kPartStride + lane) * 4),
-                                  ldsf(part + ((l + 3) * kPartStride + lane) * 4)));
+        const uint32_t base = part + (2 * lane) * 4;
+        uint2 v0, v1, v2, v3;
+        asm volatile("ld.shared.v2.b32 {%0,%1}, [%2];" : "=r"(v0.x), "=r"(v0.y) : "r"(base + (l + 0) * kPartStride * 4));
+        asm volatile("ld.shared.v2.b32 {%0,%1}, [%2];" : "=r"(v1.x), "=r"(v1.y) : "r"(base + (l + 1) * kPartStride * 4));
+        asm volatile("ld.shared.v2.b32 {%0,%1}, [%2];" : "=r"(v2.x), "=r"(v2.y) : "r"(base + (l + 2) * kPartStride * 4));
+        asm volatile("ld.shared.v2.b32 {%0,%1}, [%2];" : "=r"(v3.x), "=r"(v3.y) : "r"(base + (l + 3) * kPartStride * 4));
+        s0 = add2(s0, make_float2(__uint_as_float(v0.x), __uint_as_float(v0.y)));
+        s1 = add2(s1, make_float2(__uint_as_float(v1.x), __uint_as_float(v1.y)));
+        s2 = add2(s2, make_float2(__uint_as_float(v2.x), __uint_as_float(v2.y)));
+        s3 = add2(s3, make_float2(__uint_as_float(v3.x), __uint_as_float(v3.y)));
     }
     __syncwarp();
-    const float2 t = add2(s0, s1);
-    return t.x + t.y;
+    return add2(add2(s0, s1), add2(s2, s3));
 }
 
 __device__ __forceinline__ float bf16_at(uint32_t base, int i) {
@@ -189,6 +195,8 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
     // low-tier row operands of this lane (zero weights for lanes past the last row)
     float2 kk[R], qq[R], bk[R];
     float aa[R];
+    float unit_beta = 0.f, unit_g = 0.f, bkq = 0.f;
+    int unit = 0;
     int s = 0;
     uint32_t parity = 0;
     bool timed_out = false, bad_slot = false;
@@ -208,36 +216,54 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
 
         // ---- per-(slot, head) operands, gathered into calibrated key order ----
         if (t == t0 || c == 0) {
-            const float beta = p.beta[(int64_t)b * H + h];
-            const float alpha = KDA ? 0.f : expf(p.g[(int64_t)b * H + h]);
+            // beta (and the GDN log-decay) of the next 32 (slot, head) units are
+            // loaded one per lane, long before they are needed
+            if ((unit & 31) == 0) {
+                const int64_t ul = (int64_t)b * H + h + lane;
+                unit_beta = ul < (int64_t)p.batch * H ? p.beta[ul] : 0.f;
+                if (!KDA) unit_g = ul < (int64_t)p.batch * H ? p.g[ul] : 0.f;
+            }
+            const float beta = __shfl_sync(kFull, unit_beta, unit & 31);
+            const float alpha = KDA ? 0.f : expf(__shfl_sync(kFull, unit_g, unit & 31));
+            ++unit;
             // d_k is a power of two: masking keeps a malformed permutation in bounds
             auto chan = [&](int u) { return (int)(lds32(st + p.off_perm + (u & ~3)) >> (8 * (u & 3))) & (p.dk - 1); };
             auto kv_at = [&](int ch) { return BF16 ? bf16_at(st + p.off_k, ch) : ldsf(st + p.off_k + 4 * ch); };
             auto qv_at = [&](int ch) { return BF16 ? bf16_at(st + p.off_q, ch) : ldsf(st + p.off_q + 4 * ch); };
             auto av_at = [&](int ch) { return KDA ? expf(ldsf(st + p.off_g + 4 * ch)) : alpha; };
+            float kq = 0.f;  // this lane's share of k^T q (all d_k channels)
 #pragma unroll
             for (int i = 0; i < R; ++i) {
                 const int r = lane + 32 * i;
                 const bool live = r < lo;
                 const int ch = chan(live ? K + r : (lo > 0 ? K + lo - 1 : 0));  // stays inside perm
                 const float kv = live ? kv_at(ch) : 0.f;
+                const float qv = live ? qv_at(ch) : 0.f;
                 kk[i] = splat2(kv);
-                qq[i] = splat2(live ? qv_at(ch) : 0.f);
-                bk[i] = splat2(beta * kv);
-                aa[i] = av_at(ch);
+                qq[i] = splat2(qv);
+                bk[i] = splat2(beta * kv * kDown);  // working scale of the low tier
+                aa[i] = av_at(ch) * kDown;
+                kq = fmaf(kv, qv, kq);
             }
-            // FP16 rows in pairs: {a_u, a_u+1, k_u, k_u+1} {q_u, q_u+1, bk_u, bk_u+1}
-            for (int u = 2 * lane; u < K; u += 64) {
-                const int c0 = chan(u);
-                const bool two = u + 1 < K;
-                const int c1 = two ? chan(u + 1) : c0;
-                const float k0 = kv_at(c0), k1 = two ? kv_at(c1) : 0.f;
-                sts128(hops + 16 * u, make_uint4(__float_as_uint(av_at(c0)), __float_as_uint(two ? av_at(c1) : 0.f),
-                                                 __float_as_uint(k0), __float_as_uint(k1)));
-                sts128(hops + 16 * u + 16,
-                       make_uint4(__float_as_uint(qv_at(c0)), __float_as_uint(two ? qv_at(c1) : 0.f),
-                                  __float_as_uint(beta * k0), __float_as_uint(beta * k1)));
+            // FP16 rows in pairs: {a_u, a_u+1, k_u, k_u+1} {q_u, q_u+1, bk_u, bk_u+1};
+            // rows K .. K4-1 (padding to a multiple of 4) carry zero weights
+            const int K4 = (K + 3) & ~3;
+            for (int u = 2 * lane; u < K4; u += 64) {
+                const bool one = u < K, two = u + 1 < K;
+                const int c0 = one ? chan(u) : 0;
+                const int c1 = two ? chan(u + 1) : 0;
+                const float k0 = one ? kv_at(c0) : 0.f, k1 = two ? kv_at(c1) : 0.f;
+                sts128(hops + 16 * u, make_uint4(__float_as_uint(one ? av_at(c0) : 0.f),
+                                                 __float_as_uint(two ? av_at(c1) : 0.f), __float_as_uint(k0),
+                                                 __float_as_uint(k1)));
+                const float q0 = one ? qv_at(c0) : 0.f, q1 = two ? qv_at(c1) : 0.f;
+                sts128(hops + 16 * u + 16, make_uint4(__float_as_uint(q0), __float_as_uint(q1),
+                                                      __float_as_uint(beta * k0), __float_as_uint(beta * k1)));
+                kq = fmaf(k0, q0, fmaf(k1, q1, kq));
             }
+#pragma unroll
+            for (int m = 16; m >= 1; m >>= 1) kq += __shfl_xor_sync(kFull, kq, m);
+            bkq = beta * kq;  // beta k^T q: o = S_bar^T q + beta (k^T q) d
             __syncwarp();
         }
 
@@ -246,8 +272,9 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
         if (ok) {
             const float vt = HAD ? hadamard_lanes(vj, lane) : vj;  // H v
             float2 x[R][16];
-            float2 acc[16];
-            // ---- phase 1, low tier: reconstruct, decay, partial r~ = S~_bar^T k ----
+            float2 acc[16], accp[16];
+            // ---- phase 1, low tier: reconstruct and decay (scaled by 2^-39), partial
+            //      r~ = S~_bar^T k and p~ = S~_bar^T q ----
 #pragma unroll
             for (int i = 0; i < RL; ++i) {
                 const int r = min(lane + 32 * i, lo - 1);
@@ -257,56 +284,63 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
                 const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
                 dequantize_group(w, sz, aa[i], x[i]);
 #pragma unroll
-                for (int j = 0; j < 16; ++j) acc[j] = (i == 0) ? mul2(x[i][j], kk[i]) : fma2(x[i][j], kk[i], acc[j]);
+                for (int j = 0; j < 16; ++j) {
+                    acc[j] = (i == 0) ? mul2(x[i][j], kk[i]) : fma2(x[i][j], kk[i], acc[j]);
+                    accp[j] = (i == 0) ? mul2(x[i][j], qq[i]) : fma2(x[i][j], qq[i], accp[j]);
+                }
             }
             if (RL == 0) {
 #pragma unroll
-                for (int j = 0; j < 16; ++j) acc[j] = make_float2(0.f, 0.f);
+                for (int j = 0; j < 16; ++j) acc[j] = accp[j] = make_float2(0.f, 0.f);
             }
 
-            // ---- phase 1, FP16 tier (lane = column), two rows per step ----
+            // ---- phase 1, FP16 tier (lane = column), four rows per step ----
             const uint32_t col = st + 2 * lane;
-            float2 rh = make_float2(0.f, 0.f);
-            for (int u = 0; u < K; u += 2) {
-                const uint4 op = lds128(hops + 16 * u);
-                uint16_t h0, h1 = 0;
-                asm volatile("ld.shared.u16 %0, [%1];" : "=h"(h0) : "r"(col + 64 * u));
-                if (u + 1 < K) asm volatile("ld.shared.u16 %0, [%1];" : "=h"(h1) : "r"(col + 64 * u + 64));
-                const float2 xh = mul2(make_float2(h16_to_f32(h0), h16_to_f32(h1)),
-                                       make_float2(__uint_as_float(op.x), __uint_as_float(op.y)));
-                rh = fma2(xh, make_float2(__uint_as_float(op.z), __uint_as_float(op.w)), rh);
+            const int K4 = (K + 3) & ~3;
+            auto hrow = [&](int u) -> float {  // FP16 value of row min(u, K-1), this lane's column
+                uint16_t hv;
+                asm volatile("ld.shared.u16 %0, [%1];" : "=h"(hv) : "r"(col + 64 * min(u, K - 1)));
+                return h16_to_f32(hv);
+            };
+            float2 rh = make_float2(0.f, 0.f), rh2 = rh, ph = rh, ph2 = rh;
+            for (int u = 0; u < K4; u += 4) {
+                const uint4 opa = lds128(hops + 16 * u);
+                const uint4 opb = lds128(hops + 16 * u + 32);
+                const uint4 oqa = lds128(hops + 16 * u + 16);
+                const uint4 oqb = lds128(hops + 16 * u + 48);
+                const float2 xa = mul2(make_float2(hrow(u), hrow(u + 1)), make_float2(__uint_as_float(opa.x), __uint_as_float(opa.y)));
+                const float2 xb = mul2(make_float2(hrow(u + 2), hrow(u + 3)), make_float2(__uint_as_float(opb.x), __uint_as_float(opb.y)));
+                rh = fma2(xa, make_float2(__uint_as_float(opa.z), __uint_as_float(opa.w)), rh);
+                rh2 = fma2(xb, make_float2(__uint_as_float(opb.z), __uint_as_float(opb.w)), rh2);
+                ph = fma2(xa, make_float2(__uint_as_float(oqa.x), __uint_as_float(oqa.y)), ph);
+                ph2 = fma2(xb, make_float2(__uint_as_float(oqb.x), __uint_as_float(oqb.y)), ph2);
             }
-            const float rhi = rh.x + rh.y;
-            const float rlo = column_sum(acc, part, lane);  // r~_lo (transformed domain when HAD)
+            rh = add2(rh, rh2);
+            ph = add2(ph, ph2);
+            const float rhi = rh.x + rh.y, phi = ph.x + ph.y;
+            const float2 lo_sums = column_sum2(acc, accp, part, lane);
+            const float rlo = lo_sums.x * kUp, plo = lo_sums.y * kUp;  // back from the working scale
 
-            // r = H r~_lo + r_hi;  d = v - r (natural, FP16 rows);  H d = H v - r~_lo - H r_hi (low tier)
-            float dj, dt;
+            // r = H r~_lo + r_hi;  d = v - r (natural, FP16 rows);  H d = H v - r~_lo - H r_hi (low tier);
+            // o = S_t^T q = S_bar^T q + beta (k^T q) d, with S_bar^T q = H p~_lo + p_hi
+            float dj, dt, pj;
             if (HAD) {
-                if (K > 0) {
-                    const float hr_lo = hadamard_lanes(rlo, lane);
-                    const float hr_hi = hadamard_lanes(rhi, lane);
-                    dj = vj - (hr_lo + rhi);
-                    dt = vt - (rlo + hr_hi);
-                } else {
-                    dj = 0.f;
-                    dt = vt - rlo;
-                }
+                const float hr_lo = hadamard_lanes(rlo, lane);
+                const float hp_lo = hadamard_lanes(plo, lane);
+                const float hr_hi = K > 0 ? hadamard_lanes(rhi, lane) : 0.f;
+                dj = vj - (hr_lo + rhi);
+                dt = vt - (rlo + hr_hi);
+                pj = hp_lo + phi;
             } else {
                 dj = vj - (rlo + rhi);
                 dt = dj;
+                pj = plo + phi;
             }
+            p.o[((int64_t)b * H + h) * p.dv + c * kG + lane] = fmaf(bkq, dj, pj);
             sts32(dvec + 4 * lane, __float_as_uint(dt));
-
-            // ---- keep the ring full: next load goes into the stage of tile t-1 ----
-            if (lane == 0 && t_pre < t1) {
-                bulk_wait_read_all();
-                issue(t_pre, pre, (s + p.nstage - 1) % p.nstage);
-                ++t_pre;
-                advance(pre, H, V);
-            }
             __syncwarp();
 
-            // ---- phase 2, low tier: rank-1 correction, partial o~, requantize in place ----
+            // ---- phase 2, low tier: rank-1 correction, requantize in place ----
             float2 d[16];
 #pragma unroll
             for (int jj = 0; jj < 8; ++jj) {
@@ -314,49 +348,50 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
                 d[2 * jj] = make_float2(__uint_as_float(w.x), __uint_as_float(w.y));
                 d[2 * jj + 1] = make_float2(__uint_as_float(w.z), __uint_as_float(w.w));
             }
+            // each stage runs over all row slots before the next starts, so the short
+            // dependent chains of the rows (extrema -> scale -> codes) overlap
+#pragma unroll
+            for (int i = 0; i < RL; ++i) {
+#pragma unroll
+                for (int j = 0; j < 16; ++j) x[i][j] = fma2(bk[i], d[j], x[i][j]);
+            }
+            float mn[R], mx[R], inv[R], zq[R];
+            uint32_t szw[R];
+#pragma unroll
+            for (int i = 0; i < RL; ++i) minmax32(x[i], mn[i], mx[i]);
+#pragma unroll
+            for (int i = 0; i < RL; ++i) szw[i] = affine_params_scaled(mn[i], mx[i], inv[i], zq[i]);
 #pragma unroll
             for (int i = 0; i < RL; ++i) {
                 const int r = lane + 32 * i;
-#pragma unroll
-                for (int j = 0; j < 16; ++j) {
-                    x[i][j] = fma2(bk[i], d[j], x[i][j]);
-                    acc[j] = (i == 0) ? mul2(x[i][j], qq[i]) : fma2(x[i][j], qq[i], acc[j]);
-                }
+                const float2 inv2 = splat2(inv[i] * 0x1p-110f), zc2 = splat2(zq[i] * 0x1p-149f);
                 uint32_t w[8];
-                const uint32_t sz = quantize_group(x[i], w);
+#pragma unroll
+                for (int m = 0; m < 8; ++m) w[m] = encode4(x[i][2 * m], x[i][2 * m + 1], inv2, zc2);
                 // a lane past the last row writes into its own slice of the (idle)
                 // partial-sum buffer instead of branching around the stores
                 const bool live = r < lo;
                 const uint32_t trash = part + lane * kPartStride * 4;
                 sts128(live ? st + p.codes_off + lo_chunk_off(r, 0) : trash, make_uint4(w[0], w[1], w[2], w[3]));
                 sts128(live ? st + p.codes_off + lo_chunk_off(r, 1) : trash + 16, make_uint4(w[4], w[5], w[6], w[7]));
-                sts32(live ? st + p.meta_off + 4 * r : trash + 32, sz);
+                sts32(live ? st + p.meta_off + 4 * r : trash + 32, szw[i]);
             }
-            if (RL == 0) {
-#pragma unroll
-                for (int j = 0; j < 16; ++j) acc[j] = make_float2(0.f, 0.f);
-            }
-            __syncwarp();
 
-            // ---- phase 2, FP16 tier: S = S_bar + beta k d, o_hi, FP16 store ----
-            float2 oh = make_float2(0.f, 0.f);
-            for (int u = 0; u < K; u += 2) {
+            // ---- phase 2, FP16 tier: S = S_bar + beta k d, FP16 store ----
+            const uint32_t trash_h = part + lane * kPartStride * 4 + 48;
+            auto hpair = [&](int u) {
                 const uint4 op0 = lds128(hops + 16 * u);
                 const uint4 op1 = lds128(hops + 16 * u + 16);
-                uint16_t h0, h1 = 0;
-                asm volatile("ld.shared.u16 %0, [%1];" : "=h"(h0) : "r"(col + 64 * u));
-                if (u + 1 < K) asm volatile("ld.shared.u16 %0, [%1];" : "=h"(h1) : "r"(col + 64 * u + 64));
-                const float2 xh = mul2(make_float2(h16_to_f32(h0), h16_to_f32(h1)),
-                                       make_float2(__uint_as_float(op0.x), __uint_as_float(op0.y)));
+                const float2 xh = mul2(make_float2(hrow(u), hrow(u + 1)), make_float2(__uint_as_float(op0.x), __uint_as_float(op0.y)));
                 const float2 y = fma2(make_float2(__uint_as_float(op1.z), __uint_as_float(op1.w)), splat2(dj), xh);
-                oh = fma2(y, make_float2(__uint_as_float(op1.x), __uint_as_float(op1.y)), oh);
                 const uint32_t hy = f2_to_h2(y.x, y.y);
-                sts16(col + 64 * u, (unsigned short)(hy & 0xffffu));
-                if (u + 1 < K) sts16(col + 64 * u + 64, (unsigned short)(hy >> 16));
+                sts16(u < K ? col + 64 * u : trash_h, (unsigned short)(hy & 0xffffu));
+                sts16(u + 1 < K ? col + 64 * u + 64 : trash_h + 2, (unsigned short)(hy >> 16));
+            };
+            for (int u = 0; u < K4; u += 4) {
+                hpair(u);
+                hpair(u + 2);
             }
-            const float olo = column_sum(acc, part, lane);
-            const float oj = (HAD ? hadamard_lanes(olo, lane) : olo) + (oh.x + oh.y);
-            p.o[((int64_t)b * H + h) * p.dv + c * kG + lane] = oj;
 
             // ---- write the updated record back ----
             fence_proxy_async_smem();
@@ -365,8 +400,13 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
                 bulk_s2g(p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * p.rec_bytes, st, p.rec_bytes);
                 bulk_commit();
             }
-        } else if (lane == 0 && t_pre < t1) {
-            bulk_wait_read_all();
+        } else if (lane == 0) {
+            bulk_commit();  // an empty group keeps one group per tile
+        }
+        // ---- keep the ring full: the next load reuses the stage of tile t-1, whose
+        // store was committed one tile ago (every group but the newest has been read)
+        if (lane == 0 && t_pre < t1) {
+            bulk_wait_read_all_but_newest();
             issue(t_pre, pre, (s + p.nstage - 1) % p.nstage);
             ++t_pre;
             advance(pre, H, V);
