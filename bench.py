@@ -210,7 +210,9 @@ def gpu_arm(args, rank: int, world: int):
         return float(t.item())
 
     with ClockSampler(dev.index) as clk:
+        torch.cuda.nvtx.range_push("timed_packed_step")
         total_ms, launch_ms = timed(run_packed, args.steps, args.warmup)
+        torch.cuda.nvtx.range_pop()
     total_ms = max_over_ranks(total_ms)
     launch_ms = max_over_ranks(launch_ms)
     if damp.device_status() != 0:
