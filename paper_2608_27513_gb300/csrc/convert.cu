@@ -60,6 +60,7 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
 #pragma unroll
         for (int i = 0; i < R; ++i) {
             const int u = lane + 32 * i;
+            if (u < K) continue;  // FP16 rows: column-mapped loop below
             if (OP == kQuantize || OP == kDequantize) {
                 const int n = p.perm[(int64_t)h * p.dk + u] & (p.dk - 1);  // d_k is a power of two
                 float *row = p.S + ((((int64_t)b * p.H + h) * p.dk + n) * p.dv + c * kG);
@@ -71,17 +72,7 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
                         x[2 * m] = make_float2(f.x, f.y);
                         x[2 * m + 1] = make_float2(f.z, f.w);
                     }
-                    if (u < K) {
-#pragma unroll
-                        for (int m = 0; m < 4; ++m) {
-                            uint4 w;
-                            w.x = f2_to_h2(x[4 * m].x, x[4 * m].y);
-                            w.y = f2_to_h2(x[4 * m + 1].x, x[4 * m + 1].y);
-                            w.z = f2_to_h2(x[4 * m + 2].x, x[4 * m + 2].y);
-                            w.w = f2_to_h2(x[4 * m + 3].x, x[4 * m + 3].y);
-                            *reinterpret_cast<uint4 *>(rec + hi_chunk_off(u, m)) = w;
-                        }
-                    } else {
+                    {
                         const int r = u - K;
                         if (HAD) hadamard_pairs(x);
 #pragma unroll
@@ -95,16 +86,7 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
                         *reinterpret_cast<uint32_t *>(rec + p.meta_off + 4 * r) = sz;
                     }
                 } else {
-                    if (u < K) {
-#pragma unroll
-                        for (int m = 0; m < 4; ++m) {
-                            const uint4 w = *reinterpret_cast<const uint4 *>(rec + hi_chunk_off(u, m));
-                            x[4 * m] = h2_to_f2(w.x);
-                            x[4 * m + 1] = h2_to_f2(w.y);
-                            x[4 * m + 2] = h2_to_f2(w.z);
-                            x[4 * m + 3] = h2_to_f2(w.w);
-                        }
-                    } else {
+                    {
                         const int r = u - K;
                         const uint4 c0 = *reinterpret_cast<const uint4 *>(rec + p.codes_off + lo_chunk_off(r, 0));
                         const uint4 c1 = *reinterpret_cast<const uint4 *>(rec + p.codes_off + lo_chunk_off(r, 1));
@@ -118,19 +100,8 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
                         reinterpret_cast<float4 *>(row)[m] = make_float4(x[2 * m].x, x[2 * m].y, x[2 * m + 1].x, x[2 * m + 1].y);
                 }
             } else {
-                // logical tiers <-> record, 32-bit words
-                if (u < K) {
-                    uint32_t *trow = reinterpret_cast<uint32_t *>(p.hi + ((((int64_t)b * p.H + h) * K + u) * p.dv + c * kG));
-#pragma unroll
-                    for (int m = 0; m < 4; ++m) {
-                        uint32_t *r4 = reinterpret_cast<uint32_t *>(rec + hi_chunk_off(u, m));
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            if (OP == kPackTiers) r4[e] = trow[4 * m + e];
-                            else trow[4 * m + e] = r4[e];
-                        }
-                    }
-                } else {
+                // logical tiers <-> record, 32-bit words (FP16 rows: column-mapped loop below)
+                {
                     const int r = u - K;
                     uint32_t *crow = reinterpret_cast<uint32_t *>(p.codes + ((((int64_t)b * p.H + h) * lo + r) * p.dv + c * kG));
                     uint32_t *mrow = reinterpret_cast<uint32_t *>(p.meta + ((((int64_t)b * p.H + h) * lo + r) * p.V + c) * 2);
@@ -146,6 +117,32 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
                     uint32_t *mr = reinterpret_cast<uint32_t *>(rec + p.meta_off + 4 * r);
                     if (OP == kPackTiers) *mr = *mrow;
                     else *mrow = *mr;
+                }
+            }
+        }
+        // ---- FP16 rows, lane = column, two rows per 32-bit word ----
+        for (int u = 0; u < K; u += 2) {
+            const bool two = u + 1 < K;
+            uint32_t *word = reinterpret_cast<uint32_t *>(rec + hi_elem_off(u, lane));
+            if (OP == kQuantize || OP == kDequantize) {
+                float *r0 = p.S + ((((int64_t)b * p.H + h) * p.dk + (p.perm[(int64_t)h * p.dk + u] & (p.dk - 1))) * p.dv + c * kG + lane);
+                float *r1 = two ? p.S + ((((int64_t)b * p.H + h) * p.dk + (p.perm[(int64_t)h * p.dk + u + 1] & (p.dk - 1))) * p.dv + c * kG + lane) : nullptr;
+                if (OP == kQuantize) {
+                    *word = f2_to_h2(*r0, two ? *r1 : 0.f);
+                } else {
+                    const float2 f = h2_to_f2(*word);
+                    *r0 = f.x;
+                    if (two) *r1 = f.y;
+                }
+            } else {
+                uint16_t *t0 = p.hi + ((((int64_t)b * p.H + h) * K + u) * p.dv + c * kG + lane);
+                uint16_t *t1 = two ? t0 + p.dv : nullptr;
+                if (OP == kPackTiers) {
+                    *word = (uint32_t)*t0 | ((uint32_t)(two ? *t1 : 0) << 16);
+                } else {
+                    const uint32_t w = *word;
+                    *t0 = (uint16_t)(w & 0xffffu);
+                    if (two) *t1 = (uint16_t)(w >> 16);
                 }
             }
         }

@@ -20,7 +20,10 @@ enum : uint32_t { kDevWaitTimeout = 1u, kDevBadSlot = 2u };
 
 // ---------------------------------------------------------------------------
 // Packed record geometry (one (slot, head, value block) record).
-//   hi rows:   K x 64 B   at 0;   row-major binary16 (lanes read one column each)
+//   hi rows:   ceil(K/2) pairs x 128 B at 0: pair i holds rows 2i and 2i+1 as
+//              32 column words (binary16 of row 2i in the low half); an odd K
+//              leaves the last high half zero.  A lane reads two FP16 rows of its
+//              column with one 32-bit load.
 //   codes:     (d_k-K) x 32 B;    16-B chunk m of lo row r at 16 * (m ^ ((r >> 2) & 1))
 //   meta:      (d_k-K) x 4 B      (s, z) as two binary16
 // The chunk permutation of the codes makes the 8 consecutive rows that a
@@ -32,13 +35,14 @@ struct RecGeom {
 
 __host__ __device__ inline RecGeom rec_geom(int d_k, int k_hi) {
     RecGeom g;
-    g.codes_off = 64 * k_hi;
+    g.codes_off = 128 * ((k_hi + 1) / 2);
     g.meta_off = g.codes_off + 32 * (d_k - k_hi);
     g.bytes = (g.meta_off + 4 * (d_k - k_hi) + 15) & ~15;
     return g;
 }
 
-__host__ __device__ inline int hi_chunk_off(int u, int m) { return 64 * u + 16 * m; }
+// byte offset of FP16 row u, column j (0..31) inside a record
+__host__ __device__ inline int hi_elem_off(int u, int j) { return 128 * (u >> 1) + 4 * j + 2 * (u & 1); }
 __host__ __device__ inline int lo_chunk_off(int r, int m) { return 32 * r + 16 * (m ^ ((r >> 2) & 1)); }
 
 // ---------------------------------------------------------------------------

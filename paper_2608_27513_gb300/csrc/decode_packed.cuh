@@ -294,22 +294,21 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
                 for (int j = 0; j < 16; ++j) acc[j] = accp[j] = make_float2(0.f, 0.f);
             }
 
-            // ---- phase 1, FP16 tier (lane = column), four rows per step ----
-            const uint32_t col = st + 2 * lane;
-            const int K4 = (K + 3) & ~3;
-            auto hrow = [&](int u) -> float {  // FP16 value of row min(u, K-1), this lane's column
-                uint16_t hv;
-                asm volatile("ld.shared.u16 %0, [%1];" : "=h"(hv) : "r"(col + 64 * min(u, K - 1)));
-                return h16_to_f32(hv);
-            };
+            // ---- phase 1, FP16 tier (lane = column): one 32-bit load per row pair ----
+            const uint32_t col = st + 4 * lane;  // this lane's word in FP16 row pair 0
+            const int KP = (K + 1) >> 1;         // row pairs in the record
             float2 rh = make_float2(0.f, 0.f), rh2 = rh, ph = rh, ph2 = rh;
-            for (int u = 0; u < K4; u += 4) {
-                const uint4 opa = lds128(hops + 16 * u);
-                const uint4 opb = lds128(hops + 16 * u + 32);
-                const uint4 oqa = lds128(hops + 16 * u + 16);
-                const uint4 oqb = lds128(hops + 16 * u + 48);
-                const float2 xa = mul2(make_float2(hrow(u), hrow(u + 1)), make_float2(__uint_as_float(opa.x), __uint_as_float(opa.y)));
-                const float2 xb = mul2(make_float2(hrow(u + 2), hrow(u + 3)), make_float2(__uint_as_float(opb.x), __uint_as_float(opb.y)));
+            for (int pi = 0; pi < KP; pi += 2) {
+                // pair pi + 1 may be the zero-weight padding pair (hops rows up to K4):
+                // read a valid word and let the zero weights cancel it
+                const uint32_t wa = lds32(col + 128 * pi);
+                const uint32_t wb = lds32(col + 128 * min(pi + 1, KP - 1));
+                const uint4 opa = lds128(hops + 32 * pi);
+                const uint4 oqa = lds128(hops + 32 * pi + 16);
+                const uint4 opb = lds128(hops + 32 * pi + 32);
+                const uint4 oqb = lds128(hops + 32 * pi + 48);
+                const float2 xa = mul2(h2_to_f2(wa), make_float2(__uint_as_float(opa.x), __uint_as_float(opa.y)));
+                const float2 xb = mul2(h2_to_f2(wb), make_float2(__uint_as_float(opb.x), __uint_as_float(opb.y)));
                 rh = fma2(xa, make_float2(__uint_as_float(opa.z), __uint_as_float(opa.w)), rh);
                 rh2 = fma2(xb, make_float2(__uint_as_float(opb.z), __uint_as_float(opb.w)), rh2);
                 ph = fma2(xa, make_float2(__uint_as_float(oqa.x), __uint_as_float(oqa.y)), ph);
@@ -377,20 +376,15 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
                 sts32(live ? st + p.meta_off + 4 * r : trash + 32, szw[i]);
             }
 
-            // ---- phase 2, FP16 tier: S = S_bar + beta k d, FP16 store ----
-            const uint32_t trash_h = part + lane * kPartStride * 4 + 48;
-            auto hpair = [&](int u) {
-                const uint4 op0 = lds128(hops + 16 * u);
-                const uint4 op1 = lds128(hops + 16 * u + 16);
-                const float2 xh = mul2(make_float2(hrow(u), hrow(u + 1)), make_float2(__uint_as_float(op0.x), __uint_as_float(op0.y)));
-                const float2 y = fma2(make_float2(__uint_as_float(op1.z), __uint_as_float(op1.w)), splat2(dj), xh);
-                const uint32_t hy = f2_to_h2(y.x, y.y);
-                sts16(u < K ? col + 64 * u : trash_h, (unsigned short)(hy & 0xffffu));
-                sts16(u + 1 < K ? col + 64 * u + 64 : trash_h + 2, (unsigned short)(hy >> 16));
-            };
-            for (int u = 0; u < K4; u += 4) {
-                hpair(u);
-                hpair(u + 2);
+            // ---- phase 2, FP16 tier: S = S_bar + beta k d, FP16 store (two rows per word) ----
+            const float2 dj2 = splat2(dj);
+            for (int pi = 0; pi < KP; ++pi) {
+                const uint32_t wa = lds32(col + 128 * pi);
+                const uint4 opa = lds128(hops + 32 * pi);
+                const uint4 oqa = lds128(hops + 32 * pi + 16);
+                const float2 xa = mul2(h2_to_f2(wa), make_float2(__uint_as_float(opa.x), __uint_as_float(opa.y)));
+                const float2 y = fma2(make_float2(__uint_as_float(oqa.z), __uint_as_float(oqa.w)), dj2, xa);
+                sts32(col + 128 * pi, f2_to_h2(y.x, y.y));  // an odd K's padding half stays 0
             }
 
             // ---- write the updated record back ----
