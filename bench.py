@@ -136,6 +136,62 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def max_over_ranks(x: float, world: int, device) -> float:
+    """The maximum of x over all ranks (the slowest rank sets the step time)."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def make_line(r: dict, steps: int, warmup: int, world: int) -> dict:
+    """The bench's JSON line from one rank-0 result (times already maxed over ranks)."""
+    w = r["w"]
+    bytes_step = algorithmic_bytes(w)
+    bytes_fp32 = algorithmic_bytes(w, packed=False)
+    ms = r["total_ms"] / steps
+    value = world * bytes_step / (ms * 1e-3) / 1e12
+    peaks = measured_peaks()
+    peak_gbs = peaks.get("hbm_gbs")
+    peak_note = "measured" if peak_gbs else "fallback"
+    peak_gbs = peak_gbs or 6800.0
+    achieved_gbs = bytes_step / (r["launch_ms"] * 1e-3) / 1e9
+    return {
+        "metric": METRIC, "value": value, "unit": "TB/s", "n_gpus": world, "steps": steps,
+        "warmup": warmup, "ms_per_step": ms, "us_per_step": ms * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": workload_config(w, r.get("bits")),
+        "clocks": r.get("clocks"),
+        "e2e": {"value": world * bytes_step / (r["e2e_ms"] * 1e-3) / 1e12, "unit": "TB/s",
+                "us_per_step": r["e2e_ms"] * 1e3, "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]},
+        "gpu_launches": steps,
+        "roofline": {"bound": "hbm", "achieved": achieved_gbs, "peak": peak_gbs, "unit": "GB/s",
+                     "frac": achieved_gbs / peak_gbs, "peak_source": f"{peak_note} copy bandwidth",
+                     "frac_of_8TBs": achieved_gbs / 8000.0,
+                     "traffic": ncu_traffic("packed_step_kda_b256"),
+                     "kernel": "packed_step_kernel<4,KDA,H32,BF16>", "algorithmic_bytes": bytes_step},
+        "fp32_state_kernel": {"us_per_step": r["fp32_launch_ms"] * 1e3,
+                              "achieved_gbs": bytes_fp32 / (r["fp32_launch_ms"] * 1e-3) / 1e9,
+                              "bytes_per_step": bytes_fp32,
+                              "speedup_of_packed": r["fp32_launch_ms"] / r["launch_ms"]},
+        "device": r.get("dev_name"),
+    }
+
+
+def workload_config(w: wl.Workload, bits=None) -> dict:
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    return {"workload": w.name, "kind": w.kind, "batch": w.batch, "heads": w.heads, "qk_heads": w.qk_heads,
+            "d_k": w.d_k, "d_v": w.d_v, "k_hi": w.k_hi, "lo_format": "uint8 affine G32 + H32",
+            "bits_per_value": bits, "in_dtype": w.in_dtype, "bytes_per_step": algorithmic_bytes(w),
+            "l2": f"inputs larger than L2: {POOLS} packed state pools of "
+                  f"{algorithmic_bytes(w) / 2 / 1e6:.0f} MB each rotated per step (> 129 MB L2)",
+            "permutation": "seeded random pi per head (throughput does not depend on which)",
+            "parallelism": f"{world} independent replica(s), one batch per GPU"}
+
+
 # ------------------------------------------------------------------ GPU arm ---
 
 def gpu_arm(args, rank: int, world: int):
@@ -202,26 +258,22 @@ def gpu_arm(args, rank: int, world: int):
         launch_ms = statistics.mean(a.elapsed_time(b) for a, b in ev) if per_launch else total_ms / steps
         return total_ms, launch_ms
 
-    def max_over_ranks(x):
-        if world == 1:
-            return x
-        t = torch.tensor([x], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+    def max_over_ranks_(x):
+        return max_over_ranks(x, world, dev)
 
     with ClockSampler(dev.index) as clk:
         torch.cuda.nvtx.range_push("timed_packed_step")
         total_ms, launch_ms = timed(run_packed, args.steps, args.warmup)
         torch.cuda.nvtx.range_pop()
-    total_ms = max_over_ranks(total_ms)
-    launch_ms = max_over_ranks(launch_ms)
+    total_ms = max_over_ranks_(total_ms)
+    launch_ms = max_over_ranks_(launch_ms)
     if damp.device_status() != 0:
         raise RuntimeError("device status word set during the timed region")
 
     # ---- the in-house FP32-state kernel on the same inputs (speedup reference) ----
     fp_steps = max(args.steps // 4, 10)
     fp_total, fp_launch = timed(run_fp32, fp_steps, max(args.warmup, 3))
-    fp_launch = max_over_ranks(fp_launch)
+    fp_launch = max_over_ranks_(fp_launch)
 
     # ---- end to end through the C ABI from pinned host buffers ----
     host_in = [{k: v.cpu().pin_memory() for k, v in d.items()} for d in inputs[:2]]
@@ -240,7 +292,7 @@ def gpu_arm(args, rank: int, world: int):
 
     e2e_steps = max(args.steps // 10, 10)
     e2e_total, _ = timed(run_e2e, e2e_steps, max(args.warmup, 3), per_launch=False)
-    e2e_total = max_over_ranks(e2e_total)
+    e2e_total = max_over_ranks_(e2e_total)
     return {
         "w": w, "total_ms": total_ms, "launch_ms": launch_ms, "fp32_launch_ms": fp_launch,
         "e2e_ms": e2e_total / e2e_steps, "h2d": h2d, "d2h": d2h, "clocks": clk.summary(),
@@ -312,13 +364,75 @@ def reference_arm(args, rank: int, world: int):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic",
-            "config": {"workload": w.name, "kind": "kda", "batch": w.batch, "heads": w.heads, "d_k": w.d_k,
-                       "d_v": w.d_v, "k_hi": w.k_hi, "lo_format": "uint8 affine G32 + H32",
-                       "reference": "CPU oracle (plain C, FP32, one thread)"},
+            "config": dict(workload_config(w, 9.0 + 7.0 * w.k_hi / w.d_k),
+                           reference="CPU oracle (plain C, FP32, one thread) in place of a reference implementation"),
             "cpu_baseline": {"value": value, "unit": "TB/s", "cores": 1, "kind": "oracle",
                              "sample": f"{heads} of the 8192 (slot, head) updates of a step, per step"},
             "e2e": {"value": value, "unit": "TB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+def sweep_arm(steps: int, warmup: int):
+    """K_hi sweep at B=256, H=32, d=128 (GDN and KDA) against the FP32-state kernel and
+    uniform INT8 (K_hi = 0) with and without H_32: bits/value, bytes and us per step."""
+    import torch
+
+    import paper_2608_27513_gb300 as damp
+    from paper_2608_27513_gb300 import build
+    build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    out = []
+    for kind in ("gdn", "kda"):
+        base = wl.sweep(kind, 0)
+        inputs = wl.torch_step_inputs(base, 4, dev)
+        S = 0.3 * torch.randn((base.batch, base.heads, base.d_k, base.d_v), device=dev)
+        o = torch.empty((base.batch, base.heads, base.d_v), device=dev)
+
+        def timeit(fn, n):
+            for i in range(warmup):
+                fn(i)
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for i in range(n):
+                fn(i)
+            e1.record()
+            torch.cuda.synchronize()
+            return e0.elapsed_time(e1) / n * 1e3
+
+        L0 = damp.Layout(base.heads, base.qk_heads, base.d_k, base.d_v, 0, 0)
+        fp = [S.clone(), S.clone()]
+        step32 = damp.fp32_kda_decode_step if kind == "kda" else damp.fp32_gdn_decode_step
+        us = timeit(lambda i: step32(L0, fp[i % 2], inputs[i % 4]["q"], inputs[i % 4]["k"], inputs[i % 4]["v"],
+                                     inputs[i % 4]["g"], inputs[i % 4]["beta"], o=o), max(steps // 4, 10))
+        nb = algorithmic_bytes(base, packed=False)
+        out.append({"kind": kind, "format": "fp32 state", "k_hi": None, "bits_per_value": 32.0,
+                    "bytes_per_step": nb, "us_per_step": us, "tb_s": nb / us / 1e6})
+        del fp
+        perm = torch.from_numpy(wl.random_perm(base)).to(dev)
+        points = [(0, 1, "uniform int8 (no H32)"), (0, 0, "uniform int8 + H32")] + \
+                 [(k, 0, "damp fp16 + int8 + H32") for k in wl.SWEEP_K_HI if k > 0]
+        for k, fmt, name in points:
+            w = wl.sweep(kind, k, fmt)
+            L = damp.Layout(w.heads, w.qk_heads, w.d_k, w.d_v, k, fmt)
+            pools = [damp.new_state(L, w.batch, dev) for _ in range(2)]
+            for pl in pools:
+                damp.quantize_state(L, S, perm, pl)
+            if k == 0:
+                step = damp.u8_kda_decode_step if kind == "kda" else damp.u8_gdn_decode_step
+            else:
+                step = damp.kda_decode_step if kind == "kda" else damp.gdn_decode_step
+            us = timeit(lambda i: step(L, pools[i % 2], perm, inputs[i % 4]["q"], inputs[i % 4]["k"],
+                                       inputs[i % 4]["v"], inputs[i % 4]["g"], inputs[i % 4]["beta"], o=o), steps)
+            nb = algorithmic_bytes(w)
+            out.append({"kind": kind, "format": name, "k_hi": k, "bits_per_value": damp.bits_per_value(L),
+                        "bytes_per_step": nb, "us_per_step": us, "tb_s": nb / us / 1e6})
+            del pools
+    if damp.device_status() != 0:
+        raise RuntimeError("device status word set during the sweep")
+    for row in out:
+        print(json.dumps(row), flush=True)
 
 
 def main():
@@ -328,6 +442,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=50)
     ap.add_argument("--impl", default="damp", choices=["damp", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true", help="K_hi sweep (GDN and KDA, B=256) instead of the bench line")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -336,6 +451,9 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     if args.impl == "reference":
         reference_arm(args, rank, world)
+        return
+    if args.sweep:
+        sweep_arm(args.steps, args.warmup)
         return
     import torch
     import torch.distributed as dist
@@ -347,42 +465,7 @@ def main():
         if world > 1 and dist.is_initialized():
             pass
     if rank == 0:
-        w = r["w"]
-        bytes_step = algorithmic_bytes(w)
-        bytes_fp32 = algorithmic_bytes(w, packed=False)
-        ms = r["total_ms"] / args.steps
-        value = world * bytes_step / (ms * 1e-3) / 1e12
-        peaks = measured_peaks()
-        peak_gbs = peaks.get("hbm_gbs")
-        peak_note = "measured" if peak_gbs else "fallback"
-        peak_gbs = peak_gbs or 6800.0
-        achieved_gbs = bytes_step / (r["launch_ms"] * 1e-3) / 1e9
-        line = {
-            "metric": METRIC, "value": value, "unit": "TB/s", "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms, "us_per_step": ms * 1e3, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": w.name, "kind": "kda", "batch": w.batch, "heads": w.heads, "qk_heads": w.qk_heads,
-                       "d_k": w.d_k, "d_v": w.d_v, "k_hi": w.k_hi, "lo_format": "uint8 affine G32 + H32",
-                       "bits_per_value": r["bits"], "in_dtype": "bf16", "bytes_per_step": bytes_step,
-                       "l2": f"inputs larger than L2: {POOLS} packed state pools of "
-                             f"{bytes_step / 2 / 1e6:.0f} MB each rotated per step (> 129 MB L2)",
-                       "permutation": "seeded random pi per head (throughput does not depend on which)",
-                       "parallelism": f"{world} independent replica(s), one batch per GPU"},
-            "clocks": r["clocks"],
-            "e2e": {"value": world * bytes_step / (r["e2e_ms"] * 1e-3) / 1e12, "unit": "TB/s",
-                    "us_per_step": r["e2e_ms"] * 1e3, "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]},
-            "gpu_launches": args.steps,
-            "roofline": {"bound": "hbm", "achieved": achieved_gbs, "peak": peak_gbs, "unit": "GB/s",
-                         "frac": achieved_gbs / peak_gbs, "peak_source": f"{peak_note} copy bandwidth",
-                         "frac_of_8TBs": achieved_gbs / 8000.0,
-                         "traffic": ncu_traffic("packed_step_kda_b256"),
-                         "kernel": "packed_step_kernel<4,KDA,H32,BF16>", "algorithmic_bytes": bytes_step},
-            "fp32_state_kernel": {"us_per_step": r["fp32_launch_ms"] * 1e3,
-                                  "achieved_gbs": bytes_fp32 / (r["fp32_launch_ms"] * 1e-3) / 1e9,
-                                  "bytes_per_step": bytes_fp32,
-                                  "speedup_of_packed": r["fp32_launch_ms"] / r["launch_ms"]},
-            "device": r["dev_name"],
-        }
+        line = make_line(r, args.steps, args.warmup, world)
         if not args.no_cpu_baseline and world == 1:
             line["cpu_baseline"] = cpu_baseline()
         print(json.dumps(line), flush=True)
