@@ -122,6 +122,14 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+// 16-byte asynchronous copy global -> shared through the load/store path (not the
+// bulk-copy engine); completion per thread with cp.async.wait_group.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
 __device__ __forceinline__ uint4 lds128(uint32_t a) {
     uint4 v;
     asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
@@ -268,17 +276,42 @@ __device__ __forceinline__ uint32_t encode4(float2 x01, float2 x23, float2 inv2,
     return pack_sat_u8(__float_as_uint(a.y), __float_as_uint(a.x), upper);
 }
 
+// Extrema of 32 values with three-input min/max only: 32 -> 11 -> 4 -> 2 -> 1
+// (16 operations each for min and max).
 __device__ __forceinline__ void minmax32(const float2 (&y)[16], float &mn, float &mx) {
-    float a[6], b[6];
+    float v[32];
 #pragma unroll
-    for (int i = 0; i < 5; ++i) {  // pairs 3i .. 3i+2 hold six values
-        a[i] = fmin3(fmin3(y[3 * i].x, y[3 * i].y, y[3 * i + 1].x), y[3 * i + 1].y, fminf(y[3 * i + 2].x, y[3 * i + 2].y));
-        b[i] = fmax3(fmax3(y[3 * i].x, y[3 * i].y, y[3 * i + 1].x), y[3 * i + 1].y, fmaxf(y[3 * i + 2].x, y[3 * i + 2].y));
+    for (int j = 0; j < 16; ++j) {
+        v[2 * j] = y[j].x;
+        v[2 * j + 1] = y[j].y;
     }
-    a[5] = fminf(y[15].x, y[15].y);
-    b[5] = fmaxf(y[15].x, y[15].y);
-    mn = fmin3(fmin3(a[0], a[1], a[2]), fmin3(a[3], a[4], a[5]), a[5]);
-    mx = fmax3(fmax3(b[0], b[1], b[2]), fmax3(b[3], b[4], b[5]), b[5]);
+    float a[11], b[11];
+#pragma unroll
+    for (int i = 0; i < 10; ++i) {
+        a[i] = fmin3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+        b[i] = fmax3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+    }
+    a[10] = fminf(v[30], v[31]);
+    b[10] = fmaxf(v[30], v[31]);
+    const float a0 = fmin3(a[0], a[1], a[2]), a1 = fmin3(a[3], a[4], a[5]), a2 = fmin3(a[6], a[7], a[8]);
+    const float b0 = fmax3(b[0], b[1], b[2]), b1 = fmax3(b[3], b[4], b[5]), b2 = fmax3(b[6], b[7], b[8]);
+    mn = fmin3(fmin3(a0, a1, a2), a[9], a[10]);
+    mx = fmax3(fmax3(b0, b1, b2), b[9], b[10]);
+}
+
+// Scale and zero point from the scale s already known to be nonzero (the common
+// case): returns the packed (s, z) pair, inv ~ 1/s and z.
+__device__ __forceinline__ uint32_t affine_finish(float s, float mn, float &inv_out, float &z_out) {
+    const float inv = rcp_approx(s);
+    const __half zh = __float2half_rn(rintf(-mn * (inv * kUp)));
+    z_out = __half2float(zh);
+    inv_out = inv;
+    return (uint32_t)__half_as_ushort(__float2half_rn(s)) | ((uint32_t)__half_as_ushort(zh) << 16);
+}
+
+// binary16 scale of a scaled range: fp16((max - min) / 255)
+__device__ __forceinline__ float scale_of(float mn, float mx) {
+    return __half2float(__float2half_rn((mx - mn) * (kUp / 255.0f)));
 }
 
 // Quantize y' (one lo row, one value block, 16 pairs, scaled by 2^-39) into

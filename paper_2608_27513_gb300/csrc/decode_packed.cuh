@@ -47,6 +47,8 @@ struct PackedParams {
     int32_t rec_bytes, codes_off, meta_off;
     int64_t slot_bytes;
     int32_t nstage, stage_bytes, warp_smem, stage0_off;
+    // per-(slot, head) operand buffer (two per warp): [v row][q][k][g (KDA)][perm]
+    int32_t ops_off, ops_bytes;
     int32_t off_v, off_q, off_k, off_g, off_perm;
     int32_t bytes_v, bytes_qk, bytes_g, bytes_perm;
     int64_t total_tiles;
@@ -157,31 +159,46 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
 
     auto slot_of = [&](int b) -> int64_t { return p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b; };
 
-    // ---- producer (lane 0): bulk copies of tile t (cursor k) into stage s ----
+    // ---- producer (lane 0): one bulk copy of the record of tile t (cursor k) into stage s ----
     auto issue = [&](int64_t t, const Cursor &k, int s) {
         const int64_t slot = slot_of(k.b);
         const bool ok = slot >= 0 && slot < p.num_slots;
-        const bool ops = (t == t0) || (k.c == 0);
         const uint32_t st = stage0 + (uint32_t)(s * p.stage_bytes);
         const uint32_t bar = bar0 + 8 * s;
-        uint32_t bytes = (uint32_t)p.bytes_v;
-        if (ok) bytes += (uint32_t)p.rec_bytes;
-        if (ops) bytes += 2u * p.bytes_qk + p.bytes_g + p.bytes_perm;
-        mbar_arrive_expect_tx(bar, bytes);
-        const int64_t bh = (int64_t)k.b * H + k.h;
+        mbar_arrive_expect_tx(bar, ok ? (uint32_t)p.rec_bytes : 0u);
         if (ok) bulk_g2s(st, p.state + slot * p.slot_bytes + (int64_t)(k.h * V + k.c) * p.rec_bytes, p.rec_bytes, bar);
-        bulk_g2s(st + p.off_v, (const uint8_t *)p.v + (bh * p.dv + k.c * kG) * esz, p.bytes_v, bar);
-        if (ops) {
-            const int hq = (k.h * p.Hqk) / H;
-            const int64_t qoff = ((int64_t)k.b * p.Hqk + hq) * p.dk * esz;
-            bulk_g2s(st + p.off_q, (const uint8_t *)p.q + qoff, p.bytes_qk, bar);
-            bulk_g2s(st + p.off_k, (const uint8_t *)p.k + qoff, p.bytes_qk, bar);
-            if (KDA) bulk_g2s(st + p.off_g, p.g + bh * p.dk, p.bytes_g, bar);
-            bulk_g2s(st + p.off_perm, p.perm + (int64_t)k.h * p.dk, p.bytes_perm, bar);
+    };
+
+    // ---- per-(slot, head) operands: 16-byte copies by all lanes, one head ahead ----
+    const uint32_t ops0 = ws + p.ops_off;
+    auto load_ops = [&](int ub, int uh, uint32_t dst) {
+        const int64_t bh = (int64_t)ub * H + uh;
+        const int hq = (uh * p.Hqk) / H;
+        const int nv = p.bytes_v >> 4, nq = p.bytes_qk >> 4, ng = p.bytes_g >> 4, np = p.bytes_perm >> 4;
+        const int total = nv + 2 * nq + ng + np;
+        const uint8_t *qrow = (const uint8_t *)p.q + ((int64_t)ub * p.Hqk + hq) * p.dk * esz;
+        const uint8_t *krow = (const uint8_t *)p.k + ((int64_t)ub * p.Hqk + hq) * p.dk * esz;
+        for (int ci = lane; ci < total; ci += 32) {
+            int j = ci;
+            const uint8_t *src;
+            if (j < nv) {
+                src = (const uint8_t *)p.v + bh * p.dv * esz + 16 * j;
+            } else if ((j -= nv) < nq) {
+                src = qrow + 16 * j;
+            } else if ((j -= nq) < nq) {
+                src = krow + 16 * j;
+            } else if ((j -= nq) < ng) {
+                src = (const uint8_t *)(p.g + bh * p.dk) + 16 * j;
+            } else {
+                src = p.perm + (int64_t)uh * p.dk + 16 * (j - ng);
+            }
+            cp_async16(dst + 16 * ci, src);
         }
+        cp_async_commit();
     };
 
     Cursor cur = cursor_at(t0, H, V);
+    load_ops(cur.b, cur.h, ops0);
     Cursor pre = cur;  // next tile to load (lane 0)
     int64_t t_pre = t0;
     if (lane == 0) {
@@ -197,6 +214,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
     float aa[R];
     float unit_beta = 0.f, unit_g = 0.f, bkq = 0.f;
     int unit = 0;
+    uint32_t ob = ops0;  // operand buffer of the current (slot, head)
     int s = 0;
     uint32_t parity = 0;
     bool timed_out = false, bad_slot = false;
@@ -216,6 +234,9 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
 
         // ---- per-(slot, head) operands, gathered into calibrated key order ----
         if (t == t0 || c == 0) {
+            ob = ops0 + (uint32_t)((unit & 1) * p.ops_bytes);
+            cp_async_wait_all();
+            __syncwarp();
             // beta (and the GDN log-decay) of the next 32 (slot, head) units are
             // loaded one per lane, long before they are needed
             if ((unit & 31) == 0) {
@@ -227,10 +248,10 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             const float alpha = KDA ? 0.f : expf(__shfl_sync(kFull, unit_g, unit & 31));
             ++unit;
             // d_k is a power of two: masking keeps a malformed permutation in bounds
-            auto chan = [&](int u) { return (int)(lds32(st + p.off_perm + (u & ~3)) >> (8 * (u & 3))) & (p.dk - 1); };
-            auto kv_at = [&](int ch) { return BF16 ? bf16_at(st + p.off_k, ch) : ldsf(st + p.off_k + 4 * ch); };
-            auto qv_at = [&](int ch) { return BF16 ? bf16_at(st + p.off_q, ch) : ldsf(st + p.off_q + 4 * ch); };
-            auto av_at = [&](int ch) { return KDA ? expf(ldsf(st + p.off_g + 4 * ch)) : alpha; };
+            auto chan = [&](int u) { return (int)(lds32(ob + p.off_perm + (u & ~3)) >> (8 * (u & 3))) & (p.dk - 1); };
+            auto kv_at = [&](int ch) { return BF16 ? bf16_at(ob + p.off_k, ch) : ldsf(ob + p.off_k + 4 * ch); };
+            auto qv_at = [&](int ch) { return BF16 ? bf16_at(ob + p.off_q, ch) : ldsf(ob + p.off_q + 4 * ch); };
+            auto av_at = [&](int ch) { return KDA ? expf(ldsf(ob + p.off_g + 4 * ch)) : alpha; };
             float kq = 0.f;  // this lane's share of k^T q (all d_k channels)
 #pragma unroll
             for (int i = 0; i < R; ++i) {
@@ -265,9 +286,14 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             for (int m = 16; m >= 1; m >>= 1) kq += __shfl_xor_sync(kFull, kq, m);
             bkq = beta * kq;  // beta k^T q: o = S_bar^T q + beta (k^T q) d
             __syncwarp();
+            // operands of the next (slot, head) go into the other buffer
+            if (t + (V - c) < t1) {
+                const int nb = h + 1 == H ? b + 1 : b, nh = h + 1 == H ? 0 : h + 1;
+                load_ops(nb, nh, ops0 + (uint32_t)((unit & 1) * p.ops_bytes));  // unit was incremented above
+            }
         }
 
-        const float vj = BF16 ? bf16_at(st + p.off_v, lane) : ldsf(st + p.off_v + 4 * lane);
+        const float vj = BF16 ? bf16_at(ob + p.off_v + c * kG * 2, lane) : ldsf(ob + p.off_v + c * kG * 4 + 4 * lane);
 
         if (ok) {
             const float vt = HAD ? hadamard_lanes(vj, lane) : vj;  // H v
@@ -358,8 +384,21 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             uint32_t szw[R];
 #pragma unroll
             for (int i = 0; i < RL; ++i) minmax32(x[i], mn[i], mx[i]);
+            // scales; a block whose scale rounds to 0 (rare) takes the general path
+            float sc[R];
+            bool any_zero = false;
 #pragma unroll
-            for (int i = 0; i < RL; ++i) szw[i] = affine_params_scaled(mn[i], mx[i], inv[i], zq[i]);
+            for (int i = 0; i < RL; ++i) {
+                sc[i] = scale_of(mn[i], mx[i]);
+                any_zero |= sc[i] == 0.0f;
+            }
+            if (__any_sync(kFull, any_zero)) {
+#pragma unroll
+                for (int i = 0; i < RL; ++i) szw[i] = affine_params_scaled(mn[i], mx[i], inv[i], zq[i]);
+            } else {
+#pragma unroll
+                for (int i = 0; i < RL; ++i) szw[i] = affine_finish(sc[i], mn[i], inv[i], zq[i]);
+            }
 #pragma unroll
             for (int i = 0; i < RL; ++i) {
                 const int r = lane + 32 * i;
@@ -420,6 +459,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             mbar_wait_bounded(bar0 + 8 * (int)(idx % p.nstage), (uint32_t)((idx / p.nstage) & 1));
         }
     }
+    cp_async_wait_all();  // operand copies of a (slot, head) that will not run
     if (lane == 0) {
         bulk_wait_all();
         const uint32_t bits = (timed_out ? kDevWaitTimeout : 0u) | (bad_slot ? kDevBadSlot : 0u);

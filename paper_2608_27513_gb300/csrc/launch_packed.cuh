@@ -42,12 +42,12 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
     p.codes_off = rg.codes_off;
     p.meta_off = rg.meta_off;
     p.slot_bytes = (int64_t)a.H * V * rg.bytes;
-    p.bytes_v = kG * esz;
+    p.bytes_v = a.dv * esz;  // the whole v row of a (slot, head)
     p.bytes_qk = a.dk * esz;
     p.bytes_g = KDA ? a.dk * 4 : 0;
     p.bytes_perm = a.dk;
-    // stage: [record][v][q][k][g][perm], each 16-B aligned
-    int off = rg.bytes;
+    // operand buffer: [v][q][k][g][perm], every part a multiple of 16 B
+    int off = 0;
     p.off_v = off;
     off += p.bytes_v;
     p.off_q = off;
@@ -58,9 +58,11 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
     off += p.bytes_g;
     p.off_perm = off;
     off += p.bytes_perm;
-    p.stage_bytes = (off + 127) & ~127;
+    p.ops_bytes = off;
+    p.ops_off = (scratch_bytes(a.K) + 15) & ~15;
+    p.stage_bytes = (rg.bytes + 127) & ~127;
     p.nstage = kPackedStages;
-    p.stage0_off = (scratch_bytes(a.K) + 127) & ~127;
+    p.stage0_off = (p.ops_off + 2 * p.ops_bytes + 127) & ~127;
     p.warp_smem = p.stage0_off + p.nstage * p.stage_bytes;
     p.total_tiles = (int64_t)a.batch * a.H * V;
     p.status = status;
