@@ -42,7 +42,9 @@ POOLS = 2
 def algorithmic_bytes(w: wl.Workload, packed: bool = True) -> int:
     """Bytes a step must move: every state read and written once, operands read once, o written."""
     B, H, Hq, dk, dv, K = w.batch, w.heads, w.qk_heads, w.d_k, w.d_v, w.k_hi
-    if packed:
+    if packed and w.lo_format == 2:  # row-absmax INT8: one FP32 scale per row
+        state = 2 * K * dv + (dk - K) * dv + 4 * (dk - K)
+    elif packed:
         state = 2 * K * dv + (dk - K) * dv + 4 * (dk - K) * (dv // 32)
     else:
         state = 4 * dk * dv
@@ -412,7 +414,8 @@ def sweep_arm(steps: int, warmup: int):
         del fp
         perm = torch.from_numpy(wl.random_perm(base)).to(dev)
         points = [(0, 1, "uniform int8 (no H32)"), (0, 0, "uniform int8 + H32")] + \
-                 [(k, 0, "damp fp16 + int8 + H32") for k in wl.SWEEP_K_HI if k > 0]
+                 [(k, 0, "damp fp16 + int8 + H32") for k in wl.SWEEP_K_HI if k > 0] + \
+                 [(0, 2, "uniform int8 row-absmax"), (16, 2, "fp16 + int8 row-absmax")]
         for k, fmt, name in points:
             w = wl.sweep(kind, k, fmt)
             L = damp.Layout(w.heads, w.qk_heads, w.d_k, w.d_v, k, fmt)

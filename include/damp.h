@@ -77,7 +77,13 @@ typedef enum {
 typedef enum {
     DAMP_LO_U8_AFFINE_G32_H32 = 0, /* UINT8 affine, G = 32 along d_v, FP16 (s, z), H_32 first:
                                       the paper's DAMP low tier ("INT8+Hadamard", 9.0 bits) */
-    DAMP_LO_U8_AFFINE_G32 = 1      /* the same without H_32 (the paper's "INT8" row, 9.0 bits) */
+    DAMP_LO_U8_AFFINE_G32 = 1,     /* the same without H_32 (the paper's "INT8" row, 9.0 bits) */
+    DAMP_LO_S8_ABSMAX_ROW = 2      /* per-row symmetric absmax INT8, one FP32 scale per row over
+                                      all d_v values: s = max|x|/127, q = sat_[-127,127](rne(x/s)),
+                                      s = 0 -> q = 0; no H_32 (8 + 32/d_v bits).  A fallback
+                                      for a low tier whose scales are left open, not the paper's
+                                      format.  Its step sweeps each head twice (the row scale
+                                      spans every value block) and is not tuned. */
 } damp_lo_format;
 
 /* Element type of q, k and v. */
@@ -115,9 +121,12 @@ DAMP_API damp_status damp_validate_layout(const damp_layout *layout);
  * point).  Record (slot, h, c) starts at byte
  *     slot * damp_slot_bytes + (h * d_v/32 + c) * damp_record_bytes
  * and holds, for value columns 32c .. 32c+31 of all d_k packed rows:
- *     [K_hi x 32 FP16][(d_k-K_hi) x 32 UINT8 codes][(d_k-K_hi) x (s, z) FP16][padding to 16 B]
- * with the 16-byte chunks inside each row permuted for conflict-free shared-memory
- * access.  The byte order inside a record is private to libdamp: move logical
+ *     [ceil(K_hi/2) FP16 row pairs x 128 B][(d_k-K_hi) x 32 codes][(d_k-K_hi) x 4 B metadata]
+ *     [padding to 16 B]
+ * FP16 row pair i interleaves rows 2i and 2i+1 column by column; the 16-byte chunks
+ * inside each code row are permuted for conflict-free shared-memory access.  The
+ * metadata word of a row is its (s, z) FP16 pair (formats 0, 1) or its FP32 row
+ * scale (format 2, the same value in each of the head's d_v/32 records).  The byte order inside a record is private to libdamp: move logical
  * tiers in and out with damp_pack_tiers / damp_unpack_tiers.
  * The pool pointer must be 16-byte aligned.
  */
@@ -125,9 +134,11 @@ DAMP_API size_t damp_record_bytes(const damp_layout *layout); /* 0 if the layout
 DAMP_API size_t damp_slot_bytes(const damp_layout *layout);   /* 0 if the layout is invalid */
 
 /* Storage bits per state value counted from the logical tiers (FP16 rows, codes and
- * FP16 metadata; record padding excluded).  Equals Eq. budgeted_allocation,
+ * metadata; record padding excluded).  Equals Eq. budgeted_allocation,
  * b(K_hi) = b_lo + (K_hi/d_k)(b_hi - b_lo) with b_hi = 16 and b_lo = 8 + 32/32 = 9:
- * 9.875 at K_hi = 16, d_k = 128 (Sec. 5.1).  Returns -1.0 for an invalid layout. */
+ * 9.875 at K_hi = 16, d_k = 128 (Sec. 5.1).  Format 2 counts one FP32 scale per row
+ * (b_lo = 8 + 32/d_v), although its records hold d_v/32 copies of it.
+ * Returns -1.0 for an invalid layout. */
 DAMP_API double damp_bits_per_value(const damp_layout *layout);
 
 /*
@@ -148,7 +159,7 @@ DAMP_API double damp_bits_per_value(const damp_layout *layout);
  *   o          float [B][H][d_v]: output S_t^T q_t from the FP32 post-update state,
  *              before requantization.  4-B aligned; must not overlap the pool.
  *   in_dtype   damp_in_dtype of q, k, v
- * lo_format must be DAMP_LO_U8_AFFINE_G32_H32 or DAMP_LO_U8_AFFINE_G32.
+ * Any lo_format; DAMP_LO_S8_ABSMAX_ROW runs the two-sweep step of that format.
  */
 DAMP_API damp_status damp_gdn_decode_step(const damp_layout *layout, void *state, int64_t num_slots,
                                  const int32_t *slot_idx, int32_t batch, const uint8_t *perm,
@@ -200,7 +211,7 @@ DAMP_API damp_status damp_fp32_kda_decode_step(const damp_layout *layout, float 
  * state (App. A.5 "Prefill path": the chunk-final state is written directly into
  * the packed cache).  Row i of packed head h takes natural row perm[h][i];
  * rows < K_hi are rounded to FP16, the others H_32-transformed (format 0) and
- * quantized as above.
+ * quantized as their lo_format says.
  *   S      float [batch][H][d_k][d_v], natural key order, 16-B aligned, read only
  *   state, num_slots, slot_idx, batch, perm as in damp_gdn_decode_step
  */
@@ -209,7 +220,7 @@ DAMP_API damp_status damp_quantize_state(const damp_layout *layout, const float 
                                 int32_t batch, void *stream);
 
 /* Reconstruct FP32 states from the packed cache (the inverse map: FP16 rows widened,
- * codes dequantized s (q - z) and H_32-transformed back for format 0).
+ * codes dequantized s (q - z) (format 2: s q) and H_32-transformed back for format 0).
  *   S      float [batch][H][d_k][d_v] output, natural key order, 16-B aligned */
 DAMP_API damp_status damp_dequantize_state(const damp_layout *layout, const void *state, int64_t num_slots,
                                   const int32_t *slot_idx, int32_t batch, const uint8_t *perm,
@@ -218,9 +229,11 @@ DAMP_API damp_status damp_dequantize_state(const damp_layout *layout, const void
 /*
  * Copy logical tiers into / out of packed slots, bit for bit (no arithmetic).
  *   hi     uint16 [batch][H][K_hi][d_v]            FP16 bit patterns (S_hi)
- *   codes  uint8  [batch][H][d_k-K_hi][d_v]        UINT8 codes (Q_lo)
- *   meta   uint16 [batch][H][d_k-K_hi][d_v/32][2]  FP16 (s, z) (M_lo)
- * All three 4-B aligned.  NULL is allowed for an empty tier.
+ *   codes  uint8  [batch][H][d_k-K_hi][d_v]        UINT8 codes (Q_lo); int8 for format 2
+ *   meta   uint16 [batch][H][d_k-K_hi][d_v/32][2]  FP16 (s, z) (M_lo); for format 2
+ *          float  [batch][H][d_k-K_hi]             FP32 row scales, through the same pointer
+ * All three 4-B aligned.  NULL is allowed for an empty tier.  Unpacking format 2
+ * returns the scale copy of each row's first record.
  */
 DAMP_API damp_status damp_pack_tiers(const damp_layout *layout, const uint16_t *hi, const uint8_t *codes,
                             const uint16_t *meta, void *state, int64_t num_slots,

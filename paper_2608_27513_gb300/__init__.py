@@ -19,7 +19,7 @@ from dataclasses import dataclass
 from ._lib import DampLayout, DampLibraryError, lib
 
 __all__ = [
-    "Layout", "DampError", "DampLibraryError", "LO_U8_AFFINE_G32_H32", "LO_U8_AFFINE_G32",
+    "Layout", "DampError", "DampLibraryError", "LO_U8_AFFINE_G32_H32", "LO_U8_AFFINE_G32", "LO_S8_ABSMAX_ROW",
     "record_bytes", "slot_bytes", "bits_per_value", "new_state", "new_fp32_state",
     "gdn_decode_step", "kda_decode_step", "u8_gdn_decode_step", "u8_kda_decode_step",
     "fp32_gdn_decode_step", "fp32_kda_decode_step", "quantize_state", "dequantize_state",
@@ -28,6 +28,7 @@ __all__ = [
 
 LO_U8_AFFINE_G32_H32 = 0
 LO_U8_AFFINE_G32 = 1
+LO_S8_ABSMAX_ROW = 2  # per-row symmetric absmax INT8, FP32 row scale
 IN_BF16 = 0
 IN_FP32 = 1
 DEV_WAIT_TIMEOUT = 1
@@ -192,7 +193,8 @@ def dequantize_state(layout, state, perm, batch=None, S=None, slot_idx=None, num
 
 def pack_tiers(layout, hi, codes, meta, state, slot_idx=None, num_slots=None, stream=None):
     """Copy logical tiers (hi uint16/fp16 [B,H,K,d_v], codes uint8 [B,H,d_k-K,d_v],
-    meta uint16/fp16 [B,H,d_k-K,d_v/32,2]) into packed slots, bit for bit."""
+    meta uint16/fp16 [B,H,d_k-K,d_v/32,2]; row-absmax format: codes int8, meta float32
+    [B,H,d_k-K]) into packed slots, bit for bit."""
     for n, t in (("hi", hi), ("codes", codes), ("meta", meta), ("state", state), ("slot_idx", slot_idx)):
         _cuda_contig(n, t)
     B = codes.shape[0] if codes is not None else hi.shape[0]
@@ -205,7 +207,8 @@ def pack_tiers(layout, hi, codes, meta, state, slot_idx=None, num_slots=None, st
 
 
 def unpack_tiers(layout, state, batch=None, slot_idx=None, num_slots=None, stream=None):
-    """Logical tiers (hi int16 bits, codes uint8, meta int16 bits) of `batch` packed slots."""
+    """Logical tiers (hi int16 bits, codes uint8, meta int16 bits; row-absmax format: codes
+    int8, meta float32 [B,H,d_k-K]) of `batch` packed slots."""
     import torch
     _cuda_contig("state", state)
     _cuda_contig("slot_idx", slot_idx)
@@ -213,8 +216,12 @@ def unpack_tiers(layout, state, batch=None, slot_idx=None, num_slots=None, strea
     H, dk, dv, K = layout.num_heads, layout.d_k, layout.d_v, layout.k_hi
     dev = state.device
     hi = torch.empty((B, H, K, dv), dtype=torch.int16, device=dev)
-    codes = torch.empty((B, H, dk - K, dv), dtype=torch.uint8, device=dev)
-    meta = torch.empty((B, H, dk - K, dv // 32, 2), dtype=torch.int16, device=dev)
+    if layout.lo_format == LO_S8_ABSMAX_ROW:
+        codes = torch.empty((B, H, dk - K, dv), dtype=torch.int8, device=dev)
+        meta = torch.empty((B, H, dk - K), dtype=torch.float32, device=dev)
+    else:
+        codes = torch.empty((B, H, dk - K, dv), dtype=torch.uint8, device=dev)
+        meta = torch.empty((B, H, dk - K, dv // 32, 2), dtype=torch.int16, device=dev)
     c = layout.c()
     _check(lib().damp_unpack_tiers(ctypes.byref(c), _ptr(state), state.shape[0] if num_slots is None else num_slots,
                                    _ptr(slot_idx), B, _ptr(hi if hi.numel() else None),

@@ -43,7 +43,9 @@ damp_status check_layout(const damp_layout *L) {
     if (L->d_k != 32 && L->d_k != 64 && L->d_k != 128) return DAMP_ERR_SHAPE;
     if (L->d_v < 32 || L->d_v > 1024 || L->d_v % 32) return DAMP_ERR_SHAPE;
     if (L->k_hi < 0 || L->k_hi > L->d_k) return DAMP_ERR_SHAPE;
-    if (L->lo_format != DAMP_LO_U8_AFFINE_G32_H32 && L->lo_format != DAMP_LO_U8_AFFINE_G32) return DAMP_ERR_FORMAT;
+    if (L->lo_format != DAMP_LO_U8_AFFINE_G32_H32 && L->lo_format != DAMP_LO_U8_AFFINE_G32 &&
+        L->lo_format != DAMP_LO_S8_ABSMAX_ROW)
+        return DAMP_ERR_FORMAT;
     return DAMP_OK;
 }
 
@@ -67,6 +69,7 @@ damp_status check_pool(const void *state, int64_t num_slots, const int32_t *slot
 
 cudaError_t launch_step(const StepArgs &a, bool packed, cudaStream_t s) {
     if (!packed) return launch_fp32_step(a, s);
+    if (a.fmt == DAMP_LO_S8_ABSMAX_ROW) return launch_rowabs_step(a, s);
     return a.kda ? launch_packed_kda(a, s) : launch_packed_gdn(a, s);
 }
 
@@ -148,7 +151,8 @@ damp_status convert(const damp_layout *L, void *state, int64_t num_slots, const 
             overlap(rs, range_of(slot_idx, slot_idx ? B * 4 : 0)) || overlap(pool, range_of(perm, H * dk)))
             return DAMP_ERR_ALIAS;
     } else {
-        const int64_t nh = B * H * K * dv * 2, nc = B * H * (dk - K) * dv, nm = B * H * (dk - K) * (dv / 32) * 4;
+        const int64_t nh = B * H * K * dv * 2, nc = B * H * (dk - K) * dv;
+        const int64_t nm = B * H * (dk - K) * (L->lo_format == DAMP_LO_S8_ABSMAX_ROW ? 1 : dv / 32) * 4;
         if ((nh && !hi) || (nc && !codes) || (nm && !meta)) return DAMP_ERR_NULL;
         if ((hi && !aligned(hi, 4)) || (codes && !aligned(codes, 4)) || (meta && !aligned(meta, 4)))
             return DAMP_ERR_ALIGN;
@@ -174,6 +178,8 @@ damp_status convert(const damp_layout *L, void *state, int64_t num_slots, const 
     a.codes = codes;
     a.meta = meta;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (a.fmt == DAMP_LO_S8_ABSMAX_ROW)
+        return launch_rowabs_convert(a, (int)kind, s) == cudaSuccess ? DAMP_OK : DAMP_ERR_CUDA;
     cudaError_t e = kind == kQ ? launch_quantize(a, s)
                     : kind == kDQ ? launch_dequantize(a, s)
                     : kind == kPack ? launch_pack_tiers(a, s)
@@ -262,7 +268,9 @@ size_t damp_slot_bytes(const damp_layout *layout) {
 double damp_bits_per_value(const damp_layout *L) {
     if (check_layout(L) != DAMP_OK) return -1.0;
     const double hi = 16.0 * L->k_hi * L->d_v;
-    const double lo = (8.0 + 32.0 / 32.0) * (double)(L->d_k - L->k_hi) * L->d_v;  // UINT8 + FP16 (s,z) per 32
+    const double lo = L->lo_format == DAMP_LO_S8_ABSMAX_ROW
+                          ? (8.0 * L->d_v + 32.0) * (double)(L->d_k - L->k_hi)             // int8 + one FP32 scale
+                          : (8.0 + 32.0 / 32.0) * (double)(L->d_k - L->k_hi) * L->d_v;  // UINT8 + FP16 (s,z) per 32
     return (hi + lo) / ((double)L->d_k * L->d_v);
 }
 
@@ -348,6 +356,8 @@ damp_status damp_device_status(uint32_t *status) {
     if (take_status_fp32(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     if (take_status_convert(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_rowabs(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     *status = all;
     return DAMP_OK;

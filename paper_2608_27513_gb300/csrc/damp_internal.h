@@ -44,12 +44,16 @@ cudaError_t launch_quantize(const ConvArgs &a, cudaStream_t s);
 cudaError_t launch_dequantize(const ConvArgs &a, cudaStream_t s);
 cudaError_t launch_pack_tiers(const ConvArgs &a, cudaStream_t s);
 cudaError_t launch_unpack_tiers(const ConvArgs &a, cudaStream_t s);
+// Row-absmax INT8 low tier (lo_format 2); op: 0 quantize, 1 dequantize, 2 pack, 3 unpack.
+cudaError_t launch_rowabs_step(const StepArgs &a, cudaStream_t s);
+cudaError_t launch_rowabs_convert(const ConvArgs &a, int op, cudaStream_t s);
 
 // Read-and-clear of each translation unit's device status word.
 cudaError_t take_status_packed_gdn(uint32_t *bits);
 cudaError_t take_status_packed_kda(uint32_t *bits);
 cudaError_t take_status_fp32(uint32_t *bits);
 cudaError_t take_status_convert(uint32_t *bits);
+cudaError_t take_status_rowabs(uint32_t *bits);
 
 // Streaming multiprocessors / opt-in shared memory per block of the current device (cached per device).
 int sm_count();

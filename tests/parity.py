@@ -46,14 +46,20 @@ def inputs_to_dev(w: wl.Workload, inp: dict, dev) -> dict:
 def tiers_to_dev(w: wl.Workload, tiers, rows: int, dev):
     hi, codes, meta = tiers
     H, dk, dv, K = w.heads, w.d_k, w.d_v, w.k_hi
+    if w.lo_format == core.FMT_S8_ROW:
+        m = to_dev(meta.astype(np.float32).reshape(rows, H, dk - K), dev)
+    else:
+        m = to_dev(meta.view(np.int16).reshape(rows, H, dk - K, dv // 32, 2), dev)
     return (to_dev(hi.view(np.int16).reshape(rows, H, K, dv), dev),
-            to_dev(codes.reshape(rows, H, dk - K, dv), dev),
-            to_dev(meta.view(np.int16).reshape(rows, H, dk - K, dv // 32, 2), dev))
+            to_dev(codes.reshape(rows, H, dk - K, dv), dev), m)
 
 
 def tiers_from_dev(w: wl.Workload, dev_tiers, units: int):
     hi, codes, meta = (t.cpu().numpy() for t in dev_tiers)
     H, dk, dv, K = w.heads, w.d_k, w.d_v, w.k_hi
+    if w.lo_format == core.FMT_S8_ROW:
+        return (hi.view(np.uint16).reshape(units, K, dv), codes.view(np.int8).reshape(units, dk - K, dv),
+                meta.astype(np.float32).reshape(units, dk - K))
     return (hi.view(np.uint16).reshape(units, K, dv), codes.reshape(units, dk - K, dv),
             meta.view(np.uint16).reshape(units, dk - K, dv // 32, 2))
 
@@ -101,6 +107,9 @@ def compare_tiers(w: wl.Workload, ref, gpu, lo_pre, stats: CodeStats, what=""):
         assert not bad.any(), f"{what}: FP16 tier differs at {np.argwhere(bad)[:5].tolist()}"
     if not codes_r.size:
         return
+    if w.lo_format == core.FMT_S8_ROW:
+        _compare_s8_rows(ref, gpu, lo_pre, stats, what)
+        return
     n, lo, dv = codes_r.shape
     G = dv // 32
     cr = codes_r.reshape(n, lo, G, 32).astype(np.int64)
@@ -143,6 +152,30 @@ def compare_tiers(w: wl.Workload, ref, gpu, lo_pre, stats: CodeStats, what=""):
     stats.meta_mismatched += int(meta_diff.sum())
 
 
+S8_SCALE_REL = 1e-5  # a row scale is max|x|/127 of values that may differ by float ordering
+
+
+def _compare_s8_rows(ref, gpu, lo_pre, stats: CodeStats, what):
+    """Row-absmax INT8 rows: scales within S8_SCALE_REL, codes within 1 and only at
+    ties of the oracle's own x/s."""
+    _, codes_r, s_r = ref
+    _, codes_g, s_g = gpu
+    s_r64, s_g64 = s_r.astype(np.float64), s_g.astype(np.float64)
+    assert np.all(np.abs(s_g64 - s_r64) <= S8_SCALE_REL * np.abs(s_r64) + 1e-30), \
+        f"{what}: a row scale differs beyond float ordering"
+    d = np.abs(codes_r.astype(np.int64) - codes_g.astype(np.int64))
+    assert np.all(d <= 1), f"{what}: a code differs by more than 1 LSB"
+    with np.errstate(divide="ignore", invalid="ignore"):
+        t = np.where(s_r64[..., None] > 0, lo_pre.astype(np.float64) / s_r64[..., None], 0.0)
+    near = np.abs(np.abs(t - np.floor(t)) - 0.5) < TIE
+    bad = (d > 0) & ~near
+    assert not bad.any(), f"{what}: codes differ away from a rounding tie at {np.argwhere(bad)[:5].tolist()}"
+    stats.codes += d.size
+    stats.mismatched += int((d > 0).sum())
+    stats.groups += s_r.size
+    stats.meta_mismatched += int((s_r != s_g).sum())
+
+
 def compare_o(o_gpu, o_ref, what=""):
     bad = np.abs(o_gpu - o_ref) > ATOL + RTOL * np.abs(o_ref)
     assert not bad.any(), (f"{what}: o differs at {np.argwhere(bad)[:5].tolist()} "
@@ -155,3 +188,37 @@ def initial_tiers(w: wl.Workload, rows, perms, prefix=None):
     S0 = runs.prefix_states(w, rows, steps=prefix).reshape(len(rows) * w.heads, w.d_k, w.d_v)
     perm_units = np.tile(perms, (len(rows), 1))
     return perm_units, core.pack_heads(perm_units, S0, w.k_hi, w.lo_format)
+
+
+def run_teacher_forced(w: wl.Workload, steps: int, dev, rows=None, n_docs=2, n_tokens=16, slot_of=None, pool=None,
+                       u8=False):
+    """Teacher-forced steps through the C ABI against the oracle: every GPU step starts
+    from the oracle's packed state, so one rounding tie never compounds."""
+    rows = list(range(w.batch)) if rows is None else list(rows)
+    perms, _ = runs.calibrate_layout(w, n_docs=n_docs, n_tokens=n_tokens)
+    perm_units, tiers = initial_tiers(w, rows, perms, prefix=min(w.prefix, 32))
+    L = layout_of(w)
+    n_slots = pool or len(rows)
+    state = damp.new_state(L, n_slots, dev)
+    slot_idx = None if slot_of is None else torch.tensor([slot_of[b] for b in range(len(rows))],
+                                                         dtype=torch.int32, device=dev)
+    dperm = to_dev(perms, dev)
+    stats = CodeStats()
+    if u8:
+        step = damp.u8_kda_decode_step if w.kind == "kda" else damp.u8_gdn_decode_step
+    else:
+        step = damp.kda_decode_step if w.kind == "kda" else damp.gdn_decode_step
+    for t in range(steps):
+        inp = wl.step_inputs(w, t, rows=rows)
+        u = runs.unit_operands(w, inp)
+        o_ref, new_ref, lo_pre = oracle_step(w, perm_units, tiers, u)
+        damp.pack_tiers(L, *tiers_to_dev(w, tiers, len(rows), dev), state, slot_idx=slot_idx)
+        d = inputs_to_dev(w, inp, dev)
+        o = step(L, state, dperm, d["q"], d["k"], d["v"], d["g"], d["beta"], slot_idx=slot_idx)
+        got = tiers_from_dev(w, damp.unpack_tiers(L, state, batch=len(rows), slot_idx=slot_idx),
+                             len(rows) * w.heads)
+        compare_o(o.cpu().numpy().reshape(-1, w.d_v), o_ref, f"{w.name} step {t}")
+        compare_tiers(w, new_ref, got, lo_pre, stats, f"{w.name} step {t}")
+        tiers = new_ref
+    stats.check_fraction()
+    return stats

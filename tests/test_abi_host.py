@@ -9,6 +9,7 @@ import pytest
 
 import paper_2608_27513_gb300 as damp
 from paper_2608_27513_gb300 import _lib, build
+from oracle import core
 from tests.golden.load import paper_values
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
@@ -60,12 +61,18 @@ def test_record_geometry_and_bits(L):
         assert damp.slot_bytes(lay) == 32 * 4 * damp.record_bytes(lay)
         assert damp.bits_per_value(lay) == 8.0 * logical / (128 * 32)
     assert damp.bits_per_value(_layout(k_hi=16)) == pv["damp_bits_k16_dk128"]
+    # row-absmax INT8: one FP32 scale per row counted once, as the oracle's logical tiers
+    for K in (0, 5, 16, 128):
+        for dv in (64, 128, 1024):
+            lay = _layout(k_hi=K, lo_format=2, d_v=dv)
+            assert damp.bits_per_value(lay) == pytest.approx(core.bits_per_value(128, dv, K, core.FMT_S8_ROW), rel=1e-12)
+            assert damp.record_bytes(lay) == damp.record_bytes(_layout(k_hi=K, d_v=dv))
     assert damp.bits_per_value(_layout(k_hi=0)) == pv["bits_int8_hadamard"]
 
 
 @pytest.mark.parametrize("kw,status", [
     (dict(d_k=96), 2), (dict(d_k=256), 2), (dict(d_v=48), 2), (dict(d_v=2048), 2), (dict(k_hi=129), 2),
-    (dict(k_hi=-1), 2), (dict(num_qk_heads=5), 2), (dict(num_heads=0), 2), (dict(lo_format=2), 5)])
+    (dict(k_hi=-1), 2), (dict(num_qk_heads=5), 2), (dict(num_heads=0), 2), (dict(lo_format=3), 5)])
 def test_layout_validation(L, kw, status):
     c = _layout(**kw).c()
     assert L.damp_validate_layout(ctypes.byref(c)) == status

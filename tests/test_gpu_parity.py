@@ -114,35 +114,8 @@ def test_fp32_step_matches_oracle(w):
 
 # --------------------------------------------------- fused packed step ---
 
-def _run_teacher_forced(w, steps, rows=None, n_docs=2, n_tokens=16, slot_of=None, pool=None, u8=False):
-    rows = list(range(w.batch)) if rows is None else list(rows)
-    perms, _ = runs.calibrate_layout(w, n_docs=n_docs, n_tokens=n_tokens)
-    perm_units, tiers = P.initial_tiers(w, rows, perms, prefix=min(w.prefix, 32))
-    L = P.layout_of(w)
-    n_slots = pool or len(rows)
-    state = damp.new_state(L, n_slots, DEV)
-    slot_idx = None if slot_of is None else torch.tensor([slot_of[b] for b in range(len(rows))],
-                                                         dtype=torch.int32, device=DEV)
-    dperm = P.to_dev(perms, DEV)
-    stats = P.CodeStats()
-    if u8:
-        step = damp.u8_kda_decode_step if w.kind == "kda" else damp.u8_gdn_decode_step
-    else:
-        step = damp.kda_decode_step if w.kind == "kda" else damp.gdn_decode_step
-    for t in range(steps):
-        inp = wl.step_inputs(w, t, rows=rows)
-        u = runs.unit_operands(w, inp)
-        o_ref, new_ref, lo_pre = P.oracle_step(w, perm_units, tiers, u)
-        damp.pack_tiers(L, *P.tiers_to_dev(w, tiers, len(rows), DEV), state, slot_idx=slot_idx)
-        d = P.inputs_to_dev(w, inp, DEV)
-        o = step(L, state, dperm, d["q"], d["k"], d["v"], d["g"], d["beta"], slot_idx=slot_idx)
-        got = P.tiers_from_dev(w, damp.unpack_tiers(L, state, batch=len(rows), slot_idx=slot_idx),
-                               len(rows) * w.heads)
-        P.compare_o(o.cpu().numpy().reshape(-1, w.d_v), o_ref, f"{w.name} step {t}")
-        P.compare_tiers(w, new_ref, got, lo_pre, stats, f"{w.name} step {t}")
-        tiers = new_ref
-    stats.check_fraction()
-    return stats
+def _run_teacher_forced(w, steps, **kw):
+    return P.run_teacher_forced(w, steps, DEV, **kw)
 
 
 def test_gdn_b1_d64_k8_matches_oracle():
