@@ -79,17 +79,17 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
                         for (int m = 0; m < 16; ++m) x[m] = mul2(x[m], splat2(kDown));  // working scale
                         uint32_t w[8];
                         const uint32_t sz = quantize_group(x, w);
-                        *reinterpret_cast<uint4 *>(rec + p.codes_off + lo_chunk_off(r, 0)) =
+                        *reinterpret_cast<uint4 *>(rec + p.codes_off + lo_chunk_off(r, 0, lo)) =
                             make_uint4(w[0], w[1], w[2], w[3]);
-                        *reinterpret_cast<uint4 *>(rec + p.codes_off + lo_chunk_off(r, 1)) =
+                        *reinterpret_cast<uint4 *>(rec + p.codes_off + lo_chunk_off(r, 1, lo)) =
                             make_uint4(w[4], w[5], w[6], w[7]);
                         *reinterpret_cast<uint32_t *>(rec + p.meta_off + 4 * r) = sz;
                     }
                 } else {
                     {
                         const int r = u - K;
-                        const uint4 c0 = *reinterpret_cast<const uint4 *>(rec + p.codes_off + lo_chunk_off(r, 0));
-                        const uint4 c1 = *reinterpret_cast<const uint4 *>(rec + p.codes_off + lo_chunk_off(r, 1));
+                        const uint4 c0 = *reinterpret_cast<const uint4 *>(rec + p.codes_off + lo_chunk_off(r, 0, lo));
+                        const uint4 c1 = *reinterpret_cast<const uint4 *>(rec + p.codes_off + lo_chunk_off(r, 1, lo));
                         const uint32_t sz = *reinterpret_cast<const uint32_t *>(rec + p.meta_off + 4 * r);
                         const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
                         dequantize_group(w, sz, 1.0f, x);
@@ -107,7 +107,7 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
                     uint32_t *mrow = reinterpret_cast<uint32_t *>(p.meta + ((((int64_t)b * p.H + h) * lo + r) * p.V + c) * 2);
 #pragma unroll
                     for (int m = 0; m < 2; ++m) {
-                        uint32_t *r4 = reinterpret_cast<uint32_t *>(rec + p.codes_off + lo_chunk_off(r, m));
+                        uint32_t *r4 = reinterpret_cast<uint32_t *>(rec + p.codes_off + lo_chunk_off(r, m, lo));
 #pragma unroll
                         for (int e = 0; e < 4; ++e) {
                             if (OP == kPackTiers) r4[e] = crow[4 * m + e];

@@ -24,10 +24,12 @@ enum : uint32_t { kDevWaitTimeout = 1u, kDevBadSlot = 2u };
 //              32 column words (binary16 of row 2i in the low half); an odd K
 //              leaves the last high half zero.  A lane reads two FP16 rows of its
 //              column with one 32-bit load.
-//   codes:     (d_k-K) x 32 B;    16-B chunk m of lo row r at 16 * (m ^ ((r >> 2) & 1))
+//   codes:     (d_k-K) x 32 B, chunk-major: 16-B chunk m (columns 16m .. 16m+15)
+//              of lo row r at 16 * (m * (d_k-K) + r)
 //   meta:      (d_k-K) x 4 B      (s, z) as two binary16
-// The chunk permutation of the codes makes the 8 consecutive rows that a
-// quarter warp reads with 128-bit loads hit distinct shared-memory banks.
+// With one lane per lo row, a warp's 128-bit access to chunk m of 32 consecutive
+// rows covers 512 contiguous bytes: conflict-free in shared memory, whole
+// sectors in global memory.
 // ---------------------------------------------------------------------------
 struct RecGeom {
     int codes_off, meta_off, bytes;
@@ -43,7 +45,7 @@ __host__ __device__ inline RecGeom rec_geom(int d_k, int k_hi) {
 
 // byte offset of FP16 row u, column j (0..31) inside a record
 __host__ __device__ inline int hi_elem_off(int u, int j) { return 128 * (u >> 1) + 4 * j + 2 * (u & 1); }
-__host__ __device__ inline int lo_chunk_off(int r, int m) { return 32 * r + 16 * (m ^ ((r >> 2) & 1)); }
+__host__ __device__ inline int lo_chunk_off(int r, int m, int lo) { return 16 * (m * lo + r); }
 
 // ---------------------------------------------------------------------------
 // PTX wrappers
@@ -129,6 +131,14 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void *src) {
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
+__device__ __forceinline__ void stg128(void *p, uint4 v) {
+    asm volatile("st.global.v4.b32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+__device__ __forceinline__ void stg32(void *p, uint32_t v) {
+    asm volatile("st.global.b32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
 
 __device__ __forceinline__ uint4 lds128(uint32_t a) {
     uint4 v;

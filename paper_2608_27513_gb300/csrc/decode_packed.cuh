@@ -60,7 +60,7 @@ constexpr int kPartOff = 64;                              // after NSTAGE (<= 8)
 constexpr int kPartStride = 68;                           // floats per lane row: 32 (r, p) pairs + padding
 constexpr int kDvecOff = kPartOff + 32 * kPartStride * 4; // 32 floats: H d for the low tier
 constexpr int kHopsOff = kDvecOff + 32 * 4;               // FP16-row operands, 32 B per row pair
-__host__ __device__ constexpr int scratch_bytes(int k_hi) { return kHopsOff + 16 * ((k_hi + 3) & ~3); }
+__host__ __device__ constexpr int scratch_bytes(int k_hi) { return kHopsOff + 16 * ((k_hi + 7) & ~7); }
 
 __device__ __forceinline__ float ldsf(uint32_t a) { return __uint_as_float(lds32(a)); }
 
@@ -202,7 +202,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
     Cursor pre = cur;  // next tile to load (lane 0)
     int64_t t_pre = t0;
     if (lane == 0) {
-        for (int j = 0; j < p.nstage - 1 && t_pre < t1; ++j) {
+        for (int j = 0; j < p.nstage && t_pre < t1; ++j) {
             issue(t_pre, pre, j);
             ++t_pre;
             advance(pre, H, V);
@@ -231,6 +231,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
         const int64_t slot = slot_of(b);
         const bool ok = slot >= 0 && slot < p.num_slots;
         bad_slot |= !ok;
+        uint8_t *const grec = p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * p.rec_bytes;  // written in place
 
         // ---- per-(slot, head) operands, gathered into calibrated key order ----
         if (t == t0 || c == 0) {
@@ -266,22 +267,25 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
                 aa[i] = av_at(ch) * kDown;
                 kq = fmaf(kv, qv, kq);
             }
-            // FP16 rows in pairs: {a_u, a_u+1, k_u, k_u+1} {q_u, q_u+1, bk_u, bk_u+1};
-            // rows K .. K4-1 (padding to a multiple of 4) carry zero weights
-            const int K4 = (K + 3) & ~3;
-            for (int u = 2 * lane; u < K4; u += 64) {
+            // FP16 rows in pairs: {a_u, a_u+1, bk_u, bk_u+1} {k_u, k_u+1, q_u, q_u+1};
+            // rows K .. K8-1 (padding to whole chunks of 4 pairs) carry zero weights.
+            // Lane l writes pair l (and pair l + 32 when K_hi > 64), straight-line.
+            const int K8 = (K + 7) & ~7;
+            auto hop_pair = [&](int u) {
                 const bool one = u < K, two = u + 1 < K;
-                const int c0 = one ? chan(u) : 0;
-                const int c1 = two ? chan(u + 1) : 0;
+                const int c0 = chan(one ? u : 0);
+                const int c1 = chan(two ? u + 1 : 0);
                 const float k0 = one ? kv_at(c0) : 0.f, k1 = two ? kv_at(c1) : 0.f;
-                sts128(hops + 16 * u, make_uint4(__float_as_uint(one ? av_at(c0) : 0.f),
-                                                 __float_as_uint(two ? av_at(c1) : 0.f), __float_as_uint(k0),
-                                                 __float_as_uint(k1)));
                 const float q0 = one ? qv_at(c0) : 0.f, q1 = two ? qv_at(c1) : 0.f;
-                sts128(hops + 16 * u + 16, make_uint4(__float_as_uint(q0), __float_as_uint(q1),
-                                                      __float_as_uint(beta * k0), __float_as_uint(beta * k1)));
+                const float a0 = av_at(c0), a1 = av_at(c1);
+                sts128(hops + 16 * u, make_uint4(__float_as_uint(one ? a0 : 0.f), __float_as_uint(two ? a1 : 0.f),
+                                                 __float_as_uint(beta * k0), __float_as_uint(beta * k1)));
+                sts128(hops + 16 * u + 16, make_uint4(__float_as_uint(k0), __float_as_uint(k1), __float_as_uint(q0),
+                                                      __float_as_uint(q1)));
                 kq = fmaf(k0, q0, fmaf(k1, q1, kq));
-            }
+            };
+            if (2 * lane < K8) hop_pair(2 * lane);
+            if (K8 > 64 && 2 * lane + 64 < K8) hop_pair(2 * lane + 64);
 #pragma unroll
             for (int m = 16; m >= 1; m >>= 1) kq += __shfl_xor_sync(kFull, kq, m);
             bkq = beta * kq;  // beta k^T q: o = S_bar^T q + beta (k^T q) d
@@ -304,8 +308,8 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
 #pragma unroll
             for (int i = 0; i < RL; ++i) {
                 const int r = min(lane + 32 * i, lo - 1);
-                const uint4 c0 = lds128(st + p.codes_off + lo_chunk_off(r, 0));
-                const uint4 c1 = lds128(st + p.codes_off + lo_chunk_off(r, 1));
+                const uint4 c0 = lds128(st + p.codes_off + lo_chunk_off(r, 0, lo));
+                const uint4 c1 = lds128(st + p.codes_off + lo_chunk_off(r, 1, lo));
                 const uint32_t sz = lds32(st + p.meta_off + 4 * r);
                 const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
                 dequantize_group(w, sz, aa[i], x[i]);
@@ -323,26 +327,30 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             // ---- phase 1, FP16 tier (lane = column): one 32-bit load per row pair ----
             const uint32_t col = st + 4 * lane;  // this lane's word in FP16 row pair 0
             const int KP = (K + 1) >> 1;         // row pairs in the record
-            float2 rh = make_float2(0.f, 0.f), rh2 = rh, ph = rh, ph2 = rh;
-            for (int pi = 0; pi < KP; pi += 2) {
-                // pair pi + 1 may be the zero-weight padding pair (hops rows up to K4):
-                // read a valid word and let the zero weights cancel it
-                const uint32_t wa = lds32(col + 128 * pi);
-                const uint32_t wb = lds32(col + 128 * min(pi + 1, KP - 1));
-                const uint4 opa = lds128(hops + 32 * pi);
-                const uint4 oqa = lds128(hops + 32 * pi + 16);
-                const uint4 opb = lds128(hops + 32 * pi + 32);
-                const uint4 oqb = lds128(hops + 32 * pi + 48);
-                const float2 xa = mul2(h2_to_f2(wa), make_float2(__uint_as_float(opa.x), __uint_as_float(opa.y)));
-                const float2 xb = mul2(h2_to_f2(wb), make_float2(__uint_as_float(opb.x), __uint_as_float(opb.y)));
-                rh = fma2(xa, make_float2(__uint_as_float(opa.z), __uint_as_float(opa.w)), rh);
-                rh2 = fma2(xb, make_float2(__uint_as_float(opb.z), __uint_as_float(opb.w)), rh2);
-                ph = fma2(xa, make_float2(__uint_as_float(oqa.x), __uint_as_float(oqa.y)), ph);
-                ph2 = fma2(xb, make_float2(__uint_as_float(oqb.x), __uint_as_float(oqb.y)), ph2);
+            // chunks of 4 pairs, loads first; pairs past the last carry zero weights
+            // and read a zero word
+            float2 rh[4], ph[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) rh[q] = ph[q] = make_float2(0.f, 0.f);
+            for (int p0 = 0; p0 < KP; p0 += 4) {
+                uint32_t wv[4];
+                uint4 oa[4], ok[4];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    wv[q] = p0 + q < KP ? lds32(col + 128 * (p0 + q)) : 0u;
+                    oa[q] = lds128(hops + 32 * (p0 + q));
+                    ok[q] = lds128(hops + 32 * (p0 + q) + 16);
+                }
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float2 xa = mul2(h2_to_f2(wv[q]), make_float2(__uint_as_float(oa[q].x), __uint_as_float(oa[q].y)));
+                    rh[q] = fma2(xa, make_float2(__uint_as_float(ok[q].x), __uint_as_float(ok[q].y)), rh[q]);
+                    ph[q] = fma2(xa, make_float2(__uint_as_float(ok[q].z), __uint_as_float(ok[q].w)), ph[q]);
+                }
             }
-            rh = add2(rh, rh2);
-            ph = add2(ph, ph2);
-            const float rhi = rh.x + rh.y, phi = ph.x + ph.y;
+            rh[0] = add2(add2(rh[0], rh[1]), add2(rh[2], rh[3]));
+            ph[0] = add2(add2(ph[0], ph[1]), add2(ph[2], ph[3]));
+            const float rhi = rh[0].x + rh[0].y, phi = ph[0].x + ph[0].y;
             const float2 lo_sums = column_sum2(acc, accp, part, lane);
             const float rlo = lo_sums.x * kUp, plo = lo_sums.y * kUp;  // back from the working scale
 
@@ -384,67 +392,67 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             uint32_t szw[R];
 #pragma unroll
             for (int i = 0; i < RL; ++i) minmax32(x[i], mn[i], mx[i]);
-            // scales; a block whose scale rounds to 0 (rare) takes the general path
+            // scales: the common path assumes s != 0; a block whose scale rounds to 0
+            // (rare) is encoded again below with the general path, over its first stores
             float sc[R];
             bool any_zero = false;
 #pragma unroll
             for (int i = 0; i < RL; ++i) {
                 sc[i] = scale_of(mn[i], mx[i]);
                 any_zero |= sc[i] == 0.0f;
+                szw[i] = affine_finish(sc[i], mn[i], inv[i], zq[i]);
             }
-            if (__any_sync(kFull, any_zero)) {
-#pragma unroll
-                for (int i = 0; i < RL; ++i) szw[i] = affine_params_scaled(mn[i], mx[i], inv[i], zq[i]);
-            } else {
-#pragma unroll
-                for (int i = 0; i < RL; ++i) szw[i] = affine_finish(sc[i], mn[i], inv[i], zq[i]);
-            }
-#pragma unroll
-            for (int i = 0; i < RL; ++i) {
+            auto encode_store = [&](int i) {
                 const int r = lane + 32 * i;
                 const float2 inv2 = splat2(inv[i] * 0x1p-110f), zc2 = splat2(zq[i] * 0x1p-149f);
                 uint32_t w[8];
 #pragma unroll
                 for (int m = 0; m < 8; ++m) w[m] = encode4(x[i][2 * m], x[i][2 * m + 1], inv2, zc2);
-                // a lane past the last row writes into its own slice of the (idle)
-                // partial-sum buffer instead of branching around the stores
-                const bool live = r < lo;
-                const uint32_t trash = part + lane * kPartStride * 4;
-                sts128(live ? st + p.codes_off + lo_chunk_off(r, 0) : trash, make_uint4(w[0], w[1], w[2], w[3]));
-                sts128(live ? st + p.codes_off + lo_chunk_off(r, 1) : trash + 16, make_uint4(w[4], w[5], w[6], w[7]));
-                sts32(live ? st + p.meta_off + 4 * r : trash + 32, szw[i]);
+                if (r < lo) {
+                    stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                    stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
+                    stg32(grec + p.meta_off + 4 * r, szw[i]);
+                }
+            };
+#pragma unroll
+            for (int i = 0; i < RL; ++i) encode_store(i);
+            if (__any_sync(kFull, any_zero)) {
+#pragma unroll
+                for (int i = 0; i < RL; ++i) {
+                    if (sc[i] == 0.0f) {
+                        szw[i] = affine_params_scaled(mn[i], mx[i], inv[i], zq[i]);
+                        encode_store(i);
+                    }
+                }
             }
 
             // ---- phase 2, FP16 tier: S = S_bar + beta k d, FP16 store (two rows per word) ----
             const float2 dj2 = splat2(dj);
-            for (int pi = 0; pi < KP; ++pi) {
-                const uint32_t wa = lds32(col + 128 * pi);
-                const uint4 opa = lds128(hops + 32 * pi);
-                const uint4 oqa = lds128(hops + 32 * pi + 16);
-                const float2 xa = mul2(h2_to_f2(wa), make_float2(__uint_as_float(opa.x), __uint_as_float(opa.y)));
-                const float2 y = fma2(make_float2(__uint_as_float(oqa.z), __uint_as_float(oqa.w)), dj2, xa);
-                sts32(col + 128 * pi, f2_to_h2(y.x, y.y));  // an odd K's padding half stays 0
+            for (int p0 = 0; p0 < KP; p0 += 4) {
+                uint32_t wv[4];
+                uint4 oa[4];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    wv[q] = p0 + q < KP ? lds32(col + 128 * (p0 + q)) : 0u;
+                    oa[q] = lds128(hops + 32 * (p0 + q));
+                }
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float2 xa = mul2(h2_to_f2(wv[q]), make_float2(__uint_as_float(oa[q].x), __uint_as_float(oa[q].y)));
+                    const float2 y = fma2(make_float2(__uint_as_float(oa[q].z), __uint_as_float(oa[q].w)), dj2, xa);
+                    // an odd K's padding half stays 0
+                    if (p0 + q < KP) stg32(grec + 128 * (p0 + q) + 4 * lane, f2_to_h2(y.x, y.y));
+                }
             }
-
-            // ---- write the updated record back ----
-            fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) {
-                bulk_s2g(p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * p.rec_bytes, st, p.rec_bytes);
-                bulk_commit();
-            }
-        } else if (lane == 0) {
-            bulk_commit();  // an empty group keeps one group per tile
         }
-        // ---- keep the ring full: the next load reuses the stage of tile t-1, whose
-        // store was committed one tile ago (every group but the newest has been read)
+        // ---- the stage has been read: refill it with tile t + nstage ----
+        __syncwarp();
         if (lane == 0 && t_pre < t1) {
-            bulk_wait_read_all_but_newest();
-            issue(t_pre, pre, (s + p.nstage - 1) % p.nstage);
+            fence_proxy_async_smem();  // the warp's reads of the stage before the bulk copy's writes
+            issue(t_pre, pre, s);
             ++t_pre;
             advance(pre, H, V);
         }
-        __syncwarp();
         if (++s == p.nstage) {
             s = 0;
             parity ^= 1u;
@@ -453,15 +461,14 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
     if (timed_out) {
         // let the loads already in flight land (each wait bounded) before the CTA's
         // shared memory goes away
-        const int64_t last = min(t1 - 1, t_fail + p.nstage - 2);
-        for (int64_t tt = t_fail + 1; tt <= last; ++tt) {
+        const int64_t last = min(t1 - 1, t_fail + p.nstage - 1);
+        for (int64_t tt = t_fail; tt <= last; ++tt) {
             const int64_t idx = tt - t0;
             mbar_wait_bounded(bar0 + 8 * (int)(idx % p.nstage), (uint32_t)((idx / p.nstage) & 1));
         }
     }
     cp_async_wait_all();  // operand copies of a (slot, head) that will not run
     if (lane == 0) {
-        bulk_wait_all();
         const uint32_t bits = (timed_out ? kDevWaitTimeout : 0u) | (bad_slot ? kDevBadSlot : 0u);
         if (bits) atomicOr(p.status, bits);
     }

@@ -64,10 +64,10 @@ __device__ __forceinline__ float transpose_sum32(float (&v)[32], int lane) {
 }
 
 // Reconstructed and decayed low-tier row r of one record: a * (s * q_j).
-__device__ __forceinline__ void lo_row_decayed(const uint8_t *rec, int codes_off, int meta_off, int r, float a,
-                                               float (&x)[32]) {
-    const uint4 c0 = *reinterpret_cast<const uint4 *>(rec + codes_off + lo_chunk_off(r, 0));
-    const uint4 c1 = *reinterpret_cast<const uint4 *>(rec + codes_off + lo_chunk_off(r, 1));
+__device__ __forceinline__ void lo_row_decayed(const uint8_t *rec, int codes_off, int meta_off, int lo, int r,
+                                               float a, float (&x)[32]) {
+    const uint4 c0 = *reinterpret_cast<const uint4 *>(rec + codes_off + lo_chunk_off(r, 0, lo));
+    const uint4 c1 = *reinterpret_cast<const uint4 *>(rec + codes_off + lo_chunk_off(r, 1, lo));
     const float s = *reinterpret_cast<const float *>(rec + meta_off + 4 * r);
     const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
 #pragma unroll
@@ -133,7 +133,7 @@ __global__ void __launch_bounds__(32 * kRaWarps) rowabs_step_kernel(const RowAbs
             const int r = lane + 32 * i;
             if (r < lo) {
                 float x[32];
-                lo_row_decayed(rec, p.codes_off, p.meta_off, r, as[K + r], x);
+                lo_row_decayed(rec, p.codes_off, p.meta_off, lo, r, as[K + r], x);
                 const float kv = ks[K + r], qv = qs[K + r];
 #pragma unroll
                 for (int e = 0; e < 32; ++e) {
@@ -166,7 +166,7 @@ __global__ void __launch_bounds__(32 * kRaWarps) rowabs_step_kernel(const RowAbs
             const int r = lane + 32 * i;
             if (r < lo) {
                 float x[32];
-                lo_row_decayed(rec, p.codes_off, p.meta_off, r, as[K + r], x);
+                lo_row_decayed(rec, p.codes_off, p.meta_off, lo, r, as[K + r], x);
                 const float bk = __fmul_rn(beta, ks[K + r]);
 #pragma unroll
                 for (int e = 0; e < 32; ++e)
@@ -186,7 +186,7 @@ __global__ void __launch_bounds__(32 * kRaWarps) rowabs_step_kernel(const RowAbs
             const int r = lane + 32 * i;
             if (r < lo) {
                 float x[32];
-                lo_row_decayed(rec, p.codes_off, p.meta_off, r, as[K + r], x);
+                lo_row_decayed(rec, p.codes_off, p.meta_off, lo, r, as[K + r], x);
                 const float bk = __fmul_rn(beta, ks[K + r]);
                 uint32_t w[8] = {0, 0, 0, 0, 0, 0, 0, 0};
 #pragma unroll
@@ -194,8 +194,8 @@ __global__ void __launch_bounds__(32 * kRaWarps) rowabs_step_kernel(const RowAbs
                     const float xn = __fadd_rn(x[e], __fmul_rn(bk, dsm[kG * c + e]));
                     w[e >> 2] |= (uint32_t)(uint8_t)encode_s8(xn, scale[i]) << (8 * (e & 3));
                 }
-                *reinterpret_cast<uint4 *>(rec + p.codes_off + lo_chunk_off(r, 0)) = make_uint4(w[0], w[1], w[2], w[3]);
-                *reinterpret_cast<uint4 *>(rec + p.codes_off + lo_chunk_off(r, 1)) = make_uint4(w[4], w[5], w[6], w[7]);
+                *reinterpret_cast<uint4 *>(rec + p.codes_off + lo_chunk_off(r, 0, lo)) = make_uint4(w[0], w[1], w[2], w[3]);
+                *reinterpret_cast<uint4 *>(rec + p.codes_off + lo_chunk_off(r, 1, lo)) = make_uint4(w[4], w[5], w[6], w[7]);
                 *reinterpret_cast<float *>(rec + p.meta_off + 4 * r) = scale[i];
             }
         }
@@ -266,7 +266,7 @@ __global__ void __launch_bounds__(256) rowabs_convert_kernel(const RowAbsConv p)
             const int r = u - K;
             auto code_at = [&](int j) -> int8_t * {
                 uint8_t *rec = head + (int64_t)(j >> 5) * p.rec_bytes;
-                return reinterpret_cast<int8_t *>(rec + p.codes_off + lo_chunk_off(r, (j & 31) >> 4) + (j & 15));
+                return reinterpret_cast<int8_t *>(rec + p.codes_off + lo_chunk_off(r, (j & 31) >> 4, lo) + (j & 15));
             };
             auto meta_at = [&](int c) {
                 return reinterpret_cast<float *>(head + (int64_t)c * p.rec_bytes + p.meta_off + 4 * r);
