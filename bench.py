@@ -191,6 +191,8 @@ def workload_config(w: wl.Workload, bits=None) -> dict:
             "l2": f"inputs larger than L2: {POOLS} packed state pools of "
                   f"{algorithmic_bytes(w) / 2 / 1e6:.0f} MB each rotated per step (> 129 MB L2)",
             "permutation": "seeded random pi per head (throughput does not depend on which)",
+            "timing": "CUDA events around K back-to-back launches on the launching stream; "
+                      "roofline.achieved uses the same average launch time",
             "parallelism": f"{world} independent replica(s), one batch per GPU"}
 
 
@@ -236,7 +238,9 @@ def gpu_arm(args, rank: int, world: int):
         d = inputs[i % N_INPUT_SETS]
         damp.fp32_kda_decode_step(L, fp32_pools[i % POOLS], d["q"], d["k"], d["v"], d["g"], d["beta"], o=o_buf)
 
-    def timed(fn, steps, warmup, per_launch=True):
+    def timed(fn, steps, warmup, per_launch=False):
+        # Back-to-back launches between two CUDA events: an event pair around every
+        # launch would add a gap per launch to the timeline being measured.
         for i in range(warmup):
             fn(i, o)
         if world > 1:

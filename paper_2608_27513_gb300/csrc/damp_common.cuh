@@ -187,11 +187,22 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
 // ---------------------------------------------------------------------------
 
 // Across the 32 lanes of a warp: lane j holds x_j, returns (H_32 x)_j.
-__device__ __forceinline__ float hadamard_lanes(float x, int lane) {
+// Butterfly signs of a lane: round m (partner lane ^ 2^m) adds for bit m clear
+// and subtracts for bit m set; fma(x, sign, y) is then y - x or x + y, rounded once.
+struct LaneSigns {
+    float s[5];
+};
+__device__ __forceinline__ LaneSigns lane_signs(int lane) {
+    LaneSigns g;
 #pragma unroll
-    for (int m = 1; m < 32; m <<= 1) {
-        const float y = __shfl_xor_sync(kFull, x, m);
-        x = (lane & m) ? (y - x) : (x + y);
+    for (int i = 0; i < 5; ++i) g.s[i] = (lane >> i) & 1 ? -1.0f : 1.0f;
+    return g;
+}
+__device__ __forceinline__ float hadamard_lanes(float x, const LaneSigns &g) {
+#pragma unroll
+    for (int i = 0; i < 5; ++i) {
+        const float y = __shfl_xor_sync(kFull, x, 1 << i);
+        x = __fmaf_rn(x, g.s[i], y);
     }
     return x * kInvSqrt32;
 }

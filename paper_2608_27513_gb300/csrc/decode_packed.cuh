@@ -127,13 +127,17 @@ __device__ __forceinline__ void advance(Cursor &k, int H, int V) {
 
 // RL = ceil((d_k - K_hi) / 32): low-tier row slots per lane, fixed at compile time
 // so that the row loops unroll into one basic block.
-template <int RL, bool KDA, bool HAD, bool BF16>
+// KC >= 0 fixes K_hi at compile time (KC = 0: no FP16 tier) and DKC > 0 fixes d_k:
+// with both fixed, the record geometry and every row offset are constants and the
+// FP16 tier runs as straight-line code.  KC = -1, DKC = 0 is the general kernel.
+template <int RL, int DKC, int KC, bool KDA, bool HAD, bool BF16>
 __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams p) {
     constexpr int R = RL > 0 ? RL : 1;
     extern __shared__ __align__(128) uint8_t smem[];
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     const int nw = blockDim.x >> 5;
+    const LaneSigns sg = lane_signs(lane);
     const uint32_t ws = smem_u32(smem) + (uint32_t)(warp * p.warp_smem);
     const uint32_t bar0 = ws;
     const uint32_t part = ws + kPartOff;
@@ -141,8 +145,14 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
     const uint32_t hops = ws + kHopsOff;
     const uint32_t stage0 = ws + p.stage0_off;
     const int esz = BF16 ? 2 : 4;
-    const int K = p.K;
-    const int lo = p.dk - K;  // low-tier rows
+    constexpr bool KFIX = KC >= 0, DFIX = DKC > 0;
+    const int K = KFIX ? KC : p.K;
+    const int dk = DFIX ? DKC : p.dk;
+    const int lo = dk - K;  // low-tier rows
+    // record geometry (constants for a fixed layout)
+    const int codes_off = KFIX ? 128 * ((KC + 1) / 2) : p.codes_off;
+    const int meta_off = (KFIX && DFIX) ? 128 * ((KC + 1) / 2) + 32 * (DKC - KC) : p.meta_off;
+    const int rec_bytes = (KFIX && DFIX) ? (128 * ((KC + 1) / 2) + 36 * (DKC - KC) + 15) & ~15 : p.rec_bytes;
     const int H = p.H, V = p.V;
 
     const int64_t gw = (int64_t)blockIdx.x * nw + warp;
@@ -165,8 +175,8 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
         const bool ok = slot >= 0 && slot < p.num_slots;
         const uint32_t st = stage0 + (uint32_t)(s * p.stage_bytes);
         const uint32_t bar = bar0 + 8 * s;
-        mbar_arrive_expect_tx(bar, ok ? (uint32_t)p.rec_bytes : 0u);
-        if (ok) bulk_g2s(st, p.state + slot * p.slot_bytes + (int64_t)(k.h * V + k.c) * p.rec_bytes, p.rec_bytes, bar);
+        mbar_arrive_expect_tx(bar, ok ? (uint32_t)rec_bytes : 0u);
+        if (ok) bulk_g2s(st, p.state + slot * p.slot_bytes + (int64_t)(k.h * V + k.c) * rec_bytes, rec_bytes, bar);
     };
 
     // ---- per-(slot, head) operands: 16-byte copies by all lanes, one head ahead ----
@@ -176,8 +186,8 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
         const int hq = (uh * p.Hqk) / H;
         const int nv = p.bytes_v >> 4, nq = p.bytes_qk >> 4, ng = p.bytes_g >> 4, np = p.bytes_perm >> 4;
         const int total = nv + 2 * nq + ng + np;
-        const uint8_t *qrow = (const uint8_t *)p.q + ((int64_t)ub * p.Hqk + hq) * p.dk * esz;
-        const uint8_t *krow = (const uint8_t *)p.k + ((int64_t)ub * p.Hqk + hq) * p.dk * esz;
+        const uint8_t *qrow = (const uint8_t *)p.q + ((int64_t)ub * p.Hqk + hq) * dk * esz;
+        const uint8_t *krow = (const uint8_t *)p.k + ((int64_t)ub * p.Hqk + hq) * dk * esz;
         for (int ci = lane; ci < total; ci += 32) {
             int j = ci;
             const uint8_t *src;
@@ -188,9 +198,9 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             } else if ((j -= nq) < nq) {
                 src = krow + 16 * j;
             } else if ((j -= nq) < ng) {
-                src = (const uint8_t *)(p.g + bh * p.dk) + 16 * j;
+                src = (const uint8_t *)(p.g + bh * dk) + 16 * j;
             } else {
-                src = p.perm + (int64_t)uh * p.dk + 16 * (j - ng);
+                src = p.perm + (int64_t)uh * dk + 16 * (j - ng);
             }
             cp_async16(dst + 16 * ci, src);
         }
@@ -231,7 +241,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
         const int64_t slot = slot_of(b);
         const bool ok = slot >= 0 && slot < p.num_slots;
         bad_slot |= !ok;
-        uint8_t *const grec = p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * p.rec_bytes;  // written in place
+        uint8_t *const grec = p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * rec_bytes;  // written in place
 
         // ---- per-(slot, head) operands, gathered into calibrated key order ----
         if (t == t0 || c == 0) {
@@ -249,7 +259,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             const float alpha = KDA ? 0.f : expf(__shfl_sync(kFull, unit_g, unit & 31));
             ++unit;
             // d_k is a power of two: masking keeps a malformed permutation in bounds
-            auto chan = [&](int u) { return (int)(lds32(ob + p.off_perm + (u & ~3)) >> (8 * (u & 3))) & (p.dk - 1); };
+            auto chan = [&](int u) { return (int)(lds32(ob + p.off_perm + (u & ~3)) >> (8 * (u & 3))) & (dk - 1); };
             auto kv_at = [&](int ch) { return BF16 ? bf16_at(ob + p.off_k, ch) : ldsf(ob + p.off_k + 4 * ch); };
             auto qv_at = [&](int ch) { return BF16 ? bf16_at(ob + p.off_q, ch) : ldsf(ob + p.off_q + 4 * ch); };
             auto av_at = [&](int ch) { return KDA ? expf(ldsf(ob + p.off_g + 4 * ch)) : alpha; };
@@ -300,7 +310,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
         const float vj = BF16 ? bf16_at(ob + p.off_v + c * kG * 2, lane) : ldsf(ob + p.off_v + c * kG * 4 + 4 * lane);
 
         if (ok) {
-            const float vt = HAD ? hadamard_lanes(vj, lane) : vj;  // H v
+            const float vt = HAD ? hadamard_lanes(vj, sg) : vj;  // H v
             float2 x[R][16];
             float2 acc[16], accp[16];
             // ---- phase 1, low tier: reconstruct and decay (scaled by 2^-39), partial
@@ -308,9 +318,9 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
 #pragma unroll
             for (int i = 0; i < RL; ++i) {
                 const int r = min(lane + 32 * i, lo - 1);
-                const uint4 c0 = lds128(st + p.codes_off + lo_chunk_off(r, 0, lo));
-                const uint4 c1 = lds128(st + p.codes_off + lo_chunk_off(r, 1, lo));
-                const uint32_t sz = lds32(st + p.meta_off + 4 * r);
+                const uint4 c0 = lds128(st + codes_off + lo_chunk_off(r, 0, lo));
+                const uint4 c1 = lds128(st + codes_off + lo_chunk_off(r, 1, lo));
+                const uint32_t sz = lds32(st + meta_off + 4 * r);
                 const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
                 dequantize_group(w, sz, aa[i], x[i]);
 #pragma unroll
@@ -327,25 +337,33 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             // ---- phase 1, FP16 tier (lane = column): one 32-bit load per row pair ----
             const uint32_t col = st + 4 * lane;  // this lane's word in FP16 row pair 0
             const int KP = (K + 1) >> 1;         // row pairs in the record
-            // chunks of 4 pairs, loads first; pairs past the last carry zero weights
-            // and read a zero word
+            // pair pi accumulates into rh[pi & 3], ph[pi & 3] (four independent chains)
             float2 rh[4], ph[4];
 #pragma unroll
             for (int q = 0; q < 4; ++q) rh[q] = ph[q] = make_float2(0.f, 0.f);
-            for (int p0 = 0; p0 < KP; p0 += 4) {
-                uint32_t wv[4];
-                uint4 oa[4], ok[4];
+            auto hi_pair1 = [&](int pi, uint32_t wv, const uint4 &oa, const uint4 &ok) {
+                const float2 xa = mul2(h2_to_f2(wv), make_float2(__uint_as_float(oa.x), __uint_as_float(oa.y)));
+                rh[pi & 3] = fma2(xa, make_float2(__uint_as_float(ok.x), __uint_as_float(ok.y)), rh[pi & 3]);
+                ph[pi & 3] = fma2(xa, make_float2(__uint_as_float(ok.z), __uint_as_float(ok.w)), ph[pi & 3]);
+            };
+            if constexpr (KFIX) {
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    wv[q] = p0 + q < KP ? lds32(col + 128 * (p0 + q)) : 0u;
-                    oa[q] = lds128(hops + 32 * (p0 + q));
-                    ok[q] = lds128(hops + 32 * (p0 + q) + 16);
-                }
+                for (int pi = 0; pi < (KC + 1) / 2; ++pi)
+                    hi_pair1(pi, lds32(col + 128 * pi), lds128(hops + 32 * pi), lds128(hops + 32 * pi + 16));
+            } else {
+                // chunks of 4 pairs, loads first; pairs past the last carry zero
+                // weights and read a zero word
+                for (int p0 = 0; p0 < KP; p0 += 4) {
+                    uint32_t wv[4];
+                    uint4 oa[4], ok[4];
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const float2 xa = mul2(h2_to_f2(wv[q]), make_float2(__uint_as_float(oa[q].x), __uint_as_float(oa[q].y)));
-                    rh[q] = fma2(xa, make_float2(__uint_as_float(ok[q].x), __uint_as_float(ok[q].y)), rh[q]);
-                    ph[q] = fma2(xa, make_float2(__uint_as_float(ok[q].z), __uint_as_float(ok[q].w)), ph[q]);
+                    for (int q = 0; q < 4; ++q) {
+                        wv[q] = p0 + q < KP ? lds32(col + 128 * (p0 + q)) : 0u;
+                        oa[q] = lds128(hops + 32 * (p0 + q));
+                        ok[q] = lds128(hops + 32 * (p0 + q) + 16);
+                    }
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) hi_pair1(q, wv[q], oa[q], ok[q]);
                 }
             }
             rh[0] = add2(add2(rh[0], rh[1]), add2(rh[2], rh[3]));
@@ -358,9 +376,9 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             // o = S_t^T q = S_bar^T q + beta (k^T q) d, with S_bar^T q = H p~_lo + p_hi
             float dj, dt, pj;
             if (HAD) {
-                const float hr_lo = hadamard_lanes(rlo, lane);
-                const float hp_lo = hadamard_lanes(plo, lane);
-                const float hr_hi = K > 0 ? hadamard_lanes(rhi, lane) : 0.f;
+                const float hr_lo = hadamard_lanes(rlo, sg);
+                const float hp_lo = hadamard_lanes(plo, sg);
+                const float hr_hi = K > 0 ? hadamard_lanes(rhi, sg) : 0.f;
                 dj = vj - (hr_lo + rhi);
                 dt = vt - (rlo + hr_hi);
                 pj = hp_lo + phi;
@@ -409,9 +427,9 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
 #pragma unroll
                 for (int m = 0; m < 8; ++m) w[m] = encode4(x[i][2 * m], x[i][2 * m + 1], inv2, zc2);
                 if (r < lo) {
-                    stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
-                    stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
-                    stg32(grec + p.meta_off + 4 * r, szw[i]);
+                    stg128(grec + codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                    stg128(grec + codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
+                    stg32(grec + meta_off + 4 * r, szw[i]);
                 }
             };
 #pragma unroll
@@ -428,20 +446,26 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
 
             // ---- phase 2, FP16 tier: S = S_bar + beta k d, FP16 store (two rows per word) ----
             const float2 dj2 = splat2(dj);
-            for (int p0 = 0; p0 < KP; p0 += 4) {
-                uint32_t wv[4];
-                uint4 oa[4];
+            auto hi_pair2 = [&](int pi, uint32_t wv, const uint4 &oa) {
+                const float2 xa = mul2(h2_to_f2(wv), make_float2(__uint_as_float(oa.x), __uint_as_float(oa.y)));
+                const float2 y = fma2(make_float2(__uint_as_float(oa.z), __uint_as_float(oa.w)), dj2, xa);
+                stg32(grec + 128 * pi + 4 * lane, f2_to_h2(y.x, y.y));  // an odd K's padding half stays 0
+            };
+            if constexpr (KFIX) {
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    wv[q] = p0 + q < KP ? lds32(col + 128 * (p0 + q)) : 0u;
-                    oa[q] = lds128(hops + 32 * (p0 + q));
-                }
+                for (int pi = 0; pi < (KC + 1) / 2; ++pi) hi_pair2(pi, lds32(col + 128 * pi), lds128(hops + 32 * pi));
+            } else {
+                for (int p0 = 0; p0 < KP; p0 += 4) {
+                    uint32_t wv[4];
+                    uint4 oa[4];
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const float2 xa = mul2(h2_to_f2(wv[q]), make_float2(__uint_as_float(oa[q].x), __uint_as_float(oa[q].y)));
-                    const float2 y = fma2(make_float2(__uint_as_float(oa[q].z), __uint_as_float(oa[q].w)), dj2, xa);
-                    // an odd K's padding half stays 0
-                    if (p0 + q < KP) stg32(grec + 128 * (p0 + q) + 4 * lane, f2_to_h2(y.x, y.y));
+                    for (int q = 0; q < 4; ++q) {
+                        wv[q] = p0 + q < KP ? lds32(col + 128 * (p0 + q)) : 0u;
+                        oa[q] = lds128(hops + 32 * (p0 + q));
+                    }
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        if (p0 + q < KP) hi_pair2(p0 + q, wv[q], oa[q]);
                 }
             }
         }

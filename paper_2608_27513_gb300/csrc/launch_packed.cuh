@@ -83,20 +83,42 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
 
     void (*kern)(PackedParams) = nullptr;
     const bool had = a.fmt == 0;
-#define DAMP_PICK(RL_)                                                                         \
-    if (rl == RL_) {                                                                           \
-        if (had) kern = a.in_bf16 ? packed_step_kernel<RL_, KDA, true, true>                   \
-                                  : packed_step_kernel<RL_, KDA, true, false>;                 \
-        else kern = a.in_bf16 ? packed_step_kernel<RL_, KDA, false, true>                      \
-                              : packed_step_kernel<RL_, KDA, false, false>;                    \
+#define DAMP_PICK4(RL_, DKC_, KC_)                                                                \
+    if (had) kern = a.in_bf16 ? packed_step_kernel<RL_, DKC_, KC_, KDA, true, true>               \
+                              : packed_step_kernel<RL_, DKC_, KC_, KDA, true, false>;             \
+    else kern = a.in_bf16 ? packed_step_kernel<RL_, DKC_, KC_, KDA, false, true>                  \
+                          : packed_step_kernel<RL_, DKC_, KC_, KDA, false, false>;
+    // compile-time layouts: d_k = 128 with the K_hi values below
+#define DAMP_FIXED(KC_)                                                                           \
+    if (!kern && a.dk == 128 && a.K == KC_) {                                                     \
+        DAMP_PICK4((128 - KC_ + 31) / 32, 128, KC_)                                               \
     }
+    DAMP_FIXED(0)
+    DAMP_FIXED(4)
+    DAMP_FIXED(8)
+    DAMP_FIXED(10)
+    DAMP_FIXED(16)
+    DAMP_FIXED(32)
+    // general kernels: K_hi = 0 (no FP16 tier) or any K_hi, runtime d_k
     const int rl = (a.dk - a.K + 31) / 32;
-    DAMP_PICK(0)
-    DAMP_PICK(1)
-    DAMP_PICK(2)
-    DAMP_PICK(3)
-    DAMP_PICK(4)
-#undef DAMP_PICK
+#define DAMP_GENERAL(RL_)                                                                         \
+    if (!kern && rl == RL_) {                                                                     \
+        if (a.K == 0) {                                                                           \
+            DAMP_PICK4(RL_, 0, 0)                                                                 \
+        } else {                                                                                  \
+            DAMP_PICK4(RL_, 0, -1)                                                                \
+        }                                                                                         \
+    }
+    if (!kern && rl == 0) {
+        DAMP_PICK4(0, 0, -1)
+    }
+    DAMP_GENERAL(1)
+    DAMP_GENERAL(2)
+    DAMP_GENERAL(3)
+    DAMP_GENERAL(4)
+#undef DAMP_GENERAL
+#undef DAMP_FIXED
+#undef DAMP_PICK4
     if (!kern) return cudaErrorInvalidValue;
     cudaError_t e = ensure_smem_limit(reinterpret_cast<const void *>(kern), smem);
     if (e != cudaSuccess) return e;
