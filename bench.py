@@ -168,13 +168,14 @@ def make_line(r: dict, steps: int, warmup: int, world: int) -> dict:
         "config": workload_config(w, r.get("bits")),
         "clocks": r.get("clocks"),
         "e2e": {"value": world * bytes_step / (r["e2e_ms"] * 1e-3) / 1e12, "unit": "TB/s",
-                "us_per_step": r["e2e_ms"] * 1e3, "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"]},
+                "us_per_step": r["e2e_ms"] * 1e3, "h2d_bytes_per_step": r["h2d"], "d2h_bytes_per_step": r["d2h"],
+                "pipeline": "uploads and read-backs on a copy stream overlapping the previous/next step"},
         "gpu_launches": steps,
         "roofline": {"bound": "hbm", "achieved": achieved_gbs, "peak": peak_gbs, "unit": "GB/s",
                      "frac": achieved_gbs / peak_gbs, "peak_source": f"{peak_note} copy bandwidth",
                      "frac_of_8TBs": achieved_gbs / 8000.0,
                      "traffic": ncu_traffic("packed_step_kda_b256"),
-                     "kernel": "packed_step_kernel<4,KDA,H32,BF16>", "algorithmic_bytes": bytes_step},
+                     "kernel": "packed_step_kernel<RL=4,d_k=128,K_hi=10,KDA,H32,BF16>", "algorithmic_bytes": bytes_step},
         "fp32_state_kernel": {"us_per_step": r["fp32_launch_ms"] * 1e3,
                               "achieved_gbs": bytes_fp32 / (r["fp32_launch_ms"] * 1e-3) / 1e9,
                               "bytes_per_step": bytes_fp32,
@@ -281,24 +282,62 @@ def gpu_arm(args, rank: int, world: int):
     fp_total, fp_launch = timed(run_fp32, fp_steps, max(args.warmup, 3))
     fp_launch = max_over_ranks_(fp_launch)
 
-    # ---- end to end through the C ABI from pinned host buffers ----
+    # ---- end to end through the C ABI from pinned host buffers.  Every step uploads its
+    # own inputs and reads its output back; a copy stream overlaps step i+1's upload and
+    # step i's read-back with step i's kernel (inputs and outputs double-buffered on the
+    # device, events order every reuse). ----
+    copy_stream = torch.cuda.Stream(dev)
     host_in = [{k: v.cpu().pin_memory() for k, v in d.items()} for d in inputs[:2]]
     dev_in = [{k: torch.empty_like(v) for k, v in d.items()} for d in inputs[:2]]
-    o_host = torch.empty((w.batch, w.heads, w.d_v), dtype=torch.float32).pin_memory()
+    o_dev = [torch.empty_like(o) for _ in range(2)]
+    o_host = [torch.empty(o.shape, dtype=torch.float32).pin_memory() for _ in range(2)]
     h2d = sum(v.numel() * v.element_size() for v in host_in[0].values())
-    d2h = o_host.numel() * 4
+    d2h = o_host[0].numel() * 4
+    up_done = [torch.cuda.Event() for _ in range(2)]
+    step_done = [torch.cuda.Event() for _ in range(2)]
+    down_done = [torch.cuda.Event() for _ in range(2)]
 
-    def run_e2e(i, o_buf):
-        src, dst = host_in[i % 2], dev_in[i % 2]
-        for k in dst:
-            dst[k].copy_(src[k], non_blocking=True)
-        damp.kda_decode_step(L, pools[i % POOLS], perm, dst["q"], dst["k"], dst["v"], dst["g"], dst["beta"],
-                             o=o_buf)
-        o_host.copy_(o_buf, non_blocking=True)
+    def upload(i):
+        j = i % 2
+        with torch.cuda.stream(copy_stream):
+            if i >= 2:
+                copy_stream.wait_event(step_done[j])  # step i-2 has read dev_in[j]
+            for k in dev_in[j]:
+                dev_in[j][k].copy_(host_in[j][k], non_blocking=True)
+            up_done[j].record(copy_stream)
+
+    def run_e2e(i):
+        j = i % 2
+        upload(i + 1)
+        stream.wait_event(up_done[j])
+        if i >= 2:
+            stream.wait_event(down_done[j])  # step i-2's output has been read back
+        d = dev_in[j]
+        damp.kda_decode_step(L, pools[i % POOLS], perm, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o_dev[j])
+        step_done[j].record(stream)
+        with torch.cuda.stream(copy_stream):
+            copy_stream.wait_event(step_done[j])
+            o_host[j].copy_(o_dev[j], non_blocking=True)
+            down_done[j].record(copy_stream)
 
     e2e_steps = max(args.steps // 10, 10)
-    e2e_total, _ = timed(run_e2e, e2e_steps, max(args.warmup, 3), per_launch=False)
-    e2e_total = max_over_ranks_(e2e_total)
+    e2e_warm = max(args.warmup, 3)
+    upload(0)
+    for i in range(e2e_warm):
+        run_e2e(i)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(e2e_warm, e2e_warm + e2e_steps):
+        run_e2e(i)
+    stream.wait_event(down_done[(e2e_warm + e2e_steps - 1) % 2])  # the last read-back is inside
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e2e_total = max_over_ranks_(e0.elapsed_time(e1))
     return {
         "w": w, "total_ms": total_ms, "launch_ms": launch_ms, "fp32_launch_ms": fp_launch,
         "e2e_ms": e2e_total / e2e_steps, "h2d": h2d, "d2h": d2h, "clocks": clk.summary(),
