@@ -369,25 +369,36 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             rh[0] = add2(add2(rh[0], rh[1]), add2(rh[2], rh[3]));
             ph[0] = add2(add2(ph[0], ph[1]), add2(ph[2], ph[3]));
             const float rhi = rh[0].x + rh[0].y, phi = ph[0].x + ph[0].y;
+            // fixed layouts: H r_hi overlaps the column sums, and the butterflies for d and o
+            // run during the requantization (the general kernel keeps the plain order:
+            // deferring them costs it registers)
+            constexpr bool kLateD = KFIX && DFIX;
+            const float hr_hi_early = (kLateD && HAD && K > 0) ? hadamard_lanes(rhi, sg) : 0.f;
             const float2 lo_sums = column_sum2(acc, accp, part, lane);
             const float rlo = lo_sums.x * kUp, plo = lo_sums.y * kUp;  // back from the working scale
 
             // r = H r~_lo + r_hi;  d = v - r (natural, FP16 rows);  H d = H v - r~_lo - H r_hi (low tier);
-            // o = S_t^T q = S_bar^T q + beta (k^T q) d, with S_bar^T q = H p~_lo + p_hi
-            float dj, dt, pj;
-            if (HAD) {
-                const float hr_lo = hadamard_lanes(rlo, sg);
-                const float hp_lo = hadamard_lanes(plo, sg);
-                const float hr_hi = K > 0 ? hadamard_lanes(rhi, sg) : 0.f;
-                dj = vj - (hr_lo + rhi);
-                dt = vt - (rlo + hr_hi);
-                pj = hp_lo + phi;
+            // o = S_t^T q = S_bar^T q + beta (k^T q) d, with S_bar^T q = H p~_lo + p_hi.
+            // H d goes out first: the low tier's requantization waits on it; the butterflies
+            // for d and o run while it proceeds.
+            float dj = 0.f, pj = 0.f, dt;
+            auto natural_d_and_o = [&]() {
+                if (HAD) {
+                    dj = vj - (hadamard_lanes(rlo, sg) + rhi);
+                    pj = hadamard_lanes(plo, sg) + phi;
+                } else {
+                    dj = vj - (rlo + rhi);
+                    pj = plo + phi;
+                }
+                p.o[((int64_t)b * H + h) * p.dv + c * kG + lane] = fmaf(bkq, dj, pj);
+            };
+            if constexpr (kLateD) {
+                dt = HAD ? vt - (rlo + hr_hi_early) : vj - (rlo + rhi);
             } else {
-                dj = vj - (rlo + rhi);
-                dt = dj;
-                pj = plo + phi;
+                const float hr_hi = (HAD && K > 0) ? hadamard_lanes(rhi, sg) : 0.f;
+                natural_d_and_o();
+                dt = HAD ? vt - (rlo + hr_hi) : dj;
             }
-            p.o[((int64_t)b * H + h) * p.dv + c * kG + lane] = fmaf(bkq, dj, pj);
             sts32(dvec + 4 * lane, __float_as_uint(dt));
             __syncwarp();
 
@@ -406,6 +417,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
 #pragma unroll
                 for (int j = 0; j < 16; ++j) x[i][j] = fma2(bk[i], d[j], x[i][j]);
             }
+            if constexpr (kLateD) natural_d_and_o();
             float mn[R], mx[R], inv[R], zq[R];
             uint32_t szw[R];
 #pragma unroll

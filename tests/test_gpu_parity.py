@@ -162,6 +162,13 @@ def test_k_hi_spanning_two_row_slots():
     _run_teacher_forced(w, 2)
 
 
+@pytest.mark.parametrize("K,fmt", [(12, 0), (5, 0), (12, 1)])
+def test_general_kernel_at_d128(K, fmt):
+    """d_k = 128 layouts outside the compile-time list run the general kernel."""
+    w = wl.KDA_B256.replace(batch=2, heads=4, qk_heads=4, k_hi=K, lo_format=fmt)
+    _run_teacher_forced(w, 2)
+
+
 def test_slot_indirection_into_a_larger_pool():
     w = wl.KDA_B256.replace(batch=3, heads=4, qk_heads=4)
     _run_teacher_forced(w, 2, slot_of={0: 6, 1: 1, 2: 3}, pool=7)
