@@ -44,6 +44,7 @@ def lib() -> ctypes.CDLL:
             "dor_delta_step": (None, [i32, i32, P, P, P, P, P, f32, P]),
             "dor_delta_step_heads": (None, [i64, i32, i32, i32, P, P, P, P, P, P, P]),
             "dor_mixed_step_heads": (i32, [i64, i32, i32, i32, i32, i32, P, P, P, P, P, P, P, P, P, P]),
+            "dor_prefill_chunk_heads": (i32, [i64, i32, i32, i32, i32, i32, P, P, P, P, i32, P, P, P, P, P, P, P]),
             "dor_pack_heads": (i32, [i64, i32, i32, i32, i32, P, P, P, P, P]),
             "dor_unpack_heads": (i32, [i64, i32, i32, i32, i32, P, P, P, P, P]),
         }
@@ -193,6 +194,29 @@ def mixed_step_heads(perm, hi, codes, meta, q, k, v, g, beta, k_hi: int, fmt: in
                                     _p(q), _p(k), _p(v), _p(g), _p(beta), _p(o))
     if rc:
         raise ValueError("oracle mixed step: invalid permutation or sizes")
+    return o
+
+
+def prefill_chunk_heads(perm, hi, codes, meta, q, k, v, g, beta, k_hi: int, fmt: int, kind: str,
+                        lengths=None) -> np.ndarray:
+    """One prefill chunk per head on packed tiers (updated in place; App. A.5 prefill path).
+
+    q, k [n, T, d_k]; v [n, T, d_v]; g [n, T] (GDN) or [n, T, d_k] (KDA); beta [n, T];
+    lengths [n] (default T) = tokens of each head's chunk.  Returns o [n, T, d_v]
+    (rows past a head's length are zero)."""
+    for a in (hi, codes, meta):
+        assert a.flags["C_CONTIGUOUS"]
+    perm = np.ascontiguousarray(perm, dtype=np.uint8)
+    n, d_k = perm.shape
+    q, k, v, g, beta = _f32(q), _f32(k), _f32(v), _f32(g), _f32(beta)
+    T = q.shape[1]
+    d_v = v.shape[-1]
+    lens = np.full(n, T, np.int32) if lengths is None else np.ascontiguousarray(lengths, dtype=np.int32)
+    o = np.zeros((n, T, d_v), np.float32)
+    rc = lib().dor_prefill_chunk_heads(n, d_k, d_v, k_hi, fmt, KINDS[kind], _p(perm), _p(hi), _p(codes), _p(meta),
+                                       T, _p(lens), _p(q), _p(k), _p(v), _p(g), _p(beta), _p(o))
+    if rc:
+        raise ValueError("oracle prefill: invalid permutation, sizes or lengths")
     return o
 
 

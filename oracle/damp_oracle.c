@@ -362,6 +362,34 @@ int dor_mixed_step(int dk, int dv, int K, int fmt, int kind, const uint8_t *perm
 }
 
 /* ------------------------------------------------------------------------- */
+/* One prefill chunk of one head (App. A.5, "Prefill path"): reconstruct the */
+/* packed state, evaluate the exact FP32 recurrence over the chunk's T       */
+/* tokens (Eq. delta_update per token, o_t = S_t^T q_t), then quantize the   */
+/* chunk-final state once into the packed tiers.  T = 0 leaves the tiers     */
+/* untouched.  Token t reads q + t*dk, k + t*dk, v + t*dv, g + t*gdim and    */
+/* beta[t]; o receives T rows of d_v values.                                 */
+/* ------------------------------------------------------------------------- */
+
+int dor_prefill_chunk(int dk, int dv, int K, int fmt, int kind, const uint8_t *perm,
+                      uint16_t *hi, void *codes, void *meta, int T,
+                      const float *q, const float *k, const float *v, const float *g, const float *beta,
+                      float *o)
+{
+    static float S[256 * 4096];
+    float a[256];
+    int gdim = kind == DOR_GDN ? 1 : dk;
+    if (check_args(dk, dv, K, fmt, perm)) return -1;
+    if (T <= 0) return 0;
+    if (dor_unpack_head(dk, dv, K, fmt, perm, hi, codes, meta, S)) return -1;
+    for (int t = 0; t < T; t++) {
+        decay_from_log(kind, dk, g + (int64_t)t * gdim, a);
+        dor_delta_step(dk, dv, S, q + (int64_t)t * dk, k + (int64_t)t * dk, v + (int64_t)t * dv, a, beta[t],
+                       o + (int64_t)t * dv);
+    }
+    return dor_pack_head(dk, dv, K, fmt, perm, S, hi, codes, meta);
+}
+
+/* ------------------------------------------------------------------------- */
 /* Plain loops over n independent heads (each head: its own permutation,     */
 /* operands and state).  Arrays are dense, head-major.                       */
 /* ------------------------------------------------------------------------- */
@@ -378,6 +406,27 @@ int dor_mixed_step_heads(int64_t n, int dk, int dv, int K, int fmt, int kind, co
         int rc = dor_mixed_step(dk, dv, K, fmt, kind, perm + h * dk, hi + h * (int64_t)K * dv,
                                 (uint8_t *)codes + h * code_b, (uint8_t *)meta + h * meta_b,
                                 q + h * dk, k + h * dk, v + h * dv, g + h * gdim, beta[h], o + h * dv);
+        if (rc) return rc;
+    }
+    return 0;
+}
+
+/* n heads, each with its own chunk length T[h] <= Tmax: operands head-major
+ * [n][Tmax][...], o [n][Tmax][dv] (rows t >= T[h] untouched). */
+int dor_prefill_chunk_heads(int64_t n, int dk, int dv, int K, int fmt, int kind, const uint8_t *perm,
+                            uint16_t *hi, void *codes, void *meta, int Tmax, const int32_t *T,
+                            const float *q, const float *k, const float *v, const float *g,
+                            const float *beta, float *o)
+{
+    int64_t code_b = (int64_t)(dk - K) * dv * 1;
+    int64_t meta_b = (int64_t)(dk - K) * meta_row_bytes(dv, fmt);
+    int64_t gdim = kind == DOR_GDN ? 1 : dk;
+    for (int64_t h = 0; h < n; h++) {
+        if (T[h] < 0 || T[h] > Tmax) return -1;
+        int rc = dor_prefill_chunk(dk, dv, K, fmt, kind, perm + h * dk, hi + h * (int64_t)K * dv,
+                                   (uint8_t *)codes + h * code_b, (uint8_t *)meta + h * meta_b, T[h],
+                                   q + h * Tmax * dk, k + h * Tmax * dk, v + h * Tmax * dv,
+                                   g + h * Tmax * gdim, beta + h * Tmax, o + h * Tmax * dv);
         if (rc) return rc;
     }
     return 0;
