@@ -207,6 +207,40 @@ DAMP_API damp_status damp_fp32_kda_decode_step(const damp_layout *layout, float 
                                       const float *beta, float *o, int32_t in_dtype, void *stream);
 
 /*
+ * One GDN prefill chunk on the packed state (App. A.5, "Prefill path"): for each
+ * batch row, the packed slot is reconstructed, the recurrence runs in FP32 over the
+ * chunk's tokens (Sec. 3.1 Eq. delta_update per token, o_t = S_t^T q_t) and the
+ * chunk-final state is quantized once, in place, into the same packed cache that
+ * decode steps and later chunks read.  An all-zero slot is the zero state (start of
+ * a sequence).
+ *   chunk_len  T >= 0 tokens per row (0 enqueues nothing)
+ *   lengths    int32 [batch]: row b runs its first min(max(lengths[b], 0), T) tokens;
+ *              NULL means T for every row.  A row with length 0 keeps its state.
+ *              4-B aligned.
+ *   q, k       [B][T][H_qk][d_k] of in_dtype, natural key order, 16-B aligned
+ *   v          [B][T][H][d_v] of in_dtype, 16-B aligned
+ *   g          float [B][T][H]: log-decay per token, 4-B aligned
+ *   beta       float [B][T][H], 4-B aligned
+ *   o          float [B][T][H][d_v]: o_t from the FP32 state after token t; rows past
+ *              a row's length are not written.  Must not overlap the pool or inputs.
+ * Other arguments as in damp_gdn_decode_step.  lo_format must be 0 or 1
+ * (DAMP_ERR_FORMAT for the row-absmax format).
+ */
+DAMP_API damp_status damp_gdn_prefill_chunk(const damp_layout *layout, void *state, int64_t num_slots,
+                                            const int32_t *slot_idx, int32_t batch, int32_t chunk_len,
+                                            const int32_t *lengths, const uint8_t *perm, const void *q,
+                                            const void *k, const void *v, const float *g, const float *beta,
+                                            float *o, int32_t in_dtype, void *stream);
+
+/* One KDA prefill chunk, as damp_gdn_prefill_chunk except
+ *   g          float [B][T][H][d_k]: per-key-channel log-decay per token, 16-B aligned. */
+DAMP_API damp_status damp_kda_prefill_chunk(const damp_layout *layout, void *state, int64_t num_slots,
+                                            const int32_t *slot_idx, int32_t batch, int32_t chunk_len,
+                                            const int32_t *lengths, const uint8_t *perm, const void *q,
+                                            const void *k, const void *v, const float *g, const float *beta,
+                                            float *o, int32_t in_dtype, void *stream);
+
+/*
  * Write FP32 states into the packed cache: the hand-off from an FP32 prefix
  * state (App. A.5 "Prefill path": the chunk-final state is written directly into
  * the packed cache).  Row i of packed head h takes natural row perm[h][i];

@@ -21,7 +21,7 @@ from ._lib import DampLayout, DampLibraryError, lib
 __all__ = [
     "Layout", "DampError", "DampLibraryError", "LO_U8_AFFINE_G32_H32", "LO_U8_AFFINE_G32", "LO_S8_ABSMAX_ROW",
     "record_bytes", "slot_bytes", "bits_per_value", "new_state", "new_fp32_state",
-    "gdn_decode_step", "kda_decode_step", "u8_gdn_decode_step", "u8_kda_decode_step",
+    "gdn_decode_step", "kda_decode_step", "gdn_prefill_chunk", "kda_prefill_chunk", "u8_gdn_decode_step", "u8_kda_decode_step",
     "fp32_gdn_decode_step", "fp32_kda_decode_step", "quantize_state", "dequantize_state",
     "pack_tiers", "unpack_tiers", "device_status", "version", "DEV_WAIT_TIMEOUT", "DEV_BAD_SLOT",
 ]
@@ -164,6 +164,38 @@ def fp32_gdn_decode_step(layout, state, q, k, v, g, beta, o=None, slot_idx=None,
 
 def fp32_kda_decode_step(layout, state, q, k, v, g, beta, o=None, slot_idx=None, num_slots=None, stream=None):
     return _step("damp_fp32_kda_decode_step", layout, state, None, q, k, v, g, beta, o, slot_idx, num_slots, stream)
+
+
+def _prefill(fn_name, layout, state, perm, q, k, v, g, beta, o, lengths, slot_idx, num_slots, stream):
+    import torch
+    for n, t in (("state", state), ("perm", perm), ("q", q), ("k", k), ("v", v), ("g", g), ("beta", beta),
+                 ("o", o), ("lengths", lengths), ("slot_idx", slot_idx)):
+        _cuda_contig(n, t)
+    B, T = v.shape[0], v.shape[1]
+    if o is None:
+        o = torch.zeros((B, T, layout.num_heads, layout.d_v), dtype=torch.float32, device=v.device)
+    if num_slots is None:
+        num_slots = state.shape[0]
+    c = layout.c()
+    _check(getattr(lib(), fn_name)(ctypes.byref(c), _ptr(state), num_slots, _ptr(slot_idx), B, T, _ptr(lengths),
+                                   _ptr(perm), _ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(beta), _ptr(o),
+                                   _in_dtype(q, k, v), _stream(stream)), fn_name)
+    return o
+
+
+def gdn_prefill_chunk(layout, state, perm, q, k, v, g, beta, o=None, lengths=None, slot_idx=None, num_slots=None,
+                      stream=None):
+    """One GDN prefill chunk on the packed state (in place): q, k [B, T, H_qk, d_k], v [B, T, H, d_v],
+    g, beta [B, T, H]; returns o [B, T, H, d_v] float32."""
+    return _prefill("damp_gdn_prefill_chunk", layout, state, perm, q, k, v, g, beta, o, lengths, slot_idx,
+                    num_slots, stream)
+
+
+def kda_prefill_chunk(layout, state, perm, q, k, v, g, beta, o=None, lengths=None, slot_idx=None, num_slots=None,
+                      stream=None):
+    """One KDA prefill chunk on the packed state (in place): as gdn_prefill_chunk with g [B, T, H, d_k]."""
+    return _prefill("damp_kda_prefill_chunk", layout, state, perm, q, k, v, g, beta, o, lengths, slot_idx,
+                    num_slots, stream)
 
 
 def quantize_state(layout, S, perm, state, slot_idx=None, num_slots=None, stream=None):

@@ -40,6 +40,8 @@ SIGNATURES = {
     "damp_u8_kda_decode_step": (_status, _STEP),
     "damp_fp32_gdn_decode_step": (_status, _FP32_STEP),
     "damp_fp32_kda_decode_step": (_status, _FP32_STEP),
+    "damp_gdn_prefill_chunk": (_status, [_L, _P, _i64, _P, _i32, _i32, _P, _P, _P, _P, _P, _P, _P, _P, _i32, _P]),
+    "damp_kda_prefill_chunk": (_status, [_L, _P, _i64, _P, _i32, _i32, _P, _P, _P, _P, _P, _P, _P, _P, _i32, _P]),
     "damp_quantize_state": (_status, [_L, _P, _P, _P, _i64, _P, _i32, _P]),
     "damp_dequantize_state": (_status, [_L, _P, _i64, _P, _i32, _P, _P, _P]),
     "damp_pack_tiers": (_status, [_L, _P, _P, _P, _P, _i64, _P, _i32, _P]),

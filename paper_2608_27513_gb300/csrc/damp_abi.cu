@@ -131,6 +131,59 @@ damp_status step(const damp_layout *L, void *state, int64_t num_slots, const int
     return launch_step(a, packed, static_cast<cudaStream_t>(stream)) == cudaSuccess ? DAMP_OK : DAMP_ERR_CUDA;
 }
 
+damp_status prefill(const damp_layout *L, void *state, int64_t num_slots, const int32_t *slot_idx, int32_t batch,
+                    int32_t chunk_len, const int32_t *lengths, const uint8_t *perm, const void *q, const void *k,
+                    const void *v, const float *g, const float *beta, float *o, int32_t in_dtype, void *stream,
+                    bool kda) {
+    damp_status st = check_layout(L);
+    if (st != DAMP_OK) return st;
+    if (L->lo_format == DAMP_LO_S8_ABSMAX_ROW) return DAMP_ERR_FORMAT;
+    if (in_dtype != DAMP_IN_BF16 && in_dtype != DAMP_IN_FP32) return DAMP_ERR_FORMAT;
+    if (batch < 0 || chunk_len < 0) return DAMP_ERR_SHAPE;
+    if (batch == 0 || chunk_len == 0) return DAMP_OK;
+    Range pool;
+    if ((st = check_pool(state, num_slots, slot_idx, batch, slot_bytes_of(L), &pool)) != DAMP_OK) return st;
+    if (!perm || !q || !k || !v || !g || !beta || !o) return DAMP_ERR_NULL;
+    if (!aligned(perm, 16) || !aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(g, kda ? 16 : 4) ||
+        !aligned(beta, 4) || !aligned(o, 4) || (lengths && !aligned(lengths, 4)))
+        return DAMP_ERR_ALIGN;
+    const int64_t B = batch, T = chunk_len, H = L->num_heads, Hq = L->num_qk_heads, dk = L->d_k, dv = L->d_v;
+    const int64_t esz = in_dtype == DAMP_IN_BF16 ? 2 : 4;
+    const Range ro = range_of(o, B * T * H * dv * 4);
+    const Range inputs[] = {range_of(q, B * T * Hq * dk * esz), range_of(k, B * T * Hq * dk * esz),
+                            range_of(v, B * T * H * dv * esz), range_of(g, B * T * H * (kda ? dk : 1) * 4),
+                            range_of(beta, B * T * H * 4), range_of(perm, H * dk),
+                            range_of(slot_idx, slot_idx ? B * 4 : 0), range_of(lengths, lengths ? B * 4 : 0)};
+    if (overlap(ro, pool)) return DAMP_ERR_ALIAS;
+    for (const Range &r : inputs)
+        if (overlap(ro, r) || overlap(pool, r)) return DAMP_ERR_ALIAS;
+
+    StepArgs a{};
+    a.H = L->num_heads;
+    a.Hqk = L->num_qk_heads;
+    a.dk = L->d_k;
+    a.dv = L->d_v;
+    a.K = L->k_hi;
+    a.fmt = L->lo_format;
+    a.state = state;
+    a.num_slots = num_slots;
+    a.slot_idx = slot_idx;
+    a.batch = batch;
+    a.perm = perm;
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.g = g;
+    a.beta = beta;
+    a.o = o;
+    a.in_bf16 = in_dtype == DAMP_IN_BF16;
+    a.kda = kda;
+    a.T = chunk_len;
+    a.lengths = lengths;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    return (kda ? launch_prefill_kda(a, s) : launch_prefill_gdn(a, s)) == cudaSuccess ? DAMP_OK : DAMP_ERR_CUDA;
+}
+
 enum ConvKind { kQ, kDQ, kPack, kUnpack };
 
 damp_status convert(const damp_layout *L, void *state, int64_t num_slots, const int32_t *slot_idx, int32_t batch,
@@ -320,6 +373,22 @@ damp_status damp_fp32_kda_decode_step(const damp_layout *layout, float *state, i
                 false, false);
 }
 
+damp_status damp_gdn_prefill_chunk(const damp_layout *layout, void *state, int64_t num_slots, const int32_t *slot_idx,
+                                   int32_t batch, int32_t chunk_len, const int32_t *lengths, const uint8_t *perm,
+                                   const void *q, const void *k, const void *v, const float *g, const float *beta,
+                                   float *o, int32_t in_dtype, void *stream) {
+    return prefill(layout, state, num_slots, slot_idx, batch, chunk_len, lengths, perm, q, k, v, g, beta, o, in_dtype,
+                   stream, false);
+}
+
+damp_status damp_kda_prefill_chunk(const damp_layout *layout, void *state, int64_t num_slots, const int32_t *slot_idx,
+                                   int32_t batch, int32_t chunk_len, const int32_t *lengths, const uint8_t *perm,
+                                   const void *q, const void *k, const void *v, const float *g, const float *beta,
+                                   float *o, int32_t in_dtype, void *stream) {
+    return prefill(layout, state, num_slots, slot_idx, batch, chunk_len, lengths, perm, q, k, v, g, beta, o, in_dtype,
+                   stream, true);
+}
+
 damp_status damp_quantize_state(const damp_layout *layout, const float *S, const uint8_t *perm, void *state,
                                 int64_t num_slots, const int32_t *slot_idx, int32_t batch, void *stream) {
     return convert(layout, state, num_slots, slot_idx, batch, perm, const_cast<float *>(S), nullptr, nullptr,
@@ -358,6 +427,10 @@ damp_status damp_device_status(uint32_t *status) {
     if (take_status_convert(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     if (take_status_rowabs(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_prefill_gdn(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_prefill_kda(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     *status = all;
     return DAMP_OK;

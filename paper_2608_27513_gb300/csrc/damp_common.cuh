@@ -129,6 +129,9 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void *src) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
 }
+__device__ __forceinline__ void cp_async4(uint32_t dst, const void *src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");
+}
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
@@ -387,6 +390,44 @@ __device__ __forceinline__ uint32_t f2_to_h2(float a, float b) {
     uint32_t w;
     memcpy(&w, &h, 4);
     return w;
+}
+
+// Per-warp partial-sum buffer of column_sum2: 32 lane rows of 32 (r, p) pairs + padding.
+constexpr int kPartStride = 68;  // floats per lane row
+
+__device__ __forceinline__ float ldsf(uint32_t a) { return __uint_as_float(lds32(a)); }
+
+// Column sums of two per-lane 32-vectors at once: lane j returns
+// (sum_l a_l[j], sum_l b_l[j]) over the 32 lanes l.
+__device__ __forceinline__ float2 column_sum2(const float2 (&a)[16], const float2 (&b)[16], uint32_t part, int lane) {
+#pragma unroll
+    for (int m = 0; m < 16; ++m) {  // row of lane l: (a_j, b_j) pairs in column order
+        sts128(part + (lane * kPartStride + 4 * m) * 4,
+               make_uint4(__float_as_uint(a[m].x), __float_as_uint(b[m].x), __float_as_uint(a[m].y),
+                          __float_as_uint(b[m].y)));
+    }
+    __syncwarp();
+    float2 s0 = make_float2(0.f, 0.f), s1 = s0, s2 = s0, s3 = s0;
+#pragma unroll
+    for (int l = 0; l < 32; l += 4) {
+        const uint32_t base = part + (2 * lane) * 4;
+        uint2 v0, v1, v2, v3;
+        asm volatile("ld.shared.v2.b32 {%0,%1}, [%2];" : "=r"(v0.x), "=r"(v0.y) : "r"(base + (l + 0) * kPartStride * 4));
+        asm volatile("ld.shared.v2.b32 {%0,%1}, [%2];" : "=r"(v1.x), "=r"(v1.y) : "r"(base + (l + 1) * kPartStride * 4));
+        asm volatile("ld.shared.v2.b32 {%0,%1}, [%2];" : "=r"(v2.x), "=r"(v2.y) : "r"(base + (l + 2) * kPartStride * 4));
+        asm volatile("ld.shared.v2.b32 {%0,%1}, [%2];" : "=r"(v3.x), "=r"(v3.y) : "r"(base + (l + 3) * kPartStride * 4));
+        s0 = add2(s0, make_float2(__uint_as_float(v0.x), __uint_as_float(v0.y)));
+        s1 = add2(s1, make_float2(__uint_as_float(v1.x), __uint_as_float(v1.y)));
+        s2 = add2(s2, make_float2(__uint_as_float(v2.x), __uint_as_float(v2.y)));
+        s3 = add2(s3, make_float2(__uint_as_float(v3.x), __uint_as_float(v3.y)));
+    }
+    __syncwarp();
+    return add2(add2(s0, s1), add2(s2, s3));
+}
+
+__device__ __forceinline__ float bf16_at(uint32_t base, int i) {
+    const uint32_t w = lds32(base + 2 * (i & ~1));
+    return __uint_as_float((i & 1) ? (w & 0xffff0000u) : (w << 16));
 }
 
 __device__ __forceinline__ float load_in(const void *p, int64_t i, bool bf16) {

@@ -21,6 +21,10 @@ struct StepArgs {
     float *o;
     int32_t in_bf16;  // 1: q/k/v are bf16, 0: fp32
     int32_t kda;      // 1: per-channel decay g[B][H][d_k], 0: scalar g[B][H]
+    // prefill chunks only: tokens per chunk (operands gain a [T] axis after the batch
+    // axis) and optional per-row lengths
+    int32_t T;
+    const int32_t *lengths;
 };
 
 struct ConvArgs {
@@ -44,6 +48,9 @@ cudaError_t launch_quantize(const ConvArgs &a, cudaStream_t s);
 cudaError_t launch_dequantize(const ConvArgs &a, cudaStream_t s);
 cudaError_t launch_pack_tiers(const ConvArgs &a, cudaStream_t s);
 cudaError_t launch_unpack_tiers(const ConvArgs &a, cudaStream_t s);
+// One prefill chunk on the packed state (formats 0 and 1).
+cudaError_t launch_prefill_gdn(const StepArgs &a, cudaStream_t s);
+cudaError_t launch_prefill_kda(const StepArgs &a, cudaStream_t s);
 // Row-absmax INT8 low tier (lo_format 2); op: 0 quantize, 1 dequantize, 2 pack, 3 unpack.
 cudaError_t launch_rowabs_step(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_rowabs_convert(const ConvArgs &a, int op, cudaStream_t s);
@@ -54,6 +61,8 @@ cudaError_t take_status_packed_kda(uint32_t *bits);
 cudaError_t take_status_fp32(uint32_t *bits);
 cudaError_t take_status_convert(uint32_t *bits);
 cudaError_t take_status_rowabs(uint32_t *bits);
+cudaError_t take_status_prefill_gdn(uint32_t *bits);
+cudaError_t take_status_prefill_kda(uint32_t *bits);
 
 // Streaming multiprocessors / opt-in shared memory per block of the current device (cached per device).
 int sm_count();

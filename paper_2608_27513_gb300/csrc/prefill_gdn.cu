@@ -1,0 +1,24 @@
+// prefill_gdn.cu -- instantiations of the prefill chunk kernel for
+// GDN (scalar decay per head).
+#include "launch_prefill.cuh"
+
+namespace damp {
+
+static __device__ uint32_t g_status_prefill_gdn;
+
+cudaError_t launch_prefill_gdn(const StepArgs &a, cudaStream_t s) {
+    static uint32_t *cache[64];
+    uint32_t *status = nullptr;
+    cudaError_t e = symbol_address_cached(&g_status_prefill_gdn, cache, &status);
+    if (e != cudaSuccess) return e;
+    return launch_prefill_impl<false>(a, s, status);
+}
+
+cudaError_t take_status_prefill_gdn(uint32_t *bits) {
+    uint32_t zero = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(bits, g_status_prefill_gdn, sizeof(uint32_t));
+    if (e != cudaSuccess) return e;
+    return cudaMemcpyToSymbol(g_status_prefill_gdn, &zero, sizeof(uint32_t));
+}
+
+}  // namespace damp

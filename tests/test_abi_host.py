@@ -123,6 +123,30 @@ def test_step_rejects_bad_arguments_before_launch(L):
                                                         fb[6], fb[7], 0, None]) == 2
 
 
+def _call_prefill(L, lay, fb, **over):
+    c = lay.c()
+    args = dict(layout=ctypes.byref(c), state=fb[0], num_slots=4, slot_idx=None, batch=4, chunk_len=8, lengths=None,
+                perm=fb[1], q=fb[2], k=fb[3], v=fb[4], g=fb[5], beta=fb[6], o=fb[7], in_dtype=0, stream=None)
+    args.update(over)
+    return L.damp_kda_prefill_chunk(*args.values())
+
+
+def test_prefill_rejects_bad_arguments_before_launch(L):
+    fb = FakeBuffers()
+    lay = _layout()
+    off = lambda i, d: ctypes.c_void_p(fb.ptrs[i] + d)
+    assert _call_prefill(L, lay, fb, batch=0) == 0                   # nothing enqueued
+    assert _call_prefill(L, lay, fb, chunk_len=0) == 0
+    assert _call_prefill(L, lay, fb, chunk_len=-1) == 2
+    assert _call_prefill(L, lay, fb, v=None) == 1
+    assert _call_prefill(L, lay, fb, lengths=off(8, 2)) == 3
+    assert _call_prefill(L, lay, fb, q=off(2, 8)) == 3
+    assert _call_prefill(L, lay, fb, o=off(0, 64)) == 4               # o inside the pool
+    assert _call_prefill(L, lay, fb, lengths=off(7, 0)) == 4          # lengths under o
+    assert _call_prefill(L, _layout(lo_format=2), fb) == 5            # row-absmax: no prefill kernel
+    assert _call_prefill(L, lay, fb, in_dtype=3) == 5
+
+
 def test_gdn_gate_alignment_is_4_bytes(L):
     fb = FakeBuffers()
     c = _layout().c()

@@ -1,0 +1,136 @@
+"""GPU parity of the prefill chunk (App. A.5 "Prefill path") through the C ABI against
+the oracle: outputs of every token within the decode tolerance, the chunk-final
+packed state within the tie rules of the decode step."""
+import numpy as np
+import pytest
+import torch
+
+import paper_2608_27513_gb300 as damp
+import workloads as wl
+from oracle import core, runs
+from tests import parity as P
+
+pytestmark = pytest.mark.gpu
+DEV = torch.device("cuda:0")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2608_27513_gb300 import build
+    build.build()
+    torch.cuda.init()
+    assert damp.device_status() == 0
+    yield
+    assert damp.device_status() == 0
+
+
+def _chunk_inputs(w, t0, T, rows):
+    """Per-token draws of the decode stream, stacked on a token axis after the batch axis."""
+    steps = [wl.step_inputs(w, t0 + t, rows=rows) for t in range(T)]
+    return {key: np.stack([s[key] for s in steps], axis=1) for key in steps[0]}
+
+
+def _unit_chunk(w, inp, T):
+    """Per-(slot, head) operands [n, T, ...] (GQA expanded) for the oracle."""
+    per_t = [runs.unit_operands(w, {key: val[:, t] for key, val in inp.items()}) for t in range(T)]
+    return {key: np.stack([u[key] for u in per_t], axis=1) for key in per_t[0]}
+
+
+def _oracle_chunk(w, perm_units, tiers, u, lens_units):
+    """The oracle's chunk, plus its chunk-final FP32 state for the tie rules."""
+    n = perm_units.shape[0]
+    S = core.unpack_heads(perm_units, *tiers, w.k_hi, w.lo_format, w.d_k, w.d_v)
+    for t in range(u["q"].shape[1]):
+        live = lens_units > t
+        if live.any():
+            sub = np.ascontiguousarray(S[live])
+            core.delta_step_heads(sub, u["q"][live, t], u["k"][live, t], u["v"][live, t], u["g"][live, t],
+                                  u["beta"][live, t], w.kind)
+            S[live] = sub
+    new = tuple(np.ascontiguousarray(t).copy() for t in tiers)
+    o = core.prefill_chunk_heads(perm_units, *new, u["q"], u["k"], u["v"], u["g"], u["beta"], w.k_hi, w.lo_format,
+                                 w.kind, lengths=lens_units)
+    assert np.array_equal(core.unpack_heads(perm_units, *new, w.k_hi, w.lo_format, w.d_k, w.d_v)[lens_units > 0],
+                          core.unpack_heads(perm_units, *core.pack_heads(perm_units, S, w.k_hi, w.lo_format),
+                                            w.k_hi, w.lo_format, w.d_k, w.d_v)[lens_units > 0])
+    lo_rows = np.stack([S[i][perm_units[i][w.k_hi:]] for i in range(n)])
+    if w.lo_format == core.FMT_U8_H32 and lo_rows.size:
+        lo_rows = core.hadamard32(lo_rows.reshape(-1, 32)).reshape(lo_rows.shape)
+    return o, new, lo_rows
+
+
+def _run(w, T, lengths=None, slot_of=None, pool=None, chunks=1):
+    rows = list(range(w.batch))
+    perms, _ = runs.calibrate_layout(w, n_docs=2, n_tokens=16)
+    perm_units, tiers = P.initial_tiers(w, rows, perms, prefix=min(w.prefix, 24))
+    L = P.layout_of(w)
+    state = damp.new_state(L, pool or len(rows), DEV)
+    slot_idx = None if slot_of is None else torch.tensor([slot_of[b] for b in rows], dtype=torch.int32, device=DEV)
+    lens = np.full(len(rows), T, np.int32) if lengths is None else np.asarray(lengths, np.int32)
+    lens_units = np.repeat(lens, w.heads)
+    dperm = P.to_dev(perms, DEV)
+    stats = P.CodeStats()
+    fn = damp.kda_prefill_chunk if w.kind == "kda" else damp.gdn_prefill_chunk
+    dt = torch.bfloat16 if w.in_dtype == "bf16" else torch.float32
+    for ch in range(chunks):
+        # teacher-forced: every chunk starts from the oracle's packed state
+        damp.pack_tiers(L, *P.tiers_to_dev(w, tiers, len(rows), DEV), state, slot_idx=slot_idx)
+        inp = _chunk_inputs(w, ch * T, T, rows)
+        u = _unit_chunk(w, inp, T)
+        o_ref, tiers, lo_pre = _oracle_chunk(w, perm_units, tiers, u, lens_units)
+        d = {key: P.to_dev(val, DEV, dt if key in ("q", "k", "v") else None) for key, val in inp.items()}
+        o = fn(L, state, dperm, d["q"], d["k"], d["v"], d["g"], d["beta"],
+               lengths=None if lengths is None else P.to_dev(lens, DEV), slot_idx=slot_idx)
+        torch.cuda.synchronize()
+        o = o.cpu().numpy().transpose(0, 2, 1, 3).reshape(len(rows) * w.heads, T, w.d_v)
+        for i in range(o.shape[0]):
+            P.compare_o(o[i, :lens_units[i]], o_ref[i, :lens_units[i]], f"{w.name} chunk {ch} unit {i}")
+        got = P.tiers_from_dev(w, damp.unpack_tiers(L, state, batch=len(rows), slot_idx=slot_idx),
+                               len(rows) * w.heads)
+        P.compare_tiers(w, tiers, got, lo_pre, stats, f"{w.name} chunk {ch}")
+    stats.check_fraction()
+    return state, L, dperm, slot_idx
+
+
+def test_kda_chunk_matches_oracle():
+    """KDA, H = 8, d = 128, K_hi = 10, BF16 inputs, 16-token chunks, two chunks in a row."""
+    _run(wl.KDA_B256.replace(batch=2, heads=8, qk_heads=8), 16, chunks=2)
+
+
+def test_gdn_gqa_chunk_matches_oracle():
+    _run(wl.GDN_B64_GQA.replace(batch=2), 8)
+
+
+def test_ragged_lengths_and_slot_indirection():
+    """Rows of 9, 3 and 0 tokens in a 9-token chunk, scattered over a larger pool; the
+    zero-length row's slot stays as it was."""
+    w = wl.KDA_B256.replace(batch=3, heads=4, qk_heads=4)
+    _run(w, 9, lengths=[9, 3, 0], slot_of={0: 5, 1: 0, 2: 2}, pool=6)
+
+
+@pytest.mark.parametrize("w", [
+    wl.Workload("gdn_d64_dv96_k5_f1", "gdn", 2, 4, 2, 64, 96, 5, 4, 8, "fp32", 21, 1),
+    wl.Workload("kda_uniform", "kda", 1, 4, 4, 128, 64, 0, 4, 8, "bf16", 22, 0),
+    wl.Workload("kda_all_fp16", "kda", 1, 2, 2, 32, 64, 32, 4, 8, "fp32", 23, 0),
+    wl.Workload("gdn_d32_k3", "gdn", 2, 2, 1, 32, 32, 3, 4, 8, "bf16", 24, 0),
+], ids=lambda w: w.name)
+def test_layouts(w):
+    _run(w, 6)
+
+
+def test_decode_after_prefill_reads_the_chunk_state():
+    """The decode step continues from the chunk-final packed state that the GPU chunk
+    wrote (the hand-off of the prefill path), matching the oracle's step from it."""
+    w = wl.KDA_B256.replace(batch=2, heads=4, qk_heads=4)
+    state, L, dperm, _ = _run(w, 5)
+    got_tiers = P.tiers_from_dev(w, damp.unpack_tiers(L, state), w.batch * w.heads)
+    inp = wl.step_inputs(w, 5, rows=list(range(w.batch)))
+    perms = dperm.cpu().numpy()
+    o_ref, new_ref, lo_pre = P.oracle_step(w, np.tile(perms, (w.batch, 1)), got_tiers, runs.unit_operands(w, inp))
+    d = P.inputs_to_dev(w, inp, DEV)
+    o = damp.kda_decode_step(L, state, dperm, d["q"], d["k"], d["v"], d["g"], d["beta"])
+    P.compare_o(o.cpu().numpy().reshape(-1, w.d_v), o_ref, "decode after prefill")
+    stats = P.CodeStats()
+    P.compare_tiers(w, new_ref, P.tiers_from_dev(w, damp.unpack_tiers(L, state), w.batch * w.heads), lo_pre, stats,
+                    "decode after prefill")
+    stats.check_fraction()
