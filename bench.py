@@ -481,6 +481,70 @@ def sweep_arm(steps: int, warmup: int):
         print(json.dumps(row), flush=True)
 
 
+def prefill_arm(steps: int, warmup: int, T: int = 64):
+    """Prefill chunks (App. A.5 prefill path) at B = 256, H = 32, d = 128: one launch per
+    chunk of T tokens per slot.  The chunk keeps each tile's FP32 state on chip, so it
+    is bound by FP32 FMA throughput, not HBM: achieved = algorithmic FLOPs / time against
+    the FP32 FMA peak (SMs x 4 sub-partitions x 32 lanes x 2 flops x SM clock)."""
+    import torch
+
+    import paper_2608_27513_gb300 as damp
+    from paper_2608_27513_gb300 import build
+    build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    out = []
+    for w in (wl.KDA_B256, wl.sweep("gdn", 16)):
+        L = damp.Layout(w.heads, w.qk_heads, w.d_k, w.d_v, w.k_hi, w.lo_format)
+        per_t = wl.torch_step_inputs(w, T, dev)
+        chunk = {key: torch.stack([d[key] for d in per_t], dim=1).contiguous() for key in per_t[0]}
+        del per_t
+        perm = torch.from_numpy(wl.random_perm(w)).to(dev)
+        S = 0.3 * torch.randn((w.batch, w.heads, w.d_k, w.d_v), device=dev)
+        pools = [damp.new_state(L, w.batch, dev) for _ in range(2)]
+        for pl in pools:
+            damp.quantize_state(L, S, perm, pl)
+        del S
+        o = torch.empty((w.batch, T, w.heads, w.d_v), device=dev)
+        fn = damp.kda_prefill_chunk if w.kind == "kda" else damp.gdn_prefill_chunk
+
+        def run(i):
+            fn(L, pools[i % 2], perm, chunk["q"], chunk["k"], chunk["v"], chunk["g"], chunk["beta"], o=o)
+
+        for i in range(warmup):
+            run(i)
+        torch.cuda.synchronize()
+        n = max(steps // 100, 5)
+        with ClockSampler(dev.index) as clk:
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for i in range(n):
+                run(i)
+            e1.record()
+            torch.cuda.synchronize()
+        us = e0.elapsed_time(e1) / n * 1e3
+        flops = 7.0 * w.d_k * w.d_v * w.batch * w.heads * T  # decay 1, r 2, p 2, update 2 per state element
+        clocks = clk.summary()
+        mhz = (clocks or {}).get("sm_mhz") or 2070.0
+        peak = sms * 4 * 32 * 2 * mhz * 1e6
+        esz = 2 if w.in_dtype == "bf16" else 4
+        hbm = (2 * w.batch * w.heads * damp.slot_bytes(L) // w.heads
+               + w.batch * T * (2 * w.qk_heads * w.d_k * esz + w.heads * w.d_v * (esz + 4)
+                                + w.heads * 4 * ((w.d_k if w.kind == "kda" else 1) + 1)))
+        out.append({"mode": "prefill_chunk", "kind": w.kind, "workload": w.name, "chunk_tokens": T,
+                    "us_per_chunk": us, "tokens_per_s": w.batch * T / (us * 1e-6),
+                    "roofline": {"bound": "fma", "achieved": flops / (us * 1e-6) / 1e12, "peak": peak / 1e12,
+                                 "unit": "TFLOP/s", "frac": flops / (us * 1e-6) / peak,
+                                 "peak_source": f"FP32 FMA: {sms} SMs x 128 lanes x 2 flops x {mhz:.0f} MHz"},
+                    "hbm_gbs": hbm / (us * 1e-6) / 1e9, "clocks": clocks})
+        del pools, chunk, o
+    if damp.device_status() != 0:
+        raise RuntimeError("device status word set during the prefill runs")
+    for row in out:
+        print(json.dumps(row), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -489,6 +553,7 @@ def main():
     ap.add_argument("--impl", default="damp", choices=["damp", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true", help="K_hi sweep (GDN and KDA, B=256) instead of the bench line")
+    ap.add_argument("--prefill", action="store_true", help="prefill chunks (64 tokens, B=256) instead of the bench line")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -500,6 +565,9 @@ def main():
         return
     if args.sweep:
         sweep_arm(args.steps, args.warmup)
+        return
+    if args.prefill:
+        prefill_arm(args.steps, args.warmup)
         return
     import torch
     import torch.distributed as dist
