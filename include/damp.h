@@ -276,6 +276,38 @@ DAMP_API damp_status damp_unpack_tiers(const damp_layout *layout, const void *st
                               const int32_t *slot_idx, int32_t batch, uint16_t *hi, uint8_t *codes,
                               uint16_t *meta, void *stream);
 
+/*
+ * Offline key-channel selection (Sec. 5.1 Eq. error_energy, persistence,
+ * budgeted_selection; App. A.2 Eq. empirical_error_energy, empirical_persistence;
+ * Algorithm 1), run on the GPU over calibration trajectories the caller produces
+ * (for example with damp_fp32_*_decode_step on calibration documents).
+ *
+ * damp_calib_error_energy: E_acc[h][u] += sum_b || Q_lo(S_b,h)_{u:} - S_b,h,u: ||^2,
+ *   the squared round-trip error of every key-channel row of the sampled FP32 states
+ *   under layout->lo_format (H_32 + UINT8 G32, UINT8 G32, or row absmax INT8).
+ *   S      float [batch][H][d_k][d_v] natural key order, 16-B aligned, read only
+ *   E_acc  float [H][d_k], 4-B aligned, accumulated (the caller zeroes it first)
+ * damp_calib_log_decay: G_acc[h][u] += sum_b g_b,h,u (KDA, g float [batch][H][d_k]) or
+ *   sum_b g_b,h (GDN, g float [batch][H]: the head's log-decay counts for every channel).
+ *   G_acc  float [H][d_k], 4-B aligned, accumulated
+ * damp_calib_select: E = E_acc / n_samples, a_eff = exp(G_acc / n_tokens),
+ *   P = 1 / max(1 - a_eff^2, tau), C = E P (FP32), H = TopK_{K_hi}(C) with ties to the
+ *   lower channel index, pi = the protected channels in ascending order, then the rest
+ *   in ascending order.
+ *   C_out     float [H][d_k] the scores (4-B aligned)
+ *   perm_out  uint8 [H][d_k] pi per head, ready for the decode and prefill calls
+ *   tau       the persistence cap, 0 < tau <= 1 (the paper uses 1e-4)
+ * Each accumulator entry has one writer and a fixed summation order: repeated runs
+ * give identical bits.  No call allocates or uses global scratch memory.
+ */
+DAMP_API damp_status damp_calib_error_energy(const damp_layout *layout, const float *S, int32_t batch, float *E_acc,
+                                             void *stream);
+DAMP_API damp_status damp_calib_log_decay(const damp_layout *layout, const float *g, int32_t batch, int32_t kda,
+                                          float *G_acc, void *stream);
+DAMP_API damp_status damp_calib_select(const damp_layout *layout, const float *E_acc, int64_t n_samples,
+                                       const float *G_acc, int64_t n_tokens, float tau, float *C_out,
+                                       uint8_t *perm_out, void *stream);
+
 /* Reads and clears the device status word of the current device (DAMP_DEV_* bits).
  * Synchronous with respect to the device.  DAMP_ERR_NULL if status is NULL. */
 DAMP_API damp_status damp_device_status(uint32_t *status);

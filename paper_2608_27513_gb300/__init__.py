@@ -21,7 +21,7 @@ from ._lib import DampLayout, DampLibraryError, lib
 __all__ = [
     "Layout", "DampError", "DampLibraryError", "LO_U8_AFFINE_G32_H32", "LO_U8_AFFINE_G32", "LO_S8_ABSMAX_ROW",
     "record_bytes", "slot_bytes", "bits_per_value", "new_state", "new_fp32_state",
-    "gdn_decode_step", "kda_decode_step", "gdn_prefill_chunk", "kda_prefill_chunk", "u8_gdn_decode_step", "u8_kda_decode_step",
+    "gdn_decode_step", "kda_decode_step", "gdn_prefill_chunk", "kda_prefill_chunk", "calib_error_energy", "calib_log_decay", "calib_select", "u8_gdn_decode_step", "u8_kda_decode_step",
     "fp32_gdn_decode_step", "fp32_kda_decode_step", "quantize_state", "dequantize_state",
     "pack_tiers", "unpack_tiers", "device_status", "version", "DEV_WAIT_TIMEOUT", "DEV_BAD_SLOT",
 ]
@@ -196,6 +196,36 @@ def kda_prefill_chunk(layout, state, perm, q, k, v, g, beta, o=None, lengths=Non
     """One KDA prefill chunk on the packed state (in place): as gdn_prefill_chunk with g [B, T, H, d_k]."""
     return _prefill("damp_kda_prefill_chunk", layout, state, perm, q, k, v, g, beta, o, lengths, slot_idx,
                     num_slots, stream)
+
+
+def calib_error_energy(layout, S, E_acc, stream=None):
+    """E_acc [H, d_k] += per-channel squared low-tier round-trip error of S [B, H, d_k, d_v]."""
+    _cuda_contig("S", S)
+    _cuda_contig("E_acc", E_acc)
+    _check(lib().damp_calib_error_energy(ctypes.byref(layout.c()), _ptr(S), S.shape[0], _ptr(E_acc), _stream(stream)),
+           "damp_calib_error_energy")
+    return E_acc
+
+
+def calib_log_decay(layout, g, G_acc, stream=None):
+    """G_acc [H, d_k] += log-decay g summed over the batch (g [B, H] GDN or [B, H, d_k] KDA)."""
+    _cuda_contig("g", g)
+    _cuda_contig("G_acc", G_acc)
+    _check(lib().damp_calib_log_decay(ctypes.byref(layout.c()), _ptr(g), g.shape[0], 1 if g.dim() == 3 else 0,
+                                      _ptr(G_acc), _stream(stream)), "damp_calib_log_decay")
+    return G_acc
+
+
+def calib_select(layout, E_acc, n_samples, G_acc, n_tokens, tau=1e-4, stream=None):
+    """Scores C [H, d_k] float32 and permutations pi [H, d_k] uint8 (Algorithm 1)."""
+    import torch
+    _cuda_contig("E_acc", E_acc)
+    _cuda_contig("G_acc", G_acc)
+    C = torch.empty((layout.num_heads, layout.d_k), dtype=torch.float32, device=E_acc.device)
+    perm = torch.empty((layout.num_heads, layout.d_k), dtype=torch.uint8, device=E_acc.device)
+    _check(lib().damp_calib_select(ctypes.byref(layout.c()), _ptr(E_acc), int(n_samples), _ptr(G_acc), int(n_tokens),
+                                   float(tau), _ptr(C), _ptr(perm), _stream(stream)), "damp_calib_select")
+    return C, perm
 
 
 def quantize_state(layout, S, perm, state, slot_idx=None, num_slots=None, stream=None):

@@ -1,0 +1,31 @@
+"""Calibration run on the GPU (Algorithm 1, App. A.2): FP32 trajectories of the
+calibration documents, error energy of the states sampled every `every` tokens,
+mean log-decay over every token, then the selection of K_hi protected channels and
+the permutation pi per head.  Every step is a libdamp call; this module only orders
+them."""
+from __future__ import annotations
+
+import paper_2608_27513_gb300 as damp
+
+
+def calibrate(layout, kind: str, token_inputs, every: int = 8, tau: float = 1e-4, stream=None):
+    """token_inputs: sequence of per-token dicts of device tensors (q, k, v, g, beta) for
+    the calibration documents (rows = documents), in token order.  Returns (C, perm):
+    float32 [H, d_k] scores and uint8 [H, d_k] permutations."""
+    import torch
+    inputs = list(token_inputs)
+    n_docs = inputs[0]["v"].shape[0]
+    dev = inputs[0]["v"].device
+    S = damp.new_fp32_state(layout, n_docs, dev)
+    o = torch.empty((n_docs, layout.num_heads, layout.d_v), dtype=torch.float32, device=dev)
+    E_acc = torch.zeros((layout.num_heads, layout.d_k), dtype=torch.float32, device=dev)
+    G_acc = torch.zeros_like(E_acc)
+    step = damp.fp32_kda_decode_step if kind == "kda" else damp.fp32_gdn_decode_step
+    n_samples = 0
+    for t, d in enumerate(inputs):
+        step(layout, S, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o, stream=stream)
+        damp.calib_log_decay(layout, d["g"], G_acc, stream=stream)
+        if (t + 1) % every == 0:
+            damp.calib_error_energy(layout, S, E_acc, stream=stream)
+            n_samples += n_docs
+    return damp.calib_select(layout, E_acc, max(n_samples, 1), G_acc, n_docs * len(inputs), tau, stream=stream)

@@ -1,0 +1,161 @@
+// calib.cu -- offline key-channel selection on the GPU (Sec. 5.1; App. A.2; Algorithm 1).
+//
+//   calib_error_energy   E_acc[h][u] += sum_b || Q_lo(S_b,h)_{u:} - S_b,h,u: ||^2
+//                        (Eq. empirical_error_energy: the low-tier round trip of every
+//                        key-channel row of the sampled states, in the layout's format)
+//   calib_log_decay      G_acc[h][u] += sum_b log a_{b,h,u}   (GDN: the head's scalar)
+//   calib_select         E = E_acc / n_samples, a_eff = exp(G_acc / n_tokens),
+//                        P = 1 / max(1 - a_eff^2, tau), C = E P, H = TopK_{K_hi}(C)
+//                        (ties to the lower channel), pi = stable partition (H first,
+//                        each part in ascending channel order)
+//
+// Every accumulator entry has exactly one writer per call and sums in a fixed order,
+// so repeated runs give the same bits; no global scratch is used.
+#include "damp_common.cuh"
+#include "damp_internal.h"
+
+#include <algorithm>
+
+namespace damp {
+
+namespace {
+
+// One warp per (head, 32 key channels): lane u accumulates its row's error over the
+// batch and the value blocks.
+template <int FMT>
+__global__ void __launch_bounds__(256) calib_error_energy_kernel(const float *S, int32_t batch, int32_t H,
+                                                                 int32_t dk, int32_t dv, float *E_acc) {
+    const int lane = threadIdx.x & 31;
+    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int groups = (dk + 31) / 32;
+    if (gw >= (int64_t)H * groups) return;
+    const int h = (int)(gw / groups);
+    const int u = (int)(gw % groups) * 32 + lane;
+    if (u >= dk) return;
+    float err = 0.f;
+    for (int b = 0; b < batch; ++b) {
+        const float *row = S + (((int64_t)b * H + h) * dk + u) * dv;
+        if (FMT == 2) {
+            // per-row symmetric absmax INT8: s = max|x| / 127, q = sat(rne(x / s)), x^ = s q
+            float amax = 0.f;
+            for (int j = 0; j < dv; ++j) amax = fmaxf(amax, fabsf(row[j]));
+            const float s = __fdiv_rn(amax, 127.f);
+            for (int j = 0; j < dv; ++j) {
+                float t = s == 0.f ? 0.f : rintf(__fdiv_rn(row[j], s));
+                t = fminf(fmaxf(t, -127.f), 127.f);
+                const float dlt = __fmul_rn(s, t) - row[j];
+                err = fmaf(dlt, dlt, err);
+            }
+            continue;
+        }
+        for (int c = 0; c < dv / kG; ++c) {
+            float2 x[16], y[16];
+#pragma unroll
+            for (int m = 0; m < 8; ++m) {
+                const float4 f = reinterpret_cast<const float4 *>(row + kG * c)[m];
+                x[2 * m] = make_float2(f.x, f.y);
+                x[2 * m + 1] = make_float2(f.z, f.w);
+            }
+#pragma unroll
+            for (int m = 0; m < 16; ++m) y[m] = x[m];
+            if (FMT == 0) hadamard_pairs(y);
+#pragma unroll
+            for (int m = 0; m < 16; ++m) y[m] = mul2(y[m], splat2(kDown));  // working scale of the quantizer
+            uint32_t w[8];
+            const uint32_t sz = quantize_group(y, w);
+            dequantize_group(w, sz, 1.0f, y);
+            if (FMT == 0) hadamard_pairs(y);
+#pragma unroll
+            for (int m = 0; m < 16; ++m) {
+                const float d0 = y[m].x - x[m].x, d1 = y[m].y - x[m].y;
+                err = fmaf(d0, d0, fmaf(d1, d1, err));
+            }
+        }
+    }
+    E_acc[(int64_t)h * dk + u] += err;
+}
+
+__global__ void calib_log_decay_kernel(const float *g, int32_t batch, int32_t H, int32_t dk, int32_t kda,
+                                       float *G_acc) {
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= (int64_t)H * dk) return;
+    const int h = (int)(i / dk), u = (int)(i % dk);
+    float s = 0.f;
+    for (int b = 0; b < batch; ++b) s += kda ? g[((int64_t)b * H + h) * dk + u] : g[(int64_t)b * H + h];
+    G_acc[i] += s;
+}
+
+// One warp per head: scores, rank of every channel, then the stable partition.
+__global__ void __launch_bounds__(32) calib_select_kernel(const float *E_acc, float inv_samples, const float *G_acc,
+                                                          float inv_tokens, float tau, int32_t H, int32_t dk,
+                                                          int32_t k_hi, float *C_out, uint8_t *perm_out) {
+    __shared__ float sc[256];
+    const int lane = threadIdx.x & 31;
+    const int h = blockIdx.x;
+    if (h >= H) return;
+    for (int u = lane; u < dk; u += 32) {
+        const float E = E_acc[(int64_t)h * dk + u] * inv_samples;
+        // 1 - a_eff^2 = 1 - exp(2 mean log a) = -expm1(2 mean log a): no cancellation near a = 1
+        const float one_minus_a2 = -expm1f(2.0f * (G_acc[(int64_t)h * dk + u] * inv_tokens));
+        const float P = 1.0f / fmaxf(one_minus_a2, tau);
+        const float C = E * P;
+        sc[u] = C;
+        C_out[(int64_t)h * dk + u] = C;
+    }
+    __syncwarp();
+    // protected: fewer than K_hi channels rank above u (larger score, or equal score at a lower index)
+    unsigned prot_words[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    for (int u0 = 0; u0 < dk; u0 += 32) {
+        const int u = u0 + lane;
+        const float cu = sc[u];
+        int above = 0;
+        for (int v = 0; v < dk; ++v) {
+            const float cv = sc[v];
+            above += (cv > cu) || (cv == cu && v < u);
+        }
+        prot_words[u0 / 32] = __ballot_sync(kFull, above < k_hi);
+    }
+    // stable partition: protected channels in ascending order, then the rest
+    int n_prot = 0;
+    for (int i = 0; i < dk / 32; ++i) n_prot += __popc(prot_words[i]);
+    int before_p = 0, before_r = 0;
+    for (int i = 0; i < dk / 32; ++i) {
+        const unsigned m = prot_words[i];
+        const unsigned below = (1u << lane) - 1u;
+        const int u = 32 * i + lane;
+        const bool p = (m >> lane) & 1u;
+        const int pos = p ? before_p + __popc(m & below) : n_prot + before_r + __popc(~m & below);
+        perm_out[(int64_t)h * dk + pos] = (uint8_t)u;
+        before_p += __popc(m);
+        before_r += 32 - __popc(m);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_calib_error_energy(const float *S, int32_t batch, int32_t H, int32_t dk, int32_t dv, int32_t fmt,
+                                      float *E_acc, cudaStream_t stream) {
+    const int64_t warps = (int64_t)H * ((dk + 31) / 32);
+    const int grid = (int)((warps + 7) / 8);
+    void (*kern)(const float *, int32_t, int32_t, int32_t, int32_t, float *) =
+        fmt == 0 ? calib_error_energy_kernel<0> : fmt == 1 ? calib_error_energy_kernel<1> : calib_error_energy_kernel<2>;
+    kern<<<grid, 256, 0, stream>>>(S, batch, H, dk, dv, E_acc);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_calib_log_decay(const float *g, int32_t batch, int32_t H, int32_t dk, int32_t kda, float *G_acc,
+                                   cudaStream_t stream) {
+    const int64_t n = (int64_t)H * dk;
+    calib_log_decay_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(g, batch, H, dk, kda, G_acc);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_calib_select(const float *E_acc, int64_t n_samples, const float *G_acc, int64_t n_tokens, float tau,
+                                int32_t H, int32_t dk, int32_t k_hi, float *C_out, uint8_t *perm_out,
+                                cudaStream_t stream) {
+    calib_select_kernel<<<H, 32, 0, stream>>>(E_acc, 1.0f / (float)n_samples, G_acc, 1.0f / (float)n_tokens, tau, H,
+                                               dk, k_hi, C_out, perm_out);
+    return cudaGetLastError();
+}
+
+}  // namespace damp

@@ -415,6 +415,60 @@ damp_status damp_unpack_tiers(const damp_layout *layout, const void *state, int6
                    stream, kUnpack);
 }
 
+damp_status damp_calib_error_energy(const damp_layout *layout, const float *S, int32_t batch, float *E_acc,
+                                    void *stream) {
+    damp_status st = check_layout(layout);
+    if (st != DAMP_OK) return st;
+    if (batch < 0) return DAMP_ERR_SHAPE;
+    if (!E_acc) return DAMP_ERR_NULL;
+    if (batch == 0) return DAMP_OK;
+    if (!S) return DAMP_ERR_NULL;
+    if (!aligned(S, 16) || !aligned(E_acc, 4)) return DAMP_ERR_ALIGN;
+    const int64_t H = layout->num_heads, dk = layout->d_k, dv = layout->d_v;
+    if (overlap(range_of(S, (int64_t)batch * H * dk * dv * 4), range_of(E_acc, H * dk * 4))) return DAMP_ERR_ALIAS;
+    return launch_calib_error_energy(S, batch, (int32_t)H, (int32_t)dk, (int32_t)dv, layout->lo_format, E_acc,
+                                     static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? DAMP_OK
+               : DAMP_ERR_CUDA;
+}
+
+damp_status damp_calib_log_decay(const damp_layout *layout, const float *g, int32_t batch, int32_t kda, float *G_acc,
+                                 void *stream) {
+    damp_status st = check_layout(layout);
+    if (st != DAMP_OK) return st;
+    if (batch < 0) return DAMP_ERR_SHAPE;
+    if (!G_acc) return DAMP_ERR_NULL;
+    if (batch == 0) return DAMP_OK;
+    if (!g) return DAMP_ERR_NULL;
+    if (!aligned(g, 4) || !aligned(G_acc, 4)) return DAMP_ERR_ALIGN;
+    const int64_t H = layout->num_heads, dk = layout->d_k;
+    if (overlap(range_of(g, (int64_t)batch * H * (kda ? dk : 1) * 4), range_of(G_acc, H * dk * 4)))
+        return DAMP_ERR_ALIAS;
+    return launch_calib_log_decay(g, batch, (int32_t)H, (int32_t)dk, kda ? 1 : 0, G_acc,
+                                  static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? DAMP_OK
+               : DAMP_ERR_CUDA;
+}
+
+damp_status damp_calib_select(const damp_layout *layout, const float *E_acc, int64_t n_samples, const float *G_acc,
+                              int64_t n_tokens, float tau, float *C_out, uint8_t *perm_out, void *stream) {
+    damp_status st = check_layout(layout);
+    if (st != DAMP_OK) return st;
+    if (!E_acc || !G_acc || !C_out || !perm_out) return DAMP_ERR_NULL;
+    if (n_samples < 1 || n_tokens < 1 || !(tau > 0.0f) || !(tau <= 1.0f)) return DAMP_ERR_SHAPE;
+    if (!aligned(E_acc, 4) || !aligned(G_acc, 4) || !aligned(C_out, 4)) return DAMP_ERR_ALIGN;
+    const int64_t H = layout->num_heads, dk = layout->d_k;
+    const Range rc = range_of(C_out, H * dk * 4), rp = range_of(perm_out, H * dk);
+    const Range ins[] = {range_of(E_acc, H * dk * 4), range_of(G_acc, H * dk * 4)};
+    if (overlap(rc, rp)) return DAMP_ERR_ALIAS;
+    for (const Range &r : ins)
+        if (overlap(r, rc) || overlap(r, rp)) return DAMP_ERR_ALIAS;
+    return launch_calib_select(E_acc, n_samples, G_acc, n_tokens, tau, (int32_t)H, (int32_t)dk, layout->k_hi, C_out,
+                               perm_out, static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? DAMP_OK
+               : DAMP_ERR_CUDA;
+}
+
 damp_status damp_device_status(uint32_t *status) {
     if (!status) return DAMP_ERR_NULL;
     uint32_t all = 0, bits = 0;

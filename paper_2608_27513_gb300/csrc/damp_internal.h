@@ -51,6 +51,13 @@ cudaError_t launch_unpack_tiers(const ConvArgs &a, cudaStream_t s);
 // One prefill chunk on the packed state (formats 0 and 1).
 cudaError_t launch_prefill_gdn(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_prefill_kda(const StepArgs &a, cudaStream_t s);
+// Offline key-channel selection (Sec. 5.1, Algorithm 1).
+cudaError_t launch_calib_error_energy(const float *S, int32_t batch, int32_t H, int32_t dk, int32_t dv, int32_t fmt,
+                                      float *E_acc, cudaStream_t s);
+cudaError_t launch_calib_log_decay(const float *g, int32_t batch, int32_t H, int32_t dk, int32_t kda, float *G_acc,
+                                   cudaStream_t s);
+cudaError_t launch_calib_select(const float *E_acc, int64_t n_samples, const float *G_acc, int64_t n_tokens, float tau,
+                                int32_t H, int32_t dk, int32_t k_hi, float *C_out, uint8_t *perm_out, cudaStream_t s);
 // Row-absmax INT8 low tier (lo_format 2); op: 0 quantize, 1 dequantize, 2 pack, 3 unpack.
 cudaError_t launch_rowabs_step(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_rowabs_convert(const ConvArgs &a, int op, cudaStream_t s);

@@ -147,6 +147,25 @@ def test_prefill_rejects_bad_arguments_before_launch(L):
     assert _call_prefill(L, lay, fb, in_dtype=3) == 5
 
 
+def test_calibration_calls_reject_bad_arguments(L):
+    fb = FakeBuffers()
+    c = _layout().c()
+    off = lambda i, d: ctypes.c_void_p(fb.ptrs[i] + d)
+    assert L.damp_calib_error_energy(ctypes.byref(c), fb[0], 0, fb[1], None) == 0   # empty batch
+    assert L.damp_calib_error_energy(ctypes.byref(c), None, 4, fb[1], None) == 1
+    assert L.damp_calib_error_energy(ctypes.byref(c), off(0, 4), 4, fb[1], None) == 3
+    assert L.damp_calib_error_energy(ctypes.byref(c), fb[0], 4, off(0, 64), None) == 4  # accumulator inside S
+    assert L.damp_calib_log_decay(ctypes.byref(c), fb[0], -1, 1, fb[1], None) == 2
+    assert L.damp_calib_log_decay(ctypes.byref(c), fb[0], 4, 1, off(1, 2), None) == 3
+    sel = lambda **kw: L.damp_calib_select(ctypes.byref(c), *dict(dict(E=fb[0], ns=4, G=fb[1], nt=8,
+                                                                       tau=ctypes.c_float(1e-4), C=fb[2],
+                                                                       perm=fb[3], stream=None), **kw).values())
+    assert sel(ns=0) == 2
+    assert sel(tau=ctypes.c_float(0.0)) == 2
+    assert sel(perm=None) == 1
+    assert sel(perm=off(2, 16)) == 4                                                  # pi over the scores
+
+
 def test_gdn_gate_alignment_is_4_bytes(L):
     fb = FakeBuffers()
     c = _layout().c()
