@@ -545,6 +545,56 @@ def prefill_arm(steps: int, warmup: int, T: int = 64):
         print(json.dumps(row), flush=True)
 
 
+def calibrate_arm(steps: int, warmup: int, n_docs: int = 32, n_tokens: int = 256):
+    """Calibration run (Algorithm 1, App. A.2) on the GPU for one layer of H = 32 heads,
+    d = 128: FP32 trajectories of n_docs documents over n_tokens tokens, error energy of
+    the states every 8 tokens, mean log-decay, selection.  Reports the whole run and the
+    error-energy pass alone (HBM-bound: it reads the sampled states once)."""
+    import torch
+
+    import paper_2608_27513_gb300 as damp
+    from paper_2608_27513_gb300 import build, calibration
+    build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    peak = measured_peaks().get("hbm_gbs") or 6800.0
+    out = []
+    for w in (wl.stack_layer(1, 16), wl.stack_layer(0, 16)):
+        w = w.replace(batch=n_docs)
+        L = damp.Layout(w.heads, w.qk_heads, w.d_k, w.d_v, w.k_hi, w.lo_format)
+        inputs = wl.torch_step_inputs(w, n_tokens, dev)
+        calibration.calibrate(L, w.kind, inputs[:16])  # warm-up
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        C, perm = calibration.calibrate(L, w.kind, inputs)
+        e1.record()
+        torch.cuda.synchronize()
+        run_ms = e0.elapsed_time(e1)
+        S = 0.3 * torch.randn((n_docs, w.heads, w.d_k, w.d_v), device=dev)
+        E = torch.zeros((w.heads, w.d_k), device=dev)
+        for _ in range(max(warmup, 3)):
+            damp.calib_error_energy(L, S, E)
+        n = max(steps // 20, 10)
+        torch.cuda.synchronize()
+        e0.record()
+        for _ in range(n):
+            damp.calib_error_energy(L, S, E)
+        e1.record()
+        torch.cuda.synchronize()
+        ee_us = e0.elapsed_time(e1) / n * 1e3
+        gbs = S.numel() * 4 / (ee_us * 1e-6) / 1e9
+        out.append({"mode": "calibration", "kind": w.kind, "docs": n_docs, "tokens": n_tokens, "heads": w.heads,
+                    "d": w.d_k, "k_hi": w.k_hi, "run_ms": run_ms, "error_energy_us_per_call": ee_us,
+                    "error_energy_roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s",
+                                              "frac": gbs / peak, "bytes_per_call": S.numel() * 4}})
+        del inputs, S
+    if damp.device_status() != 0:
+        raise RuntimeError("device status word set during the calibration runs")
+    for row in out:
+        print(json.dumps(row), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -554,6 +604,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true", help="K_hi sweep (GDN and KDA, B=256) instead of the bench line")
     ap.add_argument("--prefill", action="store_true", help="prefill chunks (64 tokens, B=256) instead of the bench line")
+    ap.add_argument("--calibrate", action="store_true", help="GPU calibration run instead of the bench line")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -568,6 +619,9 @@ def main():
         return
     if args.prefill:
         prefill_arm(args.steps, args.warmup)
+        return
+    if args.calibrate:
+        calibrate_arm(args.steps, args.warmup)
         return
     import torch
     import torch.distributed as dist

@@ -10,7 +10,8 @@
 //                        each part in ascending channel order)
 //
 // Every accumulator entry has exactly one writer per call and sums in a fixed order,
-// so repeated runs give the same bits; no global scratch is used.
+// so repeated runs give the same bits; no global scratch is used (partials of the
+// error energy meet in shared memory).
 #include "damp_common.cuh"
 #include "damp_internal.h"
 
@@ -20,20 +21,22 @@ namespace damp {
 
 namespace {
 
-// One warp per (head, 32 key channels): lane u accumulates its row's error over the
-// batch and the value blocks.
+// One CTA per (head, 32 key channels); warp w takes batch rows w, w + 8, ...; lane u
+// accumulates its row's error over those rows and the value blocks; the eight warp
+// partials are added in warp order (a fixed order: the result does not depend on
+// scheduling).
+constexpr int kEeWarps = 8;
+
 template <int FMT>
-__global__ void __launch_bounds__(256) calib_error_energy_kernel(const float *S, int32_t batch, int32_t H,
-                                                                 int32_t dk, int32_t dv, float *E_acc) {
-    const int lane = threadIdx.x & 31;
-    const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+__global__ void __launch_bounds__(32 * kEeWarps) calib_error_energy_kernel(const float *S, int32_t batch, int32_t H,
+                                                                           int32_t dk, int32_t dv, float *E_acc) {
+    __shared__ float partial[kEeWarps][32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int groups = (dk + 31) / 32;
-    if (gw >= (int64_t)H * groups) return;
-    const int h = (int)(gw / groups);
-    const int u = (int)(gw % groups) * 32 + lane;
-    if (u >= dk) return;
+    const int h = (int)(blockIdx.x / groups);
+    const int u = (int)(blockIdx.x % groups) * 32 + lane;  // d_k is a multiple of 32
     float err = 0.f;
-    for (int b = 0; b < batch; ++b) {
+    for (int b = warp; b < batch; b += kEeWarps) {
         const float *row = S + (((int64_t)b * H + h) * dk + u) * dv;
         if (FMT == 2) {
             // per-row symmetric absmax INT8: s = max|x| / 127, q = sat(rne(x / s)), x^ = s q
@@ -72,7 +75,14 @@ __global__ void __launch_bounds__(256) calib_error_energy_kernel(const float *S,
             }
         }
     }
-    E_acc[(int64_t)h * dk + u] += err;
+    partial[warp][lane] = err;
+    __syncthreads();
+    if (warp == 0) {
+        float sum = 0.f;
+#pragma unroll
+        for (int i = 0; i < kEeWarps; ++i) sum += partial[i][lane];
+        E_acc[(int64_t)h * dk + u] += sum;
+    }
 }
 
 __global__ void calib_log_decay_kernel(const float *g, int32_t batch, int32_t H, int32_t dk, int32_t kda,
@@ -135,11 +145,10 @@ __global__ void __launch_bounds__(32) calib_select_kernel(const float *E_acc, fl
 
 cudaError_t launch_calib_error_energy(const float *S, int32_t batch, int32_t H, int32_t dk, int32_t dv, int32_t fmt,
                                       float *E_acc, cudaStream_t stream) {
-    const int64_t warps = (int64_t)H * ((dk + 31) / 32);
-    const int grid = (int)((warps + 7) / 8);
+    const int64_t grid = (int64_t)H * ((dk + 31) / 32);
     void (*kern)(const float *, int32_t, int32_t, int32_t, int32_t, float *) =
         fmt == 0 ? calib_error_energy_kernel<0> : fmt == 1 ? calib_error_energy_kernel<1> : calib_error_energy_kernel<2>;
-    kern<<<grid, 256, 0, stream>>>(S, batch, H, dk, dv, E_acc);
+    kern<<<(unsigned)grid, 32 * kEeWarps, 0, stream>>>(S, batch, H, dk, dv, E_acc);
     return cudaGetLastError();
 }
 
