@@ -27,6 +27,8 @@ import subprocess
 import sys
 import time
 
+import numpy as np
+
 ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
@@ -595,6 +597,73 @@ def calibrate_arm(steps: int, warmup: int, n_docs: int = 32, n_tokens: int = 256
         print(json.dumps(row), flush=True)
 
 
+def drift_arm(layers: int = 30, steps: int = 1024, every: int = 64):
+    """Free-running drift of the 30-layer stack (15 GDN + 15 KDA, alternating; B = 256,
+    H = 32, d = 128): per layer, pi from a GPU calibration run (32 documents x 256
+    tokens), a 256-token FP32 prefix, then `steps` decode steps of the FP32 state, of
+    DAMP (K_hi = 16, calibrated pi) and of uniform INT8 + H_32 (K_hi = 0) on the same
+    inputs.  Drift = held-out trajectory RRMSE (App. E): output RRMSE over every step,
+    state RRMSE over the states every `every` steps."""
+    import torch
+
+    import paper_2608_27513_gb300 as damp
+    from paper_2608_27513_gb300 import build, calibration
+    build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    rows = []
+    block = 64
+    for layer in range(layers):
+        w = wl.stack_layer(layer, 16)
+        Ld = damp.Layout(w.heads, w.qk_heads, w.d_k, w.d_v, 16, 0)
+        Lu = damp.Layout(w.heads, w.qk_heads, w.d_k, w.d_v, 0, 0)
+        calib = wl.torch_step_inputs(w.replace(batch=32), 256, dev, seed_offset=7_000_000)
+        _, perm_d = calibration.calibrate(Ld, w.kind, calib)
+        del calib
+        perm_u = torch.arange(w.d_k, dtype=torch.uint8, device=dev).repeat(w.heads, 1)
+        fp32 = damp.fp32_kda_decode_step if w.kind == "kda" else damp.fp32_gdn_decode_step
+        packed = damp.kda_decode_step if w.kind == "kda" else damp.gdn_decode_step
+        S = damp.new_fp32_state(Ld, w.batch, dev)
+        o = torch.empty((w.batch, w.heads, w.d_v), device=dev)
+        for t0 in range(0, w.prefix, block):
+            for d in wl.torch_step_inputs(w, min(block, w.prefix - t0), dev, seed_offset=1_000_000 + t0):
+                fp32(Ld, S, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o)
+        st_d = damp.new_state(Ld, w.batch, dev)
+        st_u = damp.new_state(Lu, w.batch, dev)
+        damp.quantize_state(Ld, S, perm_d, st_d)
+        damp.quantize_state(Lu, S, perm_u, st_u)
+        acc = torch.zeros(6, dtype=torch.float64, device=dev)  # o: err_d, err_u, ref; state: err_d, err_u, ref
+        od = torch.empty_like(o)
+        ou = torch.empty_like(o)
+        for t0 in range(0, steps, block):
+            for i, d in enumerate(wl.torch_step_inputs(w, min(block, steps - t0), dev, seed_offset=2_000_000 + t0)):
+                fp32(Ld, S, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o)
+                packed(Ld, st_d, perm_d, d["q"], d["k"], d["v"], d["g"], d["beta"], o=od)
+                packed(Lu, st_u, perm_u, d["q"], d["k"], d["v"], d["g"], d["beta"], o=ou)
+                acc[0] += ((od - o).double() ** 2).sum()
+                acc[1] += ((ou - o).double() ** 2).sum()
+                acc[2] += (o.double() ** 2).sum()
+                if (t0 + i + 1) % every == 0:
+                    Sd = damp.dequantize_state(Ld, st_d, perm_d)
+                    acc[3] += ((Sd - S).double() ** 2).sum()
+                    del Sd
+                    Su = damp.dequantize_state(Lu, st_u, perm_u)
+                    acc[4] += ((Su - S).double() ** 2).sum()
+                    del Su
+                    acc[5] += (S.double() ** 2).sum()
+        a = acc.cpu().numpy()
+        rows.append({"mode": "drift", "layer": layer, "kind": w.kind, "steps": steps,
+                     "damp_k16": {"o_rrmse": float(np.sqrt(a[0] / a[2])), "state_rrmse": float(np.sqrt(a[3] / a[5]))},
+                     "uniform_int8_h32": {"o_rrmse": float(np.sqrt(a[1] / a[2])),
+                                          "state_rrmse": float(np.sqrt(a[4] / a[5]))},
+                     "bits_per_value": {"damp_k16": damp.bits_per_value(Ld), "uniform": damp.bits_per_value(Lu)}})
+        print(json.dumps(rows[-1]), flush=True)
+        del S, st_d, st_u, o, od, ou
+        torch.cuda.empty_cache()
+    if damp.device_status() != 0:
+        raise RuntimeError("device status word set during the drift run")
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -605,6 +674,7 @@ def main():
     ap.add_argument("--sweep", action="store_true", help="K_hi sweep (GDN and KDA, B=256) instead of the bench line")
     ap.add_argument("--prefill", action="store_true", help="prefill chunks (64 tokens, B=256) instead of the bench line")
     ap.add_argument("--calibrate", action="store_true", help="GPU calibration run instead of the bench line")
+    ap.add_argument("--drift", action="store_true", help="30-layer free-running drift run instead of the bench line")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -622,6 +692,9 @@ def main():
         return
     if args.calibrate:
         calibrate_arm(args.steps, args.warmup)
+        return
+    if args.drift:
+        drift_arm()
         return
     import torch
     import torch.distributed as dist
