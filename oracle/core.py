@@ -3,9 +3,12 @@
 Array conventions (all dense, C order):
   perm  uint8  [n, d_k]           packed row i holds natural key channel perm[i]
   hi    uint16 [n, K, d_v]        binary16 bit patterns of the FP16 tier S_hi
-  codes uint8  [n, d_k-K, d_v]    UINT8 codes Q_lo (int8 for the row-absmax format)
+  codes uint8  [n, d_k-K, d_v]    UINT8 codes Q_lo (int8 for the row-absmax format; E4M3
+        bit patterns for FP8; [n, d_k-K, d_v/2] two UINT4 codes per byte, even value
+        index in the low nibble, for the 4-bit formats)
   meta  uint16 [n, d_k-K, d_v/32, 2]  binary16 (s, z) per 32-group (M_lo);
-        float32 [n, d_k-K] scales for the row-absmax format
+        float32 [n, d_k-K] scales for the row-absmax format,
+        float32 [n, d_k-K, d_v/32] scales for FP8
   S     float32 [n, d_k, d_v]     natural-order state
 """
 from __future__ import annotations
@@ -19,6 +22,9 @@ from . import build as _build
 FMT_U8_H32 = 0
 FMT_U8 = 1
 FMT_S8_ROW = 2
+FMT_U4_H32 = 3
+FMT_U4 = 4
+FMT_E4M3 = 5
 KINDS = {"gdn": 0, "kda": 1}
 
 _lib = None
@@ -39,6 +45,12 @@ def lib() -> ctypes.CDLL:
             "dor_quant_group_u8": (None, [P, P, P]),
             "dor_dequant_group_u8": (None, [P, P, P]),
             "dor_quant_row_s8": (None, [P, i32, P, P]),
+            "dor_quant_group_u4": (None, [P, P, P]),
+            "dor_dequant_group_u4": (None, [P, P, P]),
+            "dor_e4m3_to_f32": (f32, [ctypes.c_uint8]),
+            "dor_f32_to_e4m3": (ctypes.c_uint8, [f32]),
+            "dor_quant_group_e4m3": (None, [P, P, P]),
+            "dor_dequant_group_e4m3": (None, [P, f32, P]),
             "dor_dequant_row_s8": (None, [P, i32, f32, P]),
             "dor_qdq_rows": (None, [i64, i32, i32, P, P]),
             "dor_delta_step": (None, [i32, i32, P, P, P, P, P, f32, P]),
@@ -110,6 +122,47 @@ def dequant_group_u8(q, sz) -> np.ndarray:
     return x
 
 
+def quant_group_u4(x):
+    """UINT4 affine quantizer of one 32-group: returns (codes uint8[16] nibble pairs, sz uint16[2])."""
+    x = _f32(x).reshape(32)
+    q = np.empty(16, np.uint8)
+    sz = np.empty(2, np.uint16)
+    lib().dor_quant_group_u4(_p(x), _p(q), _p(sz))
+    return q, sz
+
+
+def dequant_group_u4(q, sz) -> np.ndarray:
+    q = np.ascontiguousarray(q, dtype=np.uint8).reshape(16)
+    sz = np.ascontiguousarray(sz, dtype=np.uint16).reshape(2)
+    x = np.empty(32, np.float32)
+    lib().dor_dequant_group_u4(_p(q), _p(sz), _p(x))
+    return x
+
+
+def e4m3_to_f32(b: int) -> float:
+    return float(lib().dor_e4m3_to_f32(int(b)))
+
+
+def f32_to_e4m3(x: float) -> int:
+    return int(lib().dor_f32_to_e4m3(float(x)))
+
+
+def quant_group_e4m3(x):
+    """FP8 E4M3 group quantizer: returns (codes uint8[32] E4M3 bits, s float)."""
+    x = _f32(x).reshape(32)
+    q = np.empty(32, np.uint8)
+    s = np.empty(1, np.float32)
+    lib().dor_quant_group_e4m3(_p(x), _p(q), _p(s))
+    return q, float(s[0])
+
+
+def dequant_group_e4m3(q, s: float) -> np.ndarray:
+    q = np.ascontiguousarray(q, dtype=np.uint8).reshape(32)
+    x = np.empty(32, np.float32)
+    lib().dor_dequant_group_e4m3(_p(q), float(s), _p(x))
+    return x
+
+
 def quant_row_s8(x):
     x = _f32(x).reshape(-1)
     q = np.empty(x.size, np.int8)
@@ -139,6 +192,12 @@ def tier_arrays(n: int, d_k: int, d_v: int, k_hi: int, fmt: int):
     if fmt == FMT_S8_ROW:
         codes = np.zeros((n, lo, d_v), np.int8)
         meta = np.zeros((n, lo), np.float32)
+    elif fmt in (FMT_U4_H32, FMT_U4):
+        codes = np.zeros((n, lo, d_v // 2), np.uint8)
+        meta = np.zeros((n, lo, d_v // 32, 2), np.uint16)
+    elif fmt == FMT_E4M3:
+        codes = np.zeros((n, lo, d_v), np.uint8)
+        meta = np.zeros((n, lo, d_v // 32), np.float32)
     else:
         codes = np.zeros((n, lo, d_v), np.uint8)
         meta = np.zeros((n, lo, d_v // 32, 2), np.uint16)
@@ -187,7 +246,7 @@ def mixed_step_heads(perm, hi, codes, meta, q, k, v, g, beta, k_hi: int, fmt: in
         assert a.flags["C_CONTIGUOUS"]
     perm = np.ascontiguousarray(perm, dtype=np.uint8)
     n, d_k = perm.shape
-    d_v = codes.shape[-1] if codes.ndim == 3 else hi.shape[-1]
+    d_v = np.shape(v)[-1]
     q, k, v, g, beta = _f32(q), _f32(k), _f32(v), _f32(g), _f32(beta)
     o = np.empty((n, d_v), np.float32)
     rc = lib().dor_mixed_step_heads(n, d_k, d_v, k_hi, fmt, KINDS[kind], _p(perm), _p(hi), _p(codes), _p(meta),

@@ -41,7 +41,7 @@
 
 #define DOR_G 32 /* group size along d_v (App. A.1) */
 
-enum { DOR_FMT_U8_H32 = 0, DOR_FMT_U8 = 1, DOR_FMT_S8_ROW = 2 };
+enum { DOR_FMT_U8_H32 = 0, DOR_FMT_U8 = 1, DOR_FMT_S8_ROW = 2, DOR_FMT_U4_H32 = 3, DOR_FMT_U4 = 4, DOR_FMT_E4M3 = 5 };
 enum { DOR_GDN = 0, DOR_KDA = 1 };
 
 /* ------------------------------------------------------------------------- */
@@ -139,18 +139,19 @@ void dor_hadamard32(const float *x, float *y)
 /* sz[0] = s, sz[1] = z, both binary16 bit patterns.                         */
 /* ------------------------------------------------------------------------- */
 
-void dor_quant_group_u8(const float *x, uint8_t *q, uint16_t *sz)
+/* The affine rule for b-bit codes (levels = 2^b - 1); q receives the codes as ints. */
+static void quant_group_affine(const float *x, float levels, int *q, uint16_t *sz)
 {
     float x_min = x[0], x_max = x[0];
     for (int i = 1; i < DOR_G; i++) {
         if (x[i] < x_min) x_min = x[i];
         if (x[i] > x_max) x_max = x[i];
     }
-    float s = f16_round((x_max - x_min) / 255.0f);
+    float s = f16_round((x_max - x_min) / levels);
     if (s == 0.0f) { /* degenerate block: widen the range to contain 0 */
         if (x_min > 0.0f) x_min = 0.0f;
         if (x_max < 0.0f) x_max = 0.0f;
-        s = f16_round((x_max - x_min) / 255.0f);
+        s = f16_round((x_max - x_min) / levels);
     }
     if (s == 0.0f) s = 1.0f; /* all (near-)zero block */
     uint16_t z16 = dor_f32_to_f16(rintf(-x_min / s));
@@ -158,11 +159,18 @@ void dor_quant_group_u8(const float *x, uint8_t *q, uint16_t *sz)
     for (int i = 0; i < DOR_G; i++) {
         float t = rintf(x[i] / s) + z;
         if (t < 0.0f) t = 0.0f;
-        if (t > 255.0f) t = 255.0f;
-        q[i] = (uint8_t)t;
+        if (t > levels) t = levels;
+        q[i] = (int)t;
     }
     sz[0] = dor_f32_to_f16(s);
     sz[1] = z16;
+}
+
+void dor_quant_group_u8(const float *x, uint8_t *q, uint16_t *sz)
+{
+    int c[DOR_G];
+    quant_group_affine(x, 255.0f, c, sz);
+    for (int i = 0; i < DOR_G; i++) q[i] = (uint8_t)c[i];
 }
 
 void dor_dequant_group_u8(const uint8_t *q, const uint16_t *sz, float *x)
@@ -170,6 +178,88 @@ void dor_dequant_group_u8(const uint8_t *q, const uint16_t *sz, float *x)
     float s = dor_f16_to_f32(sz[0]);
     float z = dor_f16_to_f32(sz[1]);
     for (int i = 0; i < DOR_G; i++) x[i] = s * ((float)q[i] - z);
+}
+
+/* UINT4 variant (Eq. integer_quantizer with b = 4, App. A.1): levels 0..15, FP16
+ * (s, z); the 32 codes are packed two per byte, value 2i in the low nibble of q[i]. */
+void dor_quant_group_u4(const float *x, uint8_t *q, uint16_t *sz)
+{
+    int c[DOR_G];
+    quant_group_affine(x, 15.0f, c, sz);
+    for (int i = 0; i < DOR_G / 2; i++) q[i] = (uint8_t)(c[2 * i] | (c[2 * i + 1] << 4));
+}
+
+void dor_dequant_group_u4(const uint8_t *q, const uint16_t *sz, float *x)
+{
+    float s = dor_f16_to_f32(sz[0]);
+    float z = dor_f16_to_f32(sz[1]);
+    for (int i = 0; i < DOR_G; i++) x[i] = s * ((float)((q[i / 2] >> (4 * (i & 1))) & 15) - z);
+}
+
+/* ------------------------------------------------------------------------- */
+/* FP8 E4M3: sign, 4 exponent bits (bias 7), 3 mantissa bits.  Exponent field */
+/* e = 1..15 gives 2^(e-7) (1 + m/8), e = 0 the subnormals 2^-6 (m/8); e = 15 */
+/* with m = 7 is NaN, so the largest finite magnitude is 448; no infinities.  */
+/* ------------------------------------------------------------------------- */
+
+float dor_e4m3_to_f32(uint8_t b)
+{
+    int sign = b >> 7, e = (b >> 3) & 15, m = b & 7;
+    double v;
+    if (e == 15 && m == 7) return NAN;
+    if (e == 0) v = ldexp(m / 8.0, -6);
+    else v = ldexp(1.0 + m / 8.0, e - 7);
+    return (float)(sign ? -v : v);
+}
+
+/* Nearest E4M3 value of a finite float, ties to the even mantissa, magnitudes of
+ * 448 and above saturating to 448. */
+uint8_t dor_f32_to_e4m3(float x)
+{
+    int sign = signbit(x) ? 1 : 0;
+    double a = fabs((double)x);
+    if (a >= 448.0) return (uint8_t)(sign << 7 | 0x7E);
+    int e = -6;                       /* binade of a (values below 2^-6 share the subnormal spacing) */
+    while (e < 8 && a >= ldexp(1.0, e + 1)) e++;
+    double quantum = ldexp(1.0, e - 3); /* spacing of E4M3 values in [2^e, 2^(e+1)) */
+    double v = nearbyint(a / quantum) * quantum; /* a / quantum is exact; ties to even */
+    if (v == 0.0) return (uint8_t)(sign << 7);
+    int ev = -6;
+    while (ev < 8 && v >= ldexp(1.0, ev + 1)) ev++;
+    int field, m;
+    if (v < ldexp(1.0, -6)) {
+        field = 0;
+        m = (int)(v / ldexp(1.0, -9));
+    } else {
+        field = ev + 7;
+        m = (int)((v / ldexp(1.0, ev) - 1.0) * 8.0);
+    }
+    return (uint8_t)(sign << 7 | field << 3 | m);
+}
+
+/* FP8 group quantizer (App. A.1, Eq. fp8_storage): one FP32 scale per 32 values,
+ *   s = max(max_i |x_i|, 1e-10) / 448,  q_i = E4M3(clip(x_i / s, -448, 448)),
+ *   Q(x_i) = s * FP32(q_i). */
+void dor_quant_group_e4m3(const float *x, uint8_t *q, float *s_out)
+{
+    float amax = 0.0f;
+    for (int i = 0; i < DOR_G; i++) {
+        float a = fabsf(x[i]);
+        if (a > amax) amax = a;
+    }
+    float s = (amax > 1e-10f ? amax : 1e-10f) / 448.0f;
+    for (int i = 0; i < DOR_G; i++) {
+        float t = x[i] / s;
+        if (t < -448.0f) t = -448.0f;
+        if (t > 448.0f) t = 448.0f;
+        q[i] = dor_f32_to_e4m3(t);
+    }
+    *s_out = s;
+}
+
+void dor_dequant_group_e4m3(const uint8_t *q, float s, float *x)
+{
+    for (int i = 0; i < DOR_G; i++) x[i] = s * dor_e4m3_to_f32(q[i]);
 }
 
 /* Per-row symmetric absmax INT8 with an FP32 scale and round-to-nearest-even:
@@ -202,6 +292,9 @@ void dor_dequant_row_s8(const int8_t *q, int n, float s, float *x)
 /* (the deployed low-tier mapping of App. A.1 / App. A.2).                   */
 /* ------------------------------------------------------------------------- */
 
+static int code_bits(int fmt) { return fmt == DOR_FMT_U4_H32 || fmt == DOR_FMT_U4 ? 4 : 8; }
+static int uses_h32(int fmt) { return fmt == DOR_FMT_U8_H32 || fmt == DOR_FMT_U4_H32; }
+
 static void lo_encode_row(int dv, int fmt, const float *x, void *codes_row, void *meta_row)
 {
     if (fmt == DOR_FMT_S8_ROW) {
@@ -210,9 +303,12 @@ static void lo_encode_row(int dv, int fmt, const float *x, void *codes_row, void
     }
     for (int g = 0; g < dv / DOR_G; g++) {
         float xt[DOR_G];
-        if (fmt == DOR_FMT_U8_H32) dor_hadamard32(x + g * DOR_G, xt);
+        if (uses_h32(fmt)) dor_hadamard32(x + g * DOR_G, xt);
         else memcpy(xt, x + g * DOR_G, sizeof xt);
-        dor_quant_group_u8(xt, (uint8_t *)codes_row + g * DOR_G, (uint16_t *)meta_row + 2 * g);
+        uint8_t *cg = (uint8_t *)codes_row + g * DOR_G * code_bits(fmt) / 8;
+        if (fmt == DOR_FMT_E4M3) dor_quant_group_e4m3(xt, cg, (float *)meta_row + g);
+        else if (code_bits(fmt) == 4) dor_quant_group_u4(xt, cg, (uint16_t *)meta_row + 2 * g);
+        else dor_quant_group_u8(xt, cg, (uint16_t *)meta_row + 2 * g);
     }
 }
 
@@ -224,8 +320,11 @@ static void lo_decode_row(int dv, int fmt, const void *codes_row, const void *me
     }
     for (int g = 0; g < dv / DOR_G; g++) {
         float xt[DOR_G];
-        dor_dequant_group_u8((const uint8_t *)codes_row + g * DOR_G, (const uint16_t *)meta_row + 2 * g, xt);
-        if (fmt == DOR_FMT_U8_H32) dor_hadamard32(xt, x + g * DOR_G);
+        const uint8_t *cg = (const uint8_t *)codes_row + g * DOR_G * code_bits(fmt) / 8;
+        if (fmt == DOR_FMT_E4M3) dor_dequant_group_e4m3(cg, ((const float *)meta_row)[g], xt);
+        else if (code_bits(fmt) == 4) dor_dequant_group_u4(cg, (const uint16_t *)meta_row + 2 * g, xt);
+        else dor_dequant_group_u8(cg, (const uint16_t *)meta_row + 2 * g, xt);
+        if (uses_h32(fmt)) dor_hadamard32(xt, x + g * DOR_G);
         else memcpy(x + g * DOR_G, xt, sizeof xt);
     }
 }
@@ -234,6 +333,8 @@ static int64_t meta_row_bytes(int dv, int fmt)
 {
     return fmt == DOR_FMT_S8_ROW ? 4 : (int64_t)(dv / DOR_G) * 4;
 }
+
+static int64_t code_row_bytes(int dv, int fmt) { return (int64_t)dv * code_bits(fmt) / 8; }
 
 void dor_qdq_rows(int64_t n_rows, int dv, int fmt, const float *x, float *out)
 {
@@ -257,7 +358,7 @@ void dor_qdq_rows(int64_t n_rows, int dv, int fmt, const float *x, float *out)
 static int check_args(int dk, int dv, int K, int fmt, const uint8_t *perm)
 {
     if (dk <= 0 || dk > 256 || dv <= 0 || dv > 4096 || dv % DOR_G) return -1;
-    if (K < 0 || K > dk || fmt < 0 || fmt > 2) return -1;
+    if (K < 0 || K > dk || fmt < 0 || fmt > 5) return -1;
     int seen[256] = {0};
     for (int i = 0; i < dk; i++) {
         if (perm[i] >= dk || seen[perm[i]]) return -1;
@@ -277,7 +378,7 @@ int dor_pack_head(int dk, int dv, int K, int fmt, const uint8_t *perm, const flo
             for (int j = 0; j < dv; j++) hi[(int64_t)i * dv + j] = dor_f32_to_f16(row[j]);
         } else {
             int r = i - K;
-            lo_encode_row(dv, fmt, row, (uint8_t *)codes + (int64_t)r * dv, (uint8_t *)meta + r * mrow);
+            lo_encode_row(dv, fmt, row, (uint8_t *)codes + r * code_row_bytes(dv, fmt), (uint8_t *)meta + r * mrow);
         }
     }
     return 0;
@@ -294,7 +395,7 @@ int dor_unpack_head(int dk, int dv, int K, int fmt, const uint8_t *perm, const u
             for (int j = 0; j < dv; j++) row[j] = dor_f16_to_f32(hi[(int64_t)i * dv + j]);
         } else {
             int r = i - K;
-            lo_decode_row(dv, fmt, (const uint8_t *)codes + (int64_t)r * dv, (const uint8_t *)meta + r * mrow, row);
+            lo_decode_row(dv, fmt, (const uint8_t *)codes + r * code_row_bytes(dv, fmt), (const uint8_t *)meta + r * mrow, row);
         }
     }
     return 0;
@@ -399,7 +500,7 @@ int dor_mixed_step_heads(int64_t n, int dk, int dv, int K, int fmt, int kind, co
                          const float *q, const float *k, const float *v, const float *g,
                          const float *beta, float *o)
 {
-    int64_t code_b = (int64_t)(dk - K) * dv * 1;
+    int64_t code_b = (int64_t)(dk - K) * code_row_bytes(dv, fmt);
     int64_t meta_b = (int64_t)(dk - K) * meta_row_bytes(dv, fmt);
     int64_t gdim = kind == DOR_GDN ? 1 : dk;
     for (int64_t h = 0; h < n; h++) {
@@ -418,7 +519,7 @@ int dor_prefill_chunk_heads(int64_t n, int dk, int dv, int K, int fmt, int kind,
                             const float *q, const float *k, const float *v, const float *g,
                             const float *beta, float *o)
 {
-    int64_t code_b = (int64_t)(dk - K) * dv * 1;
+    int64_t code_b = (int64_t)(dk - K) * code_row_bytes(dv, fmt);
     int64_t meta_b = (int64_t)(dk - K) * meta_row_bytes(dv, fmt);
     int64_t gdim = kind == DOR_GDN ? 1 : dk;
     for (int64_t h = 0; h < n; h++) {
@@ -448,7 +549,7 @@ void dor_delta_step_heads(int64_t n, int dk, int dv, int kind, float *S,
 int dor_pack_heads(int64_t n, int dk, int dv, int K, int fmt, const uint8_t *perm, const float *S,
                    uint16_t *hi, void *codes, void *meta)
 {
-    int64_t code_b = (int64_t)(dk - K) * dv;
+    int64_t code_b = (int64_t)(dk - K) * code_row_bytes(dv, fmt);
     int64_t meta_b = (int64_t)(dk - K) * meta_row_bytes(dv, fmt);
     for (int64_t h = 0; h < n; h++) {
         int rc = dor_pack_head(dk, dv, K, fmt, perm + h * dk, S + h * (int64_t)dk * dv,
@@ -462,7 +563,7 @@ int dor_pack_heads(int64_t n, int dk, int dv, int K, int fmt, const uint8_t *per
 int dor_unpack_heads(int64_t n, int dk, int dv, int K, int fmt, const uint8_t *perm, const uint16_t *hi,
                      const void *codes, const void *meta, float *S)
 {
-    int64_t code_b = (int64_t)(dk - K) * dv;
+    int64_t code_b = (int64_t)(dk - K) * code_row_bytes(dv, fmt);
     int64_t meta_b = (int64_t)(dk - K) * meta_row_bytes(dv, fmt);
     for (int64_t h = 0; h < n; h++) {
         int rc = dor_unpack_head(dk, dv, K, fmt, perm + h * dk, hi + h * (int64_t)K * dv,
