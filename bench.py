@@ -46,8 +46,9 @@ def algorithmic_bytes(w: wl.Workload, packed: bool = True) -> int:
     B, H, Hq, dk, dv, K = w.batch, w.heads, w.qk_heads, w.d_k, w.d_v, w.k_hi
     if packed and w.lo_format == 2:  # row-absmax INT8: one FP32 scale per row
         state = 2 * K * dv + (dk - K) * dv + 4 * (dk - K)
-    elif packed:
-        state = 2 * K * dv + (dk - K) * dv + 4 * (dk - K) * (dv // 32)
+    elif packed:  # codes (8 or 4 bits) + 4 bytes of metadata per 32-group
+        bits = 4 if w.lo_format in (3, 4) else 8
+        state = 2 * K * dv + (dk - K) * dv * bits // 8 + 4 * (dk - K) * (dv // 32)
     else:
         state = 4 * dk * dv
     esz = 2 if w.in_dtype == "bf16" else 4
@@ -460,7 +461,9 @@ def sweep_arm(steps: int, warmup: int):
         perm = torch.from_numpy(wl.random_perm(base)).to(dev)
         points = [(0, 1, "uniform int8 (no H32)"), (0, 0, "uniform int8 + H32")] + \
                  [(k, 0, "damp fp16 + int8 + H32") for k in wl.SWEEP_K_HI if k > 0] + \
-                 [(0, 2, "uniform int8 row-absmax"), (16, 2, "fp16 + int8 row-absmax")]
+                 [(0, 2, "uniform int8 row-absmax"), (16, 2, "fp16 + int8 row-absmax"),
+                  (0, 3, "uniform int4 + H32"), (0, 4, "uniform int4 (no H32)"), (0, 5, "uniform fp8 e4m3"),
+                  (16, 3, "fp16 + int4 + H32")]
         for k, fmt, name in points:
             w = wl.sweep(kind, k, fmt)
             L = damp.Layout(w.heads, w.qk_heads, w.d_k, w.d_v, k, fmt)

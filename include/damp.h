@@ -78,12 +78,19 @@ typedef enum {
     DAMP_LO_U8_AFFINE_G32_H32 = 0, /* UINT8 affine, G = 32 along d_v, FP16 (s, z), H_32 first:
                                       the paper's DAMP low tier ("INT8+Hadamard", 9.0 bits) */
     DAMP_LO_U8_AFFINE_G32 = 1,     /* the same without H_32 (the paper's "INT8" row, 9.0 bits) */
-    DAMP_LO_S8_ABSMAX_ROW = 2      /* per-row symmetric absmax INT8, one FP32 scale per row over
+    DAMP_LO_S8_ABSMAX_ROW = 2,     /* per-row symmetric absmax INT8, one FP32 scale per row over
                                       all d_v values: s = max|x|/127, q = sat_[-127,127](rne(x/s)),
                                       s = 0 -> q = 0; no H_32 (8 + 32/d_v bits).  A fallback
                                       for a low tier whose scales are left open, not the paper's
                                       format.  Its step sweeps each head twice (the row scale
                                       spans every value block) and is not tuned. */
+    DAMP_LO_U4_AFFINE_G32_H32 = 3, /* UINT4 affine (b = 4), G = 32, FP16 (s, z), H_32 first (5.0 bits) */
+    DAMP_LO_U4_AFFINE_G32 = 4,     /* the same without H_32 (the paper's "INT4" row, 5.0 bits) */
+    DAMP_LO_FP8_E4M3_G32 = 5       /* FP8 E4M3, G = 32, one FP32 scale per group, natural domain:
+                                      s = max(max|x|, 1e-10)/448, q = E4M3(clip(x/s, +-448)) (9.0 bits).
+                                      Formats 3-5 are the paper's comparison tiers (App. A.1): their
+                                      decode step runs as a one-token chunk of the prefill kernel
+                                      and is not tuned like formats 0 and 1. */
 } damp_lo_format;
 
 /* Element type of q, k and v. */
@@ -123,10 +130,13 @@ DAMP_API damp_status damp_validate_layout(const damp_layout *layout);
  * and holds, for value columns 32c .. 32c+31 of all d_k packed rows:
  *     [ceil(K_hi/2) FP16 row pairs x 128 B][(d_k-K_hi) x 32 codes][(d_k-K_hi) x 4 B metadata]
  *     [padding to 16 B]
- * FP16 row pair i interleaves rows 2i and 2i+1 column by column; the 16-byte chunks
- * inside each code row are permuted for conflict-free shared-memory access.  The
- * metadata word of a row is its (s, z) FP16 pair (formats 0, 1) or its FP32 row
- * scale (format 2, the same value in each of the head's d_v/32 records).  The byte order inside a record is private to libdamp: move logical
+ * FP16 row pair i interleaves rows 2i and 2i+1 column by column; code rows are stored
+ * chunk-major (16-byte chunk m of every row, then chunk m + 1), so that a warp's
+ * 128-bit accesses to one chunk of 32 consecutive rows are contiguous.  The
+ * metadata word of a row is its (s, z) FP16 pair (formats 0, 1, 3, 4), the FP32 group
+ * scale (format 5) or its FP32 row scale (format 2, the same value in each of the
+ * head's d_v/32 records).  4-bit formats store a code row in 16 bytes (value 2i in the
+ * low nibble of byte i).  The byte order inside a record is private to libdamp: move logical
  * tiers in and out with damp_pack_tiers / damp_unpack_tiers.
  * The pool pointer must be 16-byte aligned.
  */
@@ -223,7 +233,7 @@ DAMP_API damp_status damp_fp32_kda_decode_step(const damp_layout *layout, float 
  *   beta       float [B][T][H], 4-B aligned
  *   o          float [B][T][H][d_v]: o_t from the FP32 state after token t; rows past
  *              a row's length are not written.  Must not overlap the pool or inputs.
- * Other arguments as in damp_gdn_decode_step.  lo_format must be 0 or 1
+ * Other arguments as in damp_gdn_decode_step.  Any lo_format except 2
  * (DAMP_ERR_FORMAT for the row-absmax format).
  */
 DAMP_API damp_status damp_gdn_prefill_chunk(const damp_layout *layout, void *state, int64_t num_slots,
@@ -263,9 +273,12 @@ DAMP_API damp_status damp_dequantize_state(const damp_layout *layout, const void
 /*
  * Copy logical tiers into / out of packed slots, bit for bit (no arithmetic).
  *   hi     uint16 [batch][H][K_hi][d_v]            FP16 bit patterns (S_hi)
- *   codes  uint8  [batch][H][d_k-K_hi][d_v]        UINT8 codes (Q_lo); int8 for format 2
+ *   codes  uint8  [batch][H][d_k-K_hi][d_v]        UINT8 codes (Q_lo); int8 for format 2,
+ *                                                   E4M3 bit patterns for format 5,
+ *          uint8  [batch][H][d_k-K_hi][d_v/2]      two UINT4 codes per byte for formats 3, 4
  *   meta   uint16 [batch][H][d_k-K_hi][d_v/32][2]  FP16 (s, z) (M_lo); for format 2
- *          float  [batch][H][d_k-K_hi]             FP32 row scales, through the same pointer
+ *          float  [batch][H][d_k-K_hi]             FP32 row scales, for format 5
+ *          float  [batch][H][d_k-K_hi][d_v/32]     FP32 group scales, through the same pointer
  * All three 4-B aligned.  NULL is allowed for an empty tier.  Unpacking format 2
  * returns the scale copy of each row's first record.
  */

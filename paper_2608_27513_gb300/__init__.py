@@ -19,7 +19,8 @@ from dataclasses import dataclass
 from ._lib import DampLayout, DampLibraryError, lib
 
 __all__ = [
-    "Layout", "DampError", "DampLibraryError", "LO_U8_AFFINE_G32_H32", "LO_U8_AFFINE_G32", "LO_S8_ABSMAX_ROW",
+    "Layout", "DampError", "DampLibraryError", "LO_U8_AFFINE_G32_H32", "LO_U8_AFFINE_G32", "LO_S8_ABSMAX_ROW", "LO_U4_AFFINE_G32_H32",
+    "LO_U4_AFFINE_G32", "LO_FP8_E4M3_G32",
     "record_bytes", "slot_bytes", "bits_per_value", "new_state", "new_fp32_state",
     "gdn_decode_step", "kda_decode_step", "gdn_prefill_chunk", "kda_prefill_chunk", "calib_error_energy", "calib_log_decay", "calib_select", "u8_gdn_decode_step", "u8_kda_decode_step",
     "fp32_gdn_decode_step", "fp32_kda_decode_step", "quantize_state", "dequantize_state",
@@ -29,6 +30,9 @@ __all__ = [
 LO_U8_AFFINE_G32_H32 = 0
 LO_U8_AFFINE_G32 = 1
 LO_S8_ABSMAX_ROW = 2  # per-row symmetric absmax INT8, FP32 row scale
+LO_U4_AFFINE_G32_H32 = 3  # UINT4 affine G32 + H32
+LO_U4_AFFINE_G32 = 4  # UINT4 affine G32
+LO_FP8_E4M3_G32 = 5  # FP8 E4M3, FP32 scale per 32
 IN_BF16 = 0
 IN_FP32 = 1
 DEV_WAIT_TIMEOUT = 1
@@ -281,6 +285,12 @@ def unpack_tiers(layout, state, batch=None, slot_idx=None, num_slots=None, strea
     if layout.lo_format == LO_S8_ABSMAX_ROW:
         codes = torch.empty((B, H, dk - K, dv), dtype=torch.int8, device=dev)
         meta = torch.empty((B, H, dk - K), dtype=torch.float32, device=dev)
+    elif layout.lo_format in (LO_U4_AFFINE_G32_H32, LO_U4_AFFINE_G32):
+        codes = torch.empty((B, H, dk - K, dv // 2), dtype=torch.uint8, device=dev)
+        meta = torch.empty((B, H, dk - K, dv // 32, 2), dtype=torch.int16, device=dev)
+    elif layout.lo_format == LO_FP8_E4M3_G32:
+        codes = torch.empty((B, H, dk - K, dv), dtype=torch.uint8, device=dev)
+        meta = torch.empty((B, H, dk - K, dv // 32), dtype=torch.float32, device=dev)
     else:
         codes = torch.empty((B, H, dk - K, dv), dtype=torch.uint8, device=dev)
         meta = torch.empty((B, H, dk - K, dv // 32, 2), dtype=torch.int16, device=dev)

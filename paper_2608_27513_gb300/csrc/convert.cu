@@ -14,6 +14,7 @@
 // per-step path).
 #include "damp_common.cuh"
 #include "damp_internal.h"
+#include "formats.cuh"
 
 #include <algorithm>
 
@@ -38,8 +39,11 @@ struct ConvParams {
 
 enum ConvOp { kQuantize = 0, kDequantize = 1, kPackTiers = 2, kUnpackTiers = 3 };
 
-template <int R, bool HAD, int OP>
+template <int R, int FMT, int OP>
 __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
+    constexpr bool HAD = fmt_had(FMT);
+    constexpr bool U4 = fmt_u4(FMT);
+    constexpr int CB = U4 ? 16 : 32;  // code bytes per row and value block
     const int lane = threadIdx.x & 31;
     const int64_t gw = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int64_t nwt = ((int64_t)gridDim.x * blockDim.x) >> 5;
@@ -61,6 +65,10 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
         for (int i = 0; i < R; ++i) {
             const int u = lane + 32 * i;
             if (u < K) continue;  // FP16 rows: column-mapped loop below
+            const int r = u - K;
+            uint8_t *crec = rec + p.codes_off + lo_chunk_off(r, 0, lo);  // chunk 0 (the whole row for 4-bit codes)
+            uint8_t *crec1 = rec + p.codes_off + lo_chunk_off(r, 1, lo);
+            uint32_t *mrec = reinterpret_cast<uint32_t *>(rec + p.meta_off + 4 * r);
             if (OP == kQuantize || OP == kDequantize) {
                 const int n = p.perm[(int64_t)h * p.dk + u] & (p.dk - 1);  // d_k is a power of two
                 float *row = p.S + ((((int64_t)b * p.H + h) * p.dk + n) * p.dv + c * kG);
@@ -72,52 +80,59 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
                         x[2 * m] = make_float2(f.x, f.y);
                         x[2 * m + 1] = make_float2(f.z, f.w);
                     }
-                    {
-                        const int r = u - K;
-                        if (HAD) hadamard_pairs(x);
+                    if (HAD) hadamard_pairs(x);
+                    if (FMT == kFmtE4M3) {
+                        uint32_t w[8];
+                        const float sc = quantize_group_e4m3(x, w);
+                        *reinterpret_cast<uint4 *>(crec) = make_uint4(w[0], w[1], w[2], w[3]);
+                        *reinterpret_cast<uint4 *>(crec1) = make_uint4(w[4], w[5], w[6], w[7]);
+                        *mrec = __float_as_uint(sc);
+                    } else {
 #pragma unroll
                         for (int m = 0; m < 16; ++m) x[m] = mul2(x[m], splat2(kDown));  // working scale
-                        uint32_t w[8];
-                        const uint32_t sz = quantize_group(x, w);
-                        *reinterpret_cast<uint4 *>(rec + p.codes_off + lo_chunk_off(r, 0, lo)) =
-                            make_uint4(w[0], w[1], w[2], w[3]);
-                        *reinterpret_cast<uint4 *>(rec + p.codes_off + lo_chunk_off(r, 1, lo)) =
-                            make_uint4(w[4], w[5], w[6], w[7]);
-                        *reinterpret_cast<uint32_t *>(rec + p.meta_off + 4 * r) = sz;
+                        if (U4) {
+                            uint32_t w[4];
+                            *mrec = quantize_group_u4(x, w);
+                            *reinterpret_cast<uint4 *>(crec) = make_uint4(w[0], w[1], w[2], w[3]);
+                        } else {
+                            uint32_t w[8];
+                            *mrec = quantize_group(x, w);
+                            *reinterpret_cast<uint4 *>(crec) = make_uint4(w[0], w[1], w[2], w[3]);
+                            *reinterpret_cast<uint4 *>(crec1) = make_uint4(w[4], w[5], w[6], w[7]);
+                        }
                     }
                 } else {
-                    {
-                        const int r = u - K;
-                        const uint4 c0 = *reinterpret_cast<const uint4 *>(rec + p.codes_off + lo_chunk_off(r, 0, lo));
-                        const uint4 c1 = *reinterpret_cast<const uint4 *>(rec + p.codes_off + lo_chunk_off(r, 1, lo));
-                        const uint32_t sz = *reinterpret_cast<const uint32_t *>(rec + p.meta_off + 4 * r);
+                    const uint4 c0 = *reinterpret_cast<const uint4 *>(crec);
+                    if (U4) {
+                        const uint32_t w[4] = {c0.x, c0.y, c0.z, c0.w};
+                        dequantize_group_u4(w, *mrec, 1.0f, x);
+                    } else {
+                        const uint4 c1 = *reinterpret_cast<const uint4 *>(crec1);
                         const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-                        dequantize_group(w, sz, 1.0f, x);
-                        if (HAD) hadamard_pairs(x);
+                        if (FMT == kFmtE4M3) dequantize_group_e4m3(w, __uint_as_float(*mrec), 1.0f, x);
+                        else dequantize_group(w, *mrec, 1.0f, x);
                     }
+                    if (HAD) hadamard_pairs(x);
 #pragma unroll
                     for (int m = 0; m < 8; ++m)
                         reinterpret_cast<float4 *>(row)[m] = make_float4(x[2 * m].x, x[2 * m].y, x[2 * m + 1].x, x[2 * m + 1].y);
                 }
             } else {
                 // logical tiers <-> record, 32-bit words (FP16 rows: column-mapped loop below)
-                {
-                    const int r = u - K;
-                    uint32_t *crow = reinterpret_cast<uint32_t *>(p.codes + ((((int64_t)b * p.H + h) * lo + r) * p.dv + c * kG));
-                    uint32_t *mrow = reinterpret_cast<uint32_t *>(p.meta + ((((int64_t)b * p.H + h) * lo + r) * p.V + c) * 2);
+                const int64_t row_bytes = (int64_t)p.V * CB;
+                uint32_t *crow = reinterpret_cast<uint32_t *>(p.codes + ((((int64_t)b * p.H + h) * lo + r) * row_bytes + c * CB));
+                uint32_t *mrow = reinterpret_cast<uint32_t *>(p.meta) + (((int64_t)b * p.H + h) * lo + r) * p.V + c;
 #pragma unroll
-                    for (int m = 0; m < 2; ++m) {
-                        uint32_t *r4 = reinterpret_cast<uint32_t *>(rec + p.codes_off + lo_chunk_off(r, m, lo));
+                for (int m = 0; m < CB / 16; ++m) {
+                    uint32_t *r4 = reinterpret_cast<uint32_t *>(m ? crec1 : crec);
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            if (OP == kPackTiers) r4[e] = crow[4 * m + e];
-                            else crow[4 * m + e] = r4[e];
-                        }
+                    for (int e = 0; e < 4; ++e) {
+                        if (OP == kPackTiers) r4[e] = crow[4 * m + e];
+                        else crow[4 * m + e] = r4[e];
                     }
-                    uint32_t *mr = reinterpret_cast<uint32_t *>(rec + p.meta_off + 4 * r);
-                    if (OP == kPackTiers) *mr = *mrow;
-                    else *mrow = *mr;
                 }
+                if (OP == kPackTiers) *mrec = *mrow;
+                else *mrow = *mrec;
             }
         }
         // ---- FP16 rows, lane = column, two rows per 32-bit word ----
@@ -161,7 +176,7 @@ static cudaError_t launch_convert(const ConvArgs &a, cudaStream_t stream) {
     static uint32_t *cache[64];
     cudaError_t e = symbol_address_cached(&g_status_convert, cache, &p.status);
     if (e != cudaSuccess) return e;
-    const RecGeom rg = rec_geom(a.dk, a.K);
+    const RecGeom rg = rec_geom(a.dk, a.K, a.fmt);
     p.state = static_cast<uint8_t *>(a.state);
     p.num_slots = a.num_slots;
     p.slot_idx = a.slot_idx;
@@ -186,9 +201,17 @@ static cudaError_t launch_convert(const ConvArgs &a, cudaStream_t stream) {
     const int64_t want = (p.total_tiles + warps - 1) / warps;
     const int grid = (int)std::min<int64_t>(want, (int64_t)sm_count() * 8);
     void (*kern)(ConvParams) = nullptr;
-    const bool had = a.fmt == 0;
 #define DAMP_PICK(R_)                                                                          \
-    if (a.dk == 32 * R_) kern = had ? convert_kernel<R_, true, OP> : convert_kernel<R_, false, OP>;
+    if (a.dk == 32 * R_) {                                                                     \
+        switch (a.fmt) {                                                                       \
+            case kFmtU8H32: kern = convert_kernel<R_, kFmtU8H32, OP>; break;                  \
+            case kFmtU8: kern = convert_kernel<R_, kFmtU8, OP>; break;                        \
+            case kFmtU4H32: kern = convert_kernel<R_, kFmtU4H32, OP>; break;                  \
+            case kFmtU4: kern = convert_kernel<R_, kFmtU4, OP>; break;                        \
+            case kFmtE4M3: kern = convert_kernel<R_, kFmtE4M3, OP>; break;                    \
+            default: break;                                                                    \
+        }                                                                                      \
+    }
     DAMP_PICK(1)
     DAMP_PICK(2)
     DAMP_PICK(4)

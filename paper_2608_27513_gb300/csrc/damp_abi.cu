@@ -43,14 +43,12 @@ damp_status check_layout(const damp_layout *L) {
     if (L->d_k != 32 && L->d_k != 64 && L->d_k != 128) return DAMP_ERR_SHAPE;
     if (L->d_v < 32 || L->d_v > 1024 || L->d_v % 32) return DAMP_ERR_SHAPE;
     if (L->k_hi < 0 || L->k_hi > L->d_k) return DAMP_ERR_SHAPE;
-    if (L->lo_format != DAMP_LO_U8_AFFINE_G32_H32 && L->lo_format != DAMP_LO_U8_AFFINE_G32 &&
-        L->lo_format != DAMP_LO_S8_ABSMAX_ROW)
-        return DAMP_ERR_FORMAT;
+    if (L->lo_format < DAMP_LO_U8_AFFINE_G32_H32 || L->lo_format > DAMP_LO_FP8_E4M3_G32) return DAMP_ERR_FORMAT;
     return DAMP_OK;
 }
 
 int64_t slot_bytes_of(const damp_layout *L) {
-    return (int64_t)L->num_heads * (L->d_v / 32) * rec_geom(L->d_k, L->k_hi).bytes;
+    return (int64_t)L->num_heads * (L->d_v / 32) * rec_geom(L->d_k, L->k_hi, L->lo_format).bytes;
 }
 
 // Slots, batch rows and the pool's byte range; shared by every call on a pool.
@@ -70,6 +68,13 @@ damp_status check_pool(const void *state, int64_t num_slots, const int32_t *slot
 cudaError_t launch_step(const StepArgs &a, bool packed, cudaStream_t s) {
     if (!packed) return launch_fp32_step(a, s);
     if (a.fmt == DAMP_LO_S8_ABSMAX_ROW) return launch_rowabs_step(a, s);
+    if (a.fmt != DAMP_LO_U8_AFFINE_G32_H32 && a.fmt != DAMP_LO_U8_AFFINE_G32) {
+        // UINT4 and FP8 tiers: a decode step is a one-token chunk of the generic kernel
+        StepArgs one = a;
+        one.T = 1;
+        one.lengths = nullptr;
+        return a.kda ? launch_prefill_kda(one, s) : launch_prefill_gdn(one, s);
+    }
     return a.kda ? launch_packed_kda(a, s) : launch_packed_gdn(a, s);
 }
 
@@ -204,7 +209,7 @@ damp_status convert(const damp_layout *L, void *state, int64_t num_slots, const 
             overlap(rs, range_of(slot_idx, slot_idx ? B * 4 : 0)) || overlap(pool, range_of(perm, H * dk)))
             return DAMP_ERR_ALIAS;
     } else {
-        const int64_t nh = B * H * K * dv * 2, nc = B * H * (dk - K) * dv;
+        const int64_t nh = B * H * K * dv * 2, nc = B * H * (dk - K) * dv * fmt_code_bits(L->lo_format) / 8;
         const int64_t nm = B * H * (dk - K) * (L->lo_format == DAMP_LO_S8_ABSMAX_ROW ? 1 : dv / 32) * 4;
         if ((nh && !hi) || (nc && !codes) || (nm && !meta)) return DAMP_ERR_NULL;
         if ((hi && !aligned(hi, 4)) || (codes && !aligned(codes, 4)) || (meta && !aligned(meta, 4)))
@@ -310,7 +315,7 @@ damp_status damp_validate_layout(const damp_layout *layout) { return check_layou
 
 size_t damp_record_bytes(const damp_layout *layout) {
     if (check_layout(layout) != DAMP_OK) return 0;
-    return (size_t)rec_geom(layout->d_k, layout->k_hi).bytes;
+    return (size_t)rec_geom(layout->d_k, layout->k_hi, layout->lo_format).bytes;
 }
 
 size_t damp_slot_bytes(const damp_layout *layout) {
@@ -322,8 +327,9 @@ double damp_bits_per_value(const damp_layout *L) {
     if (check_layout(L) != DAMP_OK) return -1.0;
     const double hi = 16.0 * L->k_hi * L->d_v;
     const double lo = L->lo_format == DAMP_LO_S8_ABSMAX_ROW
-                          ? (8.0 * L->d_v + 32.0) * (double)(L->d_k - L->k_hi)             // int8 + one FP32 scale
-                          : (8.0 + 32.0 / 32.0) * (double)(L->d_k - L->k_hi) * L->d_v;  // UINT8 + FP16 (s,z) per 32
+                          ? (8.0 * L->d_v + 32.0) * (double)(L->d_k - L->k_hi)  // int8 + one FP32 scale
+                          : (fmt_code_bits(L->lo_format) + 32.0 / 32.0) * (double)(L->d_k - L->k_hi) *
+                                L->d_v;  // codes + 32 bits of metadata per 32 values
     return (hi + lo) / ((double)L->d_k * L->d_v);
 }
 
@@ -485,6 +491,10 @@ damp_status damp_device_status(uint32_t *status) {
     if (take_status_prefill_gdn(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     if (take_status_prefill_kda(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_prefill_gdn_x(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_prefill_kda_x(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     *status = all;
     return DAMP_OK;

@@ -25,8 +25,9 @@ enum : uint32_t { kDevWaitTimeout = 1u, kDevBadSlot = 2u };
 //              leaves the last high half zero.  A lane reads two FP16 rows of its
 //              column with one 32-bit load.
 //   codes:     (d_k-K) x 32 B, chunk-major: 16-B chunk m (columns 16m .. 16m+15)
-//              of lo row r at 16 * (m * (d_k-K) + r)
-//   meta:      (d_k-K) x 4 B      (s, z) as two binary16
+//              of lo row r at 16 * (m * (d_k-K) + r); 4-bit formats: one 16-B chunk
+//              (all 32 codes) per row at 16 * r
+//   meta:      (d_k-K) x 4 B      (s, z) as two binary16, or an FP32 scale
 // With one lane per lo row, a warp's 128-bit access to chunk m of 32 consecutive
 // rows covers 512 contiguous bytes: conflict-free in shared memory, whole
 // sectors in global memory.
@@ -35,10 +36,13 @@ struct RecGeom {
     int codes_off, meta_off, bytes;
 };
 
-__host__ __device__ inline RecGeom rec_geom(int d_k, int k_hi) {
+// code bits of a low-tier format: 4 for the UINT4 formats (3, 4), 8 for the others
+__host__ __device__ constexpr int fmt_code_bits(int fmt) { return fmt == 3 || fmt == 4 ? 4 : 8; }
+
+__host__ __device__ inline RecGeom rec_geom(int d_k, int k_hi, int fmt = 0) {
     RecGeom g;
     g.codes_off = 128 * ((k_hi + 1) / 2);
-    g.meta_off = g.codes_off + 32 * (d_k - k_hi);
+    g.meta_off = g.codes_off + 4 * fmt_code_bits(fmt) * (d_k - k_hi);
     g.bytes = (g.meta_off + 4 * (d_k - k_hi) + 15) & ~15;
     return g;
 }

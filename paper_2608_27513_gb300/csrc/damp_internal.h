@@ -51,6 +51,8 @@ cudaError_t launch_unpack_tiers(const ConvArgs &a, cudaStream_t s);
 // One prefill chunk on the packed state (formats 0 and 1).
 cudaError_t launch_prefill_gdn(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_prefill_kda(const StepArgs &a, cudaStream_t s);
+cudaError_t launch_prefill_gdn_x(const StepArgs &a, cudaStream_t s);  // formats 3, 4, 5
+cudaError_t launch_prefill_kda_x(const StepArgs &a, cudaStream_t s);
 // Offline key-channel selection (Sec. 5.1, Algorithm 1).
 cudaError_t launch_calib_error_energy(const float *S, int32_t batch, int32_t H, int32_t dk, int32_t dv, int32_t fmt,
                                       float *E_acc, cudaStream_t s);
@@ -70,6 +72,8 @@ cudaError_t take_status_convert(uint32_t *bits);
 cudaError_t take_status_rowabs(uint32_t *bits);
 cudaError_t take_status_prefill_gdn(uint32_t *bits);
 cudaError_t take_status_prefill_kda(uint32_t *bits);
+cudaError_t take_status_prefill_gdn_x(uint32_t *bits);
+cudaError_t take_status_prefill_kda_x(uint32_t *bits);
 
 // Streaming multiprocessors / opt-in shared memory per block of the current device (cached per device).
 int sm_count();

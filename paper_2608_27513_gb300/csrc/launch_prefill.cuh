@@ -5,16 +5,17 @@
 #include <algorithm>
 
 #include "damp_internal.h"
+#include "formats.cuh"
 #include "prefill.cuh"
 
 namespace damp {
 
 constexpr int kPrefillWarps = 8;
 
-template <bool KDA>
+template <bool KDA, int FMT>
 static cudaError_t launch_prefill_impl(const StepArgs &a, cudaStream_t stream, uint32_t *status) {
     const int V = a.dv / kG;
-    const RecGeom rg = rec_geom(a.dk, a.K);
+    const RecGeom rg = rec_geom(a.dk, a.K, FMT);
     const int esz = a.in_bf16 ? 2 : 4;
     auto up16 = [](int x) { return (x + 15) & ~15; };
     PrefillParams p{};
@@ -78,15 +79,9 @@ static cudaError_t launch_prefill_impl(const StepArgs &a, cudaStream_t stream, u
     const int smem = p.warp_smem * warps;
 
     void (*kern)(PrefillParams) = nullptr;
-    const bool had = a.fmt == 0;
     const int rl = (a.dk - a.K + 31) / 32;
 #define DAMP_PICK(RL_)                                                                             \
-    if (rl == RL_) {                                                                               \
-        if (had) kern = a.in_bf16 ? prefill_chunk_kernel<RL_, KDA, true, true>                     \
-                                  : prefill_chunk_kernel<RL_, KDA, true, false>;                   \
-        else kern = a.in_bf16 ? prefill_chunk_kernel<RL_, KDA, false, true>                        \
-                              : prefill_chunk_kernel<RL_, KDA, false, false>;                      \
-    }
+    if (rl == RL_) kern = a.in_bf16 ? prefill_chunk_kernel<RL_, KDA, FMT, true> : prefill_chunk_kernel<RL_, KDA, FMT, false>;
     DAMP_PICK(0)
     DAMP_PICK(1)
     DAMP_PICK(2)

@@ -19,6 +19,7 @@
 #pragma once
 
 #include "damp_common.cuh"
+#include "formats.cuh"
 
 namespace damp {
 
@@ -40,9 +41,10 @@ struct PrefillParams {
     uint32_t *status;
 };
 
-template <int RL, bool KDA, bool HAD, bool BF16>
+template <int RL, bool KDA, int FMT, bool BF16>
 __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillParams p) {
     constexpr int R = RL > 0 ? RL : 1;
+    constexpr bool HAD = fmt_had(FMT);
     extern __shared__ __align__(128) uint8_t smem[];
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
@@ -116,10 +118,16 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
         for (int i = 0; i < RL; ++i) {
             const int r = min(lane + 32 * i, lo - 1);
             const uint4 c0 = *reinterpret_cast<const uint4 *>(grec + p.codes_off + lo_chunk_off(r, 0, lo));
-            const uint4 c1 = *reinterpret_cast<const uint4 *>(grec + p.codes_off + lo_chunk_off(r, 1, lo));
             const uint32_t sz = *reinterpret_cast<const uint32_t *>(grec + p.meta_off + 4 * r);
-            const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-            dequantize_group(w, sz, kDown, x[i]);
+            if constexpr (fmt_u4(FMT)) {
+                const uint32_t w[4] = {c0.x, c0.y, c0.z, c0.w};
+                dequantize_group_u4(w, sz, kDown, x[i]);
+            } else {
+                const uint4 c1 = *reinterpret_cast<const uint4 *>(grec + p.codes_off + lo_chunk_off(r, 1, lo));
+                const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+                if constexpr (FMT == kFmtE4M3) dequantize_group_e4m3(w, __uint_as_float(sz), kDown, x[i]);
+                else dequantize_group(w, sz, kDown, x[i]);
+            }
         }
         for (int u = 0; u < K; u += 2) {
             const float2 f = h2_to_f2(*reinterpret_cast<const uint32_t *>(grec + hi_elem_off(u, lane)));
@@ -236,18 +244,38 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
 #pragma unroll
         for (int i = 0; i < RL; ++i) {
             const int r = lane + 32 * i;
-            float mn, mx, inv, zq;
-            minmax32(x[i], mn, mx);
-            const float sc = scale_of(mn, mx);
-            const uint32_t szw = sc == 0.0f ? affine_params_scaled(mn, mx, inv, zq) : affine_finish(sc, mn, inv, zq);
-            const float2 inv2 = splat2(inv * 0x1p-110f), zc2 = splat2(zq * 0x1p-149f);
-            uint32_t w[8];
+            if constexpr (fmt_u4(FMT)) {
+                uint32_t w[4];
+                const uint32_t szw = quantize_group_u4(x[i], w);
+                if (r < lo) {
+                    stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                    stg32(grec + p.meta_off + 4 * r, szw);
+                }
+            } else if constexpr (FMT == kFmtE4M3) {
+                float2 xn[16];
 #pragma unroll
-            for (int m = 0; m < 8; ++m) w[m] = encode4(x[i][2 * m], x[i][2 * m + 1], inv2, zc2);
-            if (r < lo) {
-                stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
-                stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
-                stg32(grec + p.meta_off + 4 * r, szw);
+                for (int j = 0; j < 16; ++j) xn[j] = mul2(x[i][j], splat2(kUp));  // natural domain (exact)
+                uint32_t w[8];
+                const float sc = quantize_group_e4m3(xn, w);
+                if (r < lo) {
+                    stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                    stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
+                    stg32(grec + p.meta_off + 4 * r, __float_as_uint(sc));
+                }
+            } else {
+                float mn, mx, inv, zq;
+                minmax32(x[i], mn, mx);
+                const float sc = scale_of(mn, mx);
+                const uint32_t szw = sc == 0.0f ? affine_params_scaled(mn, mx, inv, zq) : affine_finish(sc, mn, inv, zq);
+                const float2 inv2 = splat2(inv * 0x1p-110f), zc2 = splat2(zq * 0x1p-149f);
+                uint32_t w[8];
+#pragma unroll
+                for (int m = 0; m < 8; ++m) w[m] = encode4(x[i][2 * m], x[i][2 * m + 1], inv2, zc2);
+                if (r < lo) {
+                    stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                    stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
+                    stg32(grec + p.meta_off + 4 * r, szw);
+                }
             }
         }
         for (int u = 0; u < K; u += 2) {

@@ -1,5 +1,6 @@
 // prefill_gdn.cu -- instantiations of the prefill chunk kernel for
-// GDN (scalar decay per head).
+// GDN (scalar decay per head), UINT8 low tiers (formats 0 and 1); the 4-bit and FP8 tiers are
+// instantiated in prefill_gdn_x.cu.
 #include "launch_prefill.cuh"
 
 namespace damp {
@@ -7,11 +8,13 @@ namespace damp {
 static __device__ uint32_t g_status_prefill_gdn;
 
 cudaError_t launch_prefill_gdn(const StepArgs &a, cudaStream_t s) {
+    if (a.fmt != kFmtU8H32 && a.fmt != kFmtU8) return launch_prefill_gdn_x(a, s);
     static uint32_t *cache[64];
     uint32_t *status = nullptr;
     cudaError_t e = symbol_address_cached(&g_status_prefill_gdn, cache, &status);
     if (e != cudaSuccess) return e;
-    return launch_prefill_impl<false>(a, s, status);
+    return a.fmt == kFmtU8H32 ? launch_prefill_impl<false, kFmtU8H32>(a, s, status)
+                              : launch_prefill_impl<false, kFmtU8>(a, s, status);
 }
 
 cudaError_t take_status_prefill_gdn(uint32_t *bits) {

@@ -43,24 +43,33 @@ def inputs_to_dev(w: wl.Workload, inp: dict, dev) -> dict:
             "g": to_dev(inp["g"], dev), "beta": to_dev(inp["beta"], dev)}
 
 
+def _code_cols(w: wl.Workload) -> int:
+    return w.d_v // 2 if w.lo_format in (core.FMT_U4_H32, core.FMT_U4) else w.d_v
+
+
 def tiers_to_dev(w: wl.Workload, tiers, rows: int, dev):
     hi, codes, meta = tiers
     H, dk, dv, K = w.heads, w.d_k, w.d_v, w.k_hi
     if w.lo_format == core.FMT_S8_ROW:
         m = to_dev(meta.astype(np.float32).reshape(rows, H, dk - K), dev)
+    elif w.lo_format == core.FMT_E4M3:
+        m = to_dev(meta.astype(np.float32).reshape(rows, H, dk - K, dv // 32), dev)
     else:
         m = to_dev(meta.view(np.int16).reshape(rows, H, dk - K, dv // 32, 2), dev)
     return (to_dev(hi.view(np.int16).reshape(rows, H, K, dv), dev),
-            to_dev(codes.reshape(rows, H, dk - K, dv), dev), m)
+            to_dev(codes.reshape(rows, H, dk - K, _code_cols(w)), dev), m)
 
 
 def tiers_from_dev(w: wl.Workload, dev_tiers, units: int):
     hi, codes, meta = (t.cpu().numpy() for t in dev_tiers)
     H, dk, dv, K = w.heads, w.d_k, w.d_v, w.k_hi
+    hi = hi.view(np.uint16).reshape(units, K, dv)
     if w.lo_format == core.FMT_S8_ROW:
-        return (hi.view(np.uint16).reshape(units, K, dv), codes.view(np.int8).reshape(units, dk - K, dv),
-                meta.astype(np.float32).reshape(units, dk - K))
-    return (hi.view(np.uint16).reshape(units, K, dv), codes.reshape(units, dk - K, dv),
+        return hi, codes.view(np.int8).reshape(units, dk - K, dv), meta.astype(np.float32).reshape(units, dk - K)
+    if w.lo_format == core.FMT_E4M3:
+        return (hi, codes.view(np.uint8).reshape(units, dk - K, dv),
+                meta.view(np.float32).reshape(units, dk - K, dv // 32))
+    return (hi, codes.view(np.uint8).reshape(units, dk - K, _code_cols(w)),
             meta.view(np.uint16).reshape(units, dk - K, dv // 32, 2))
 
 
@@ -75,7 +84,7 @@ def oracle_step(w: wl.Workload, perm_units, tiers, u: dict):
     o = core.delta_step_heads(S, u["q"], u["k"], u["v"], u["g"], u["beta"], w.kind)
     new = core.pack_heads(perm_units, S, w.k_hi, w.lo_format)
     lo_rows = np.stack([S[i][perm_units[i][w.k_hi:]] for i in range(n)])  # [n, d_k-K, d_v] natural
-    if w.lo_format == core.FMT_U8_H32 and lo_rows.size:
+    if w.lo_format in (core.FMT_U8_H32, core.FMT_U4_H32) and lo_rows.size:
         lo_rows = core.hadamard32(lo_rows.reshape(-1, 32)).reshape(lo_rows.shape)
     return o, new, lo_rows
 
@@ -110,6 +119,14 @@ def compare_tiers(w: wl.Workload, ref, gpu, lo_pre, stats: CodeStats, what=""):
     if w.lo_format == core.FMT_S8_ROW:
         _compare_s8_rows(ref, gpu, lo_pre, stats, what)
         return
+    if w.lo_format == core.FMT_E4M3:
+        _compare_e4m3(ref, gpu, lo_pre, stats, what)
+        return
+    levels = 255.0
+    if w.lo_format in (core.FMT_U4_H32, core.FMT_U4):  # nibbles to one code per value
+        levels = 15.0
+        codes_r = np.stack([codes_r & 15, codes_r >> 4], axis=-1).reshape(*codes_r.shape[:-1], -1)
+        codes_g = np.stack([codes_g & 15, codes_g >> 4], axis=-1).reshape(*codes_g.shape[:-1], -1)
     n, lo, dv = codes_r.shape
     G = dv // 32
     cr = codes_r.reshape(n, lo, G, 32).astype(np.int64)
@@ -133,7 +150,7 @@ def compare_tiers(w: wl.Workload, ref, gpu, lo_pre, stats: CodeStats, what=""):
             f"{what}: scale differs by more than one binary16 ulp"
         assert np.all(np.abs(z_g - z_r)[meta_diff] <= 1), f"{what}: zero point differs by more than 1"
         xmin, xmax = x.min(axis=-1), x.max(axis=-1)
-        s32 = (xmax - xmin) / 255.0
+        s32 = (xmax - xmin) / levels
         sp = np.spacing(s32.astype(np.float16)).astype(np.float64)
         frac_s = np.abs((s32 / sp) - np.floor(s32 / sp) - 0.5)   # 0 at a binary16 rounding midpoint
         frac_z = np.abs((-xmin / s_r) - np.floor(-xmin / s_r) - 0.5)
@@ -172,6 +189,44 @@ def _compare_s8_rows(ref, gpu, lo_pre, stats: CodeStats, what):
     assert not bad.any(), f"{what}: codes differ away from a rounding tie at {np.argwhere(bad)[:5].tolist()}"
     stats.codes += d.size
     stats.mismatched += int((d > 0).sum())
+    stats.groups += s_r.size
+    stats.meta_mismatched += int((s_r != s_g).sum())
+
+
+_E4M3 = None
+
+
+def _e4m3_magnitudes():
+    global _E4M3
+    if _E4M3 is None:
+        _E4M3 = np.array([core.e4m3_to_f32(c) for c in range(0x7F)], np.float64)
+    return _E4M3
+
+
+def _compare_e4m3(ref, gpu, lo_pre, stats: CodeStats, what):
+    """FP8 E4M3 groups: scales within S8_SCALE_REL (max|x| / 448 of values that may differ
+    by float ordering); a code may differ only where the oracle's x/s lies within TIE (in
+    units of the local E4M3 spacing) of the midpoint of two neighbouring values, and then
+    by that one step."""
+    _, codes_r, s_r = ref
+    _, codes_g, s_g = gpu
+    s_r64, s_g64 = s_r.astype(np.float64), s_g.astype(np.float64)
+    assert np.all(np.abs(s_g64 - s_r64) <= S8_SCALE_REL * np.abs(s_r64) + 1e-30), f"{what}: an FP8 scale differs"
+    mags = _e4m3_magnitudes()
+    n, lo, dv = codes_r.shape
+    vr = np.where(codes_r & 0x80, -1.0, 1.0) * mags[np.minimum(codes_r & 0x7F, 0x7E)]
+    vg = np.where(codes_g & 0x80, -1.0, 1.0) * mags[np.minimum(codes_g & 0x7F, 0x7E)]
+    diff = codes_r != codes_g
+    if diff.any():
+        t = np.abs(lo_pre.astype(np.float64) / np.repeat(s_r64, 32, axis=-1))
+        k = np.clip(np.searchsorted(mags, np.minimum(t, 448.0)), 1, mags.size - 1)
+        gap = mags[k] - mags[k - 1]
+        mid = (mags[k] + mags[k - 1]) / 2
+        near = np.abs(t - mid) < TIE * gap
+        bad = diff & ~(near & (np.abs(vr - vg) <= gap * 1.0001))
+        assert not bad.any(), f"{what}: FP8 codes differ away from a rounding tie at {np.argwhere(bad)[:5].tolist()}"
+    stats.codes += codes_r.size
+    stats.mismatched += int(diff.sum())
     stats.groups += s_r.size
     stats.meta_mismatched += int((s_r != s_g).sum())
 

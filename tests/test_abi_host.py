@@ -67,12 +67,20 @@ def test_record_geometry_and_bits(L):
             lay = _layout(k_hi=K, lo_format=2, d_v=dv)
             assert damp.bits_per_value(lay) == pytest.approx(core.bits_per_value(128, dv, K, core.FMT_S8_ROW), rel=1e-12)
             assert damp.record_bytes(lay) == damp.record_bytes(_layout(k_hi=K, d_v=dv))
+    # 4-bit and FP8 tiers: bits from the oracle's logical tiers; 4-bit code rows take 16 bytes
+    for fmt in (3, 4, 5):
+        for K in (0, 10, 16):
+            lay = _layout(k_hi=K, lo_format=fmt)
+            assert damp.bits_per_value(lay) == pytest.approx(core.bits_per_value(128, 128, K, fmt), rel=1e-12)
+            code_row = 16 if fmt in (3, 4) else 32
+            logical = 128 * ((K + 1) // 2) + (code_row + 4) * (128 - K)
+            assert damp.record_bytes(lay) == (logical + 15) // 16 * 16
     assert damp.bits_per_value(_layout(k_hi=0)) == pv["bits_int8_hadamard"]
 
 
 @pytest.mark.parametrize("kw,status", [
     (dict(d_k=96), 2), (dict(d_k=256), 2), (dict(d_v=48), 2), (dict(d_v=2048), 2), (dict(k_hi=129), 2),
-    (dict(k_hi=-1), 2), (dict(num_qk_heads=5), 2), (dict(num_heads=0), 2), (dict(lo_format=3), 5)])
+    (dict(k_hi=-1), 2), (dict(num_qk_heads=5), 2), (dict(num_heads=0), 2), (dict(lo_format=6), 5)])
 def test_layout_validation(L, kw, status):
     c = _layout(**kw).c()
     assert L.damp_validate_layout(ctypes.byref(c)) == status
@@ -117,7 +125,7 @@ def test_step_rejects_bad_arguments_before_launch(L):
     assert _call_step(L, lay, fb, o=off(0, 4096)) == 4                # o inside the pool
     assert _call_step(L, lay, fb, q=off(0, 1 << 12)) == 4             # an input inside the pool
     assert _call_step(L, lay, fb, o=fb[2]) == 4                       # o over q
-    assert _call_step(L, _layout(lo_format=3), fb) == 5
+    assert _call_step(L, _layout(lo_format=6), fb) == 5
     c = _layout(k_hi=8).c()
     assert L.damp_u8_kda_decode_step(ctypes.byref(c), *[fb[0], 4, None, 4, fb[1], fb[2], fb[3], fb[4], fb[5],
                                                         fb[6], fb[7], 0, None]) == 2

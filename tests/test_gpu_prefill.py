@@ -54,7 +54,7 @@ def _oracle_chunk(w, perm_units, tiers, u, lens_units):
                           core.unpack_heads(perm_units, *core.pack_heads(perm_units, S, w.k_hi, w.lo_format),
                                             w.k_hi, w.lo_format, w.d_k, w.d_v)[lens_units > 0])
     lo_rows = np.stack([S[i][perm_units[i][w.k_hi:]] for i in range(n)])
-    if w.lo_format == core.FMT_U8_H32 and lo_rows.size:
+    if w.lo_format in (core.FMT_U8_H32, core.FMT_U4_H32) and lo_rows.size:
         lo_rows = core.hadamard32(lo_rows.reshape(-1, 32)).reshape(lo_rows.shape)
     return o, new, lo_rows
 
