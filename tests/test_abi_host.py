@@ -174,6 +174,18 @@ def test_calibration_calls_reject_bad_arguments(L):
     assert sel(perm=off(2, 16)) == 4                                                  # pi over the scores
 
 
+def test_a_launch_failure_is_reported_not_raised(L):
+    """With no CUDA device, a call that passes every host check returns DAMP_ERR_CUDA
+    (the launcher's error, mapped at the boundary).  Skipped where a GPU is visible: the
+    fake host addresses must never reach a kernel."""
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is visible")
+    fb = FakeBuffers()
+    assert _call_step(L, _layout(), fb) == 6
+    assert L.damp_status_string(6).decode().startswith("DAMP_ERR_CUDA")
+
+
 def test_gdn_gate_alignment_is_4_bytes(L):
     fb = FakeBuffers()
     c = _layout().c()
