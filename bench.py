@@ -185,6 +185,9 @@ def make_line(r: dict, steps: int, warmup: int, world: int) -> dict:
                      "frac_of_8TBs": achieved_gbs / 8000.0,
                      "traffic": ncu_traffic("packed_step_kda_b256"),
                      "kernel": "packed_step_kernel<RL=4,d_k=128,K_hi=10,KDA,H32,BF16>", "algorithmic_bytes": bytes_step},
+        "cuda_graph": ({"us_per_step": r["graph_ms"] * 1e3,
+                        "note": "the same steps captured in one CUDA graph of 4 launches and replayed"}
+                       if r.get("graph_ms") else None),
         "fp32_state_kernel": {"us_per_step": r["fp32_launch_ms"] * 1e3,
                               "achieved_gbs": bytes_fp32 / (r["fp32_launch_ms"] * 1e-3) / 1e9,
                               "bytes_per_step": bytes_fp32,
@@ -286,6 +289,28 @@ def gpu_arm(args, rank: int, world: int):
     if damp.device_status() != 0:
         raise RuntimeError("device status word set during the timed region")
 
+    # ---- the same steps replayed from a CUDA graph (one graph of 2 * POOLS steps) ----
+    gstream = torch.cuda.Stream(dev)
+    gstream.wait_stream(stream)
+    graph = torch.cuda.CUDAGraph()
+    per_graph = 2 * POOLS
+    with torch.cuda.graph(graph, stream=gstream):
+        for i in range(per_graph):
+            run_packed(i, o)
+    stream.wait_stream(gstream)
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize()
+    n_graph = max(args.steps // per_graph, 5)
+    g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    g0.record(stream)
+    for _ in range(n_graph):
+        graph.replay()
+    g1.record(stream)
+    torch.cuda.synchronize()
+    graph_ms = max_over_ranks_(g0.elapsed_time(g1) / (n_graph * per_graph))
+    del graph
+
     # ---- the in-house FP32-state kernel on the same inputs (speedup reference) ----
     fp_steps = max(args.steps // 4, 10)
     fp_total, fp_launch = timed(run_fp32, fp_steps, max(args.warmup, 3))
@@ -348,7 +373,7 @@ def gpu_arm(args, rank: int, world: int):
         dist.barrier()
     e2e_total = max_over_ranks_(e0.elapsed_time(e1))
     return {
-        "w": w, "total_ms": total_ms, "launch_ms": launch_ms, "fp32_launch_ms": fp_launch,
+        "w": w, "total_ms": total_ms, "launch_ms": launch_ms, "fp32_launch_ms": fp_launch, "graph_ms": graph_ms,
         "e2e_ms": e2e_total / e2e_steps, "h2d": h2d, "d2h": d2h, "clocks": clk.summary(),
         "bits": damp.bits_per_value(L), "dev_name": torch.cuda.get_device_name(dev),
     }
