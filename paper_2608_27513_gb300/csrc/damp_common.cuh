@@ -109,21 +109,8 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t
         : "memory");
 }
 
-// 1-D bulk copy shared -> global, tracked by bulk groups.
-__device__ __forceinline__ void bulk_s2g(void *dst, uint32_t src, uint32_t bytes) {
-    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(src), "r"(bytes)
-                 : "memory");
-}
-__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_read_all() {
-    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-}
-__device__ __forceinline__ void bulk_wait_read_all_but_newest() {
-    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
-}
-__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-
-// Generic-proxy writes to shared memory become visible to the async proxy (bulk store).
+// Orders this thread's generic-proxy accesses of shared memory before later
+// async-proxy accesses (a bulk copy into the same stage).
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -171,12 +158,6 @@ __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
     return d;
 }
 
-// per-lane clamp of two signed 16-bit lanes to [0, 255]
-__device__ __forceinline__ uint32_t clamp_u8x2(uint32_t v) {
-    uint32_t d;
-    asm("min.relu.s16x2 %0, %1, %2;" : "=r"(d) : "r"(v), "r"(0x00FF00FFu));
-    return d;
-}
 
 __device__ __forceinline__ float fmin3(float a, float b, float c) {
     float d;

@@ -26,9 +26,13 @@
 // o~_lo do (a 5-step butterfly across the warp's lanes).
 //
 // Pipeline: a persistent grid; every warp walks a contiguous range of tiles.
-// Lane 0 keeps NSTAGE-1 tiles in flight with 1-D bulk copies (TMA engine) into a
-// per-warp ring of shared-memory stages, each with its own mbarrier; the updated
-// record is written back into its stage and returned with a bulk store.
+// Lane 0 keeps NSTAGE tile records in flight with 1-D bulk copies (TMA engine)
+// into a per-warp ring of shared-memory stages, each with its own mbarrier, and
+// refills a stage as soon as the warp has read it; the per-(slot, head) operands
+// come in by per-lane cp.async one head ahead.  The updated record goes straight
+// from registers to HBM with 128-bit stores (chunk-major code rows make them whole
+// sectors).  Layouts with d_k = 128 and the K_hi values the launcher lists compile
+// with the record geometry and the FP16-row loops fixed (KC, DKC below).
 #pragma once
 
 #include "damp_common.cuh"
@@ -60,12 +64,6 @@ constexpr int kPartOff = 64;                              // after NSTAGE (<= 8)
 constexpr int kDvecOff = kPartOff + 32 * kPartStride * 4; // 32 floats: H d for the low tier
 constexpr int kHopsOff = kDvecOff + 32 * 4;               // FP16-row operands, 32 B per row pair
 __host__ __device__ constexpr int scratch_bytes(int k_hi) { return kHopsOff + 16 * ((k_hi + 7) & ~7); }
-
-__device__ __forceinline__ float h16_to_f32(uint32_t h) { return __half2float(__ushort_as_half((unsigned short)h)); }
-
-__device__ __forceinline__ void sts16(uint32_t a, unsigned short v) {
-    asm volatile("st.shared.b16 [%0], %1;" ::"r"(a), "h"(v) : "memory");
-}
 
 // (batch row, head, value block) of a tile index, advanced without divisions.
 struct Cursor {

@@ -11,7 +11,7 @@
 namespace damp {
 
 // Launch shape: one CTA per SM with kPackedWarps warps; every warp owns a
-// contiguous range of tiles and keeps kPackedStages-1 tile loads in flight.
+// contiguous range of tiles and keeps kPackedStages tile loads in flight.
 constexpr int kPackedWarps = 8;
 constexpr int kPackedStages = 3;
 
