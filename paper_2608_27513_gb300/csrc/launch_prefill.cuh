@@ -44,16 +44,12 @@ static cudaError_t launch_prefill_impl(const StepArgs &a, cudaStream_t stream, u
     p.slot_bytes = (int64_t)a.H * V * rg.bytes;
     p.total_tiles = (int64_t)a.batch * a.H * V;
     p.status = status;
-    // per-warp shared memory: [column-sum buffer][H d][FP16-row operands][pi][FP16 rows][2 token buffers]
+    // per-warp shared memory: [column-sum buffer][H d][pi][2 token buffers]
     int off = 32 * kPartStride * 4;
     p.dvec_off = off;
     off += 32 * 4;
-    p.hops_off = off;
-    off += up16(16 * a.K);
     p.perm_off = off;
     off += up16(a.dk);
-    p.hbuf_off = off;
-    off += 128 * a.K;
     p.ops_off = off;
     int t = 0;
     p.off_q = t;
@@ -79,13 +75,10 @@ static cudaError_t launch_prefill_impl(const StepArgs &a, cudaStream_t stream, u
     const int smem = p.warp_smem * warps;
 
     void (*kern)(PrefillParams) = nullptr;
-    const int rl = (a.dk - a.K + 31) / 32;
-#define DAMP_PICK(RL_)                                                                             \
-    if (rl == RL_) kern = a.in_bf16 ? prefill_chunk_kernel<RL_, KDA, FMT, true> : prefill_chunk_kernel<RL_, KDA, FMT, false>;
-    DAMP_PICK(0)
+#define DAMP_PICK(R_)                                                                              \
+    if (a.dk == 32 * R_) kern = a.in_bf16 ? prefill_chunk_kernel<R_, KDA, FMT, true> : prefill_chunk_kernel<R_, KDA, FMT, false>;
     DAMP_PICK(1)
     DAMP_PICK(2)
-    DAMP_PICK(3)
     DAMP_PICK(4)
 #undef DAMP_PICK
     if (!kern) return cudaErrorInvalidValue;

@@ -6,16 +6,19 @@
 //
 // Work unit = tile (slot, head, value block c): all d_k rows x 32 columns, for the
 // whole chunk of that slot.  One warp owns a tile from load to store, so its FP32
-// state never leaves the SM between tokens:
-//   low-tier rows  lane l holds rows l, l+32, ... (32 columns each) in registers,
-//                  in the H_32 domain and scaled by 2^-39 as in the decode step
-//                  (decay and the rank-1 update are row/column scalings there too);
-//   FP16 rows      lane j holds column j of every FP16 row in shared memory as FP32.
-// Per token: decay, partial sums of r~ = S~^T k and p~ = S~^T q, column sums, the
-// lane butterflies for r, d, p (as in the decode step), o_t, and the update.  The
-// next token's operands (q, k, g, v block, beta) stream into a double buffer by
-// cp.async while the current token runs.  After the last token the tile is
-// requantized like a decode step and stored with plain 128-bit stores.
+// state never leaves the SM between tokens.  Lane l holds packed rows l, l+32, ...
+// (32 columns each) in registers, FP16 rows and low-tier rows alike, all scaled by
+// 2^-39 as in the decode step.  With the H_32 formats every row is kept in the
+// transformed domain S~ = S H while the chunk runs: the low-tier rows are stored
+// that way, and the FP16 rows are transformed once on load and back once on store
+// (H_32 is symmetric and orthonormal, and decay and the rank-1 update are
+// row/column scalings that commute with it), so the per-token work is the same for
+// every row: decay, partial sums of r~ = S~^T k and p~ = S~^T q, column sums, the
+// lane butterflies r = H r~, p = H p~, H d, o_t and the update.  The next token's
+// operands (q, k, g, v block, beta) stream into a double buffer by cp.async while
+// the current token runs.  After the last token the low-tier rows are requantized
+// like a decode step and the FP16 rows rounded once; both go back with plain
+// stores.
 #pragma once
 
 #include "damp_common.cuh"
@@ -36,14 +39,64 @@ struct PrefillParams {
     int32_t rec_bytes, codes_off, meta_off;
     int64_t slot_bytes, total_tiles;
     // per-warp shared memory
-    int32_t warp_smem, dvec_off, hops_off, perm_off, hbuf_off, ops_off, ops_bytes;
+    int32_t warp_smem, dvec_off, perm_off, ops_off, ops_bytes;
     int32_t off_q, off_k, off_g, off_v, off_beta;
     uint32_t *status;
 };
 
-template <int RL, bool KDA, int FMT, bool BF16>
+// FP16 row u of a record -> 32 FP32 values (component j of the group is y[j/2].x
+// or .y).  Row pair u>>1 holds one 32-bit word per column, row u in half u & 1.
+__device__ __forceinline__ void load_hi_row(const uint8_t *grec, int u, float2 (&y)[16]) {
+    const uint8_t *pr = grec + hi_elem_off(u & ~1, 0);
+    const uint32_t sel = (u & 1) ? 0x7632u : 0x5410u;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+        const uint4 w = *reinterpret_cast<const uint4 *>(pr + 16 * q);
+        y[2 * q] = h2_to_f2(prmt(w.x, w.y, sel));
+        y[2 * q + 1] = h2_to_f2(prmt(w.z, w.w, sel));
+    }
+}
+
+// Store FP16 row u (binary16 pairs own[m] = columns 2m, 2m+1) into its row pair.
+// Lanes 2i and 2i+1 (u = lane + 32 i) hold the two rows of a pair: they swap half
+// of their words so that the even lane writes columns 0..15 and the odd lane
+// columns 16..31, each as 64 contiguous bytes.  Every lane of the warp must call
+// this (shuffles); pairs past the FP16 tier store nothing, and the odd half of the
+// last pair of an odd K (row K, padding) is written as 0.
+__device__ __forceinline__ void store_hi_row(uint8_t *grec, int u, int K, int lane, const uint32_t (&own)[16]) {
+    const bool odd = lane & 1;
+    uint32_t recv[8];
+#pragma unroll
+    for (int m = 0; m < 8; ++m) recv[m] = __shfl_xor_sync(kFull, odd ? own[m] : own[8 + m], 1);
+    const int ue = u & ~1;  // even row of the pair
+    if (ue >= K) return;
+    const bool pad = ue + 1 >= K;
+    uint32_t w[16];
+#pragma unroll
+    for (int m = 0; m < 8; ++m) {
+        const uint32_t ev = odd ? recv[m] : own[m];
+        const uint32_t od = pad ? 0u : (odd ? own[8 + m] : recv[m]);
+        w[2 * m] = prmt(ev, od, 0x5410u);
+        w[2 * m + 1] = prmt(ev, od, 0x7632u);
+    }
+    uint8_t *pr = grec + hi_elem_off(u & ~1, 0) + (odd ? 64 : 0);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) stg128(pr + 16 * q, make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]));
+}
+
+// the 32-vector H d of the pending update (lane j wrote component j)
+__device__ __forceinline__ void load_dvec(uint32_t dvec, float2 (&d)[16]) {
+#pragma unroll
+    for (int jj = 0; jj < 8; ++jj) {
+        const uint4 w = lds128(dvec + 16 * jj);
+        d[2 * jj] = make_float2(__uint_as_float(w.x), __uint_as_float(w.y));
+        d[2 * jj + 1] = make_float2(__uint_as_float(w.z), __uint_as_float(w.w));
+    }
+}
+
+// R = d_k / 32: packed rows per lane (row u = lane + 32 i), fixed at compile time.
+template <int R, bool KDA, int FMT, bool BF16>
 __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillParams p) {
-    constexpr int R = RL > 0 ? RL : 1;
     constexpr bool HAD = fmt_had(FMT);
     extern __shared__ __align__(128) uint8_t smem[];
     const int lane = threadIdx.x & 31;
@@ -53,12 +106,11 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
     const uint32_t ws = smem_u32(smem) + (uint32_t)(warp * p.warp_smem);
     const uint32_t part = ws;  // column_sum2 buffer at the start of the warp's area
     const uint32_t dvec = ws + p.dvec_off;
-    const uint32_t hops = ws + p.hops_off;
     const uint32_t perm_s = ws + p.perm_off;
-    const uint32_t hbuf = ws + p.hbuf_off;
     const uint32_t ops0 = ws + p.ops_off;
     const int esz = BF16 ? 2 : 4;
-    const int K = p.K, dk = p.dk, lo = dk - K, H = p.H, V = p.V, T = p.T;
+    constexpr int dk = 32 * R;
+    const int K = p.K, lo = dk - K, H = p.H, V = p.V, T = p.T;
 
     const int64_t gw = (int64_t)blockIdx.x * nw + warp;
     const int64_t nwt = (int64_t)gridDim.x * nw;
@@ -112,156 +164,151 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
         for (int ci = lane; ci < dk / 16; ci += 32) cp_async16(perm_s + 16 * ci, p.perm + (int64_t)h * dk + 16 * ci);
         load_token(b, h, c, 0, ops0);
 
-        // ---- reconstruct the tile in FP32 (undecayed; low tier in the H domain at 2^-39) ----
+        // ---- reconstruct the tile in FP32, undecayed, scaled by 2^-39; with H_32 in
+        //      the transformed domain (FP16 rows transformed here) ----
+        // low-tier words of every row slot first (rows of the FP16 tier load a valid
+        // low row and ignore it), so that all loads are in flight before the branches
         float2 x[R][16];
+        uint4 cw0[R], cw1[R];
+        uint32_t szw[R];
 #pragma unroll
-        for (int i = 0; i < RL; ++i) {
-            const int r = min(lane + 32 * i, lo - 1);
-            const uint4 c0 = *reinterpret_cast<const uint4 *>(grec + p.codes_off + lo_chunk_off(r, 0, lo));
-            const uint32_t sz = *reinterpret_cast<const uint32_t *>(grec + p.meta_off + 4 * r);
+        for (int i = 0; i < R; ++i) {
+            const int r = lo > 0 ? min(max(lane + 32 * i - K, 0), lo - 1) : 0;
+            const uint8_t *crow = grec + (lo > 0 ? p.codes_off : 0);  // lo = 0: a valid dummy address
+            cw0[i] = *reinterpret_cast<const uint4 *>(crow + lo_chunk_off(r, 0, lo));
+            cw1[i] = fmt_u4(FMT) ? cw0[i] : *reinterpret_cast<const uint4 *>(crow + lo_chunk_off(r, 1, lo));
+            szw[i] = *reinterpret_cast<const uint32_t *>(grec + (lo > 0 ? p.meta_off + 4 * r : 0));
+        }
+#pragma unroll
+        for (int i = 0; i < R; ++i) {
+            const int u = lane + 32 * i;
+            if (u < K) {
+                load_hi_row(grec, u, x[i]);
+                if (HAD) hadamard_pairs(x[i]);
+#pragma unroll
+                for (int j = 0; j < 16; ++j) x[i][j] = mul2(x[i][j], splat2(kDown));  // exact
+                continue;
+            }
             if constexpr (fmt_u4(FMT)) {
-                const uint32_t w[4] = {c0.x, c0.y, c0.z, c0.w};
-                dequantize_group_u4(w, sz, kDown, x[i]);
+                const uint32_t w[4] = {cw0[i].x, cw0[i].y, cw0[i].z, cw0[i].w};
+                dequantize_group_u4(w, szw[i], kDown, x[i]);
             } else {
-                const uint4 c1 = *reinterpret_cast<const uint4 *>(grec + p.codes_off + lo_chunk_off(r, 1, lo));
-                const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-                if constexpr (FMT == kFmtE4M3) dequantize_group_e4m3(w, __uint_as_float(sz), kDown, x[i]);
-                else dequantize_group(w, sz, kDown, x[i]);
+                const uint32_t w[8] = {cw0[i].x, cw0[i].y, cw0[i].z, cw0[i].w, cw1[i].x, cw1[i].y, cw1[i].z, cw1[i].w};
+                if constexpr (FMT == kFmtE4M3) dequantize_group_e4m3(w, __uint_as_float(szw[i]), kDown, x[i]);
+                else dequantize_group(w, szw[i], kDown, x[i]);
             }
         }
-        for (int u = 0; u < K; u += 2) {
-            const float2 f = h2_to_f2(*reinterpret_cast<const uint32_t *>(grec + hi_elem_off(u, lane)));
-            sts32(hbuf + 4 * (32 * u + lane), __float_as_uint(f.x));
-            if (u + 1 < K) sts32(hbuf + 4 * (32 * (u + 1) + lane), __float_as_uint(f.y));
-        }
 
+        // The rank-1 update of token t is applied at the start of token t+1, in the
+        // same pass over the registers as that token's decay (and after the loop for
+        // the last token): H d of the pending update waits in dvec, beta k in bkp.
+        float2 bkp[R];
+#pragma unroll
+        for (int i = 0; i < R; ++i) bkp[i] = make_float2(0.f, 0.f);
+        sts32(dvec + 4 * lane, 0u);
         for (int tok = 0; tok < Tb; ++tok) {
             const uint32_t ob = ops0 + (uint32_t)((tok & 1) * p.ops_bytes);
             cp_async_wait_all();
             __syncwarp();
             if (tok + 1 < Tb) load_token(b, h, c, tok + 1, ops0 + (uint32_t)(((tok + 1) & 1) * p.ops_bytes));
 
-            // ---- operands in calibrated order ----
+            // ---- operands of this lane's rows, in calibrated order ----
             const float beta = ldsf(ob + p.off_beta);
             const float alpha = KDA ? 0.f : expf(ldsf(ob + p.off_g));
-            auto chan = [&](int u) { return (int)(lds32(perm_s + (u & ~3)) >> (8 * (u & 3))) & (dk - 1); };
-            auto kv_at = [&](int ch) { return BF16 ? bf16_at(ob + p.off_k, ch) : ldsf(ob + p.off_k + 4 * ch); };
-            auto qv_at = [&](int ch) { return BF16 ? bf16_at(ob + p.off_q, ch) : ldsf(ob + p.off_q + 4 * ch); };
-            auto av_at = [&](int ch) { return KDA ? expf(ldsf(ob + p.off_g + 4 * ch)) : alpha; };
             float2 kk[R], qq[R], bk[R], aa[R];
             float kq = 0.f;
 #pragma unroll
             for (int i = 0; i < R; ++i) {
-                const int r = lane + 32 * i;
-                const bool live = r < lo && i < RL;
-                const int ch = chan(live ? K + r : 0);
-                const float kv = live ? kv_at(ch) : 0.f;
-                const float qv = live ? qv_at(ch) : 0.f;
+                const int u = lane + 32 * i;
+                const int ch = (int)(lds32(perm_s + (u & ~3)) >> (8 * (u & 3))) & (dk - 1);
+                const float kv = BF16 ? bf16_at(ob + p.off_k, ch) : ldsf(ob + p.off_k + 4 * ch);
+                const float qv = BF16 ? bf16_at(ob + p.off_q, ch) : ldsf(ob + p.off_q + 4 * ch);
                 kk[i] = splat2(kv);
                 qq[i] = splat2(qv);
                 bk[i] = splat2(beta * kv * kDown);
-                aa[i] = splat2(av_at(ch));
-                kq = fmaf(kv, qv, kq);
-            }
-            // FP16 rows: {a_u, k_u, q_u, beta k_u} per row
-            for (int u = lane; u < K; u += 32) {
-                const int ch = chan(u);
-                const float kv = kv_at(ch), qv = qv_at(ch);
-                sts128(hops + 16 * u, make_uint4(__float_as_uint(av_at(ch)), __float_as_uint(kv), __float_as_uint(qv),
-                                                 __float_as_uint(beta * kv)));
+                aa[i] = splat2(KDA ? expf(ldsf(ob + p.off_g + 4 * ch)) : alpha);
                 kq = fmaf(kv, qv, kq);
             }
 #pragma unroll
             for (int m = 16; m >= 1; m >>= 1) kq += __shfl_xor_sync(kFull, kq, m);
             const float bkq = beta * kq;
-            __syncwarp();
 
-            // ---- decay and partial sums ----
+            // ---- the previous token's update, decay and partial sums ----
+            float2 d[16];
+            load_dvec(dvec, d);
             float2 acc[16], accp[16];
 #pragma unroll
             for (int j = 0; j < 16; ++j) acc[j] = accp[j] = make_float2(0.f, 0.f);
 #pragma unroll
-            for (int i = 0; i < RL; ++i) {
+            for (int i = 0; i < R; ++i) {
 #pragma unroll
                 for (int j = 0; j < 16; ++j) {
-                    x[i][j] = mul2(x[i][j], aa[i]);
+                    x[i][j] = mul2(fma2(bkp[i], d[j], x[i][j]), aa[i]);
                     acc[j] = fma2(x[i][j], kk[i], acc[j]);
                     accp[j] = fma2(x[i][j], qq[i], accp[j]);
                 }
             }
-            float rhi = 0.f, phi = 0.f;
-            for (int u = 0; u < K; ++u) {
-                const uint4 op = lds128(hops + 16 * u);
-                const float hb = __uint_as_float(op.x) * ldsf(hbuf + 4 * (32 * u + lane));  // decayed FP16 row
-                sts32(hbuf + 4 * (32 * u + lane), __float_as_uint(hb));
-                rhi = fmaf(hb, __uint_as_float(op.y), rhi);
-                phi = fmaf(hb, __uint_as_float(op.z), phi);
-            }
-            const float2 lo_sums = column_sum2(acc, accp, part, lane);
-            const float rlo = lo_sums.x * kUp, plo = lo_sums.y * kUp;
+            const float2 sums = column_sum2(acc, accp, part, lane);
+            const float rs = sums.x * kUp, ps = sums.y * kUp;
 
-            // ---- d, o_t, H d ----
+            // ---- d, o_t, and the column vector of the update ----
             const float vj = BF16 ? bf16_at(ob + p.off_v, lane) : ldsf(ob + p.off_v + 4 * lane);
             float dj, dt, pj;
-            if (HAD) {
-                const float vt = hadamard_lanes(vj, sg);
-                const float hr_lo = hadamard_lanes(rlo, sg);
-                const float hp_lo = hadamard_lanes(plo, sg);
-                const float hr_hi = K > 0 ? hadamard_lanes(rhi, sg) : 0.f;
-                dj = vj - (hr_lo + rhi);
-                dt = vt - (rlo + hr_hi);
-                pj = hp_lo + phi;
+            if (HAD) {  // r = H r~, p = H p~; the rows take H d = H v - r~
+                dj = vj - hadamard_lanes(rs, sg);
+                dt = hadamard_lanes(vj, sg) - rs;
+                pj = hadamard_lanes(ps, sg);
             } else {
-                dj = vj - (rlo + rhi);
+                dj = vj - rs;
                 dt = dj;
-                pj = plo + phi;
+                pj = ps;
             }
             p.o[(((int64_t)b * T + tok) * H + h) * p.dv + kG * c + lane] = fmaf(bkq, dj, pj);
             sts32(dvec + 4 * lane, __float_as_uint(dt));
+#pragma unroll
+            for (int i = 0; i < R; ++i) bkp[i] = bk[i];
+        }
+        {  // the last token's update
             __syncwarp();
-
-            // ---- rank-1 update ----
             float2 d[16];
+            load_dvec(dvec, d);
 #pragma unroll
-            for (int jj = 0; jj < 8; ++jj) {
-                const uint4 w = lds128(dvec + 16 * jj);
-                d[2 * jj] = make_float2(__uint_as_float(w.x), __uint_as_float(w.y));
-                d[2 * jj + 1] = make_float2(__uint_as_float(w.z), __uint_as_float(w.w));
-            }
+            for (int i = 0; i < R; ++i) {
 #pragma unroll
-            for (int i = 0; i < RL; ++i) {
-#pragma unroll
-                for (int j = 0; j < 16; ++j) x[i][j] = fma2(bk[i], d[j], x[i][j]);
+                for (int j = 0; j < 16; ++j) x[i][j] = fma2(bkp[i], d[j], x[i][j]);
             }
-            for (int u = 0; u < K; ++u) {
-                const float hb = ldsf(hbuf + 4 * (32 * u + lane));
-                sts32(hbuf + 4 * (32 * u + lane), __float_as_uint(fmaf(__uint_as_float(lds128(hops + 16 * u).w), dj, hb)));
-            }
-            __syncwarp();  // dvec, hops and the token buffer are reused by the next token
         }
 
-        // ---- requantize the chunk-final tile and store it in place ----
+        // ---- the chunk-final tile: FP16 rows rounded once, low-tier rows requantized ----
 #pragma unroll
-        for (int i = 0; i < RL; ++i) {
-            const int r = lane + 32 * i;
+        for (int i = 0; i < R; ++i) {
+            const int u = lane + 32 * i;
+            if (32 * i < K) {  // warp-uniform: some lanes of this slot hold FP16 rows
+                float2 y[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) y[j] = x[i][j];
+                if (HAD) hadamard_pairs(y);  // back to the natural domain
+                uint32_t own[16];
+#pragma unroll
+                for (int j = 0; j < 16; ++j) own[j] = f2_to_h2(y[j].x * kUp, y[j].y * kUp);
+                store_hi_row(grec, u, K, lane, own);
+            }
+            if (u < K) continue;
+            const int r = u - K;
             if constexpr (fmt_u4(FMT)) {
                 uint32_t w[4];
                 const uint32_t szw = quantize_group_u4(x[i], w);
-                if (r < lo) {
-                    stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
-                    stg32(grec + p.meta_off + 4 * r, szw);
-                }
+                stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                stg32(grec + p.meta_off + 4 * r, szw);
             } else if constexpr (FMT == kFmtE4M3) {
                 float2 xn[16];
 #pragma unroll
                 for (int j = 0; j < 16; ++j) xn[j] = mul2(x[i][j], splat2(kUp));  // natural domain (exact)
                 uint32_t w[8];
                 const float sc = quantize_group_e4m3(xn, w);
-                if (r < lo) {
-                    stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
-                    stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
-                    stg32(grec + p.meta_off + 4 * r, __float_as_uint(sc));
-                }
+                stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
+                stg32(grec + p.meta_off + 4 * r, __float_as_uint(sc));
             } else {
                 float mn, mx, inv, zq;
                 minmax32(x[i], mn, mx);
@@ -271,17 +318,10 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
                 uint32_t w[8];
 #pragma unroll
                 for (int m = 0; m < 8; ++m) w[m] = encode4(x[i][2 * m], x[i][2 * m + 1], inv2, zc2);
-                if (r < lo) {
-                    stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
-                    stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
-                    stg32(grec + p.meta_off + 4 * r, szw);
-                }
+                stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
+                stg32(grec + p.meta_off + 4 * r, szw);
             }
-        }
-        for (int u = 0; u < K; u += 2) {
-            const float f0 = ldsf(hbuf + 4 * (32 * u + lane));
-            const float f1 = u + 1 < K ? ldsf(hbuf + 4 * (32 * (u + 1) + lane)) : 0.f;  // odd K: padding half 0
-            stg32(grec + hi_elem_off(u, lane), f2_to_h2(f0, f1));
         }
     }
     cp_async_wait_all();
