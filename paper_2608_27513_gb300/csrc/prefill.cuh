@@ -104,7 +104,7 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
     const int nw = blockDim.x >> 5;
     const LaneSigns sg = lane_signs(lane);
     const uint32_t ws = smem_u32(smem) + (uint32_t)(warp * p.warp_smem);
-    const uint32_t part = ws;  // column_sum2 buffer at the start of the warp's area
+    const uint32_t part = ws;  // column-sum buffer at the start of the warp's area
     const uint32_t dvec = ws + p.dvec_off;
     const uint32_t perm_s = ws + p.perm_off;
     const uint32_t ops0 = ws + p.ops_off;
@@ -115,36 +115,6 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
     const int64_t gw = (int64_t)blockIdx.x * nw + warp;
     const int64_t nwt = (int64_t)gridDim.x * nw;
     bool bad_slot = false;
-
-    // operands of token tok of (b, h) for value block c into buffer dst
-    auto load_token = [&](int b, int h, int c, int tok, uint32_t dst) {
-        const int hq = (int)(((int64_t)h * p.Hqk) / H);
-        const int64_t bt = (int64_t)b * T + tok;
-        const uint8_t *qrow = (const uint8_t *)p.q + (bt * p.Hqk + hq) * dk * esz;
-        const uint8_t *krow = (const uint8_t *)p.k + (bt * p.Hqk + hq) * dk * esz;
-        const uint8_t *grow = (const uint8_t *)(p.g + (bt * H + h) * (KDA ? dk : 1));
-        const uint8_t *vblk = (const uint8_t *)p.v + ((bt * H + h) * p.dv + kG * c) * esz;
-        const int nq = dk * esz / 16, ng = KDA ? dk * 4 / 16 : 0, nv = kG * esz / 16;
-        const int total = 2 * nq + ng + nv;
-        for (int ci = lane; ci < total; ci += 32) {
-            int j = ci;
-            if (j < nq) {
-                cp_async16(dst + p.off_q + 16 * j, qrow + 16 * j);
-            } else if ((j -= nq) < nq) {
-                cp_async16(dst + p.off_k + 16 * j, krow + 16 * j);
-            } else if ((j -= nq) < ng) {
-                cp_async16(dst + p.off_g + 16 * j, grow + 16 * j);
-            } else {
-                j -= ng;
-                cp_async16(dst + p.off_v + 16 * j, vblk + 16 * j);
-            }
-        }
-        if (lane == 0) {
-            cp_async4(dst + p.off_beta, p.beta + bt * H + h);
-            if (!KDA) cp_async4(dst + p.off_g, grow);
-        }
-        cp_async_commit();
-    };
 
     for (int64_t t = p.total_tiles * gw / nwt; t < p.total_tiles * (gw + 1) / nwt; ++t) {
         const int c = (int)(t % V);
@@ -159,10 +129,40 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
         if (Tb == 0) continue;
         uint8_t *const grec = p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * p.rec_bytes;
 
+        // token 0's operands of this tile and their per-token strides (in bytes)
+        const int hq = (int)(((int64_t)h * p.Hqk) / H);
+        const uint8_t *qt = (const uint8_t *)p.q + ((int64_t)b * T * p.Hqk + hq) * dk * esz;
+        const uint8_t *kt = (const uint8_t *)p.k + ((int64_t)b * T * p.Hqk + hq) * dk * esz;
+        const uint8_t *gt = (const uint8_t *)(p.g + ((int64_t)b * T * H + h) * (KDA ? dk : 1));
+        const uint8_t *vt = (const uint8_t *)p.v + (((int64_t)b * T * H + h) * p.dv + kG * c) * esz;
+        const uint8_t *bt = (const uint8_t *)(p.beta + (int64_t)b * T * H + h);
+        float *ot = p.o + ((int64_t)b * T * H + h) * p.dv + kG * c + lane;
+        const int64_t sqk = (int64_t)p.Hqk * dk * esz, sg4 = (int64_t)H * (KDA ? dk : 1) * 4,
+                      sv = (int64_t)H * p.dv * esz, sb = (int64_t)H * 4, so = (int64_t)H * p.dv;
+        // one token's operands into buffer dst: every copy is 16 B (beta and the GDN
+        // gate 4 B); the copy counts are compile-time constants
+        auto load_token = [&](int tok, uint32_t dst) {
+            constexpr int nq = dk * (BF16 ? 2 : 4) / 16, ng = KDA ? dk * 4 / 16 : 0, nv = kG * (BF16 ? 2 : 4) / 16;
+            const uint8_t *qs = qt + tok * sqk, *ks = kt + tok * sqk, *gs = gt + tok * sg4, *vs = vt + tok * sv;
+#pragma unroll
+            for (int j = lane; j < nq; j += 32) cp_async16(dst + p.off_q + 16 * j, qs + 16 * j);
+#pragma unroll
+            for (int j = lane; j < nq; j += 32) cp_async16(dst + p.off_k + 16 * j, ks + 16 * j);
+#pragma unroll
+            for (int j = lane; j < ng; j += 32) cp_async16(dst + p.off_g + 16 * j, gs + 16 * j);
+#pragma unroll
+            for (int j = lane; j < nv; j += 32) cp_async16(dst + p.off_v + 16 * j, vs + 16 * j);
+            if (lane == 0) {
+                cp_async4(dst + p.off_beta, bt + tok * sb);
+                if (!KDA) cp_async4(dst + p.off_g, gs);
+            }
+            cp_async_commit();
+        };
+
         // π of this head, then token 0's operands
         __syncwarp();  // the previous tile's readers of the shared buffers are done
         for (int ci = lane; ci < dk / 16; ci += 32) cp_async16(perm_s + 16 * ci, p.perm + (int64_t)h * dk + 16 * ci);
-        load_token(b, h, c, 0, ops0);
+        load_token(0, ops0);
 
         // ---- reconstruct the tile in FP32, undecayed, scaled by 2^-39; with H_32 in
         //      the transformed domain (FP16 rows transformed here) ----
@@ -210,7 +210,7 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
             const uint32_t ob = ops0 + (uint32_t)((tok & 1) * p.ops_bytes);
             cp_async_wait_all();
             __syncwarp();
-            if (tok + 1 < Tb) load_token(b, h, c, tok + 1, ops0 + (uint32_t)(((tok + 1) & 1) * p.ops_bytes));
+            if (tok + 1 < Tb) load_token(tok + 1, ops0 + (uint32_t)(((tok + 1) & 1) * p.ops_bytes));
 
             // ---- operands of this lane's rows, in calibrated order ----
             const float beta = ldsf(ob + p.off_beta);
@@ -220,9 +220,9 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
 #pragma unroll
             for (int i = 0; i < R; ++i) {
                 const int u = lane + 32 * i;
-                const int ch = (int)(lds32(perm_s + (u & ~3)) >> (8 * (u & 3))) & (dk - 1);
-                const float kv = BF16 ? bf16_at(ob + p.off_k, ch) : ldsf(ob + p.off_k + 4 * ch);
-                const float qv = BF16 ? bf16_at(ob + p.off_q, ch) : ldsf(ob + p.off_q + 4 * ch);
+                const uint32_t ch = lds_u8(perm_s + u) & (dk - 1);
+                const float kv = BF16 ? lds_bf16(ob + p.off_k + 2 * ch) : ldsf(ob + p.off_k + 4 * ch);
+                const float qv = BF16 ? lds_bf16(ob + p.off_q + 2 * ch) : ldsf(ob + p.off_q + 4 * ch);
                 kk[i] = splat2(kv);
                 qq[i] = splat2(qv);
                 bk[i] = splat2(beta * kv * kDown);
@@ -248,7 +248,7 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
                     accp[j] = fma2(x[i][j], qq[i], accp[j]);
                 }
             }
-            const float2 sums = column_sum2(acc, accp, part, lane);
+            const float2 sums = column_sum_pairs(acc, accp, part, lane);
             const float rs = sums.x * kUp, ps = sums.y * kUp;
 
             // ---- d, o_t, and the column vector of the update ----
@@ -263,7 +263,7 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
                 dt = dj;
                 pj = ps;
             }
-            p.o[(((int64_t)b * T + tok) * H + h) * p.dv + kG * c + lane] = fmaf(bkq, dj, pj);
+            ot[tok * so] = fmaf(bkq, dj, pj);
             sts32(dvec + 4 * lane, __float_as_uint(dt));
 #pragma unroll
             for (int i = 0; i < R; ++i) bkp[i] = bk[i];
