@@ -13,8 +13,8 @@
 // that way, and the FP16 rows are transformed once on load and back once on store
 // (H_32 is symmetric and orthonormal, and decay and the rank-1 update are
 // row/column scalings that commute with it), so the per-token work is the same for
-// every row: decay, partial sums of r~ = S~^T k and p~ = S~^T q, column sums, the
-// lane butterflies r = H r~, p = H p~, H d, o_t and the update.  The next token's
+// every row: decay, partial sums of r~ = S~^T k and p~ = S~^T q, column sums,
+// H d = H v - r~ and the update; o_t takes one lane butterfly.  The next token's
 // operands (q, k, g, v block, beta) stream into a double buffer by cp.async while
 // the current token runs.  After the last token the low-tier rows are requantized
 // like a decode step and the FP16 rows rounded once; both go back with plain
@@ -202,10 +202,17 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
         // The rank-1 update of token t is applied at the start of token t+1, in the
         // same pass over the registers as that token's decay (and after the loop for
         // the last token): H d of the pending update waits in dvec, beta k in bkp.
+        // o_t = H (p~ - beta (k^T q) r~) + beta (k^T q) v (all rows in the transformed
+        // domain; H = I without H_32) is finished during token t+1, off the path of
+        // the recurrence: o_pend and o_add hold its two parts.
         float2 bkp[R];
 #pragma unroll
         for (int i = 0; i < R; ++i) bkp[i] = make_float2(0.f, 0.f);
         sts32(dvec + 4 * lane, 0u);
+        float o_pend = 0.f, o_add = 0.f;
+        auto finish_o = [&](int tok) {
+            ot[tok * so] = (HAD ? hadamard_lanes(o_pend, sg) : o_pend) + o_add;
+        };
         for (int tok = 0; tok < Tb; ++tok) {
             const uint32_t ob = ops0 + (uint32_t)((tok & 1) * p.ops_bytes);
             cp_async_wait_all();
@@ -232,6 +239,9 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
 #pragma unroll
             for (int m = 16; m >= 1; m >>= 1) kq += __shfl_xor_sync(kFull, kq, m);
             const float bkq = beta * kq;
+            const float vj = BF16 ? lds_bf16(ob + p.off_v + 2 * lane) : ldsf(ob + p.off_v + 4 * lane);
+            const float hv = HAD ? hadamard_lanes(vj, sg) : vj;  // H v: independent of the state
+            if (tok > 0) finish_o(tok - 1);
 
             // ---- the previous token's update, decay and partial sums ----
             float2 d[16];
@@ -251,23 +261,14 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
             const float2 sums = column_sum_pairs(acc, accp, part, lane);
             const float rs = sums.x * kUp, ps = sums.y * kUp;
 
-            // ---- d, o_t, and the column vector of the update ----
-            const float vj = BF16 ? bf16_at(ob + p.off_v, lane) : ldsf(ob + p.off_v + 4 * lane);
-            float dj, dt, pj;
-            if (HAD) {  // r = H r~, p = H p~; the rows take H d = H v - r~
-                dj = vj - hadamard_lanes(rs, sg);
-                dt = hadamard_lanes(vj, sg) - rs;
-                pj = hadamard_lanes(ps, sg);
-            } else {
-                dj = vj - rs;
-                dt = dj;
-                pj = ps;
-            }
-            ot[tok * so] = fmaf(bkq, dj, pj);
-            sts32(dvec + 4 * lane, __float_as_uint(dt));
+            // ---- the column vector of the update, H d = H v - r~, and o_t's parts ----
+            sts32(dvec + 4 * lane, __float_as_uint(hv - rs));
+            o_pend = fmaf(-bkq, rs, ps);
+            o_add = bkq * vj;
 #pragma unroll
             for (int i = 0; i < R; ++i) bkp[i] = bk[i];
         }
+        finish_o(Tb - 1);
         {  // the last token's update
             __syncwarp();
             float2 d[16];
