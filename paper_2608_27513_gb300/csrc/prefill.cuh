@@ -44,6 +44,57 @@ struct PrefillParams {
     uint32_t *status;
 };
 
+__device__ __forceinline__ uint32_t lds_u8(uint32_t a) {
+    uint32_t v;
+    asm volatile("ld.shared.u8 %0, [%1];" : "=r"(v) : "r"(a));
+    return v;
+}
+// bf16 at shared address a, widened to FP32 (exact)
+__device__ __forceinline__ float lds_bf16(uint32_t a) {
+    uint32_t v;
+    asm volatile("ld.shared.u16 %0, [%1];" : "=r"(v) : "r"(a));
+    return __uint_as_float(v << 16);
+}
+
+// The same column sums with the pairs stored as they sit in registers (no
+// repacking into (a, b) quads).  Lane l writes its row as [a 32 floats][b 32
+// floats] at a stride of kPairStride floats (2 mod 32: a half-warp's 64-bit
+// stores cover the 32 banks once); lane j < 16 then sums columns (2j, 2j+1) of a
+// over the 32 rows and lane 16 + j the same columns of b, and four shuffles hand
+// every lane its own column.  Needs 32 * kPairStride floats at part.
+constexpr int kPairStride = 66;
+static_assert(kPairStride <= kPartStride, "column_sum_pairs uses the column_sum2 buffer");
+__device__ __forceinline__ float2 column_sum_pairs(const float2 (&a)[16], const float2 (&b)[16], uint32_t part,
+                                                   int lane) {
+    const uint32_t row = part + (uint32_t)(lane * kPairStride * 4);
+#pragma unroll
+    for (int m = 0; m < 16; ++m) {
+        asm volatile("st.shared.v2.f32 [%0], {%1,%2};" ::"r"(row + 8 * m), "f"(a[m].x), "f"(a[m].y) : "memory");
+        asm volatile("st.shared.v2.f32 [%0], {%1,%2};" ::"r"(row + 128 + 8 * m), "f"(b[m].x), "f"(b[m].y) : "memory");
+    }
+    __syncwarp();
+    const uint32_t base = part + (uint32_t)(((lane >> 4) * 32 + 2 * (lane & 15)) * 4);
+    float2 s0 = make_float2(0.f, 0.f), s1 = s0, s2 = s0, s3 = s0;
+#pragma unroll
+    for (int l = 0; l < 32; l += 4) {
+        float2 v0, v1, v2, v3;
+        asm volatile("ld.shared.v2.f32 {%0,%1}, [%2];" : "=f"(v0.x), "=f"(v0.y) : "r"(base + (l + 0) * kPairStride * 4));
+        asm volatile("ld.shared.v2.f32 {%0,%1}, [%2];" : "=f"(v1.x), "=f"(v1.y) : "r"(base + (l + 1) * kPairStride * 4));
+        asm volatile("ld.shared.v2.f32 {%0,%1}, [%2];" : "=f"(v2.x), "=f"(v2.y) : "r"(base + (l + 2) * kPairStride * 4));
+        asm volatile("ld.shared.v2.f32 {%0,%1}, [%2];" : "=f"(v3.x), "=f"(v3.y) : "r"(base + (l + 3) * kPairStride * 4));
+        s0 = add2(s0, v0);
+        s1 = add2(s1, v1);
+        s2 = add2(s2, v2);
+        s3 = add2(s3, v3);
+    }
+    __syncwarp();
+    const float2 t = add2(add2(s0, s1), add2(s2, s3));
+    const int src = lane >> 1;
+    const float ax = __shfl_sync(kFull, t.x, src), ay = __shfl_sync(kFull, t.y, src);
+    const float bx = __shfl_sync(kFull, t.x, 16 + src), by = __shfl_sync(kFull, t.y, 16 + src);
+    return (lane & 1) ? make_float2(ay, by) : make_float2(ax, bx);
+}
+
 // FP16 row u of a record -> 32 FP32 values (component j of the group is y[j/2].x
 // or .y).  Row pair u>>1 holds one 32-bit word per column, row u in half u & 1.
 __device__ __forceinline__ void load_hi_row(const uint8_t *grec, int u, float2 (&y)[16]) {
