@@ -581,6 +581,74 @@ def prefill_arm(steps: int, warmup: int, T: int = 64):
         print(json.dumps(row), flush=True)
 
 
+def multitoken_arm(steps: int, warmup: int, tokens=(1, 2, 4, 8, 16)):
+    """Fused multi-token steps at the decode workload (KDA, B = 256, H = 32, d = 128,
+    K_hi = 10): T tokens per request slot in one launch of the chunk kernel (the state is
+    read and requantized once for the T tokens), against T single-token launches of the
+    packed decode step on the same pools.  Reports us per launch and per token."""
+    import torch
+
+    import paper_2608_27513_gb300 as damp
+    from paper_2608_27513_gb300 import build
+    build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    w = wl.KDA_B256
+    L = damp.Layout(w.heads, w.qk_heads, w.d_k, w.d_v, w.k_hi, w.lo_format)
+    perm = torch.from_numpy(wl.random_perm(w)).to(dev)
+    S = 0.3 * torch.randn((w.batch, w.heads, w.d_k, w.d_v), device=dev)
+    pools = [damp.new_state(L, w.batch, dev) for _ in range(2)]
+    for pl in pools:
+        damp.quantize_state(L, S, perm, pl)
+    del S
+    per_t = wl.torch_step_inputs(w, max(tokens), dev)
+
+    def timeit(fn, n):
+        for i in range(warmup):
+            fn(i)
+        torch.cuda.synchronize()
+        with ClockSampler(dev.index) as clk:
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for i in range(n):
+                fn(i)
+            e1.record()
+            torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / n * 1e3, clk.summary()
+
+    o1 = torch.empty((w.batch, w.heads, w.d_v), device=dev)
+
+    def step(i):
+        d = per_t[i % len(per_t)]
+        damp.kda_decode_step(L, pools[i % 2], perm, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o1)
+
+    us_step, _ = timeit(step, max(steps, 200))
+    out = []
+    esz = 2 if w.in_dtype == "bf16" else 4
+    state = 2 * w.batch * damp.slot_bytes(L)
+    for T in tokens:
+        chunk = {key: torch.stack([d[key] for d in per_t[:T]], dim=1).contiguous() for key in per_t[0]}
+        o = torch.empty((w.batch, T, w.heads, w.d_v), device=dev)
+
+        def run(i):
+            damp.kda_prefill_chunk(L, pools[i % 2], perm, chunk["q"], chunk["k"], chunk["v"], chunk["g"],
+                                   chunk["beta"], o=o)
+
+        us, clocks = timeit(run, max(steps // (4 * T), 20))
+        ops = w.batch * T * (2 * w.qk_heads * w.d_k * esz + w.heads * w.d_v * (esz + 4)
+                             + w.heads * 4 * (w.d_k + 1))
+        out.append({"mode": "multi_token_step", "kind": w.kind, "workload": w.name, "tokens": T,
+                    "us_per_launch": us, "us_per_token": us / T, "tokens_per_s": w.batch * T / (us * 1e-6),
+                    "single_token_steps_us": us_step * T, "speedup_vs_single_steps": us_step * T / us,
+                    "algorithmic_bytes": state + ops, "hbm_gbs": (state + ops) / (us * 1e-6) / 1e9,
+                    "clocks": clocks})
+        del chunk, o
+    if damp.device_status() != 0:
+        raise RuntimeError("device status word set during the multi-token runs")
+    for row in out:
+        print(json.dumps(row), flush=True)
+
+
 def calibrate_arm(steps: int, warmup: int, n_docs: int = 32, n_tokens: int = 256):
     """Calibration run (Algorithm 1, App. A.2) on the GPU for one layer of H = 32 heads,
     d = 128: FP32 trajectories of n_docs documents over n_tokens tokens, error energy of
@@ -707,6 +775,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true", help="K_hi sweep (GDN and KDA, B=256) instead of the bench line")
     ap.add_argument("--prefill", action="store_true", help="prefill chunks (64 tokens, B=256) instead of the bench line")
+    ap.add_argument("--multitoken", action="store_true",
+                    help="fused multi-token steps (T = 1..16 tokens per launch, B=256) instead of the bench line")
     ap.add_argument("--calibrate", action="store_true", help="GPU calibration run instead of the bench line")
     ap.add_argument("--drift", action="store_true", help="30-layer free-running drift run instead of the bench line")
     args = ap.parse_args()
@@ -723,6 +793,9 @@ def main():
         return
     if args.prefill:
         prefill_arm(args.steps, args.warmup)
+        return
+    if args.multitoken:
+        multitoken_arm(args.steps, args.warmup)
         return
     if args.calibrate:
         calibrate_arm(args.steps, args.warmup)

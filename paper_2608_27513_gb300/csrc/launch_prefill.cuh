@@ -16,8 +16,6 @@ template <bool KDA, int FMT>
 static cudaError_t launch_prefill_impl(const StepArgs &a, cudaStream_t stream, uint32_t *status) {
     const int V = a.dv / kG;
     const RecGeom rg = rec_geom(a.dk, a.K, FMT);
-    const int esz = a.in_bf16 ? 2 : 4;
-    auto up16 = [](int x) { return (x + 15) & ~15; };
     PrefillParams p{};
     p.state = static_cast<uint8_t *>(a.state);
     p.num_slots = a.num_slots;
@@ -44,35 +42,15 @@ static cudaError_t launch_prefill_impl(const StepArgs &a, cudaStream_t stream, u
     p.slot_bytes = (int64_t)a.H * V * rg.bytes;
     p.total_tiles = (int64_t)a.batch * a.H * V;
     p.status = status;
-    // per-warp shared memory: [column-sum buffer][H d][pi][2 token buffers]
-    int off = 32 * kPartStride * 4;
-    p.dvec_off = off;
-    off += 32 * 4;
-    p.perm_off = off;
-    off += up16(a.dk);
-    p.ops_off = off;
-    int t = 0;
-    p.off_q = t;
-    t += up16(a.dk * esz);
-    p.off_k = t;
-    t += up16(a.dk * esz);
-    p.off_g = t;
-    t += KDA ? up16(a.dk * 4) : 16;
-    p.off_v = t;
-    t += up16(kG * esz);
-    p.off_beta = t;
-    t += 16;
-    p.ops_bytes = t;
-    off += 2 * t;
-    p.warp_smem = (off + 127) & ~127;
+    const int warp_smem = prefill_smem(a.dk, KDA, a.in_bf16).warp_bytes;
     if (p.total_tiles == 0 || a.T == 0) return cudaSuccess;
 
     int warps = kPrefillWarps;
-    while (warps > 1 && warps * p.warp_smem > max_smem_per_block()) --warps;
-    if (warps * p.warp_smem > max_smem_per_block()) return cudaErrorInvalidValue;
+    while (warps > 1 && warps * warp_smem > max_smem_per_block()) --warps;
+    if (warps * warp_smem > max_smem_per_block()) return cudaErrorInvalidValue;
     const int64_t want = (p.total_tiles + warps - 1) / warps;
     const int grid = (int)std::min<int64_t>(want, (int64_t)sm_count());
-    const int smem = p.warp_smem * warps;
+    const int smem = warp_smem * warps;
 
     void (*kern)(PrefillParams) = nullptr;
 #define DAMP_PICK(R_)                                                                              \

@@ -26,6 +26,21 @@
 
 namespace damp {
 
+// Per-warp shared memory of the chunk kernel, fixed by (d_k, decay kind, input type):
+// [column-sum buffer][H d][pi][token buffer 0][token buffer 1], each token buffer
+// [q][k][g (KDA: d_k floats; GDN: one)][v block][beta].
+struct PrefillSmem {
+    int dvec_off, perm_off, ops_off, off_q, off_k, off_g, off_v, off_beta, ops_bytes, warp_bytes;
+};
+__host__ __device__ constexpr int up16(int x) { return (x + 15) & ~15; }
+__host__ __device__ constexpr PrefillSmem prefill_smem(int dk, bool kda, bool bf16) {
+    const int esz = bf16 ? 2 : 4;
+    const int dvec = 32 * kPartStride * 4, perm = dvec + 32 * 4, ops = perm + up16(dk);
+    const int oq = 0, ok = up16(dk * esz), og = 2 * up16(dk * esz), ov = og + (kda ? up16(dk * 4) : 16);
+    const int ob = ov + up16(kG * esz), bytes = ob + 16;
+    return PrefillSmem{dvec, perm, ops, oq, ok, og, ov, ob, bytes, (ops + 2 * bytes + 127) & ~127};
+}
+
 struct PrefillParams {
     uint8_t *state;
     int64_t num_slots;
@@ -39,8 +54,6 @@ struct PrefillParams {
     int32_t rec_bytes, codes_off, meta_off;
     int64_t slot_bytes, total_tiles;
     // per-warp shared memory
-    int32_t warp_smem, dvec_off, perm_off, ops_off, ops_bytes;
-    int32_t off_q, off_k, off_g, off_v, off_beta;
     uint32_t *status;
 };
 
@@ -154,11 +167,12 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
     const int warp = threadIdx.x >> 5;
     const int nw = blockDim.x >> 5;
     const LaneSigns sg = lane_signs(lane);
-    const uint32_t ws = smem_u32(smem) + (uint32_t)(warp * p.warp_smem);
+    constexpr PrefillSmem SM = prefill_smem(32 * R, KDA, BF16);
+    const uint32_t ws = smem_u32(smem) + (uint32_t)(warp * SM.warp_bytes);
     const uint32_t part = ws;  // column-sum buffer at the start of the warp's area
-    const uint32_t dvec = ws + p.dvec_off;
-    const uint32_t perm_s = ws + p.perm_off;
-    const uint32_t ops0 = ws + p.ops_off;
+    const uint32_t dvec = ws + SM.dvec_off;
+    const uint32_t perm_s = ws + SM.perm_off;
+    const uint32_t ops0 = ws + SM.ops_off;
     const int esz = BF16 ? 2 : 4;
     constexpr int dk = 32 * R;
     const int K = p.K, lo = dk - K, H = p.H, V = p.V, T = p.T;
@@ -196,16 +210,16 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
             constexpr int nq = dk * (BF16 ? 2 : 4) / 16, ng = KDA ? dk * 4 / 16 : 0, nv = kG * (BF16 ? 2 : 4) / 16;
             const uint8_t *qs = qt + tok * sqk, *ks = kt + tok * sqk, *gs = gt + tok * sg4, *vs = vt + tok * sv;
 #pragma unroll
-            for (int j = lane; j < nq; j += 32) cp_async16(dst + p.off_q + 16 * j, qs + 16 * j);
+            for (int j = lane; j < nq; j += 32) cp_async16(dst + SM.off_q + 16 * j, qs + 16 * j);
 #pragma unroll
-            for (int j = lane; j < nq; j += 32) cp_async16(dst + p.off_k + 16 * j, ks + 16 * j);
+            for (int j = lane; j < nq; j += 32) cp_async16(dst + SM.off_k + 16 * j, ks + 16 * j);
 #pragma unroll
-            for (int j = lane; j < ng; j += 32) cp_async16(dst + p.off_g + 16 * j, gs + 16 * j);
+            for (int j = lane; j < ng; j += 32) cp_async16(dst + SM.off_g + 16 * j, gs + 16 * j);
 #pragma unroll
-            for (int j = lane; j < nv; j += 32) cp_async16(dst + p.off_v + 16 * j, vs + 16 * j);
+            for (int j = lane; j < nv; j += 32) cp_async16(dst + SM.off_v + 16 * j, vs + 16 * j);
             if (lane == 0) {
-                cp_async4(dst + p.off_beta, bt + tok * sb);
-                if (!KDA) cp_async4(dst + p.off_g, gs);
+                cp_async4(dst + SM.off_beta, bt + tok * sb);
+                if (!KDA) cp_async4(dst + SM.off_g, gs);
             }
             cp_async_commit();
         };
@@ -265,32 +279,32 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
             ot[tok * so] = (HAD ? hadamard_lanes(o_pend, sg) : o_pend) + o_add;
         };
         for (int tok = 0; tok < Tb; ++tok) {
-            const uint32_t ob = ops0 + (uint32_t)((tok & 1) * p.ops_bytes);
+            const uint32_t ob = ops0 + (uint32_t)((tok & 1) * SM.ops_bytes);
             cp_async_wait_all();
             __syncwarp();
-            if (tok + 1 < Tb) load_token(tok + 1, ops0 + (uint32_t)(((tok + 1) & 1) * p.ops_bytes));
+            if (tok + 1 < Tb) load_token(tok + 1, ops0 + (uint32_t)(((tok + 1) & 1) * SM.ops_bytes));
 
             // ---- operands of this lane's rows, in calibrated order ----
-            const float beta = ldsf(ob + p.off_beta);
-            const float alpha = KDA ? 0.f : expf(ldsf(ob + p.off_g));
+            const float beta = ldsf(ob + SM.off_beta);
+            const float alpha = KDA ? 0.f : expf(ldsf(ob + SM.off_g));
             float2 kk[R], qq[R], bk[R], aa[R];
             float kq = 0.f;
 #pragma unroll
             for (int i = 0; i < R; ++i) {
                 const int u = lane + 32 * i;
                 const uint32_t ch = lds_u8(perm_s + u) & (dk - 1);
-                const float kv = BF16 ? lds_bf16(ob + p.off_k + 2 * ch) : ldsf(ob + p.off_k + 4 * ch);
-                const float qv = BF16 ? lds_bf16(ob + p.off_q + 2 * ch) : ldsf(ob + p.off_q + 4 * ch);
+                const float kv = BF16 ? lds_bf16(ob + SM.off_k + 2 * ch) : ldsf(ob + SM.off_k + 4 * ch);
+                const float qv = BF16 ? lds_bf16(ob + SM.off_q + 2 * ch) : ldsf(ob + SM.off_q + 4 * ch);
                 kk[i] = splat2(kv);
                 qq[i] = splat2(qv);
                 bk[i] = splat2(beta * kv * kDown);
-                aa[i] = splat2(KDA ? expf(ldsf(ob + p.off_g + 4 * ch)) : alpha);
+                aa[i] = splat2(KDA ? expf(ldsf(ob + SM.off_g + 4 * ch)) : alpha);
                 kq = fmaf(kv, qv, kq);
             }
 #pragma unroll
             for (int m = 16; m >= 1; m >>= 1) kq += __shfl_xor_sync(kFull, kq, m);
             const float bkq = beta * kq;
-            const float vj = BF16 ? lds_bf16(ob + p.off_v + 2 * lane) : ldsf(ob + p.off_v + 4 * lane);
+            const float vj = BF16 ? lds_bf16(ob + SM.off_v + 2 * lane) : ldsf(ob + SM.off_v + 4 * lane);
             const float hv = HAD ? hadamard_lanes(vj, sg) : vj;  // H v: independent of the state
             if (tok > 0) finish_o(tok - 1);
 
