@@ -42,7 +42,8 @@ static cudaError_t launch_prefill_impl(const StepArgs &a, cudaStream_t stream, u
     p.slot_bytes = (int64_t)a.H * V * rg.bytes;
     p.total_tiles = (int64_t)a.batch * a.H * V;
     p.status = status;
-    const int warp_smem = prefill_smem(a.dk, KDA, a.in_bf16).warp_bytes;
+    const int warp_smem = prefill_smem(a.dk, KDA, a.in_bf16).warp_bytes + 128 + ((rg.bytes + 127) & ~127);
+    p.warp_stride = warp_smem;
     if (p.total_tiles == 0 || a.T == 0) return cudaSuccess;
 
     int warps = kPrefillWarps;

@@ -16,9 +16,10 @@
 // every row: decay, partial sums of r~ = S~^T k and p~ = S~^T q, column sums,
 // H d = H v - r~ and the update; o_t takes one lane butterfly.  The next token's
 // operands (q, k, g, v block, beta) stream into a double buffer by cp.async while
-// the current token runs.  After the last token the low-tier rows are requantized
-// like a decode step and the FP16 rows rounded once; both go back with plain
-// stores.
+// the current token runs, and the next tile's record comes in by one bulk copy
+// (TMA engine) while the current tile runs its tokens.  After the last token the
+// low-tier rows are requantized like a decode step and the FP16 rows rounded once;
+// both go back with plain stores.
 #pragma once
 
 #include "damp_common.cuh"
@@ -53,6 +54,7 @@ struct PrefillParams {
     int32_t batch, T, H, Hqk, dk, dv, V, K;
     int32_t rec_bytes, codes_off, meta_off;
     int64_t slot_bytes, total_tiles;
+    int32_t warp_stride;  // per-warp shared memory: the fixed buffers, an mbarrier and the record stage
     // per-warp shared memory
     uint32_t *status;
 };
@@ -108,14 +110,15 @@ __device__ __forceinline__ float2 column_sum_pairs(const float2 (&a)[16], const 
     return (lane & 1) ? make_float2(ay, by) : make_float2(ax, bx);
 }
 
-// FP16 row u of a record -> 32 FP32 values (component j of the group is y[j/2].x
-// or .y).  Row pair u>>1 holds one 32-bit word per column, row u in half u & 1.
-__device__ __forceinline__ void load_hi_row(const uint8_t *grec, int u, float2 (&y)[16]) {
-    const uint8_t *pr = grec + hi_elem_off(u & ~1, 0);
+// FP16 row u of a record held in shared memory at rec -> 32 FP32 values
+// (component j of the group is y[j/2].x or .y).  Row pair u>>1 holds one 32-bit
+// word per column, row u in half u & 1.
+__device__ __forceinline__ void load_hi_row(uint32_t rec, int u, float2 (&y)[16]) {
+    const uint32_t pr = rec + (uint32_t)hi_elem_off(u & ~1, 0);
     const uint32_t sel = (u & 1) ? 0x7632u : 0x5410u;
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
-        const uint4 w = *reinterpret_cast<const uint4 *>(pr + 16 * q);
+        const uint4 w = lds128(pr + 16 * q);
         y[2 * q] = h2_to_f2(prmt(w.x, w.y, sel));
         y[2 * q + 1] = h2_to_f2(prmt(w.z, w.w, sel));
     }
@@ -168,7 +171,9 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
     const int nw = blockDim.x >> 5;
     const LaneSigns sg = lane_signs(lane);
     constexpr PrefillSmem SM = prefill_smem(32 * R, KDA, BF16);
-    const uint32_t ws = smem_u32(smem) + (uint32_t)(warp * SM.warp_bytes);
+    const uint32_t ws = smem_u32(smem) + (uint32_t)(warp * p.warp_stride);
+    const uint32_t bar = ws + SM.warp_bytes;  // completion of the record copy
+    const uint32_t st = bar + 128;            // the record of the current tile
     const uint32_t part = ws;  // column-sum buffer at the start of the warp's area
     const uint32_t dvec = ws + SM.dvec_off;
     const uint32_t perm_s = ws + SM.perm_off;
@@ -179,20 +184,53 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
 
     const int64_t gw = (int64_t)blockIdx.x * nw + warp;
     const int64_t nwt = (int64_t)gridDim.x * nw;
-    bool bad_slot = false;
+    const int64_t t0 = p.total_tiles * gw / nwt, t1 = p.total_tiles * (gw + 1) / nwt;
+    if (t0 >= t1) return;
+    bool bad_slot = false, timed_out = false;
 
-    for (int64_t t = p.total_tiles * gw / nwt; t < p.total_tiles * (gw + 1) / nwt; ++t) {
-        const int c = (int)(t % V);
-        const int64_t bh = t / V;
-        const int h = (int)(bh % H), b = (int)(bh / H);
-        const int64_t slot = p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b;
-        if (slot < 0 || slot >= p.num_slots) {
-            bad_slot = true;
+    // The record of the next tile comes in by one bulk copy (TMA engine) while the
+    // current tile runs its tokens; tiles that are skipped (slot out of range, no
+    // tokens) complete their phase with no bytes.
+    auto rec_of = [&](int64_t tt, int &b, int &h, int &c, int64_t &slot, int &Tb) -> uint8_t * {
+        c = (int)(tt % V);
+        const int64_t bh = tt / V;
+        h = (int)(bh % H);
+        b = (int)(bh / H);
+        slot = p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b;
+        Tb = p.lengths ? min(max(p.lengths[b], 0), T) : T;
+        return p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * p.rec_bytes;
+    };
+    auto issue = [&](int64_t tt) {  // lane 0
+        int b, h, c, Tb;
+        int64_t slot;
+        uint8_t *g = rec_of(tt, b, h, c, slot, Tb);
+        const bool run = slot >= 0 && slot < p.num_slots && Tb > 0;
+        mbar_arrive_expect_tx(bar, run ? (uint32_t)p.rec_bytes : 0u);
+        if (run) bulk_g2s(st, g, (uint32_t)p.rec_bytes, bar);
+    };
+    if (lane == 0) {
+        mbar_init(bar, 1);
+        fence_mbar_init();
+        issue(t0);
+    }
+    __syncwarp();
+    uint32_t parity = 0;
+
+    for (int64_t t = t0; t < t1; ++t) {
+        if (!__all_sync(kFull, mbar_wait_bounded(bar, parity))) {
+            timed_out = true;
+            break;
+        }
+        parity ^= 1u;
+        int b, h, c, Tb;
+        int64_t slot;
+        uint8_t *const grec = rec_of(t, b, h, c, slot, Tb);  // written in place
+        const bool slot_ok = slot >= 0 && slot < p.num_slots;
+        bad_slot |= !slot_ok;
+        if (!slot_ok || Tb == 0) {  // nothing landed in the stage: fetch the next record
+            if (lane == 0 && t + 1 < t1) issue(t + 1);
             continue;
         }
-        const int Tb = p.lengths ? min(max(p.lengths[b], 0), T) : T;
-        if (Tb == 0) continue;
-        uint8_t *const grec = p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * p.rec_bytes;
 
         // token 0's operands of this tile and their per-token strides (in bytes)
         const int hq = (int)(((int64_t)h * p.Hqk) / H);
@@ -239,16 +277,16 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
 #pragma unroll
         for (int i = 0; i < R; ++i) {
             const int r = lo > 0 ? min(max(lane + 32 * i - K, 0), lo - 1) : 0;
-            const uint8_t *crow = grec + (lo > 0 ? p.codes_off : 0);  // lo = 0: a valid dummy address
-            cw0[i] = *reinterpret_cast<const uint4 *>(crow + lo_chunk_off(r, 0, lo));
-            cw1[i] = fmt_u4(FMT) ? cw0[i] : *reinterpret_cast<const uint4 *>(crow + lo_chunk_off(r, 1, lo));
-            szw[i] = *reinterpret_cast<const uint32_t *>(grec + (lo > 0 ? p.meta_off + 4 * r : 0));
+            const uint32_t crow = st + (uint32_t)(lo > 0 ? p.codes_off : 0);  // lo = 0: a valid dummy address
+            cw0[i] = lds128(crow + lo_chunk_off(r, 0, lo));
+            cw1[i] = fmt_u4(FMT) ? cw0[i] : lds128(crow + lo_chunk_off(r, 1, lo));
+            szw[i] = lds32(st + (uint32_t)(lo > 0 ? p.meta_off + 4 * r : 0));
         }
 #pragma unroll
         for (int i = 0; i < R; ++i) {
             const int u = lane + 32 * i;
             if (u < K) {
-                load_hi_row(grec, u, x[i]);
+                load_hi_row(st, u, x[i]);
                 if (HAD) hadamard_pairs(x[i]);
 #pragma unroll
                 for (int j = 0; j < 16; ++j) x[i][j] = mul2(x[i][j], splat2(kDown));  // exact
@@ -262,6 +300,13 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
                 if constexpr (FMT == kFmtE4M3) dequantize_group_e4m3(w, __uint_as_float(szw[i]), kDown, x[i]);
                 else dequantize_group(w, szw[i], kDown, x[i]);
             }
+        }
+
+        // the stage has been read: the next tile's record comes in during this one
+        __syncwarp();
+        if (lane == 0 && t + 1 < t1) {
+            fence_proxy_async_smem();  // the warp's reads of the stage before the bulk copy's writes
+            issue(t + 1);
         }
 
         // The rank-1 update of token t is applied at the start of token t+1, in the
@@ -390,8 +435,12 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
             }
         }
     }
+    if (timed_out) mbar_wait_bounded(bar, parity);  // the copy in flight lands (bounded) before the CTA ends
     cp_async_wait_all();
-    if (bad_slot && lane == 0) atomicOr(p.status, (uint32_t)kDevBadSlot);
+    if (lane == 0) {
+        const uint32_t bits = (timed_out ? kDevWaitTimeout : 0u) | (bad_slot ? kDevBadSlot : 0u);
+        if (bits) atomicOr(p.status, bits);
+    }
 }
 
 }  // namespace damp
