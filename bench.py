@@ -766,6 +766,107 @@ def drift_arm(layers: int = 30, steps: int = 1024, every: int = 64):
         raise RuntimeError("device status word set during the drift run")
 
 
+def tiered_arm(steps: int = 512, every: int = 64, batch: int = 64, timing_steps: int = 1000):
+    """Decay-tiered per-head K_hi (App. E, head-budget ablation) on a GDN layer (H = 32,
+    d = 128, B = 64): the even heads decay fast and the odd heads slowly (gate logit
+    bias +1 / -3, median alpha ~0.23 / ~0.95).  Allocations common 16/16 and
+    K_fast/K_slow in {12/20, 8/24, 4/28} (mean 16, the same bytes), each a pair of head
+    groups with pi from a GPU calibration per group; then `steps` decode steps from a
+    256-step FP32 prefix.  Drift = held-out RRMSE against the FP32 trajectory (output every
+    step, state every `every` steps).  Also times one layer step at B = 256 as one launch
+    (common) and as two group launches (4/28)."""
+    import torch
+
+    import paper_2608_27513_gb300 as damp
+    from paper_2608_27513_gb300 import build, calibration
+    build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    w = wl.sweep("gdn", 16).replace(batch=batch)
+    H = w.heads
+    fast = [h % 2 == 0 for h in range(H)]
+    bias = [1.0 if f else -3.0 for f in fast]
+    allocs = [(16, 16), (12, 20), (8, 24), (4, 28)]
+    calib = wl.torch_step_inputs(w.replace(batch=32), 256, dev, seed_offset=7_000_000, gate_bias=bias)
+    setups = []
+    for kf, ks in allocs:
+        groups = damp.head_groups([kf if f else ks for f in fast], w.qk_heads, w.d_k, w.d_v, device=dev)
+        sel = calibration.calibrate_groups(groups, "gdn", calib)
+        setups.append([(L, hs, pi) for (L, hs), (_, pi) in zip(groups, sel)])
+    del calib
+    Lf = damp.Layout(H, w.qk_heads, w.d_k, w.d_v, 0, 0)
+    S = damp.new_fp32_state(Lf, w.batch, dev)
+    o = torch.empty((w.batch, H, w.d_v), device=dev)
+    for d in wl.torch_step_inputs(w, 256, dev, seed_offset=1_000_000, gate_bias=bias):
+        damp.fp32_gdn_decode_step(Lf, S, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o)
+    pools = [[damp.new_state(L, w.batch, dev) for L, _, _ in gs] for gs in setups]
+    for gs, ps in zip(setups, pools):
+        for (L, hs, pi), pl in zip(gs, ps):
+            damp.quantize_state(L, S, pi, pl)
+    acc = torch.zeros((len(allocs), 4), dtype=torch.float64, device=dev)  # o err, o ref, state err, state ref
+    oa = torch.empty_like(o)
+    for t0 in range(0, steps, 64):
+        for i, d in enumerate(wl.torch_step_inputs(w, min(64, steps - t0), dev, seed_offset=2_000_000 + t0,
+                                                   gate_bias=bias)):
+            damp.fp32_gdn_decode_step(Lf, S, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o)
+            sample = (t0 + i + 1) % every == 0
+            for a, (gs, ps) in enumerate(zip(setups, pools)):
+                for (L, hs, pi), pl in zip(gs, ps):
+                    damp.gdn_decode_step(L, pl, pi, d["q"], d["k"], d["v"], d["g"], d["beta"], o=oa)
+                acc[a, 0] += ((oa - o).double() ** 2).sum()
+                acc[a, 1] += (o.double() ** 2).sum()
+                if sample:
+                    Sa = torch.zeros_like(S)
+                    for (L, hs, pi), pl in zip(gs, ps):
+                        damp.dequantize_state(L, pl, pi, S=Sa)
+                    acc[a, 2] += ((Sa - S).double() ** 2).sum()
+                    acc[a, 3] += (S.double() ** 2).sum()
+                    del Sa
+    a = acc.cpu().numpy()
+    rows = []
+    for i, (kf, ks) in enumerate(allocs):
+        rows.append({"mode": "decay_tiered", "kind": "gdn", "batch": w.batch, "steps": steps, "k_fast": kf,
+                     "k_slow": ks, "state_rrmse": float(np.sqrt(a[i, 2] / a[i, 3])),
+                     "o_rrmse": float(np.sqrt(a[i, 0] / a[i, 1])),
+                     "bytes_per_slot": int(sum(damp.slot_bytes(L) for L, _, _ in setups[i]))})
+    # one layer step at B = 256: the common layout (one launch) and the 4/28 groups (two launches)
+    wb = w.replace(batch=256)
+    inputs = wl.torch_step_inputs(wb, 4, dev, gate_bias=bias)
+    Lc = damp.Layout(H, w.qk_heads, w.d_k, w.d_v, 16, 0)
+    pc = [damp.new_state(Lc, 256, dev) for _ in range(2)]
+    tiered = setups[-1]
+    pt = [[damp.new_state(L, 256, dev) for L, _, _ in tiered] for _ in range(2)]
+    perm_c = setups[0][0][2]
+    o2 = torch.empty((256, H, w.d_v), device=dev)
+
+    def common(i):
+        d = inputs[i % 4]
+        damp.gdn_decode_step(Lc, pc[i % 2], perm_c, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o2)
+
+    def groups(i):
+        d = inputs[i % 4]
+        for (L, hs, pi), pl in zip(tiered, pt[i % 2]):
+            damp.gdn_decode_step(L, pl, pi, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o2)
+
+    timing = {}
+    for name, fn in (("common_k16_one_launch", common), ("tiered_4_28_two_launches", groups)):
+        for i in range(20):
+            fn(i)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for i in range(timing_steps):
+            fn(i)
+        e1.record()
+        torch.cuda.synchronize()
+        timing[name] = e0.elapsed_time(e1) / timing_steps * 1e3
+    rows.append({"mode": "decay_tiered_step_time", "kind": "gdn", "batch": 256, "us_per_step": timing})
+    if damp.device_status() != 0:
+        raise RuntimeError("device status word set during the decay-tiered run")
+    for r in rows:
+        print(json.dumps(r), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -779,6 +880,8 @@ def main():
                     help="fused multi-token steps (T = 1..16 tokens per launch, B=256) instead of the bench line")
     ap.add_argument("--calibrate", action="store_true", help="GPU calibration run instead of the bench line")
     ap.add_argument("--drift", action="store_true", help="30-layer free-running drift run instead of the bench line")
+    ap.add_argument("--tiered", action="store_true",
+                    help="decay-tiered per-head K_hi (head groups) drift and step time instead of the bench line")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -802,6 +905,9 @@ def main():
         return
     if args.drift:
         drift_arm()
+        return
+    if args.tiered:
+        tiered_arm()
         return
     import torch
     import torch.distributed as dist

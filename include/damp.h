@@ -99,15 +99,30 @@ typedef enum { DAMP_IN_BF16 = 0, DAMP_IN_FP32 = 1 } damp_in_dtype;
 /* Device status bits (damp_device_status). */
 #define DAMP_DEV_WAIT_TIMEOUT 1u
 #define DAMP_DEV_BAD_SLOT 2u
+#define DAMP_DEV_BAD_HEAD 4u
 
 /*
  * Shape of one linear-attention layer's state (Sec. 3.1; Sec. 5.1 "Key-channel budget").
- *   num_heads     H      value heads; one state per (slot, head)
- *   num_qk_heads  H_qk   q/k heads; value head h reads q/k head floor(h*H_qk/H)
- *                        (GQA; H must be a multiple of H_qk)
+ *   num_heads     H      value heads held in the pool; one state per (slot, head)
+ *   num_qk_heads  H_qk   q/k heads of the operand tensors
  *   d_k, d_v             state is d_k x d_v; d_k in {32, 64, 128}; d_v a multiple of 32, <= 1024
- *   k_hi          K_hi   FP16 key channels per head, 0 <= K_hi <= d_k (same for every head)
+ *   k_hi          K_hi   FP16 key channels per head, 0 <= K_hi <= d_k (same for every head
+ *                        of the pool)
  *   lo_format            damp_lo_format of the other d_k - K_hi channels
+ *   model_heads   H_m    value heads of the operand and output tensors (v, g, beta, o, S,
+ *                        calibration accumulators); 0 means H_m = H
+ *   head_map             device int32 [H]: the model head (0 .. H_m-1) of each held head,
+ *                        or NULL for the identity (then H_m must equal H)
+ * Held head h is model head m = head_map[h] (or h); it reads q/k head floor(m*H_qk/H_m)
+ * (GQA; H_m must be a multiple of H_qk), and its per-head operands and outputs are row m
+ * of [*][H_m][...] tensors, while its permutation and packed records are row h of the pool.
+ *
+ * Head groups.  A layer whose heads protect different numbers of key channels (the
+ * decay-tiered allocation of App. E: fast- and slow-decay heads with different K_hi)
+ * is a set of layouts, one per K_hi, whose head maps partition 0 .. H_m-1; each group
+ * has its own pool and permutation table, and one call per group updates the layer
+ * (the groups write disjoint rows of o).  A head_map entry outside 0 .. H_m-1 sets
+ * DAMP_DEV_BAD_HEAD in the device status word and that head is skipped.
  */
 typedef struct {
     int32_t num_heads;
@@ -116,6 +131,8 @@ typedef struct {
     int32_t d_v;
     int32_t k_hi;
     int32_t lo_format;
+    int32_t model_heads;
+    const int32_t *head_map;
 } damp_layout;
 
 /* Checks a layout; DAMP_OK or DAMP_ERR_NULL / DAMP_ERR_SHAPE / DAMP_ERR_FORMAT. Host only. */
@@ -163,11 +180,13 @@ DAMP_API double damp_bits_per_value(const damp_layout *layout);
  *              (protected channels first).  16-B aligned.  Must be a permutation
  *              (not checked on the device).
  *   q, k       [B][H_qk][d_k] of in_dtype, natural key order, 16-B aligned
- *   v          [B][H][d_v] of in_dtype, 16-B aligned
- *   g          float [B][H]: log-decay, alpha = exp(g).  4-B aligned.
- *   beta       float [B][H]: delta-rule step size.  4-B aligned.
- *   o          float [B][H][d_v]: output S_t^T q_t from the FP32 post-update state,
- *              before requantization.  4-B aligned; must not overlap the pool.
+ *   v          [B][H_m][d_v] of in_dtype, 16-B aligned
+ *   g          float [B][H_m]: log-decay, alpha = exp(g).  4-B aligned.
+ *   beta       float [B][H_m]: delta-rule step size.  4-B aligned.
+ *   o          float [B][H_m][d_v]: output S_t^T q_t from the FP32 post-update state,
+ *              before requantization.  4-B aligned; must not overlap the pool.  Only
+ *              the rows of the layout's heads are written (H_m = H without a head map).
+ * (Per-head rows are indexed by model head, see damp_layout.)
  *   in_dtype   damp_in_dtype of q, k, v
  * Any lo_format; DAMP_LO_S8_ABSMAX_ROW runs the two-sweep step of that format.
  */
@@ -179,7 +198,7 @@ DAMP_API damp_status damp_gdn_decode_step(const damp_layout *layout, void *state
 /*
  * One KDA decode step (Sec. 3.1 with Lambda_t = diag(exp(g_t))), as
  * damp_gdn_decode_step except:
- *   g          float [B][H][d_k]: per-key-channel log-decay in natural key order,
+ *   g          float [B][H_m][d_k]: per-key-channel log-decay in natural key order,
  *              a_u = exp(g_u).  16-B aligned.
  */
 DAMP_API damp_status damp_kda_decode_step(const damp_layout *layout, void *state, int64_t num_slots,
@@ -228,10 +247,10 @@ DAMP_API damp_status damp_fp32_kda_decode_step(const damp_layout *layout, float 
  *              NULL means T for every row.  A row with length 0 keeps its state.
  *              4-B aligned.
  *   q, k       [B][T][H_qk][d_k] of in_dtype, natural key order, 16-B aligned
- *   v          [B][T][H][d_v] of in_dtype, 16-B aligned
- *   g          float [B][T][H]: log-decay per token, 4-B aligned
- *   beta       float [B][T][H], 4-B aligned
- *   o          float [B][T][H][d_v]: o_t from the FP32 state after token t; rows past
+ *   v          [B][T][H_m][d_v] of in_dtype, 16-B aligned
+ *   g          float [B][T][H_m]: log-decay per token, 4-B aligned
+ *   beta       float [B][T][H_m], 4-B aligned
+ *   o          float [B][T][H_m][d_v]: o_t from the FP32 state after token t; rows past
  *              a row's length are not written.  Must not overlap the pool or inputs.
  * Other arguments as in damp_gdn_decode_step.  Any lo_format except 2
  * (DAMP_ERR_FORMAT for the row-absmax format).
@@ -243,7 +262,7 @@ DAMP_API damp_status damp_gdn_prefill_chunk(const damp_layout *layout, void *sta
                                             float *o, int32_t in_dtype, void *stream);
 
 /* One KDA prefill chunk, as damp_gdn_prefill_chunk except
- *   g          float [B][T][H][d_k]: per-key-channel log-decay per token, 16-B aligned. */
+ *   g          float [B][T][H_m][d_k]: per-key-channel log-decay per token, 16-B aligned. */
 DAMP_API damp_status damp_kda_prefill_chunk(const damp_layout *layout, void *state, int64_t num_slots,
                                             const int32_t *slot_idx, int32_t batch, int32_t chunk_len,
                                             const int32_t *lengths, const uint8_t *perm, const void *q,
@@ -256,7 +275,8 @@ DAMP_API damp_status damp_kda_prefill_chunk(const damp_layout *layout, void *sta
  * the packed cache).  Row i of packed head h takes natural row perm[h][i];
  * rows < K_hi are rounded to FP16, the others H_32-transformed (format 0) and
  * quantized as their lo_format says.
- *   S      float [batch][H][d_k][d_v], natural key order, 16-B aligned, read only
+ *   S      float [batch][H_m][d_k][d_v], natural key order, 16-B aligned, read only
+ *          (the rows of the layout's heads)
  *   state, num_slots, slot_idx, batch, perm as in damp_gdn_decode_step
  */
 DAMP_API damp_status damp_quantize_state(const damp_layout *layout, const float *S, const uint8_t *perm,
@@ -265,13 +285,15 @@ DAMP_API damp_status damp_quantize_state(const damp_layout *layout, const float 
 
 /* Reconstruct FP32 states from the packed cache (the inverse map: FP16 rows widened,
  * codes dequantized s (q - z) (format 2: s q) and H_32-transformed back for format 0).
- *   S      float [batch][H][d_k][d_v] output, natural key order, 16-B aligned */
+ *   S      float [batch][H_m][d_k][d_v] output, natural key order, 16-B aligned (the
+ *          rows of the layout's heads are written) */
 DAMP_API damp_status damp_dequantize_state(const damp_layout *layout, const void *state, int64_t num_slots,
                                   const int32_t *slot_idx, int32_t batch, const uint8_t *perm,
                                   float *S, void *stream);
 
 /*
- * Copy logical tiers into / out of packed slots, bit for bit (no arithmetic).
+ * Copy logical tiers into / out of packed slots, bit for bit (no arithmetic).  The
+ * tiers are indexed by the pool's own heads (no head map).
  *   hi     uint16 [batch][H][K_hi][d_v]            FP16 bit patterns (S_hi)
  *   codes  uint8  [batch][H][d_k-K_hi][d_v]        UINT8 codes (Q_lo); int8 for format 2,
  *                                                   E4M3 bit patterns for format 5,
@@ -298,17 +320,19 @@ DAMP_API damp_status damp_unpack_tiers(const damp_layout *layout, const void *st
  * damp_calib_error_energy: E_acc[h][u] += sum_b || Q_lo(S_b,h)_{u:} - S_b,h,u: ||^2,
  *   the squared round-trip error of every key-channel row of the sampled FP32 states
  *   under layout->lo_format (H_32 + UINT8 G32, UINT8 G32, or row absmax INT8).
- *   S      float [batch][H][d_k][d_v] natural key order, 16-B aligned, read only
- *   E_acc  float [H][d_k], 4-B aligned, accumulated (the caller zeroes it first)
- * damp_calib_log_decay: G_acc[h][u] += sum_b g_b,h,u (KDA, g float [batch][H][d_k]) or
- *   sum_b g_b,h (GDN, g float [batch][H]: the head's log-decay counts for every channel).
- *   G_acc  float [H][d_k], 4-B aligned, accumulated
+ *   S      float [batch][H_m][d_k][d_v] natural key order, 16-B aligned, read only
+ *   E_acc  float [H_m][d_k], 4-B aligned, accumulated (the caller zeroes it first)
+ * damp_calib_log_decay: G_acc[h][u] += sum_b g_b,h,u (KDA, g float [batch][H_m][d_k]) or
+ *   sum_b g_b,h (GDN, g float [batch][H_m]: the head's log-decay counts for every channel).
+ *   G_acc  float [H_m][d_k], 4-B aligned, accumulated
+ * (S, g, E_acc and G_acc rows are model heads: row head_map[h] for held head h.)
  * damp_calib_select: E = E_acc / n_samples, a_eff = exp(G_acc / n_tokens),
  *   P = 1 / max(1 - a_eff^2, tau), C = E P (FP32), H = TopK_{K_hi}(C) with ties to the
  *   lower channel index, pi = the protected channels in ascending order, then the rest
  *   in ascending order.
- *   C_out     float [H][d_k] the scores (4-B aligned)
- *   perm_out  uint8 [H][d_k] pi per head, ready for the decode and prefill calls
+ *   C_out     float [H][d_k] the scores of the held heads (4-B aligned)
+ *   perm_out  uint8 [H][d_k] pi per held head, ready for the decode and prefill calls
+ *   (E_acc and G_acc are read at the model-head rows of the held heads)
  *   tau       the persistence cap, 0 < tau <= 1 (the paper uses 1e-4)
  * Each accumulator entry has one writer and a fixed summation order: repeated runs
  * give identical bits.  No call allocates or uses global scratch memory.

@@ -10,11 +10,15 @@ DampLibraryError.
     state = new_state(layout, num_slots=256, device="cuda")
     quantize_state(layout, S_fp32, perm, state)            # prefill hand-off
     o = kda_decode_step(layout, state, perm, q, k, v, g, beta)
+
+A layer whose heads keep different numbers of FP16 key channels (the decay-tiered
+allocation of App. E) is a list of head groups (`head_groups`), one uniform layout,
+pool and permutation table per K_hi, each with a head map into the layer's heads.
 """
 from __future__ import annotations
 
 import ctypes
-from dataclasses import dataclass
+from dataclasses import dataclass, field
 
 from ._lib import DampLayout, DampLibraryError, lib
 
@@ -24,7 +28,8 @@ __all__ = [
     "record_bytes", "slot_bytes", "bits_per_value", "new_state", "new_fp32_state",
     "gdn_decode_step", "kda_decode_step", "gdn_prefill_chunk", "kda_prefill_chunk", "calib_error_energy", "calib_log_decay", "calib_select", "u8_gdn_decode_step", "u8_kda_decode_step",
     "fp32_gdn_decode_step", "fp32_kda_decode_step", "quantize_state", "dequantize_state",
-    "pack_tiers", "unpack_tiers", "device_status", "version", "DEV_WAIT_TIMEOUT", "DEV_BAD_SLOT",
+    "pack_tiers", "unpack_tiers", "device_status", "version", "DEV_WAIT_TIMEOUT", "DEV_BAD_SLOT", "DEV_BAD_HEAD",
+    "head_groups",
 ]
 
 LO_U8_AFFINE_G32_H32 = 0
@@ -37,6 +42,7 @@ IN_BF16 = 0
 IN_FP32 = 1
 DEV_WAIT_TIMEOUT = 1
 DEV_BAD_SLOT = 2
+DEV_BAD_HEAD = 4
 
 
 class DampError(RuntimeError):
@@ -48,15 +54,52 @@ class DampError(RuntimeError):
 
 @dataclass(frozen=True)
 class Layout:
+    """damp_layout: num_heads held heads (one state per slot and head), q/k heads of the
+    operands, d_k x d_v states, K_hi FP16 key channels, the low-tier format; for a head
+    group of a layer, model_heads (value heads of the operand tensors) and head_map
+    (int32 CUDA tensor [num_heads]: the model head of each held head)."""
     num_heads: int
     num_qk_heads: int
     d_k: int
     d_v: int
     k_hi: int
     lo_format: int = LO_U8_AFFINE_G32_H32
+    model_heads: int = 0
+    head_map: object = field(default=None, compare=False, repr=False)
+
+    def __post_init__(self):
+        if self.head_map is not None:
+            import torch
+            m = self.head_map
+            if (not isinstance(m, torch.Tensor) or m.dtype != torch.int32 or not m.is_cuda or not m.is_contiguous()
+                    or m.shape != (self.num_heads,)):
+                raise ValueError(f"head_map must be a contiguous int32 CUDA tensor of shape [{self.num_heads}]")
+
+    @property
+    def heads_of_operands(self) -> int:
+        """H_m: value heads of v, g, beta, o and S."""
+        return self.model_heads or self.num_heads
 
     def c(self) -> DampLayout:
-        return DampLayout(self.num_heads, self.num_qk_heads, self.d_k, self.d_v, self.k_hi, self.lo_format)
+        return DampLayout(self.num_heads, self.num_qk_heads, self.d_k, self.d_v, self.k_hi, self.lo_format,
+                          self.model_heads, None if self.head_map is None else self.head_map.data_ptr())
+
+
+def head_groups(k_hi_of_head, num_qk_heads: int, d_k: int, d_v: int, lo_format: int = LO_U8_AFFINE_G32_H32,
+                device="cuda"):
+    """Layouts of a layer whose heads keep different numbers of FP16 key channels
+    (App. E, decay-tiered allocation): one layout per distinct K_hi, held heads in
+    ascending model-head order, each with its head map.  Returns [(layout, heads)],
+    heads the list of model heads of the group."""
+    import torch
+    ks = [int(k) for k in k_hi_of_head]
+    H = len(ks)
+    out = []
+    for K in sorted(set(ks)):
+        heads = [h for h in range(H) if ks[h] == K]
+        m = torch.tensor(heads, dtype=torch.int32, device=device)
+        out.append((Layout(len(heads), num_qk_heads, d_k, d_v, K, lo_format, model_heads=H, head_map=m), heads))
+    return out
 
 
 def _ptr(t):
@@ -131,7 +174,9 @@ def _step(fn_name, layout, state, perm, q, k, v, g, beta, o, slot_idx, num_slots
         _cuda_contig(n, t)
     B = v.shape[0]
     if o is None:
-        o = torch.empty((B, layout.num_heads, layout.d_v), dtype=torch.float32, device=v.device)
+        # a head group writes only its heads' rows: the others start at zero
+        alloc = torch.empty if layout.head_map is None else torch.zeros
+        o = alloc((B, layout.heads_of_operands, layout.d_v), dtype=torch.float32, device=v.device)
     if num_slots is None:
         num_slots = state.shape[0]
     c = layout.c()
@@ -177,7 +222,7 @@ def _prefill(fn_name, layout, state, perm, q, k, v, g, beta, o, lengths, slot_id
         _cuda_contig(n, t)
     B, T = v.shape[0], v.shape[1]
     if o is None:
-        o = torch.zeros((B, T, layout.num_heads, layout.d_v), dtype=torch.float32, device=v.device)
+        o = torch.zeros((B, T, layout.heads_of_operands, layout.d_v), dtype=torch.float32, device=v.device)
     if num_slots is None:
         num_slots = state.shape[0]
     c = layout.c()
@@ -249,7 +294,7 @@ def dequantize_state(layout, state, perm, batch=None, S=None, slot_idx=None, num
         _cuda_contig(n, t)
     B = (slot_idx.shape[0] if slot_idx is not None else state.shape[0]) if batch is None else batch
     if S is None:
-        S = torch.empty((B, layout.num_heads, layout.d_k, layout.d_v), dtype=torch.float32, device=state.device)
+        S = torch.zeros((B, layout.heads_of_operands, layout.d_k, layout.d_v), dtype=torch.float32, device=state.device)
     c = layout.c()
     _check(lib().damp_dequantize_state(ctypes.byref(c), _ptr(state),
                                        state.shape[0] if num_slots is None else num_slots, _ptr(slot_idx), B,

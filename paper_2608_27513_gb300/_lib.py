@@ -18,7 +18,8 @@ class DampLibraryError(RuntimeError):
 
 class DampLayout(ctypes.Structure):
     _fields_ = [("num_heads", ctypes.c_int32), ("num_qk_heads", ctypes.c_int32), ("d_k", ctypes.c_int32),
-                ("d_v", ctypes.c_int32), ("k_hi", ctypes.c_int32), ("lo_format", ctypes.c_int32)]
+                ("d_v", ctypes.c_int32), ("k_hi", ctypes.c_int32), ("lo_format", ctypes.c_int32),
+                ("model_heads", ctypes.c_int32), ("head_map", ctypes.c_void_p)]
 
 
 _P = ctypes.c_void_p

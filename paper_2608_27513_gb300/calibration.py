@@ -8,10 +8,10 @@ from __future__ import annotations
 import paper_2608_27513_gb300 as damp
 
 
-def calibrate(layout, kind: str, token_inputs, every: int = 8, tau: float = 1e-4, stream=None):
-    """token_inputs: sequence of per-token dicts of device tensors (q, k, v, g, beta) for
-    the calibration documents (rows = documents), in token order.  Returns (C, perm):
-    float32 [H, d_k] scores and uint8 [H, d_k] permutations."""
+def accumulate(layout, kind: str, token_inputs, every: int = 8, stream=None):
+    """The FP32 trajectories of the calibration documents under a layout holding every
+    head of the layer (no head map): returns (E_acc, n_samples, G_acc, n_tokens), the
+    error-energy and log-decay sums over the layer's heads [H, d_k]."""
     import torch
     inputs = list(token_inputs)
     n_docs = inputs[0]["v"].shape[0]
@@ -28,4 +28,26 @@ def calibrate(layout, kind: str, token_inputs, every: int = 8, tau: float = 1e-4
         if (t + 1) % every == 0:
             damp.calib_error_energy(layout, S, E_acc, stream=stream)
             n_samples += n_docs
-    return damp.calib_select(layout, E_acc, max(n_samples, 1), G_acc, n_docs * len(inputs), tau, stream=stream)
+    return E_acc, max(n_samples, 1), G_acc, n_docs * len(inputs)
+
+
+def calibrate(layout, kind: str, token_inputs, every: int = 8, tau: float = 1e-4, stream=None):
+    """token_inputs: sequence of per-token dicts of device tensors (q, k, v, g, beta) for
+    the calibration documents (rows = documents), in token order.  Returns (C, perm):
+    float32 [H, d_k] scores and uint8 [H, d_k] permutations."""
+    E_acc, n_samples, G_acc, n_tokens = accumulate(layout, kind, token_inputs, every, stream)
+    return damp.calib_select(layout, E_acc, n_samples, G_acc, n_tokens, tau, stream=stream)
+
+
+def calibrate_groups(groups, kind: str, token_inputs, every: int = 8, tau: float = 1e-4, stream=None):
+    """Calibration of a layer split into head groups (damp.head_groups: a layout per
+    K_hi with its head map).  The trajectories and sums run once over all heads; each
+    group then selects its own K_hi channels per head.  Returns [(C, perm)] per group."""
+    g0 = groups[0][0] if isinstance(groups[0], tuple) else groups[0]
+    full = damp.Layout(g0.heads_of_operands, g0.num_qk_heads, g0.d_k, g0.d_v, 0, g0.lo_format)
+    E_acc, n_samples, G_acc, n_tokens = accumulate(full, kind, token_inputs, every, stream)
+    out = []
+    for gr in groups:
+        L = gr[0] if isinstance(gr, tuple) else gr
+        out.append(damp.calib_select(L, E_acc, n_samples, G_acc, n_tokens, tau, stream=stream))
+    return out

@@ -29,18 +29,30 @@ def save_layout(path: str, layout: "damp.Layout", perms) -> None:
     doc = {"version": LAYOUT_VERSION, "num_heads": layout.num_heads, "num_qk_heads": layout.num_qk_heads,
            "d_k": layout.d_k, "d_v": layout.d_v, "k_hi": layout.k_hi, "lo_format": layout.lo_format,
            "perm": perms.tolist()}
+    if layout.head_map is not None:  # one head group of a layer: its model heads
+        doc["model_heads"] = layout.heads_of_operands
+        doc["heads"] = [int(h) for h in layout.head_map.cpu().tolist()]
     with open(path, "w") as f:
         json.dump(doc, f)
 
 
-def load_layout(path: str):
-    """Read (Layout, perms uint8 [H, d_k]) written by save_layout; the layout is validated."""
+def load_layout(path: str, device="cuda"):
+    """Read (Layout, perms uint8 [H, d_k]) written by save_layout; the layout is validated.
+    A head group's map is placed on `device`."""
     with open(path) as f:
         doc = json.load(f)
     if doc.get("version") != LAYOUT_VERSION:
         raise ValueError(f"unknown layout file version {doc.get('version')}")
+    head_map = None
+    if "heads" in doc:
+        import torch
+        heads = [int(h) for h in doc["heads"]]
+        if len(heads) != doc["num_heads"] or len(set(heads)) != len(heads) or \
+                not all(0 <= h < doc["model_heads"] for h in heads):
+            raise ValueError("the head map does not match the layout")
+        head_map = torch.tensor(heads, dtype=torch.int32, device=device)
     layout = damp.Layout(doc["num_heads"], doc["num_qk_heads"], doc["d_k"], doc["d_v"], doc["k_hi"],
-                         doc["lo_format"])
+                         doc["lo_format"], model_heads=doc.get("model_heads", 0), head_map=head_map)
     perms = np.asarray(doc["perm"], dtype=np.uint8)
     if perms.shape != (layout.num_heads, layout.d_k):
         raise ValueError("perm table does not match the layout")

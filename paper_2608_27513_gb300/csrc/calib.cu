@@ -9,11 +9,16 @@
 //                        (ties to the lower channel), pi = stable partition (H first,
 //                        each part in ascending channel order)
 //
+// Per-head rows of S, g, E_acc and G_acc are model heads (head_map[h], or h); C_out and
+// perm_out rows are the layout's own heads.  A head_map entry outside 0 .. Hm-1 makes the
+// head's work a no-op and sets kDevBadHead in the status word.
+//
 // Every accumulator entry has exactly one writer per call and sums in a fixed order,
 // so repeated runs give the same bits; no global scratch is used (partials of the
 // error energy meet in shared memory).
 #include "damp_common.cuh"
 #include "damp_internal.h"
+#include "formats.cuh"
 
 #include <algorithm>
 
@@ -27,17 +32,32 @@ namespace {
 // scheduling).
 constexpr int kEeWarps = 8;
 
+__device__ uint32_t g_status_calib;
+
+// model head of held head h, or -1 (flagged) when the map entry is out of range
+__device__ __forceinline__ int calib_model_head(const int32_t *head_map, int h, int Hm) {
+    const int m = head_map ? head_map[h] : h;
+    if (m < 0 || m >= Hm) {
+        atomicOr(&g_status_calib, (uint32_t)kDevBadHead);
+        return -1;
+    }
+    return m;
+}
+
 template <int FMT>
 __global__ void __launch_bounds__(32 * kEeWarps) calib_error_energy_kernel(const float *S, int32_t batch, int32_t H,
+                                                                           int32_t Hm, const int32_t *head_map,
                                                                            int32_t dk, int32_t dv, float *E_acc) {
     __shared__ float partial[kEeWarps][32];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int groups = (dk + 31) / 32;
     const int h = (int)(blockIdx.x / groups);
     const int u = (int)(blockIdx.x % groups) * 32 + lane;  // d_k is a multiple of 32
+    const int m = calib_model_head(head_map, h, Hm);  // the same for the whole CTA
+    if (m < 0) return;
     float err = 0.f;
     for (int b = warp; b < batch; b += kEeWarps) {
-        const float *row = S + (((int64_t)b * H + h) * dk + u) * dv;
+        const float *row = S + (((int64_t)b * Hm + m) * dk + u) * dv;
         if (FMT == 2) {
             // per-row symmetric absmax INT8: s = max|x| / 127, q = sat(rne(x / s)), x^ = s q
             float amax = 0.f;
@@ -61,13 +81,25 @@ __global__ void __launch_bounds__(32 * kEeWarps) calib_error_energy_kernel(const
             }
 #pragma unroll
             for (int m = 0; m < 16; ++m) y[m] = x[m];
-            if (FMT == 0) hadamard_pairs(y);
+            if (fmt_had(FMT)) hadamard_pairs(y);
+            if (FMT == kFmtE4M3) {  // natural domain, one FP32 scale per group
+                uint32_t w[8];
+                const float sc = quantize_group_e4m3(y, w);
+                dequantize_group_e4m3(w, sc, 1.0f, y);
+            } else {
 #pragma unroll
-            for (int m = 0; m < 16; ++m) y[m] = mul2(y[m], splat2(kDown));  // working scale of the quantizer
-            uint32_t w[8];
-            const uint32_t sz = quantize_group(y, w);
-            dequantize_group(w, sz, 1.0f, y);
-            if (FMT == 0) hadamard_pairs(y);
+                for (int m = 0; m < 16; ++m) y[m] = mul2(y[m], splat2(kDown));  // working scale of the quantizer
+                if (fmt_u4(FMT)) {
+                    uint32_t w[4];
+                    const uint32_t sz = quantize_group_u4(y, w);
+                    dequantize_group_u4(w, sz, 1.0f, y);
+                } else {
+                    uint32_t w[8];
+                    const uint32_t sz = quantize_group(y, w);
+                    dequantize_group(w, sz, 1.0f, y);
+                }
+            }
+            if (fmt_had(FMT)) hadamard_pairs(y);
 #pragma unroll
             for (int m = 0; m < 16; ++m) {
                 const float d0 = y[m].x - x[m].x, d1 = y[m].y - x[m].y;
@@ -81,32 +113,40 @@ __global__ void __launch_bounds__(32 * kEeWarps) calib_error_energy_kernel(const
         float sum = 0.f;
 #pragma unroll
         for (int i = 0; i < kEeWarps; ++i) sum += partial[i][lane];
-        E_acc[(int64_t)h * dk + u] += sum;
+        E_acc[(int64_t)m * dk + u] += sum;
     }
 }
 
-__global__ void calib_log_decay_kernel(const float *g, int32_t batch, int32_t H, int32_t dk, int32_t kda,
-                                       float *G_acc) {
+__global__ void calib_log_decay_kernel(const float *g, int32_t batch, int32_t H, int32_t Hm, const int32_t *head_map,
+                                       int32_t dk, int32_t kda, float *G_acc) {
     const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= (int64_t)H * dk) return;
     const int h = (int)(i / dk), u = (int)(i % dk);
+    const int m = calib_model_head(head_map, h, Hm);
+    if (m < 0) return;
     float s = 0.f;
-    for (int b = 0; b < batch; ++b) s += kda ? g[((int64_t)b * H + h) * dk + u] : g[(int64_t)b * H + h];
-    G_acc[i] += s;
+    for (int b = 0; b < batch; ++b) s += kda ? g[((int64_t)b * Hm + m) * dk + u] : g[(int64_t)b * Hm + m];
+    G_acc[(int64_t)m * dk + u] += s;
 }
 
 // One warp per head: scores, rank of every channel, then the stable partition.
 __global__ void __launch_bounds__(32) calib_select_kernel(const float *E_acc, float inv_samples, const float *G_acc,
-                                                          float inv_tokens, float tau, int32_t H, int32_t dk,
-                                                          int32_t k_hi, float *C_out, uint8_t *perm_out) {
+                                                          float inv_tokens, float tau, int32_t H, int32_t Hm,
+                                                          const int32_t *head_map, int32_t dk, int32_t k_hi,
+                                                          float *C_out, uint8_t *perm_out) {
     __shared__ float sc[256];
     const int lane = threadIdx.x & 31;
     const int h = blockIdx.x;
     if (h >= H) return;
+    int m = head_map ? head_map[h] : h;  // warp-uniform
+    if (m < 0 || m >= Hm) {
+        if (lane == 0) atomicOr(&g_status_calib, (uint32_t)kDevBadHead);
+        return;
+    }
     for (int u = lane; u < dk; u += 32) {
-        const float E = E_acc[(int64_t)h * dk + u] * inv_samples;
+        const float E = E_acc[(int64_t)m * dk + u] * inv_samples;
         // 1 - a_eff^2 = 1 - exp(2 mean log a) = -expm1(2 mean log a): no cancellation near a = 1
-        const float one_minus_a2 = -expm1f(2.0f * (G_acc[(int64_t)h * dk + u] * inv_tokens));
+        const float one_minus_a2 = -expm1f(2.0f * (G_acc[(int64_t)m * dk + u] * inv_tokens));
         const float P = 1.0f / fmaxf(one_minus_a2, tau);
         const float C = E * P;
         sc[u] = C;
@@ -143,28 +183,44 @@ __global__ void __launch_bounds__(32) calib_select_kernel(const float *E_acc, fl
 
 }  // namespace
 
-cudaError_t launch_calib_error_energy(const float *S, int32_t batch, int32_t H, int32_t dk, int32_t dv, int32_t fmt,
-                                      float *E_acc, cudaStream_t stream) {
+cudaError_t launch_calib_error_energy(const float *S, int32_t batch, int32_t H, int32_t Hm, const int32_t *head_map,
+                                      int32_t dk, int32_t dv, int32_t fmt, float *E_acc, cudaStream_t stream) {
     const int64_t grid = (int64_t)H * ((dk + 31) / 32);
-    void (*kern)(const float *, int32_t, int32_t, int32_t, int32_t, float *) =
-        fmt == 0 ? calib_error_energy_kernel<0> : fmt == 1 ? calib_error_energy_kernel<1> : calib_error_energy_kernel<2>;
-    kern<<<(unsigned)grid, 32 * kEeWarps, 0, stream>>>(S, batch, H, dk, dv, E_acc);
+    void (*kern)(const float *, int32_t, int32_t, int32_t, const int32_t *, int32_t, int32_t, float *) = nullptr;
+    switch (fmt) {
+        case kFmtU8H32: kern = calib_error_energy_kernel<kFmtU8H32>; break;
+        case kFmtU8: kern = calib_error_energy_kernel<kFmtU8>; break;
+        case kFmtS8Row: kern = calib_error_energy_kernel<kFmtS8Row>; break;
+        case kFmtU4H32: kern = calib_error_energy_kernel<kFmtU4H32>; break;
+        case kFmtU4: kern = calib_error_energy_kernel<kFmtU4>; break;
+        case kFmtE4M3: kern = calib_error_energy_kernel<kFmtE4M3>; break;
+        default: return cudaErrorInvalidValue;
+    }
+    kern<<<(unsigned)grid, 32 * kEeWarps, 0, stream>>>(S, batch, H, Hm, head_map, dk, dv, E_acc);
     return cudaGetLastError();
 }
 
-cudaError_t launch_calib_log_decay(const float *g, int32_t batch, int32_t H, int32_t dk, int32_t kda, float *G_acc,
-                                   cudaStream_t stream) {
+cudaError_t launch_calib_log_decay(const float *g, int32_t batch, int32_t H, int32_t Hm, const int32_t *head_map,
+                                   int32_t dk, int32_t kda, float *G_acc, cudaStream_t stream) {
     const int64_t n = (int64_t)H * dk;
-    calib_log_decay_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(g, batch, H, dk, kda, G_acc);
+    calib_log_decay_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(g, batch, H, Hm, head_map, dk, kda,
+                                                                              G_acc);
     return cudaGetLastError();
 }
 
 cudaError_t launch_calib_select(const float *E_acc, int64_t n_samples, const float *G_acc, int64_t n_tokens, float tau,
-                                int32_t H, int32_t dk, int32_t k_hi, float *C_out, uint8_t *perm_out,
-                                cudaStream_t stream) {
+                                int32_t H, int32_t Hm, const int32_t *head_map, int32_t dk, int32_t k_hi,
+                                float *C_out, uint8_t *perm_out, cudaStream_t stream) {
     calib_select_kernel<<<H, 32, 0, stream>>>(E_acc, 1.0f / (float)n_samples, G_acc, 1.0f / (float)n_tokens, tau, H,
-                                               dk, k_hi, C_out, perm_out);
+                                               Hm, head_map, dk, k_hi, C_out, perm_out);
     return cudaGetLastError();
+}
+
+cudaError_t take_status_calib(uint32_t *bits) {
+    uint32_t zero = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(bits, g_status_calib, sizeof(uint32_t));
+    if (e != cudaSuccess) return e;
+    return cudaMemcpyToSymbol(g_status_calib, &zero, sizeof(uint32_t));
 }
 
 }  // namespace damp

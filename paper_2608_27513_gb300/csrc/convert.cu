@@ -32,6 +32,8 @@ struct ConvParams {
     uint8_t *codes;
     uint16_t *meta;
     int32_t batch, H, dk, dv, V, K;
+    int32_t Hm;                // heads of S: held head h is row head_map[h] (or h)
+    const int32_t *head_map;
     int32_t rec_bytes, codes_off, meta_off;
     int64_t slot_bytes, total_tiles;
     uint32_t *status;
@@ -49,7 +51,7 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
     const int64_t nwt = ((int64_t)gridDim.x * blockDim.x) >> 5;
     const int K = p.K;
     const int lo = p.dk - K;
-    bool bad_slot = false;
+    bool bad_slot = false, bad_head = false;
     for (int64_t t = gw; t < p.total_tiles; t += nwt) {
         const int c = (int)(t % p.V);
         const int64_t bh = t / p.V;
@@ -58,6 +60,11 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
         const int64_t slot = p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b;
         if (slot < 0 || slot >= p.num_slots) {
             bad_slot = true;
+            continue;
+        }
+        const int mh = p.head_map ? p.head_map[h] : h;  // row of S (conversions only)
+        if (mh < 0 || mh >= p.Hm) {
+            bad_head = true;
             continue;
         }
         uint8_t *rec = p.state + slot * p.slot_bytes + (int64_t)(h * p.V + c) * p.rec_bytes;
@@ -71,7 +78,7 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
             uint32_t *mrec = reinterpret_cast<uint32_t *>(rec + p.meta_off + 4 * r);
             if (OP == kQuantize || OP == kDequantize) {
                 const int n = p.perm[(int64_t)h * p.dk + u] & (p.dk - 1);  // d_k is a power of two
-                float *row = p.S + ((((int64_t)b * p.H + h) * p.dk + n) * p.dv + c * kG);
+                float *row = p.S + ((((int64_t)b * p.Hm + mh) * p.dk + n) * p.dv + c * kG);
                 float2 x[16];
                 if (OP == kQuantize) {
 #pragma unroll
@@ -140,8 +147,8 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
             const bool two = u + 1 < K;
             uint32_t *word = reinterpret_cast<uint32_t *>(rec + hi_elem_off(u, lane));
             if (OP == kQuantize || OP == kDequantize) {
-                float *r0 = p.S + ((((int64_t)b * p.H + h) * p.dk + (p.perm[(int64_t)h * p.dk + u] & (p.dk - 1))) * p.dv + c * kG + lane);
-                float *r1 = two ? p.S + ((((int64_t)b * p.H + h) * p.dk + (p.perm[(int64_t)h * p.dk + u + 1] & (p.dk - 1))) * p.dv + c * kG + lane) : nullptr;
+                float *r0 = p.S + ((((int64_t)b * p.Hm + mh) * p.dk + (p.perm[(int64_t)h * p.dk + u] & (p.dk - 1))) * p.dv + c * kG + lane);
+                float *r1 = two ? p.S + ((((int64_t)b * p.Hm + mh) * p.dk + (p.perm[(int64_t)h * p.dk + u + 1] & (p.dk - 1))) * p.dv + c * kG + lane) : nullptr;
                 if (OP == kQuantize) {
                     *word = f2_to_h2(*r0, two ? *r1 : 0.f);
                 } else {
@@ -167,7 +174,8 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
             if (lane < p.rec_bytes - used) rec[used + lane] = 0;
         }
     }
-    if (bad_slot && lane == 0) atomicOr(p.status, (uint32_t)kDevBadSlot);
+    if (lane == 0 && (bad_slot || bad_head))
+        atomicOr(p.status, (bad_slot ? (uint32_t)kDevBadSlot : 0u) | (bad_head ? (uint32_t)kDevBadHead : 0u));
 }
 
 template <int OP>
@@ -187,6 +195,8 @@ static cudaError_t launch_convert(const ConvArgs &a, cudaStream_t stream) {
     p.meta = a.meta;
     p.batch = a.batch;
     p.H = a.H;
+    p.Hm = a.head_map ? a.Hm : a.H;  // the tiers of pack / unpack are pool-indexed
+    p.head_map = a.head_map;
     p.dk = a.dk;
     p.dv = a.dv;
     p.V = a.dv / kG;

@@ -36,10 +36,17 @@ Range range_of(const void *p, int64_t bytes) {
 }
 bool overlap(Range a, Range b) { return a.lo < b.hi && b.lo < a.hi && a.hi > a.lo && b.hi > b.lo; }
 
+// value heads of the operand tensors (H_m)
+int64_t model_heads_of(const damp_layout *L) { return L->model_heads > 0 ? L->model_heads : L->num_heads; }
+
 damp_status check_layout(const damp_layout *L) {
     if (!L) return DAMP_ERR_NULL;
-    if (L->num_heads < 1 || L->num_qk_heads < 1 || L->num_heads % L->num_qk_heads) return DAMP_ERR_SHAPE;
-    if (L->num_heads > (1 << 20)) return DAMP_ERR_SHAPE;
+    if (L->num_heads < 1 || L->num_qk_heads < 1 || L->model_heads < 0) return DAMP_ERR_SHAPE;
+    const int64_t Hm = model_heads_of(L);
+    if (Hm < L->num_heads || Hm % L->num_qk_heads) return DAMP_ERR_SHAPE;
+    if (!L->head_map && Hm != L->num_heads) return DAMP_ERR_SHAPE;
+    if (L->head_map && !aligned(L->head_map, 4)) return DAMP_ERR_ALIGN;
+    if (Hm > (1 << 20)) return DAMP_ERR_SHAPE;
     if (L->d_k != 32 && L->d_k != 64 && L->d_k != 128) return DAMP_ERR_SHAPE;
     if (L->d_v < 32 || L->d_v > 1024 || L->d_v % 32) return DAMP_ERR_SHAPE;
     if (L->k_hi < 0 || L->k_hi > L->d_k) return DAMP_ERR_SHAPE;
@@ -84,12 +91,13 @@ damp_status step(const damp_layout *L, void *state, int64_t num_slots, const int
                  bool uniform) {
     damp_status st = check_layout(L);
     if (st != DAMP_OK && packed) return st;
-    if (!packed) {  // the FP32 state ignores k_hi and lo_format
+    if (!packed) {  // the FP32 state ignores k_hi and lo_format and holds every model head
         if (!L) return DAMP_ERR_NULL;
         damp_layout l2 = *L;
         l2.k_hi = 0;
         l2.lo_format = 0;
         if ((st = check_layout(&l2)) != DAMP_OK) return st;
+        if (L->head_map) return DAMP_ERR_SHAPE;
     }
     if (uniform && L->k_hi != 0) return DAMP_ERR_SHAPE;
     if (in_dtype != DAMP_IN_BF16 && in_dtype != DAMP_IN_FP32) return DAMP_ERR_FORMAT;
@@ -102,13 +110,14 @@ damp_status step(const damp_layout *L, void *state, int64_t num_slots, const int
     if ((packed && !aligned(perm, 16)) || !aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) ||
         !aligned(g, kda ? 16 : 4) || !aligned(beta, 4) || !aligned(o, 4))
         return DAMP_ERR_ALIGN;
-    const int64_t B = batch, H = L->num_heads, Hq = L->num_qk_heads, dk = L->d_k, dv = L->d_v;
+    const int64_t B = batch, H = L->num_heads, Hm = model_heads_of(L), Hq = L->num_qk_heads, dk = L->d_k,
+                  dv = L->d_v;
     const int64_t esz = in_dtype == DAMP_IN_BF16 ? 2 : 4;
-    const Range ro = range_of(o, B * H * dv * 4);
+    const Range ro = range_of(o, B * Hm * dv * 4);
     const Range inputs[] = {range_of(q, B * Hq * dk * esz), range_of(k, B * Hq * dk * esz),
-                            range_of(v, B * H * dv * esz), range_of(g, B * H * (kda ? dk : 1) * 4),
-                            range_of(beta, B * H * 4), range_of(perm, packed ? H * dk : 0),
-                            range_of(slot_idx, slot_idx ? B * 4 : 0)};
+                            range_of(v, B * Hm * dv * esz), range_of(g, B * Hm * (kda ? dk : 1) * 4),
+                            range_of(beta, B * Hm * 4), range_of(perm, packed ? H * dk : 0),
+                            range_of(slot_idx, slot_idx ? B * 4 : 0), range_of(L->head_map, L->head_map ? H * 4 : 0)};
     if (overlap(ro, pool)) return DAMP_ERR_ALIAS;
     for (const Range &r : inputs)
         if (overlap(ro, r) || overlap(pool, r)) return DAMP_ERR_ALIAS;
@@ -116,6 +125,8 @@ damp_status step(const damp_layout *L, void *state, int64_t num_slots, const int
     StepArgs a{};
     a.H = L->num_heads;
     a.Hqk = L->num_qk_heads;
+    a.Hm = (int32_t)Hm;
+    a.head_map = L->head_map;
     a.dk = L->d_k;
     a.dv = L->d_v;
     a.K = packed ? L->k_hi : 0;
@@ -152,13 +163,15 @@ damp_status prefill(const damp_layout *L, void *state, int64_t num_slots, const 
     if (!aligned(perm, 16) || !aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(g, kda ? 16 : 4) ||
         !aligned(beta, 4) || !aligned(o, 4) || (lengths && !aligned(lengths, 4)))
         return DAMP_ERR_ALIGN;
-    const int64_t B = batch, T = chunk_len, H = L->num_heads, Hq = L->num_qk_heads, dk = L->d_k, dv = L->d_v;
+    const int64_t B = batch, T = chunk_len, H = L->num_heads, Hm = model_heads_of(L), Hq = L->num_qk_heads,
+                  dk = L->d_k, dv = L->d_v;
     const int64_t esz = in_dtype == DAMP_IN_BF16 ? 2 : 4;
-    const Range ro = range_of(o, B * T * H * dv * 4);
+    const Range ro = range_of(o, B * T * Hm * dv * 4);
     const Range inputs[] = {range_of(q, B * T * Hq * dk * esz), range_of(k, B * T * Hq * dk * esz),
-                            range_of(v, B * T * H * dv * esz), range_of(g, B * T * H * (kda ? dk : 1) * 4),
-                            range_of(beta, B * T * H * 4), range_of(perm, H * dk),
-                            range_of(slot_idx, slot_idx ? B * 4 : 0), range_of(lengths, lengths ? B * 4 : 0)};
+                            range_of(v, B * T * Hm * dv * esz), range_of(g, B * T * Hm * (kda ? dk : 1) * 4),
+                            range_of(beta, B * T * Hm * 4), range_of(perm, H * dk),
+                            range_of(slot_idx, slot_idx ? B * 4 : 0), range_of(lengths, lengths ? B * 4 : 0),
+                            range_of(L->head_map, L->head_map ? H * 4 : 0)};
     if (overlap(ro, pool)) return DAMP_ERR_ALIAS;
     for (const Range &r : inputs)
         if (overlap(ro, r) || overlap(pool, r)) return DAMP_ERR_ALIAS;
@@ -166,6 +179,8 @@ damp_status prefill(const damp_layout *L, void *state, int64_t num_slots, const 
     StepArgs a{};
     a.H = L->num_heads;
     a.Hqk = L->num_qk_heads;
+    a.Hm = (int32_t)Hm;
+    a.head_map = L->head_map;
     a.dk = L->d_k;
     a.dv = L->d_v;
     a.K = L->k_hi;
@@ -200,11 +215,11 @@ damp_status convert(const damp_layout *L, void *state, int64_t num_slots, const 
     if (batch == 0) return DAMP_OK;
     Range pool;
     if ((st = check_pool(state, num_slots, slot_idx, batch, slot_bytes_of(L), &pool)) != DAMP_OK) return st;
-    const int64_t B = batch, H = L->num_heads, dk = L->d_k, dv = L->d_v, K = L->k_hi;
+    const int64_t B = batch, H = L->num_heads, Hm = model_heads_of(L), dk = L->d_k, dv = L->d_v, K = L->k_hi;
     if (kind == kQ || kind == kDQ) {
         if (!perm || !S) return DAMP_ERR_NULL;
         if (!aligned(perm, 16) || !aligned(S, 16)) return DAMP_ERR_ALIGN;
-        const Range rs = range_of(S, B * H * dk * dv * 4);
+        const Range rs = range_of(S, B * Hm * dk * dv * 4);
         if (overlap(rs, pool) || overlap(rs, range_of(perm, H * dk)) ||
             overlap(rs, range_of(slot_idx, slot_idx ? B * 4 : 0)) || overlap(pool, range_of(perm, H * dk)))
             return DAMP_ERR_ALIAS;
@@ -222,6 +237,8 @@ damp_status convert(const damp_layout *L, void *state, int64_t num_slots, const 
     }
     ConvArgs a{};
     a.H = L->num_heads;
+    a.Hm = (int32_t)Hm;
+    a.head_map = kind == kQ || kind == kDQ ? L->head_map : nullptr;  // tiers are pool-indexed
     a.dk = L->d_k;
     a.dv = L->d_v;
     a.K = L->k_hi;
@@ -430,10 +447,10 @@ damp_status damp_calib_error_energy(const damp_layout *layout, const float *S, i
     if (batch == 0) return DAMP_OK;
     if (!S) return DAMP_ERR_NULL;
     if (!aligned(S, 16) || !aligned(E_acc, 4)) return DAMP_ERR_ALIGN;
-    const int64_t H = layout->num_heads, dk = layout->d_k, dv = layout->d_v;
-    if (overlap(range_of(S, (int64_t)batch * H * dk * dv * 4), range_of(E_acc, H * dk * 4))) return DAMP_ERR_ALIAS;
-    return launch_calib_error_energy(S, batch, (int32_t)H, (int32_t)dk, (int32_t)dv, layout->lo_format, E_acc,
-                                     static_cast<cudaStream_t>(stream)) == cudaSuccess
+    const int64_t H = layout->num_heads, Hm = model_heads_of(layout), dk = layout->d_k, dv = layout->d_v;
+    if (overlap(range_of(S, (int64_t)batch * Hm * dk * dv * 4), range_of(E_acc, Hm * dk * 4))) return DAMP_ERR_ALIAS;
+    return launch_calib_error_energy(S, batch, (int32_t)H, (int32_t)Hm, layout->head_map, (int32_t)dk, (int32_t)dv,
+                                     layout->lo_format, E_acc, static_cast<cudaStream_t>(stream)) == cudaSuccess
                ? DAMP_OK
                : DAMP_ERR_CUDA;
 }
@@ -447,11 +464,11 @@ damp_status damp_calib_log_decay(const damp_layout *layout, const float *g, int3
     if (batch == 0) return DAMP_OK;
     if (!g) return DAMP_ERR_NULL;
     if (!aligned(g, 4) || !aligned(G_acc, 4)) return DAMP_ERR_ALIGN;
-    const int64_t H = layout->num_heads, dk = layout->d_k;
-    if (overlap(range_of(g, (int64_t)batch * H * (kda ? dk : 1) * 4), range_of(G_acc, H * dk * 4)))
+    const int64_t H = layout->num_heads, Hm = model_heads_of(layout), dk = layout->d_k;
+    if (overlap(range_of(g, (int64_t)batch * Hm * (kda ? dk : 1) * 4), range_of(G_acc, Hm * dk * 4)))
         return DAMP_ERR_ALIAS;
-    return launch_calib_log_decay(g, batch, (int32_t)H, (int32_t)dk, kda ? 1 : 0, G_acc,
-                                  static_cast<cudaStream_t>(stream)) == cudaSuccess
+    return launch_calib_log_decay(g, batch, (int32_t)H, (int32_t)Hm, layout->head_map, (int32_t)dk, kda ? 1 : 0,
+                                  G_acc, static_cast<cudaStream_t>(stream)) == cudaSuccess
                ? DAMP_OK
                : DAMP_ERR_CUDA;
 }
@@ -463,14 +480,15 @@ damp_status damp_calib_select(const damp_layout *layout, const float *E_acc, int
     if (!E_acc || !G_acc || !C_out || !perm_out) return DAMP_ERR_NULL;
     if (n_samples < 1 || n_tokens < 1 || !(tau > 0.0f) || !(tau <= 1.0f)) return DAMP_ERR_SHAPE;
     if (!aligned(E_acc, 4) || !aligned(G_acc, 4) || !aligned(C_out, 4)) return DAMP_ERR_ALIGN;
-    const int64_t H = layout->num_heads, dk = layout->d_k;
+    const int64_t H = layout->num_heads, Hm = model_heads_of(layout), dk = layout->d_k;
     const Range rc = range_of(C_out, H * dk * 4), rp = range_of(perm_out, H * dk);
-    const Range ins[] = {range_of(E_acc, H * dk * 4), range_of(G_acc, H * dk * 4)};
+    const Range ins[] = {range_of(E_acc, Hm * dk * 4), range_of(G_acc, Hm * dk * 4)};
     if (overlap(rc, rp)) return DAMP_ERR_ALIAS;
     for (const Range &r : ins)
         if (overlap(r, rc) || overlap(r, rp)) return DAMP_ERR_ALIAS;
-    return launch_calib_select(E_acc, n_samples, G_acc, n_tokens, tau, (int32_t)H, (int32_t)dk, layout->k_hi, C_out,
-                               perm_out, static_cast<cudaStream_t>(stream)) == cudaSuccess
+    return launch_calib_select(E_acc, n_samples, G_acc, n_tokens, tau, (int32_t)H, (int32_t)Hm, layout->head_map,
+                               (int32_t)dk, layout->k_hi, C_out, perm_out,
+                               static_cast<cudaStream_t>(stream)) == cudaSuccess
                ? DAMP_OK
                : DAMP_ERR_CUDA;
 }
@@ -495,6 +513,8 @@ damp_status damp_device_status(uint32_t *status) {
     if (take_status_prefill_gdn_x(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     if (take_status_prefill_kda_x(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_calib(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     *status = all;
     return DAMP_OK;

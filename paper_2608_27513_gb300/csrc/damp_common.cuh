@@ -16,7 +16,7 @@ constexpr int kG = 32;                        // quantization group = value bloc
 constexpr float kInvSqrt32 = 0.17677669529663687f;  // fp32(1/sqrt(32)), H_32 normalization
 constexpr unsigned kFull = 0xffffffffu;
 
-enum : uint32_t { kDevWaitTimeout = 1u, kDevBadSlot = 2u };
+enum : uint32_t { kDevWaitTimeout = 1u, kDevBadSlot = 2u, kDevBadHead = 4u };
 
 // ---------------------------------------------------------------------------
 // Packed record geometry (one (slot, head, value block) record).

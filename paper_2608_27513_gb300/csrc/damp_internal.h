@@ -8,8 +8,11 @@
 namespace damp {
 
 struct StepArgs {
-    // layout
+    // layout; per-head operands and outputs are indexed by model head
+    // m = head_map ? head_map[h] : h over Hm heads
     int32_t H, Hqk, dk, dv, K, fmt;
+    int32_t Hm;
+    const int32_t *head_map;
     // buffers
     void *state;  // packed pool or FP32 state
     int64_t num_slots;
@@ -29,6 +32,8 @@ struct StepArgs {
 
 struct ConvArgs {
     int32_t H, dk, dv, K, fmt;
+    int32_t Hm;                // heads of S (rows head_map[h], or h)
+    const int32_t *head_map;
     void *state;
     int64_t num_slots;
     const int32_t *slot_idx;
@@ -54,12 +59,14 @@ cudaError_t launch_prefill_kda(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_prefill_gdn_x(const StepArgs &a, cudaStream_t s);  // formats 3, 4, 5
 cudaError_t launch_prefill_kda_x(const StepArgs &a, cudaStream_t s);
 // Offline key-channel selection (Sec. 5.1, Algorithm 1).
-cudaError_t launch_calib_error_energy(const float *S, int32_t batch, int32_t H, int32_t dk, int32_t dv, int32_t fmt,
-                                      float *E_acc, cudaStream_t s);
-cudaError_t launch_calib_log_decay(const float *g, int32_t batch, int32_t H, int32_t dk, int32_t kda, float *G_acc,
-                                   cudaStream_t s);
+cudaError_t launch_calib_error_energy(const float *S, int32_t batch, int32_t H, int32_t Hm, const int32_t *head_map,
+                                      int32_t dk, int32_t dv, int32_t fmt, float *E_acc, cudaStream_t s);
+cudaError_t launch_calib_log_decay(const float *g, int32_t batch, int32_t H, int32_t Hm, const int32_t *head_map,
+                                   int32_t dk, int32_t kda, float *G_acc, cudaStream_t s);
 cudaError_t launch_calib_select(const float *E_acc, int64_t n_samples, const float *G_acc, int64_t n_tokens, float tau,
-                                int32_t H, int32_t dk, int32_t k_hi, float *C_out, uint8_t *perm_out, cudaStream_t s);
+                                int32_t H, int32_t Hm, const int32_t *head_map, int32_t dk, int32_t k_hi,
+                                float *C_out, uint8_t *perm_out, cudaStream_t s);
+cudaError_t take_status_calib(uint32_t *bits);
 // Row-absmax INT8 low tier (lo_format 2); op: 0 quantize, 1 dequantize, 2 pack, 3 unpack.
 cudaError_t launch_rowabs_step(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_rowabs_convert(const ConvArgs &a, int op, cudaStream_t s);

@@ -48,6 +48,8 @@ struct PackedParams {
     const float *g, *beta;
     float *o;
     int32_t batch, H, Hqk, dk, dv, V, K;
+    int32_t Hm;                // heads of the operands: held head h is model head head_map[h] (or h)
+    const int32_t *head_map;
     int32_t rec_bytes, codes_off, meta_off;
     int64_t slot_bytes;
     int32_t nstage, stage_bytes, warp_smem, stage0_off;
@@ -92,7 +94,9 @@ __device__ __forceinline__ void advance(Cursor &k, int H, int V) {
 // KC >= 0 fixes K_hi at compile time (KC = 0: no FP16 tier) and DKC > 0 fixes d_k:
 // with both fixed, the record geometry and every row offset are constants and the
 // FP16 tier runs as straight-line code.  KC = -1, DKC = 0 is the general kernel.
-template <int RL, int DKC, int KC, bool KDA, bool HAD, bool BF16>
+// HMAP: the layout is a head group (held head h reads the operands of model head
+// head_map[h]); without it the model heads are the held heads.
+template <int RL, int DKC, int KC, bool KDA, bool HAD, bool BF16, bool HMAP>
 __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams p) {
     constexpr int R = RL > 0 ? RL : 1;
     extern __shared__ __align__(128) uint8_t smem[];
@@ -130,11 +134,18 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
     __syncwarp();
 
     auto slot_of = [&](int b) -> int64_t { return p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b; };
+    // model head of the operands of held head h; -1 when the map entry is out of range
+    auto model_head = [&](int h) -> int {
+        if constexpr (!HMAP) return h;
+        const int m = p.head_map[h];
+        return (m >= 0 && m < p.Hm) ? m : -1;
+    };
+    const int Hm = HMAP ? p.Hm : H;  // heads of the operand tensors
 
     // ---- producer (lane 0): one bulk copy of the record of tile t (cursor k) into stage s ----
     auto issue = [&](int64_t t, const Cursor &k, int s) {
         const int64_t slot = slot_of(k.b);
-        const bool ok = slot >= 0 && slot < p.num_slots;
+        const bool ok = slot >= 0 && slot < p.num_slots && (!HMAP || model_head(k.h) >= 0);
         const uint32_t st = stage0 + (uint32_t)(s * p.stage_bytes);
         const uint32_t bar = bar0 + 8 * s;
         mbar_arrive_expect_tx(bar, ok ? (uint32_t)rec_bytes : 0u);
@@ -144,8 +155,9 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
     // ---- per-(slot, head) operands: 16-byte copies by all lanes, one head ahead ----
     const uint32_t ops0 = ws + p.ops_off;
     auto load_ops = [&](int ub, int uh, uint32_t dst) {
-        const int64_t bh = (int64_t)ub * H + uh;
-        const int hq = (uh * p.Hqk) / H;
+        const int mh = HMAP ? max(model_head(uh), 0) : uh;  // an invalid head's tiles are skipped
+        const int64_t bh = (int64_t)ub * Hm + mh;
+        const int hq = (mh * p.Hqk) / Hm;
         const int nv = p.bytes_v >> 4, nq = p.bytes_qk >> 4, ng = p.bytes_g >> 4, np = p.bytes_perm >> 4;
         const int total = nv + 2 * nq + ng + np;
         const uint8_t *qrow = (const uint8_t *)p.q + ((int64_t)ub * p.Hqk + hq) * dk * esz;
@@ -189,7 +201,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
     uint32_t ob = ops0;  // operand buffer of the current (slot, head)
     int s = 0;
     uint32_t parity = 0;
-    bool timed_out = false, bad_slot = false;
+    bool timed_out = false, bad_slot = false, bad_head = false;
     int64_t t_fail = t1;
 
     for (int64_t t = t0; t < t1; ++t, advance(cur, H, V)) {
@@ -201,8 +213,10 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
         }
         const int b = cur.b, h = cur.h, c = cur.c;
         const int64_t slot = slot_of(b);
-        const bool ok = slot >= 0 && slot < p.num_slots;
-        bad_slot |= !ok;
+        const int mh = model_head(h);
+        const bool slot_ok = slot >= 0 && slot < p.num_slots, ok = slot_ok && (!HMAP || mh >= 0);
+        bad_slot |= !slot_ok;
+        if (HMAP) bad_head |= mh < 0;
         uint8_t *const grec = p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * rec_bytes;  // written in place
 
         // ---- per-(slot, head) operands, gathered into calibrated key order ----
@@ -213,9 +227,15 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             // beta (and the GDN log-decay) of the next 32 (slot, head) units are
             // loaded one per lane, long before they are needed
             if ((unit & 31) == 0) {
-                const int64_t ul = (int64_t)b * H + h + lane;
-                unit_beta = ul < (int64_t)p.batch * H ? p.beta[ul] : 0.f;
-                if (!KDA) unit_g = ul < (int64_t)p.batch * H ? p.g[ul] : 0.f;
+                const int64_t ul = (int64_t)b * H + h + lane;  // unit (batch row, held head)
+                const bool in = ul < (int64_t)p.batch * H;
+                int64_t um = ul;                                // its (batch row, model head)
+                if (HMAP && in) {
+                    const int64_t ub = ul / H;
+                    um = ub * Hm + max(model_head((int)(ul - ub * H)), 0);
+                }
+                unit_beta = in ? p.beta[um] : 0.f;
+                if (!KDA) unit_g = in ? p.g[um] : 0.f;
             }
             const float beta = __shfl_sync(kFull, unit_beta, unit & 31);
             const float alpha = KDA ? 0.f : expf(__shfl_sync(kFull, unit_g, unit & 31));
@@ -352,7 +372,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
                     dj = vj - (rlo + rhi);
                     pj = plo + phi;
                 }
-                p.o[((int64_t)b * H + h) * p.dv + c * kG + lane] = fmaf(bkq, dj, pj);
+                p.o[((int64_t)b * Hm + mh) * p.dv + c * kG + lane] = fmaf(bkq, dj, pj);
             };
             if constexpr (kLateD) {
                 dt = HAD ? vt - (rlo + hr_hi_early) : vj - (rlo + rhi);
@@ -467,7 +487,8 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
     }
     cp_async_wait_all();  // operand copies of a (slot, head) that will not run
     if (lane == 0) {
-        const uint32_t bits = (timed_out ? kDevWaitTimeout : 0u) | (bad_slot ? kDevBadSlot : 0u);
+        const uint32_t bits =
+            (timed_out ? kDevWaitTimeout : 0u) | (bad_slot ? kDevBadSlot : 0u) | (bad_head ? kDevBadHead : 0u);
         if (bits) atomicOr(p.status, bits);
     }
 }

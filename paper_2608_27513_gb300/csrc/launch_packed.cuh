@@ -34,6 +34,8 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
     p.batch = a.batch;
     p.H = a.H;
     p.Hqk = a.Hqk;
+    p.Hm = a.Hm;
+    p.head_map = a.head_map;
     p.dk = a.dk;
     p.dv = a.dv;
     p.V = V;
@@ -83,11 +85,30 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
 
     void (*kern)(PackedParams) = nullptr;
     const bool had = a.fmt == 0;
+    // a head group (head map) runs the general instances with model-head indexing
+    const bool hmap = a.head_map != nullptr;
 #define DAMP_PICK4(RL_, DKC_, KC_)                                                                \
-    if (had) kern = a.in_bf16 ? packed_step_kernel<RL_, DKC_, KC_, KDA, true, true>               \
-                              : packed_step_kernel<RL_, DKC_, KC_, KDA, true, false>;             \
-    else kern = a.in_bf16 ? packed_step_kernel<RL_, DKC_, KC_, KDA, false, true>                  \
-                          : packed_step_kernel<RL_, DKC_, KC_, KDA, false, false>;
+    if (had) kern = a.in_bf16 ? packed_step_kernel<RL_, DKC_, KC_, KDA, true, true, false>        \
+                              : packed_step_kernel<RL_, DKC_, KC_, KDA, true, false, false>;      \
+    else kern = a.in_bf16 ? packed_step_kernel<RL_, DKC_, KC_, KDA, false, true, false>           \
+                          : packed_step_kernel<RL_, DKC_, KC_, KDA, false, false, false>;
+#define DAMP_PICK4_HMAP(RL_)                                                                      \
+    if (had) kern = a.in_bf16 ? packed_step_kernel<RL_, 0, -1, KDA, true, true, true>             \
+                              : packed_step_kernel<RL_, 0, -1, KDA, true, false, true>;           \
+    else kern = a.in_bf16 ? packed_step_kernel<RL_, 0, -1, KDA, false, true, true>                \
+                          : packed_step_kernel<RL_, 0, -1, KDA, false, false, true>;
+    const int rl = (a.dk - a.K + 31) / 32;
+    if (hmap) {
+        switch (rl) {
+            case 0: DAMP_PICK4_HMAP(0) break;
+            case 1: DAMP_PICK4_HMAP(1) break;
+            case 2: DAMP_PICK4_HMAP(2) break;
+            case 3: DAMP_PICK4_HMAP(3) break;
+            case 4: DAMP_PICK4_HMAP(4) break;
+            default: break;
+        }
+        if (!kern) return cudaErrorInvalidValue;
+    }
     // compile-time layouts: d_k = 128 with the K_hi values below
 #define DAMP_FIXED(KC_)                                                                           \
     if (!kern && a.dk == 128 && a.K == KC_) {                                                     \
@@ -100,7 +121,6 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
     DAMP_FIXED(16)
     DAMP_FIXED(32)
     // general kernels: K_hi = 0 (no FP16 tier) or any K_hi, runtime d_k
-    const int rl = (a.dk - a.K + 31) / 32;
 #define DAMP_GENERAL(RL_)                                                                         \
     if (!kern && rl == RL_) {                                                                     \
         if (a.K == 0) {                                                                           \
@@ -119,6 +139,7 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
 #undef DAMP_GENERAL
 #undef DAMP_FIXED
 #undef DAMP_PICK4
+#undef DAMP_PICK4_HMAP
     if (!kern) return cudaErrorInvalidValue;
     cudaError_t e = ensure_smem_limit(reinterpret_cast<const void *>(kern), smem);
     if (e != cudaSuccess) return e;

@@ -32,6 +32,8 @@ static cudaError_t launch_prefill_impl(const StepArgs &a, cudaStream_t stream, u
     p.T = a.T;
     p.H = a.H;
     p.Hqk = a.Hqk;
+    p.Hm = a.Hm;
+    p.head_map = a.head_map;
     p.dk = a.dk;
     p.dv = a.dv;
     p.V = V;

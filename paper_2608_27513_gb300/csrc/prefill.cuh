@@ -52,6 +52,8 @@ struct PrefillParams {
     const float *g, *beta;
     float *o;
     int32_t batch, T, H, Hqk, dk, dv, V, K;
+    int32_t Hm;                // heads of the operands: held head h is model head head_map[h] (or h)
+    const int32_t *head_map;
     int32_t rec_bytes, codes_off, meta_off;
     int64_t slot_bytes, total_tiles;
     int32_t warp_stride;  // per-warp shared memory: the fixed buffers, an mbarrier and the record stage
@@ -186,25 +188,26 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
     const int64_t nwt = (int64_t)gridDim.x * nw;
     const int64_t t0 = p.total_tiles * gw / nwt, t1 = p.total_tiles * (gw + 1) / nwt;
     if (t0 >= t1) return;
-    bool bad_slot = false, timed_out = false;
+    bool bad_slot = false, bad_head = false, timed_out = false;
 
     // The record of the next tile comes in by one bulk copy (TMA engine) while the
     // current tile runs its tokens; tiles that are skipped (slot out of range, no
     // tokens) complete their phase with no bytes.
-    auto rec_of = [&](int64_t tt, int &b, int &h, int &c, int64_t &slot, int &Tb) -> uint8_t * {
+    auto rec_of = [&](int64_t tt, int &b, int &h, int &c, int &mh, int64_t &slot, int &Tb) -> uint8_t * {
         c = (int)(tt % V);
         const int64_t bh = tt / V;
         h = (int)(bh % H);
         b = (int)(bh / H);
+        mh = p.head_map ? p.head_map[h] : h;  // model head of the operands
         slot = p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b;
         Tb = p.lengths ? min(max(p.lengths[b], 0), T) : T;
         return p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * p.rec_bytes;
     };
     auto issue = [&](int64_t tt) {  // lane 0
-        int b, h, c, Tb;
+        int b, h, c, mh, Tb;
         int64_t slot;
-        uint8_t *g = rec_of(tt, b, h, c, slot, Tb);
-        const bool run = slot >= 0 && slot < p.num_slots && Tb > 0;
+        uint8_t *g = rec_of(tt, b, h, c, mh, slot, Tb);
+        const bool run = slot >= 0 && slot < p.num_slots && mh >= 0 && mh < p.Hm && Tb > 0;
         mbar_arrive_expect_tx(bar, run ? (uint32_t)p.rec_bytes : 0u);
         if (run) bulk_g2s(st, g, (uint32_t)p.rec_bytes, bar);
     };
@@ -222,26 +225,28 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
             break;
         }
         parity ^= 1u;
-        int b, h, c, Tb;
+        int b, h, c, mh, Tb;
         int64_t slot;
-        uint8_t *const grec = rec_of(t, b, h, c, slot, Tb);  // written in place
-        const bool slot_ok = slot >= 0 && slot < p.num_slots;
+        uint8_t *const grec = rec_of(t, b, h, c, mh, slot, Tb);  // written in place
+        const bool slot_ok = slot >= 0 && slot < p.num_slots, head_ok = mh >= 0 && mh < p.Hm;
         bad_slot |= !slot_ok;
-        if (!slot_ok || Tb == 0) {  // nothing landed in the stage: fetch the next record
+        bad_head |= !head_ok;
+        if (!slot_ok || !head_ok || Tb == 0) {  // nothing landed in the stage: fetch the next record
             if (lane == 0 && t + 1 < t1) issue(t + 1);
             continue;
         }
 
         // token 0's operands of this tile and their per-token strides (in bytes)
-        const int hq = (int)(((int64_t)h * p.Hqk) / H);
+        const int Hm = p.Hm;
+        const int hq = (int)(((int64_t)mh * p.Hqk) / Hm);
         const uint8_t *qt = (const uint8_t *)p.q + ((int64_t)b * T * p.Hqk + hq) * dk * esz;
         const uint8_t *kt = (const uint8_t *)p.k + ((int64_t)b * T * p.Hqk + hq) * dk * esz;
-        const uint8_t *gt = (const uint8_t *)(p.g + ((int64_t)b * T * H + h) * (KDA ? dk : 1));
-        const uint8_t *vt = (const uint8_t *)p.v + (((int64_t)b * T * H + h) * p.dv + kG * c) * esz;
-        const uint8_t *bt = (const uint8_t *)(p.beta + (int64_t)b * T * H + h);
-        float *ot = p.o + ((int64_t)b * T * H + h) * p.dv + kG * c + lane;
-        const int64_t sqk = (int64_t)p.Hqk * dk * esz, sg4 = (int64_t)H * (KDA ? dk : 1) * 4,
-                      sv = (int64_t)H * p.dv * esz, sb = (int64_t)H * 4, so = (int64_t)H * p.dv;
+        const uint8_t *gt = (const uint8_t *)(p.g + ((int64_t)b * T * Hm + mh) * (KDA ? dk : 1));
+        const uint8_t *vt = (const uint8_t *)p.v + (((int64_t)b * T * Hm + mh) * p.dv + kG * c) * esz;
+        const uint8_t *bt = (const uint8_t *)(p.beta + (int64_t)b * T * Hm + mh);
+        float *ot = p.o + ((int64_t)b * T * Hm + mh) * p.dv + kG * c + lane;
+        const int64_t sqk = (int64_t)p.Hqk * dk * esz, sg4 = (int64_t)Hm * (KDA ? dk : 1) * 4,
+                      sv = (int64_t)Hm * p.dv * esz, sb = (int64_t)Hm * 4, so = (int64_t)Hm * p.dv;
         // one token's operands into buffer dst: every copy is 16 B (beta and the GDN
         // gate 4 B); the copy counts are compile-time constants
         auto load_token = [&](int tok, uint32_t dst) {
@@ -438,7 +443,8 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
     if (timed_out) mbar_wait_bounded(bar, parity);  // the copy in flight lands (bounded) before the CTA ends
     cp_async_wait_all();
     if (lane == 0) {
-        const uint32_t bits = (timed_out ? kDevWaitTimeout : 0u) | (bad_slot ? kDevBadSlot : 0u);
+        const uint32_t bits =
+            (timed_out ? kDevWaitTimeout : 0u) | (bad_slot ? kDevBadSlot : 0u) | (bad_head ? kDevBadHead : 0u);
         if (bits) atomicOr(p.status, bits);
     }
 }

@@ -41,6 +41,8 @@ struct RowAbsStep {
     const float *g, *beta;
     float *o;
     int32_t batch, H, Hqk, dk, dv, V, K;
+    int32_t Hm;                // heads of the operands: held head h is model head head_map[h] (or h)
+    const int32_t *head_map;
     int32_t rec_bytes, codes_off, meta_off;
     int64_t slot_bytes;
     uint32_t *status;
@@ -96,14 +98,20 @@ __global__ void __launch_bounds__(32 * kRaWarps) rowabs_step_kernel(const RowAbs
         if (lane == 0) atomicOr(p.status, (uint32_t)kDevBadSlot);
         return;
     }
+    const int mh = p.head_map ? p.head_map[h] : h;
+    if (mh < 0 || mh >= p.Hm) {
+        if (lane == 0) atomicOr(p.status, (uint32_t)kDevBadHead);
+        return;
+    }
+    const int64_t mu = (int64_t)b * p.Hm + mh;  // (batch row, model head) of the operands
     const int dk = p.dk, K = p.K, lo = dk - K, V = p.V;
-    const int hq = (int)(((int64_t)h * p.Hqk) / p.H);
+    const int hq = (int)(((int64_t)mh * p.Hqk) / p.Hm);
     float *dsm = sm_d[warp];
     float *ks = sm_k[warp], *qs = sm_q[warp], *as = sm_a[warp];
 
     // operands in calibrated row order (row u holds key channel perm[h][u])
-    const float beta = p.beta[unit];
-    const float alpha = KDA ? 0.f : expf(p.g[unit]);
+    const float beta = p.beta[mu];
+    const float alpha = KDA ? 0.f : expf(p.g[mu]);
     float kq = 0.f;
     for (int u = lane; u < dk; u += 32) {
         const int ch = p.perm[(int64_t)h * dk + u] & (dk - 1);  // d_k is a power of two
@@ -111,7 +119,7 @@ __global__ void __launch_bounds__(32 * kRaWarps) rowabs_step_kernel(const RowAbs
         const float qv = load_in(p.q, ((int64_t)b * p.Hqk + hq) * dk + ch, BF16);
         ks[u] = kv;
         qs[u] = qv;
-        as[u] = KDA ? expf(p.g[unit * dk + ch]) : alpha;
+        as[u] = KDA ? expf(p.g[mu * dk + ch]) : alpha;
         kq = fmaf(kv, qv, kq);
     }
 #pragma unroll
@@ -157,8 +165,8 @@ __global__ void __launch_bounds__(32 * kRaWarps) rowabs_step_kernel(const RowAbs
             }
         }
         const int j = kG * c + lane;
-        const float dj = load_in(p.v, unit * p.dv + j, BF16) - rj;
-        p.o[unit * p.dv + j] = fmaf(bkq, dj, pj);
+        const float dj = load_in(p.v, mu * p.dv + j, BF16) - rj;
+        p.o[mu * p.dv + j] = fmaf(bkq, dj, pj);
         dsm[j] = dj;
         __syncwarp();
 #pragma unroll
@@ -223,6 +231,8 @@ struct RowAbsConv {
     int8_t *codes;
     float *meta;
     int32_t batch, H, dk, dv, V, K;
+    int32_t Hm;                // heads of S: held head h is row head_map[h] (or h)
+    const int32_t *head_map;
     int32_t rec_bytes, codes_off, meta_off;
     int64_t slot_bytes;
     uint32_t *status;
@@ -237,7 +247,7 @@ __global__ void __launch_bounds__(256) rowabs_convert_kernel(const RowAbsConv p)
     const int64_t nwt = ((int64_t)gridDim.x * blockDim.x) >> 5;
     const int dk = p.dk, K = p.K, lo = dk - K, dv = p.dv;
     const int64_t total = (int64_t)p.batch * p.H * dk;
-    bool bad_slot = false;
+    bool bad_slot = false, bad_head = false;
     for (int64_t w = gw; w < total; w += nwt) {
         const int u = (int)(w % dk);
         const int64_t bh = w / dk;
@@ -247,9 +257,15 @@ __global__ void __launch_bounds__(256) rowabs_convert_kernel(const RowAbsConv p)
             bad_slot = true;
             continue;
         }
+        const int mh = p.head_map ? p.head_map[h] : h;
+        if (mh < 0 || mh >= p.Hm) {
+            bad_head = true;
+            continue;
+        }
         uint8_t *head = p.state + slot * p.slot_bytes + (int64_t)h * p.V * p.rec_bytes;
         const int n = p.perm ? (p.perm[(int64_t)h * dk + u] & (dk - 1)) : 0;
-        float *srow = (OP == kRaQuantize || OP == kRaDequantize) ? p.S + (bh * dk + n) * dv : nullptr;
+        float *srow = (OP == kRaQuantize || OP == kRaDequantize) ? p.S + (((int64_t)b * p.Hm + mh) * dk + n) * dv
+                                                                  : nullptr;
         if (u < K) {
             for (int j = lane; j < dv; j += 32) {
                 uint8_t *rec = head + (int64_t)(j >> 5) * p.rec_bytes;
@@ -298,7 +314,8 @@ __global__ void __launch_bounds__(256) rowabs_convert_kernel(const RowAbsConv p)
                 if (lane < p.rec_bytes - used) head[(int64_t)c * p.rec_bytes + used + lane] = 0;
         }
     }
-    if (bad_slot && lane == 0) atomicOr(p.status, (uint32_t)kDevBadSlot);
+    if (lane == 0 && (bad_slot || bad_head))
+        atomicOr(p.status, (bad_slot ? (uint32_t)kDevBadSlot : 0u) | (bad_head ? (uint32_t)kDevBadHead : 0u));
 }
 
 uint32_t *status_word(cudaError_t *e) {
@@ -330,6 +347,8 @@ cudaError_t launch_rowabs_step(const StepArgs &a, cudaStream_t stream) {
     p.batch = a.batch;
     p.H = a.H;
     p.Hqk = a.Hqk;
+    p.Hm = a.Hm;
+    p.head_map = a.head_map;
     p.dk = a.dk;
     p.dv = a.dv;
     p.V = a.dv / kG;
@@ -364,6 +383,8 @@ cudaError_t launch_rowabs_convert(const ConvArgs &a, int op, cudaStream_t stream
     p.meta = reinterpret_cast<float *>(a.meta);
     p.batch = a.batch;
     p.H = a.H;
+    p.Hm = a.head_map ? a.Hm : a.H;  // the tiers of pack / unpack are pool-indexed
+    p.head_map = a.head_map;
     p.dk = a.dk;
     p.dv = a.dv;
     p.V = a.dv / kG;

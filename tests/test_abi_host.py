@@ -88,6 +88,30 @@ def test_layout_validation(L, kw, status):
     assert L.damp_bits_per_value(ctypes.byref(c)) == -1.0
 
 
+def test_head_group_layouts(L):
+    """Head groups (layers with per-head K_hi): held heads, model heads and the map."""
+    fb = FakeBuffers(n=2, size=4096)
+
+    def v(H, Hq, Hm, m):
+        c = _lib.DampLayout(H, Hq, 128, 128, 16, 0, Hm, m)
+        return L.damp_validate_layout(ctypes.byref(c)), c
+
+    st, ok = v(4, 4, 8, fb[0])
+    assert st == 0
+    assert L.damp_slot_bytes(ctypes.byref(ok)) == 4 * 4 * damp.record_bytes(_layout(k_hi=16))
+    assert v(3, 4, 8, fb[0])[0] == 0                      # a group need not hold whole q/k groups
+    assert v(4, 4, 0, None)[0] == 0                       # model_heads 0: the held heads
+    assert v(4, 4, 8, None)[0] == 2                       # more model heads but no map
+    assert v(8, 4, 4, fb[0])[0] == 2                      # fewer model heads than held heads
+    assert v(4, 3, 8, fb[0])[0] == 2                      # model heads not a multiple of the q/k heads
+    assert v(4, 4, -1, fb[0])[0] == 2
+    assert v(4, 4, 8, ctypes.c_void_p(fb.ptrs[0] + 2))[0] == 3   # a misaligned map
+    # the FP32-state baseline holds every model head: a head map is rejected before launch
+    _, c = v(4, 4, 4, fb[0])
+    assert L.damp_fp32_kda_decode_step(ctypes.byref(c), fb[1], 4, None, 4, fb[1], fb[1], fb[1], fb[1], fb[1],
+                                       fb[1], 0, None) == 2
+
+
 class FakeBuffers:
     """Distinct, aligned host addresses standing in for device buffers (never dereferenced)."""
 

@@ -150,17 +150,20 @@ def random_states(seed: int, n: int, d_k: int, d_v: int, scale: float = 1.0) -> 
     return (scale * rows * cols * r.standard_normal((n, d_k, d_v))).astype(np.float32)
 
 
-def torch_step_inputs(w: Workload, n_steps: int, device, seed_offset: int = 0) -> list:
+def torch_step_inputs(w: Workload, n_steps: int, device, seed_offset: int = 0, gate_bias=None) -> list:
     """Device-resident operands for throughput runs, drawn with torch's generator.
 
     Same recipe and shapes as `step_inputs` (not the same numbers): a list of
-    n_steps dicts of torch tensors on `device`.
+    n_steps dicts of torch tensors on `device`.  gate_bias (GDN only, [H] floats)
+    shifts each head's gate logit, g = -softplus(N(0,1) + bias_h): negative biases
+    give slow-decay heads (alpha near 1), positive ones fast-decay heads.
     """
     import torch
     gen = torch.Generator(device=device)
     gen.manual_seed(w.seed * 1_000_003 + w.layer * 7919 + seed_offset)
     u = torch.from_numpy(kda_u(w)).to(device=device, dtype=torch.float32) if w.kind == "kda" else None
     dt = torch.bfloat16 if w.in_dtype == "bf16" else torch.float32
+    bias = None if gate_bias is None else torch.as_tensor(gate_bias, dtype=torch.float32, device=device)
     out = []
     for _ in range(n_steps):
         def n(*shape):
@@ -172,7 +175,8 @@ def torch_step_inputs(w: Workload, n_steps: int, device, seed_offset: int = 0) -
         v = n(w.batch, w.heads, w.d_v)
         beta = torch.sigmoid(n(w.batch, w.heads))
         if w.kind == "gdn":
-            g = -torch.nn.functional.softplus(n(w.batch, w.heads))
+            z = n(w.batch, w.heads)
+            g = -torch.nn.functional.softplus(z if bias is None else z + bias[None])
         else:
             g = -torch.exp(u)[None] * (1.0 + 0.05 * n(w.batch, w.heads, w.d_k))
         out.append({"q": q.to(dt).contiguous(), "k": k.to(dt).contiguous(), "v": v.to(dt).contiguous(),
