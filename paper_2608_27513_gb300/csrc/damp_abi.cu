@@ -75,8 +75,10 @@ damp_status check_pool(const void *state, int64_t num_slots, const int32_t *slot
 cudaError_t launch_step(const StepArgs &a, bool packed, cudaStream_t s) {
     if (!packed) return launch_fp32_step(a, s);
     if (a.fmt == DAMP_LO_S8_ABSMAX_ROW) return launch_rowabs_step(a, s);
+    if (a.fmt == DAMP_LO_U4_AFFINE_G32_H32 || a.fmt == DAMP_LO_U4_AFFINE_G32)
+        return a.kda ? launch_packed_kda_u4(a, s) : launch_packed_gdn_u4(a, s);
     if (a.fmt != DAMP_LO_U8_AFFINE_G32_H32 && a.fmt != DAMP_LO_U8_AFFINE_G32) {
-        // UINT4 and FP8 tiers: a decode step is a one-token chunk of the generic kernel
+        // FP8 tier: a decode step is a one-token chunk of the chunk kernel
         StepArgs one = a;
         one.T = 1;
         one.lengths = nullptr;
@@ -499,6 +501,10 @@ damp_status damp_device_status(uint32_t *status) {
     if (take_status_packed_gdn(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     if (take_status_packed_kda(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_packed_gdn_u4(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_packed_kda_u4(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     if (take_status_fp32(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;

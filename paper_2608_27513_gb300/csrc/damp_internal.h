@@ -48,6 +48,9 @@ struct ConvArgs {
 // Launchers (return the CUDA error of the launch; they perform no host-side argument checks).
 cudaError_t launch_packed_gdn(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_packed_kda(const StepArgs &a, cudaStream_t s);
+// the UINT4 low tiers (formats 3, 4)
+cudaError_t launch_packed_gdn_u4(const StepArgs &a, cudaStream_t s);
+cudaError_t launch_packed_kda_u4(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_fp32_step(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_quantize(const ConvArgs &a, cudaStream_t s);
 cudaError_t launch_dequantize(const ConvArgs &a, cudaStream_t s);
@@ -74,6 +77,8 @@ cudaError_t launch_rowabs_convert(const ConvArgs &a, int op, cudaStream_t s);
 // Read-and-clear of each translation unit's device status word.
 cudaError_t take_status_packed_gdn(uint32_t *bits);
 cudaError_t take_status_packed_kda(uint32_t *bits);
+cudaError_t take_status_packed_gdn_u4(uint32_t *bits);
+cudaError_t take_status_packed_kda_u4(uint32_t *bits);
 cudaError_t take_status_fp32(uint32_t *bits);
 cudaError_t take_status_convert(uint32_t *bits);
 cudaError_t take_status_rowabs(uint32_t *bits);

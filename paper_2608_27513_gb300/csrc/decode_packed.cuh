@@ -36,6 +36,7 @@
 #pragma once
 
 #include "damp_common.cuh"
+#include "formats.cuh"
 
 namespace damp {
 
@@ -96,7 +97,9 @@ __device__ __forceinline__ void advance(Cursor &k, int H, int V) {
 // FP16 tier runs as straight-line code.  KC = -1, DKC = 0 is the general kernel.
 // HMAP: the layout is a head group (held head h reads the operands of model head
 // head_map[h]); without it the model heads are the held heads.
-template <int RL, int DKC, int KC, bool KDA, bool HAD, bool BF16, bool HMAP>
+// U4: UINT4 low tier (formats 3, 4: 32 nibbles in one 16-byte chunk per row, levels 15)
+// instead of UINT8.
+template <int RL, int DKC, int KC, bool KDA, bool HAD, bool BF16, bool HMAP, bool U4 = false>
 __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams p) {
     constexpr int R = RL > 0 ? RL : 1;
     extern __shared__ __align__(128) uint8_t smem[];
@@ -117,8 +120,10 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
     const int lo = dk - K;  // low-tier rows
     // record geometry (constants for a fixed layout)
     const int codes_off = KFIX ? 128 * ((KC + 1) / 2) : p.codes_off;
-    const int meta_off = (KFIX && DFIX) ? 128 * ((KC + 1) / 2) + 32 * (DKC - KC) : p.meta_off;
-    const int rec_bytes = (KFIX && DFIX) ? (128 * ((KC + 1) / 2) + 36 * (DKC - KC) + 15) & ~15 : p.rec_bytes;
+    constexpr int kCodeRow = U4 ? 16 : 32;  // code bytes per row and record
+    const int meta_off = (KFIX && DFIX) ? 128 * ((KC + 1) / 2) + kCodeRow * (DKC - KC) : p.meta_off;
+    const int rec_bytes =
+        (KFIX && DFIX) ? (128 * ((KC + 1) / 2) + (kCodeRow + 4) * (DKC - KC) + 15) & ~15 : p.rec_bytes;
     const int H = p.H, V = p.V;
 
     const int64_t gw = (int64_t)blockIdx.x * nw + warp;
@@ -301,10 +306,15 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             for (int i = 0; i < RL; ++i) {
                 const int r = min(lane + 32 * i, lo - 1);
                 const uint4 c0 = lds128(st + codes_off + lo_chunk_off(r, 0, lo));
-                const uint4 c1 = lds128(st + codes_off + lo_chunk_off(r, 1, lo));
                 const uint32_t sz = lds32(st + meta_off + 4 * r);
-                const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-                dequantize_group(w, sz, aa[i], x[i]);
+                if constexpr (U4) {
+                    const uint32_t w[4] = {c0.x, c0.y, c0.z, c0.w};
+                    dequantize_group_u4(w, sz, aa[i], x[i]);
+                } else {
+                    const uint4 c1 = lds128(st + codes_off + lo_chunk_off(r, 1, lo));
+                    const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+                    dequantize_group(w, sz, aa[i], x[i]);
+                }
 #pragma unroll
                 for (int j = 0; j < 16; ++j) {
                     acc[j] = (i == 0) ? mul2(x[i][j], kk[i]) : fma2(x[i][j], kk[i], acc[j]);
@@ -410,30 +420,55 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             bool any_zero = false;
 #pragma unroll
             for (int i = 0; i < RL; ++i) {
-                sc[i] = scale_of(mn[i], mx[i]);
-                any_zero |= sc[i] == 0.0f;
-                szw[i] = affine_finish(sc[i], mn[i], inv[i], zq[i]);
+                if constexpr (U4) {  // levels 15; the widened rule of a degenerate block is built in
+                    szw[i] = affine_params_u4(mn[i], mx[i], inv[i], zq[i]);
+                } else {
+                    sc[i] = scale_of(mn[i], mx[i]);
+                    any_zero |= sc[i] == 0.0f;
+                    szw[i] = affine_finish(sc[i], mn[i], inv[i], zq[i]);
+                }
             }
             auto encode_store = [&](int i) {
                 const int r = lane + 32 * i;
                 const float2 inv2 = splat2(inv[i] * 0x1p-110f), zc2 = splat2(zq[i] * 0x1p-149f);
-                uint32_t w[8];
+                if constexpr (U4) {
+                    // values 8m .. 8m+7 = pairs 4m .. 4m+3; value 8m ends in the low nibble
+                    uint32_t w[4];
 #pragma unroll
-                for (int m = 0; m < 8; ++m) w[m] = encode4(x[i][2 * m], x[i][2 * m + 1], inv2, zc2);
-                if (r < lo) {
-                    stg128(grec + codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
-                    stg128(grec + codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
-                    stg32(grec + meta_off + 4 * r, szw[i]);
+                    for (int m = 0; m < 4; ++m) {
+                        uint32_t a = 0u;
+#pragma unroll
+                        for (int k = 3; k >= 0; --k) {
+                            const float2 e = fma2(x[i][4 * m + k], inv2, zc2);
+                            a = pack_sat_u4(__float_as_uint(e.y), __float_as_uint(e.x), a);
+                        }
+                        w[m] = a;
+                    }
+                    if (r < lo) {
+                        stg128(grec + codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                        stg32(grec + meta_off + 4 * r, szw[i]);
+                    }
+                } else {
+                    uint32_t w[8];
+#pragma unroll
+                    for (int m = 0; m < 8; ++m) w[m] = encode4(x[i][2 * m], x[i][2 * m + 1], inv2, zc2);
+                    if (r < lo) {
+                        stg128(grec + codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                        stg128(grec + codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
+                        stg32(grec + meta_off + 4 * r, szw[i]);
+                    }
                 }
             };
 #pragma unroll
             for (int i = 0; i < RL; ++i) encode_store(i);
-            if (__any_sync(kFull, any_zero)) {
+            if constexpr (!U4) {
+                if (__any_sync(kFull, any_zero)) {
 #pragma unroll
-                for (int i = 0; i < RL; ++i) {
-                    if (sc[i] == 0.0f) {
-                        szw[i] = affine_params_scaled(mn[i], mx[i], inv[i], zq[i]);
-                        encode_store(i);
+                    for (int i = 0; i < RL; ++i) {
+                        if (sc[i] == 0.0f) {
+                            szw[i] = affine_params_scaled(mn[i], mx[i], inv[i], zq[i]);
+                            encode_store(i);
+                        }
                     }
                 }
             }

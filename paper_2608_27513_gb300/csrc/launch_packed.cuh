@@ -7,6 +7,7 @@
 
 #include "damp_internal.h"
 #include "decode_packed.cuh"
+#include "formats.cuh"
 
 namespace damp {
 
@@ -15,10 +16,11 @@ namespace damp {
 constexpr int kPackedWarps = 8;
 constexpr int kPackedStages = 3;
 
-template <bool KDA>
+// U4: the UINT4 low tiers (formats 3, 4); otherwise UINT8 (formats 0, 1).
+template <bool KDA, bool U4>
 static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, uint32_t *status) {
     const int V = a.dv / kG;
-    const RecGeom rg = rec_geom(a.dk, a.K);
+    const RecGeom rg = rec_geom(a.dk, a.K, a.fmt);
     const int esz = a.in_bf16 ? 2 : 4;
     PackedParams p{};
     p.state = static_cast<uint8_t *>(a.state);
@@ -84,19 +86,19 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
     const int smem = p.warp_smem * warps;
 
     void (*kern)(PackedParams) = nullptr;
-    const bool had = a.fmt == 0;
+    const bool had = fmt_had(a.fmt);
     // a head group (head map) runs the general instances with model-head indexing
     const bool hmap = a.head_map != nullptr;
 #define DAMP_PICK4(RL_, DKC_, KC_)                                                                \
-    if (had) kern = a.in_bf16 ? packed_step_kernel<RL_, DKC_, KC_, KDA, true, true, false>        \
-                              : packed_step_kernel<RL_, DKC_, KC_, KDA, true, false, false>;      \
-    else kern = a.in_bf16 ? packed_step_kernel<RL_, DKC_, KC_, KDA, false, true, false>           \
-                          : packed_step_kernel<RL_, DKC_, KC_, KDA, false, false, false>;
+    if (had) kern = a.in_bf16 ? packed_step_kernel<RL_, DKC_, KC_, KDA, true, true, false, U4>    \
+                              : packed_step_kernel<RL_, DKC_, KC_, KDA, true, false, false, U4>;  \
+    else kern = a.in_bf16 ? packed_step_kernel<RL_, DKC_, KC_, KDA, false, true, false, U4>       \
+                          : packed_step_kernel<RL_, DKC_, KC_, KDA, false, false, false, U4>;
 #define DAMP_PICK4_HMAP(RL_)                                                                      \
-    if (had) kern = a.in_bf16 ? packed_step_kernel<RL_, 0, -1, KDA, true, true, true>             \
-                              : packed_step_kernel<RL_, 0, -1, KDA, true, false, true>;           \
-    else kern = a.in_bf16 ? packed_step_kernel<RL_, 0, -1, KDA, false, true, true>                \
-                          : packed_step_kernel<RL_, 0, -1, KDA, false, false, true>;
+    if (had) kern = a.in_bf16 ? packed_step_kernel<RL_, 0, -1, KDA, true, true, true, U4>         \
+                              : packed_step_kernel<RL_, 0, -1, KDA, true, false, true, U4>;       \
+    else kern = a.in_bf16 ? packed_step_kernel<RL_, 0, -1, KDA, false, true, true, U4>            \
+                          : packed_step_kernel<RL_, 0, -1, KDA, false, false, true, U4>;
     const int rl = (a.dk - a.K + 31) / 32;
     if (hmap) {
         switch (rl) {
@@ -114,20 +116,22 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
     if (!kern && a.dk == 128 && a.K == KC_) {                                                     \
         DAMP_PICK4((128 - KC_ + 31) / 32, 128, KC_)                                               \
     }
+    // (the UINT4 tiers: the paper's uniform INT4 and FP16 + INT4 at K_hi = 16)
     DAMP_FIXED(0)
-    DAMP_FIXED(4)
-    DAMP_FIXED(8)
-    DAMP_FIXED(10)
     DAMP_FIXED(16)
-    DAMP_FIXED(32)
+    if constexpr (!U4) {
+        DAMP_FIXED(4)
+        DAMP_FIXED(8)
+        DAMP_FIXED(10)
+        DAMP_FIXED(32)
+    }
     // general kernels: K_hi = 0 (no FP16 tier) or any K_hi, runtime d_k
 #define DAMP_GENERAL(RL_)                                                                         \
     if (!kern && rl == RL_) {                                                                     \
-        if (a.K == 0) {                                                                           \
-            DAMP_PICK4(RL_, 0, 0)                                                                 \
-        } else {                                                                                  \
-            DAMP_PICK4(RL_, 0, -1)                                                                \
+        if constexpr (!U4) {                                                                      \
+            if (a.K == 0) DAMP_PICK4(RL_, 0, 0)                                                   \
         }                                                                                         \
+        if (!kern) DAMP_PICK4(RL_, 0, -1)                                                         \
     }
     if (!kern && rl == 0) {
         DAMP_PICK4(0, 0, -1)
