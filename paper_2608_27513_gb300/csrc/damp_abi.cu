@@ -77,13 +77,7 @@ cudaError_t launch_step(const StepArgs &a, bool packed, cudaStream_t s) {
     if (a.fmt == DAMP_LO_S8_ABSMAX_ROW) return launch_rowabs_step(a, s);
     if (a.fmt == DAMP_LO_U4_AFFINE_G32_H32 || a.fmt == DAMP_LO_U4_AFFINE_G32)
         return a.kda ? launch_packed_kda_u4(a, s) : launch_packed_gdn_u4(a, s);
-    if (a.fmt != DAMP_LO_U8_AFFINE_G32_H32 && a.fmt != DAMP_LO_U8_AFFINE_G32) {
-        // FP8 tier: a decode step is a one-token chunk of the chunk kernel
-        StepArgs one = a;
-        one.T = 1;
-        one.lengths = nullptr;
-        return a.kda ? launch_prefill_kda(one, s) : launch_prefill_gdn(one, s);
-    }
+    if (a.fmt == DAMP_LO_FP8_E4M3_G32) return a.kda ? launch_packed_kda_f8(a, s) : launch_packed_gdn_f8(a, s);
     return a.kda ? launch_packed_kda(a, s) : launch_packed_gdn(a, s);
 }
 
@@ -505,6 +499,10 @@ damp_status damp_device_status(uint32_t *status) {
     if (take_status_packed_gdn_u4(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     if (take_status_packed_kda_u4(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_packed_gdn_f8(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_packed_kda_f8(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     if (take_status_fp32(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;

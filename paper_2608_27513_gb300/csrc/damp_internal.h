@@ -51,6 +51,9 @@ cudaError_t launch_packed_kda(const StepArgs &a, cudaStream_t s);
 // the UINT4 low tiers (formats 3, 4)
 cudaError_t launch_packed_gdn_u4(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_packed_kda_u4(const StepArgs &a, cudaStream_t s);
+// the FP8 E4M3 low tier (format 5)
+cudaError_t launch_packed_gdn_f8(const StepArgs &a, cudaStream_t s);
+cudaError_t launch_packed_kda_f8(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_fp32_step(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_quantize(const ConvArgs &a, cudaStream_t s);
 cudaError_t launch_dequantize(const ConvArgs &a, cudaStream_t s);
@@ -79,6 +82,8 @@ cudaError_t take_status_packed_gdn(uint32_t *bits);
 cudaError_t take_status_packed_kda(uint32_t *bits);
 cudaError_t take_status_packed_gdn_u4(uint32_t *bits);
 cudaError_t take_status_packed_kda_u4(uint32_t *bits);
+cudaError_t take_status_packed_gdn_f8(uint32_t *bits);
+cudaError_t take_status_packed_kda_f8(uint32_t *bits);
 cudaError_t take_status_fp32(uint32_t *bits);
 cudaError_t take_status_convert(uint32_t *bits);
 cudaError_t take_status_rowabs(uint32_t *bits);

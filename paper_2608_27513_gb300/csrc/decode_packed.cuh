@@ -97,9 +97,11 @@ __device__ __forceinline__ void advance(Cursor &k, int H, int V) {
 // FP16 tier runs as straight-line code.  KC = -1, DKC = 0 is the general kernel.
 // HMAP: the layout is a head group (held head h reads the operands of model head
 // head_map[h]); without it the model heads are the held heads.
-// U4: UINT4 low tier (formats 3, 4: 32 nibbles in one 16-byte chunk per row, levels 15)
-// instead of UINT8.
-template <int RL, int DKC, int KC, bool KDA, bool HAD, bool BF16, bool HMAP, bool U4 = false>
+// LT: the low tier's code type -- kLtU8 (formats 0, 1), kLtU4 (formats 3, 4: 32 nibbles
+// in one 16-byte chunk per row, levels 15) or kLtE4M3 (format 5: FP8 codes in the natural
+// domain, one FP32 scale per group).
+enum : int { kLtU8 = 0, kLtU4 = 1, kLtE4M3 = 2 };
+template <int RL, int DKC, int KC, bool KDA, bool HAD, bool BF16, bool HMAP, int LT = kLtU8>
 __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams p) {
     constexpr int R = RL > 0 ? RL : 1;
     extern __shared__ __align__(128) uint8_t smem[];
@@ -120,6 +122,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
     const int lo = dk - K;  // low-tier rows
     // record geometry (constants for a fixed layout)
     const int codes_off = KFIX ? 128 * ((KC + 1) / 2) : p.codes_off;
+    constexpr bool U4 = LT == kLtU4, F8 = LT == kLtE4M3;
     constexpr int kCodeRow = U4 ? 16 : 32;  // code bytes per row and record
     const int meta_off = (KFIX && DFIX) ? 128 * ((KC + 1) / 2) + kCodeRow * (DKC - KC) : p.meta_off;
     const int rec_bytes =
@@ -313,7 +316,8 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
                 } else {
                     const uint4 c1 = lds128(st + codes_off + lo_chunk_off(r, 1, lo));
                     const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-                    dequantize_group(w, sz, aa[i], x[i]);
+                    if constexpr (F8) dequantize_group_e4m3(w, __uint_as_float(sz), aa[i], x[i]);
+                    else dequantize_group(w, sz, aa[i], x[i]);
                 }
 #pragma unroll
                 for (int j = 0; j < 16; ++j) {
@@ -422,6 +426,13 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             for (int i = 0; i < RL; ++i) {
                 if constexpr (U4) {  // levels 15; the widened rule of a degenerate block is built in
                     szw[i] = affine_params_u4(mn[i], mx[i], inv[i], zq[i]);
+                } else if constexpr (F8) {
+                    // s = max(max|x|, 1e-10) / 448 (IEEE division, natural domain); codes take
+                    // x * (1/s), within an ulp of x / s: a code moves only where x / s sits at
+                    // a rounding midpoint of E4M3
+                    const float s8 = __fdiv_rn(fmaxf(fmaxf(-mn[i], mx[i]) * kUp, 1e-10f), 448.0f);
+                    szw[i] = __float_as_uint(s8);
+                    inv[i] = __frcp_rn(s8) * kUp;  // exact power-of-two scaling of 1/s
                 } else {
                     sc[i] = scale_of(mn[i], mx[i]);
                     any_zero |= sc[i] == 0.0f;
@@ -431,7 +442,20 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             auto encode_store = [&](int i) {
                 const int r = lane + 32 * i;
                 const float2 inv2 = splat2(inv[i] * 0x1p-110f), zc2 = splat2(zq[i] * 0x1p-149f);
-                if constexpr (U4) {
+                if constexpr (F8) {
+                    const float2 i2 = splat2(inv[i]);
+                    uint32_t w[8];
+#pragma unroll
+                    for (int m = 0; m < 8; ++m) {  // values 4m .. 4m+3, value 4m in byte 0
+                        const float2 a = mul2(x[i][2 * m], i2), b2 = mul2(x[i][2 * m + 1], i2);
+                        w[m] = e4m3x2_of(a.y, a.x) | (e4m3x2_of(b2.y, b2.x) << 16);
+                    }
+                    if (r < lo) {
+                        stg128(grec + codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                        stg128(grec + codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
+                        stg32(grec + meta_off + 4 * r, szw[i]);
+                    }
+                } else if constexpr (U4) {
                     // values 8m .. 8m+7 = pairs 4m .. 4m+3; value 8m ends in the low nibble
                     uint32_t w[4];
 #pragma unroll
@@ -461,7 +485,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
             };
 #pragma unroll
             for (int i = 0; i < RL; ++i) encode_store(i);
-            if constexpr (!U4) {
+            if constexpr (LT == kLtU8) {
                 if (__any_sync(kFull, any_zero)) {
 #pragma unroll
                     for (int i = 0; i < RL; ++i) {

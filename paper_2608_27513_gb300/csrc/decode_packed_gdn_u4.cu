@@ -11,7 +11,7 @@ cudaError_t launch_packed_gdn_u4(const StepArgs &a, cudaStream_t s) {
     uint32_t *status = nullptr;
     cudaError_t e = symbol_address_cached(&g_status_packed_gdn_u4, cache, &status);
     if (e != cudaSuccess) return e;
-    return launch_packed_impl<false, true>(a, s, status);
+    return launch_packed_impl<false, kLtU4>(a, s, status);
 }
 
 cudaError_t take_status_packed_gdn_u4(uint32_t *bits) {

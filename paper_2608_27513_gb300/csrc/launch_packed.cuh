@@ -16,8 +16,8 @@ namespace damp {
 constexpr int kPackedWarps = 8;
 constexpr int kPackedStages = 3;
 
-// U4: the UINT4 low tiers (formats 3, 4); otherwise UINT8 (formats 0, 1).
-template <bool KDA, bool U4>
+// LT: the low tier's code type (kLtU8: formats 0, 1; kLtU4: formats 3, 4; kLtE4M3: format 5).
+template <bool KDA, int LT>
 static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, uint32_t *status) {
     const int V = a.dv / kG;
     const RecGeom rg = rec_geom(a.dk, a.K, a.fmt);
@@ -89,16 +89,25 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
     const bool had = fmt_had(a.fmt);
     // a head group (head map) runs the general instances with model-head indexing
     const bool hmap = a.head_map != nullptr;
+    // (each pick is one compound statement; the FP8 tier has no H_32 variant)
 #define DAMP_PICK4(RL_, DKC_, KC_)                                                                \
-    if (had) kern = a.in_bf16 ? packed_step_kernel<RL_, DKC_, KC_, KDA, true, true, false, U4>    \
-                              : packed_step_kernel<RL_, DKC_, KC_, KDA, true, false, false, U4>;  \
-    else kern = a.in_bf16 ? packed_step_kernel<RL_, DKC_, KC_, KDA, false, true, false, U4>       \
-                          : packed_step_kernel<RL_, DKC_, KC_, KDA, false, false, false, U4>;
+    {                                                                                             \
+        if constexpr (LT != kLtE4M3) {                                                            \
+            if (had) kern = a.in_bf16 ? packed_step_kernel<RL_, DKC_, KC_, KDA, true, true, false, LT>   \
+                                      : packed_step_kernel<RL_, DKC_, KC_, KDA, true, false, false, LT>; \
+        }                                                                                         \
+        if (!had) kern = a.in_bf16 ? packed_step_kernel<RL_, DKC_, KC_, KDA, false, true, false, LT>     \
+                                   : packed_step_kernel<RL_, DKC_, KC_, KDA, false, false, false, LT>;   \
+    }
 #define DAMP_PICK4_HMAP(RL_)                                                                      \
-    if (had) kern = a.in_bf16 ? packed_step_kernel<RL_, 0, -1, KDA, true, true, true, U4>         \
-                              : packed_step_kernel<RL_, 0, -1, KDA, true, false, true, U4>;       \
-    else kern = a.in_bf16 ? packed_step_kernel<RL_, 0, -1, KDA, false, true, true, U4>            \
-                          : packed_step_kernel<RL_, 0, -1, KDA, false, false, true, U4>;
+    {                                                                                             \
+        if constexpr (LT != kLtE4M3) {                                                            \
+            if (had) kern = a.in_bf16 ? packed_step_kernel<RL_, 0, -1, KDA, true, true, true, LT> \
+                                      : packed_step_kernel<RL_, 0, -1, KDA, true, false, true, LT>; \
+        }                                                                                         \
+        if (!had) kern = a.in_bf16 ? packed_step_kernel<RL_, 0, -1, KDA, false, true, true, LT>   \
+                                   : packed_step_kernel<RL_, 0, -1, KDA, false, false, true, LT>; \
+    }
     const int rl = (a.dk - a.K + 31) / 32;
     if (hmap) {
         switch (rl) {
@@ -116,10 +125,10 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
     if (!kern && a.dk == 128 && a.K == KC_) {                                                     \
         DAMP_PICK4((128 - KC_ + 31) / 32, 128, KC_)                                               \
     }
-    // (the UINT4 tiers: the paper's uniform INT4 and FP16 + INT4 at K_hi = 16)
+    // (the 4-bit and FP8 tiers: uniform and FP16 + low tier at K_hi = 16)
     DAMP_FIXED(0)
     DAMP_FIXED(16)
-    if constexpr (!U4) {
+    if constexpr (LT == kLtU8) {
         DAMP_FIXED(4)
         DAMP_FIXED(8)
         DAMP_FIXED(10)
@@ -128,7 +137,7 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
     // general kernels: K_hi = 0 (no FP16 tier) or any K_hi, runtime d_k
 #define DAMP_GENERAL(RL_)                                                                         \
     if (!kern && rl == RL_) {                                                                     \
-        if constexpr (!U4) {                                                                      \
+        if constexpr (LT == kLtU8) {                                                              \
             if (a.K == 0) DAMP_PICK4(RL_, 0, 0)                                                   \
         }                                                                                         \
         if (!kern) DAMP_PICK4(RL_, 0, -1)                                                         \
