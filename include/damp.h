@@ -88,9 +88,8 @@ typedef enum {
     DAMP_LO_U4_AFFINE_G32 = 4,     /* the same without H_32 (the paper's "INT4" row, 5.0 bits) */
     DAMP_LO_FP8_E4M3_G32 = 5       /* FP8 E4M3, G = 32, one FP32 scale per group, natural domain:
                                       s = max(max|x|, 1e-10)/448, q = E4M3(clip(x/s, +-448)) (9.0 bits).
-                                      Formats 3-5 are the paper's comparison tiers (App. A.1): their
-                                      decode step runs as a one-token chunk of the prefill kernel
-                                      and is not tuned like formats 0 and 1. */
+                                      Formats 3-5 are the paper's comparison tiers (App. A.1); their
+                                      decode step is the same fused step as formats 0 and 1. */
 } damp_lo_format;
 
 /* Element type of q, k and v. */

@@ -1,6 +1,5 @@
 // prefill_gdn_x.cu -- instantiations of the prefill chunk kernel for
 // GDN (scalar decay per head) with the UINT4 (+ H_32) and FP8 E4M3 low tiers (formats 3, 4, 5).
-// Decode steps of these formats run here too, as one-token chunks.
 #include "launch_prefill.cuh"
 
 namespace damp {

@@ -1,6 +1,6 @@
 """GPU parity of the 4-bit and FP8 low tiers (formats 3-5, App. A.1) against the
 oracle: logical tiers bit for bit through pack/unpack, whole-state conversions,
-decode steps (one-token chunks of the generic kernel) and prefill chunks, at the
+decode steps (the fused packed step's 4-bit and FP8 instances) and prefill chunks, at the
 decode tolerances with each format's tie rule."""
 import numpy as np
 import pytest
