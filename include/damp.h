@@ -82,8 +82,9 @@ typedef enum {
                                       all d_v values: s = max|x|/127, q = sat_[-127,127](rne(x/s)),
                                       s = 0 -> q = 0; no H_32 (8 + 32/d_v bits).  A fallback
                                       for a low tier whose scales are left open, not the paper's
-                                      format.  Its step sweeps each head twice (the row scale
-                                      spans every value block) and is not tuned. */
+                                      format.  Its row scale spans every value block of a head:
+                                      for d_v <= 128 a step is a one-token chunk whose warps share
+                                      each row's maximum; larger d_v sweep each head twice. */
     DAMP_LO_U4_AFFINE_G32_H32 = 3, /* UINT4 affine (b = 4), G = 32, FP16 (s, z), H_32 first (5.0 bits) */
     DAMP_LO_U4_AFFINE_G32 = 4,     /* the same without H_32 (the paper's "INT4" row, 5.0 bits) */
     DAMP_LO_FP8_E4M3_G32 = 5       /* FP8 E4M3, G = 32, one FP32 scale per group, natural domain:
@@ -251,8 +252,9 @@ DAMP_API damp_status damp_fp32_kda_decode_step(const damp_layout *layout, float 
  *   beta       float [B][T][H_m], 4-B aligned
  *   o          float [B][T][H_m][d_v]: o_t from the FP32 state after token t; rows past
  *              a row's length are not written.  Must not overlap the pool or inputs.
- * Other arguments as in damp_gdn_decode_step.  Any lo_format except 2
- * (DAMP_ERR_FORMAT for the row-absmax format).
+ * Other arguments as in damp_gdn_decode_step.  Any lo_format; the row-absmax format
+ * (2) needs d_v <= 128 (DAMP_ERR_SHAPE otherwise): its row scale spans the value blocks
+ * of a head, which four warps then share.
  */
 DAMP_API damp_status damp_gdn_prefill_chunk(const damp_layout *layout, void *state, int64_t num_slots,
                                             const int32_t *slot_idx, int32_t batch, int32_t chunk_len,

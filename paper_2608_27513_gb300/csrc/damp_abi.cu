@@ -74,7 +74,13 @@ damp_status check_pool(const void *state, int64_t num_slots, const int32_t *slot
 
 cudaError_t launch_step(const StepArgs &a, bool packed, cudaStream_t s) {
     if (!packed) return launch_fp32_step(a, s);
-    if (a.fmt == DAMP_LO_S8_ABSMAX_ROW) return launch_rowabs_step(a, s);
+    if (a.fmt == DAMP_LO_S8_ABSMAX_ROW) {
+        if (a.dv > 4 * 32) return launch_rowabs_step(a, s);  // the two-sweep step for d_v > 128
+        StepArgs one = a;  // otherwise a one-token chunk: four warps share each row's maximum
+        one.T = 1;
+        one.lengths = nullptr;
+        return a.kda ? launch_prefill_kda(one, s) : launch_prefill_gdn(one, s);
+    }
     if (a.fmt == DAMP_LO_U4_AFFINE_G32_H32 || a.fmt == DAMP_LO_U4_AFFINE_G32)
         return a.kda ? launch_packed_kda_u4(a, s) : launch_packed_gdn_u4(a, s);
     if (a.fmt == DAMP_LO_FP8_E4M3_G32) return a.kda ? launch_packed_kda_f8(a, s) : launch_packed_gdn_f8(a, s);
@@ -149,7 +155,7 @@ damp_status prefill(const damp_layout *L, void *state, int64_t num_slots, const 
                     bool kda) {
     damp_status st = check_layout(L);
     if (st != DAMP_OK) return st;
-    if (L->lo_format == DAMP_LO_S8_ABSMAX_ROW) return DAMP_ERR_FORMAT;
+    if (L->lo_format == DAMP_LO_S8_ABSMAX_ROW && L->d_v > 128) return DAMP_ERR_SHAPE;
     if (in_dtype != DAMP_IN_BF16 && in_dtype != DAMP_IN_FP32) return DAMP_ERR_FORMAT;
     if (batch < 0 || chunk_len < 0) return DAMP_ERR_SHAPE;
     if (batch == 0 || chunk_len == 0) return DAMP_OK;

@@ -49,11 +49,23 @@ static cudaError_t launch_prefill_impl(const StepArgs &a, cudaStream_t stream, u
     if (p.total_tiles == 0 || a.T == 0) return cudaSuccess;
 
     int warps = kPrefillWarps;
-    while (warps > 1 && warps * warp_smem > max_smem_per_block()) --warps;
-    if (warps * warp_smem > max_smem_per_block()) return cudaErrorInvalidValue;
-    const int64_t want = (p.total_tiles + warps - 1) / warps;
+    int64_t want;
+    int extra = 0;
+    if constexpr (FMT == kFmtS8Row) {
+        // groups of four warps share each row's maximum over the value blocks of a head
+        if (V > 4) return cudaErrorInvalidValue;
+        extra = (warps / 4) * 2 * 4 * 128 * 4;  // per group: two buffers of [4 blocks][128 rows]
+        if (warps * warp_smem + extra > max_smem_per_block()) return cudaErrorInvalidValue;
+        const int64_t units = p.total_tiles / V;
+        want = (units + warps / 4 - 1) / (warps / 4);
+    } else {
+        while (warps > 1 && warps * warp_smem > max_smem_per_block()) --warps;
+        if (warps * warp_smem > max_smem_per_block()) return cudaErrorInvalidValue;
+        want = (p.total_tiles + warps - 1) / warps;
+    }
+    p.amax_off = warps * warp_smem;
     const int grid = (int)std::min<int64_t>(want, (int64_t)sm_count());
-    const int smem = warp_smem * warps;
+    const int smem = warp_smem * warps + extra;
 
     void (*kern)(PrefillParams) = nullptr;
 #define DAMP_PICK(R_)                                                                              \

@@ -57,6 +57,7 @@ struct PrefillParams {
     int32_t rec_bytes, codes_off, meta_off;
     int64_t slot_bytes, total_tiles;
     int32_t warp_stride;  // per-warp shared memory: the fixed buffers, an mbarrier and the record stage
+    int32_t amax_off;     // row-absmax format: the groups' row-maximum buffers after the warps' areas
     // per-warp shared memory
     uint32_t *status;
 };
@@ -110,6 +111,19 @@ __device__ __forceinline__ float2 column_sum_pairs(const float2 (&a)[16], const 
     const float ax = __shfl_sync(kFull, t.x, src), ay = __shfl_sync(kFull, t.y, src);
     const float bx = __shfl_sync(kFull, t.x, 16 + src), by = __shfl_sync(kFull, t.y, 16 + src);
     return (lane & 1) ? make_float2(ay, by) : make_float2(ax, bx);
+}
+
+// Row-absmax INT8 (format 2): x_j = s q_j * scale from 8 words of int8 codes (the
+// codes offset by 128 land on the UINT8 path's 2^23 + byte trick; s q is exact).
+__device__ __forceinline__ void dequantize_row_s8(const uint32_t (&w)[8], float s, float scale, float2 (&x)[16]) {
+    const float2 nzb = splat2(-(8388608.0f + 128.0f));
+    const float2 sa = splat2(s * scale);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const uint32_t u = w[i] ^ 0x80808080u;  // q + 128 in [1, 255]
+        x[2 * i] = mul2(add2(make_float2(u8_biased(u, 0), u8_biased(u, 1)), nzb), sa);
+        x[2 * i + 1] = mul2(add2(make_float2(u8_biased(u, 2), u8_biased(u, 3)), nzb), sa);
+    }
 }
 
 // FP16 row u of a record held in shared memory at rec -> 32 FP32 values
@@ -184,10 +198,31 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
     constexpr int dk = 32 * R;
     const int K = p.K, lo = dk - K, H = p.H, V = p.V, T = p.T;
 
-    const int64_t gw = (int64_t)blockIdx.x * nw + warp;
-    const int64_t nwt = (int64_t)gridDim.x * nw;
-    const int64_t t0 = p.total_tiles * gw / nwt, t1 = p.total_tiles * (gw + 1) / nwt;
-    if (t0 >= t1) return;
+    // Tiles of this warp: a contiguous range k -> t0 + k; for the row-absmax format a
+    // group of four warps takes a range of (slot, head) units, warp 4g + c the value
+    // block c of each (the row scale spans the V <= 4 blocks of a head, so the group
+    // meets at a named barrier to share each row's maximum; warps with c >= V only meet).
+    constexpr bool ROW = FMT == kFmtS8Row;
+    int64_t t0 = 0, u0 = 0, n = 0;
+    const int cw = warp & 3;
+    const bool idle = ROW && cw >= V;
+    if constexpr (ROW) {
+        const int64_t ng = (int64_t)gridDim.x * (nw >> 2), g = (int64_t)blockIdx.x * (nw >> 2) + (warp >> 2);
+        const int64_t units = p.total_tiles / V;
+        u0 = units * g / ng;
+        n = units * (g + 1) / ng - u0;
+    } else {
+        const int64_t gw = (int64_t)blockIdx.x * nw + warp;
+        const int64_t nwt = (int64_t)gridDim.x * nw;
+        t0 = p.total_tiles * gw / nwt;
+        n = p.total_tiles * (gw + 1) / nwt - t0;
+    }
+    // the tile of step k (for an idle warp: block 0 of its unit, whose batch row and head
+    // decide, as for the group's other warps, whether the unit runs)
+    auto tile_of = [&](int64_t k) -> int64_t { return ROW ? (u0 + k) * V + (idle ? 0 : cw) : t0 + k; };
+    if (n <= 0) return;  // the same for the four warps of a row-absmax group
+    const uint32_t amax_s = smem_u32(smem) + (uint32_t)(p.amax_off + (warp >> 2) * 2 * 4 * 128 * 4);
+    auto group_sync = [&]() { asm volatile("bar.sync %0, 128;" ::"r"(1 + (warp >> 2)) : "memory"); };
     bool bad_slot = false, bad_head = false, timed_out = false;
 
     // The record of the next tile comes in by one bulk copy (TMA engine) while the
@@ -203,36 +238,43 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
         Tb = p.lengths ? min(max(p.lengths[b], 0), T) : T;
         return p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * p.rec_bytes;
     };
-    auto issue = [&](int64_t tt) {  // lane 0
+    auto issue = [&](int64_t k) {  // lane 0: the record of step k
         int b, h, c, mh, Tb;
         int64_t slot;
-        uint8_t *g = rec_of(tt, b, h, c, mh, slot, Tb);
-        const bool run = slot >= 0 && slot < p.num_slots && mh >= 0 && mh < p.Hm && Tb > 0;
+        uint8_t *g = rec_of(tile_of(k), b, h, c, mh, slot, Tb);
+        const bool run = !idle && slot >= 0 && slot < p.num_slots && mh >= 0 && mh < p.Hm && Tb > 0;
         mbar_arrive_expect_tx(bar, run ? (uint32_t)p.rec_bytes : 0u);
         if (run) bulk_g2s(st, g, (uint32_t)p.rec_bytes, bar);
     };
     if (lane == 0) {
         mbar_init(bar, 1);
         fence_mbar_init();
-        issue(t0);
+        issue(0);
     }
     __syncwarp();
     uint32_t parity = 0;
 
-    for (int64_t t = t0; t < t1; ++t) {
-        if (!__all_sync(kFull, mbar_wait_bounded(bar, parity))) {
+    for (int64_t k = 0; k < n; ++k) {
+        // A lost copy ends this warp's work; in a row-absmax group it keeps meeting the
+        // other warps (no compute) so that no barrier waits for it.
+        if (!timed_out && !__all_sync(kFull, mbar_wait_bounded(bar, parity))) {
             timed_out = true;
-            break;
+            if (!ROW) break;
         }
-        parity ^= 1u;
+        if (!timed_out) parity ^= 1u;
         int b, h, c, mh, Tb;
         int64_t slot;
-        uint8_t *const grec = rec_of(t, b, h, c, mh, slot, Tb);  // written in place
+        uint8_t *const grec = rec_of(tile_of(k), b, h, c, mh, slot, Tb);  // written in place
         const bool slot_ok = slot >= 0 && slot < p.num_slots, head_ok = mh >= 0 && mh < p.Hm;
         bad_slot |= !slot_ok;
         bad_head |= !head_ok;
         if (!slot_ok || !head_ok || Tb == 0) {  // nothing landed in the stage: fetch the next record
-            if (lane == 0 && t + 1 < t1) issue(t + 1);
+            if (lane == 0 && k + 1 < n && !timed_out) issue(k + 1);
+            continue;
+        }
+        if (ROW && (idle || timed_out)) {  // the unit runs: meet the group once, at its row maxima
+            if (lane == 0 && k + 1 < n && !timed_out) issue(k + 1);
+            group_sync();
             continue;
         }
 
@@ -303,15 +345,16 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
             } else {
                 const uint32_t w[8] = {cw0[i].x, cw0[i].y, cw0[i].z, cw0[i].w, cw1[i].x, cw1[i].y, cw1[i].z, cw1[i].w};
                 if constexpr (FMT == kFmtE4M3) dequantize_group_e4m3(w, __uint_as_float(szw[i]), kDown, x[i]);
+                else if constexpr (ROW) dequantize_row_s8(w, __uint_as_float(szw[i]), kDown, x[i]);
                 else dequantize_group(w, szw[i], kDown, x[i]);
             }
         }
 
         // the stage has been read: the next tile's record comes in during this one
         __syncwarp();
-        if (lane == 0 && t + 1 < t1) {
+        if (lane == 0 && k + 1 < n) {
             fence_proxy_async_smem();  // the warp's reads of the stage before the bulk copy's writes
-            issue(t + 1);
+            issue(k + 1);
         }
 
         // The rank-1 update of token t is applied at the start of token t+1, in the
@@ -396,6 +439,18 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
         }
 
         // ---- the chunk-final tile: FP16 rows rounded once, low-tier rows requantized ----
+        if constexpr (ROW) {
+            // each row's maximum over the V value blocks of the head (buffer k & 1: a warp
+            // writes unit k+2's maxima only after the group met at unit k+1)
+            const uint32_t ab = amax_s + (uint32_t)((k & 1) * 4 * 128 * 4);
+#pragma unroll
+            for (int i = 0; i < R; ++i) {
+                float mn, mx;
+                minmax32(x[i], mn, mx);
+                sts32(ab + (uint32_t)((cw * 128 + lane + 32 * i) * 4), __float_as_uint(fmaxf(-mn, mx)));
+            }
+            group_sync();
+        }
 #pragma unroll
         for (int i = 0; i < R; ++i) {
             const int u = lane + 32 * i;
@@ -416,6 +471,22 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
                 const uint32_t szw = quantize_group_u4(x[i], w);
                 stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
                 stg32(grec + p.meta_off + 4 * r, szw);
+            } else if constexpr (ROW) {
+                // s = max|x| / 127 over the whole row (FP32, IEEE division); codes
+                // sat(rne(x / s)) taken as x * (1/s) + 128 on the denormal grid, then
+                // moved back to int8 (a code can differ from x / s only at a rounding tie)
+                const uint32_t ab = amax_s + (uint32_t)((k & 1) * 4 * 128 * 4);
+                float am = 0.f;
+                for (int c2 = 0; c2 < V; ++c2) am = fmaxf(am, ldsf(ab + (uint32_t)((c2 * 128 + u) * 4)));
+                const float sc = __fdiv_rn(am * kUp, 127.0f);
+                const float inv = sc > 0.0f ? __frcp_rn(sc) : 0.0f;
+                const float2 inv2 = splat2(inv * 0x1p-110f), zc2 = splat2(128.0f * 0x1p-149f);
+                uint32_t w[8];
+#pragma unroll
+                for (int m = 0; m < 8; ++m) w[m] = encode4(x[i][2 * m], x[i][2 * m + 1], inv2, zc2) ^ 0x80808080u;
+                stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
+                stg32(grec + p.meta_off + 4 * r, __float_as_uint(sc));
             } else if constexpr (FMT == kFmtE4M3) {
                 float2 xn[16];
 #pragma unroll

@@ -1,5 +1,5 @@
 // prefill_kda_x.cu -- instantiations of the prefill chunk kernel for
-// KDA (per-key-channel decay) with the UINT4 (+ H_32) and FP8 E4M3 low tiers (formats 3, 4, 5).
+// KDA (per-key-channel decay) with the row-absmax INT8, UINT4 (+ H_32) and FP8 E4M3 low tiers (formats 2, 3, 4, 5).
 #include "launch_prefill.cuh"
 
 namespace damp {
@@ -15,6 +15,7 @@ cudaError_t launch_prefill_kda_x(const StepArgs &a, cudaStream_t s) {
         case kFmtU4H32: return launch_prefill_impl<true, kFmtU4H32>(a, s, status);
         case kFmtU4: return launch_prefill_impl<true, kFmtU4>(a, s, status);
         case kFmtE4M3: return launch_prefill_impl<true, kFmtE4M3>(a, s, status);
+        case kFmtS8Row: return launch_prefill_impl<true, kFmtS8Row>(a, s, status);
         default: return cudaErrorInvalidValue;
     }
 }

@@ -175,7 +175,7 @@ def test_prefill_rejects_bad_arguments_before_launch(L):
     assert _call_prefill(L, lay, fb, q=off(2, 8)) == 3
     assert _call_prefill(L, lay, fb, o=off(0, 64)) == 4               # o inside the pool
     assert _call_prefill(L, lay, fb, lengths=off(7, 0)) == 4          # lengths under o
-    assert _call_prefill(L, _layout(lo_format=2), fb) == 5            # row-absmax: no prefill kernel
+    assert _call_prefill(L, _layout(lo_format=2, d_v=256), fb) == 2   # row-absmax chunks need d_v <= 128
     assert _call_prefill(L, lay, fb, in_dtype=3) == 5
 
 

@@ -112,3 +112,12 @@ def test_all_fp16_and_widest_rows():
 def test_slot_indirection_row_absmax():
     w = wl.KDA_B256.replace(batch=3, heads=4, qk_heads=4, lo_format=S8)
     P.run_teacher_forced(w, 2, DEV, slot_of={0: 5, 1: 0, 2: 2}, pool=6)
+
+
+@pytest.mark.parametrize("dv,lengths", [(128, [6, 2]), (96, [6, 0]), (64, [3, 6])])
+def test_row_absmax_prefill_chunks_match_oracle(dv, lengths):
+    """Prefill chunks of the row-absmax format: the four warps of a head share each row's
+    maximum over the value blocks (d_v = 96 and 64 leave warps without a block)."""
+    from tests.test_gpu_prefill import _run as run_chunks
+    w = wl.KDA_B256.replace(batch=2, heads=4, qk_heads=4, d_v=dv, lo_format=S8)
+    run_chunks(w, 6, lengths=lengths)
