@@ -69,7 +69,11 @@ static cudaError_t launch_prefill_impl(const StepArgs &a, cudaStream_t stream, u
 
     void (*kern)(PrefillParams) = nullptr;
 #define DAMP_PICK(R_)                                                                              \
-    if (a.dk == 32 * R_) kern = a.in_bf16 ? prefill_chunk_kernel<R_, KDA, FMT, true> : prefill_chunk_kernel<R_, KDA, FMT, false>;
+    if constexpr (FMT == kFmtS8Row) {                                                              \
+        if (a.dk == 32 * R_) kern = a.in_bf16 ? prefill_row_kernel<R_, KDA, true> : prefill_row_kernel<R_, KDA, false>; \
+    } else {                                                                                       \
+        if (a.dk == 32 * R_) kern = a.in_bf16 ? prefill_chunk_kernel<R_, KDA, FMT, true> : prefill_chunk_kernel<R_, KDA, FMT, false>; \
+    }
     DAMP_PICK(1)
     DAMP_PICK(2)
     DAMP_PICK(4)
