@@ -92,3 +92,12 @@ def test_uniform_entry_point(fmt):
 @pytest.mark.parametrize("fmt", NEW)
 def test_prefill_chunks_match_oracle(fmt):
     run_chunks(wl.KDA_B256.replace(batch=2, heads=4, qk_heads=4, lo_format=fmt), 6, lengths=[6, 2])
+
+
+@pytest.mark.parametrize("fmt", NEW)
+@pytest.mark.parametrize("dk,dv,K", [(64, 96, 5), (32, 64, 0), (32, 32, 3)])
+def test_decode_steps_small_heads(fmt, dk, dv, K):
+    """The general instances of the 4-bit and FP8 steps (fewer row slots per lane,
+    ragged value blocks)."""
+    w = wl.Workload("t", "kda", 2, 4, 2, dk, dv, K, 1, 1, "bf16", 17, fmt)
+    P.run_teacher_forced(w, 2, DEV)

@@ -121,3 +121,10 @@ def test_row_absmax_prefill_chunks_match_oracle(dv, lengths):
     from tests.test_gpu_prefill import _run as run_chunks
     w = wl.KDA_B256.replace(batch=2, heads=4, qk_heads=4, d_v=dv, lo_format=S8)
     run_chunks(w, 6, lengths=lengths)
+
+
+@pytest.mark.parametrize("dk,dv,K", [(32, 32, 4), (64, 64, 0)])
+def test_row_absmax_small_heads(dk, dv, K):
+    """One or two value blocks per head: three or two warps of each group only meet."""
+    w = wl.Workload("t", "gdn", 3, 4, 4, dk, dv, K, 1, 1, "fp32", 18, S8)
+    P.run_teacher_forced(w, 2, DEV)
