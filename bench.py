@@ -394,8 +394,9 @@ def gpu_arm(args, rank: int, world: int):
     }
 
 
-def cpu_baseline(seconds: float = 12.0) -> dict:
-    """The oracle as it stands, single thread, on a bounded sample of the workload's heads."""
+def _oracle_sample(seconds: float):
+    """(state updates done, seconds): the oracle's packed step over 2 slots x H heads of
+    the bench workload, repeated for about `seconds` (one host thread)."""
     import numpy as np
 
     from oracle import core, runs
@@ -412,11 +413,33 @@ def cpu_baseline(seconds: float = 12.0) -> dict:
         core.mixed_step_heads(perms, *tiers, units["q"], units["k"], units["v"], units["g"], units["beta"],
                               w.k_hi, w.lo_format, w.kind)
         done += n
-    el = time.perf_counter() - t0
+    return done, time.perf_counter() - t0
+
+
+def cpu_baseline(seconds: float = 12.0) -> dict:
+    """The oracle as it stands, single thread, on a bounded sample of the workload's heads."""
+    w = WORKLOAD
+    done, el = _oracle_sample(seconds)
     per_unit = algorithmic_bytes(w) / (w.batch * w.heads)
     return {"value": per_unit * done / el / 1e12, "unit": "TB/s", "cores": 1, "kind": "oracle",
             "sample": f"{done} (slot, head) state updates of the KDA B=256 workload "
-                      f"({done // n} passes over 2 slots x 32 heads), {el:.1f} s, one host thread",
+                      f"({done // (2 * w.heads)} passes over 2 slots x {w.heads} heads), {el:.1f} s, one host thread",
+            "us_per_full_step": el / done * w.batch * w.heads * 1e6}
+
+
+def cpu_baseline_all_cores(seconds: float = 8.0) -> dict:
+    """The same sample on every host core at once: one spawned process per core, each
+    running the oracle on its own copy (the (slot, head) updates are independent)."""
+    import multiprocessing as mp
+    w = WORKLOAD
+    n = os.cpu_count() or 1
+    with mp.get_context("spawn").Pool(n) as pool:
+        res = pool.map(_oracle_sample, [seconds] * n)
+    done = sum(d for d, _ in res)
+    el = max(e for _, e in res)
+    per_unit = algorithmic_bytes(w) / (w.batch * w.heads)
+    return {"value": per_unit * done / el / 1e12, "unit": "TB/s", "cores": n, "kind": "oracle",
+            "sample": f"{done} (slot, head) state updates on {n} processes, {el:.1f} s each",
             "us_per_full_step": el / done * w.batch * w.heads * 1e6}
 
 
@@ -937,6 +960,7 @@ def main():
         line = make_line(r, args.steps, args.warmup, world)
         if not args.no_cpu_baseline and world == 1:
             line["cpu_baseline"] = cpu_baseline()
+            line["cpu_baseline_all_cores"] = cpu_baseline_all_cores()
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.barrier()
