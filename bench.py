@@ -185,6 +185,10 @@ def make_line(r: dict, steps: int, warmup: int, world: int) -> dict:
                      "frac_of_8TBs": achieved_gbs / 8000.0,
                      "traffic": ncu_traffic("packed_step_kda_b256"),
                      "kernel": "packed_step_kernel<RL=4,d_k=128,K_hi=10,KDA,H32,BF16>", "algorithmic_bytes": bytes_step},
+        "repeats": ({"n": len(r["reps_ms"]), "median_us_per_step": statistics.median(r["reps_ms"]) * 1e3,
+                     "min_us_per_step": min(r["reps_ms"]) * 1e3, "max_us_per_step": max(r["reps_ms"]) * 1e3,
+                     "note": "five further timed blocks of steps/5 launches each, after 3 warm-up launches"}
+                    if r.get("reps_ms") else None),
         "cuda_graph": ({"us_per_step": r["graph_ms"] * 1e3,
                         "note": "the same steps captured in one CUDA graph of 4 launches and replayed"}
                        if r.get("graph_ms") else None),
@@ -288,6 +292,10 @@ def gpu_arm(args, rank: int, world: int):
     launch_ms = max_over_ranks_(launch_ms)
     if damp.device_status() != 0:
         raise RuntimeError("device status word set during the timed region")
+    # five more repetitions of a fifth of the steps each (spread of the measurement)
+    reps = []
+    for _ in range(5):
+        reps.append(max_over_ranks_(timed(run_packed, max(args.steps // 5, 10), 3)[1]))
 
     # ---- the same steps replayed from a CUDA graph (one graph of 2 * POOLS steps) ----
     gstream = torch.cuda.Stream(dev)
@@ -389,6 +397,7 @@ def gpu_arm(args, rank: int, world: int):
     e2e_total = max_over_ranks_(e0.elapsed_time(e1))
     return {
         "w": w, "total_ms": total_ms, "launch_ms": launch_ms, "fp32_launch_ms": fp_launch, "graph_ms": graph_ms,
+        "reps_ms": reps,
         "e2e_ms": e2e_total / e2e_steps, "h2d": h2d, "d2h": d2h, "clocks": clk.summary(),
         "bits": damp.bits_per_value(L), "dev_name": torch.cuda.get_device_name(dev),
     }
