@@ -7,10 +7,36 @@
 #include "damp_internal.h"
 #include "formats.cuh"
 #include "prefill.cuh"
+#include "prefill_cg.cuh"
 
 namespace damp {
 
 constexpr int kPrefillWarps = 8;
+// Chunks of at least this many tokens on the UINT8 tiers (d_k 64 or 128, o 16-byte
+// aligned) run prefill_cg_kernel, whose per-token work is lower and per-tile work higher;
+// shorter chunks and the other tiers run prefill_chunk_kernel.
+constexpr int kPrefillCgMinT = 32;
+
+template <bool KDA, bool HAD>
+static cudaError_t launch_prefill_cg(const PrefillParams &p0, const StepArgs &a, int rec_bytes, cudaStream_t stream) {
+    PrefillParams p = p0;
+    const int warp_smem = ((prefill_cg_smem(a.dk, KDA, a.in_bf16).stage_off + rec_bytes + 127) & ~127) + 128 * a.K;
+    p.warp_stride = warp_smem;
+    int warps = kPrefillWarps;
+    while (warps > 1 && warps * warp_smem > max_smem_per_block()) --warps;
+    if (warps * warp_smem > max_smem_per_block()) return cudaErrorInvalidValue;
+    const int64_t want = (p.total_tiles + warps - 1) / warps;
+    const int grid = (int)std::min<int64_t>(want, (int64_t)sm_count());
+    const int smem = warp_smem * warps;
+    void (*kern)(PrefillParams) = nullptr;
+    if (a.dk == 64) kern = a.in_bf16 ? prefill_cg_kernel<64, KDA, HAD, true> : prefill_cg_kernel<64, KDA, HAD, false>;
+    if (a.dk == 128) kern = a.in_bf16 ? prefill_cg_kernel<128, KDA, HAD, true> : prefill_cg_kernel<128, KDA, HAD, false>;
+    if (!kern) return cudaErrorInvalidValue;
+    cudaError_t e = ensure_smem_limit(reinterpret_cast<const void *>(kern), smem);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, 32 * warps, smem, stream>>>(p);
+    return cudaGetLastError();
+}
 
 template <bool KDA, int FMT>
 static cudaError_t launch_prefill_impl(const StepArgs &a, cudaStream_t stream, uint32_t *status) {
@@ -47,6 +73,10 @@ static cudaError_t launch_prefill_impl(const StepArgs &a, cudaStream_t stream, u
     const int warp_smem = prefill_smem(a.dk, KDA, a.in_bf16).warp_bytes + 128 + ((rg.bytes + 127) & ~127);
     p.warp_stride = warp_smem;
     if (p.total_tiles == 0 || a.T == 0) return cudaSuccess;
+    if constexpr (FMT == kFmtU8H32 || FMT == kFmtU8) {
+        if (a.T >= kPrefillCgMinT && (a.dk == 64 || a.dk == 128) && (reinterpret_cast<uintptr_t>(a.o) & 15) == 0)
+            return launch_prefill_cg<KDA, FMT == kFmtU8H32>(p, a, rg.bytes, stream);
+    }
 
     int warps = kPrefillWarps;
     int64_t want;

@@ -1,0 +1,405 @@
+// prefill_cg.cuh -- the prefill chunk for chunks of many tokens on the UINT8 tiers
+// (formats 0, 1), with the tile held in key-channel order (App. A.5 prefill path;
+// Sec. 3.1 Eq. delta_update per token, o_t = S_t^T q_t).
+//
+// One warp owns a tile (slot, head, value block c) for the whole chunk, as in
+// prefill_chunk_kernel, and all rows run in the H_32 domain the same way (FP16 rows
+// transformed once on load and once on store).  What differs is the placement:
+//   * lane l = 2 g + h holds key channels g NR .. g NR + NR - 1 (NR = d_k / 16) and
+//     value columns 16 h .. 16 h + 15 of each; the channel ch sits in row pi^-1(ch) of
+//     the packed record, so the record is read and written through pi^-1 once per tile
+//     while a lane's per-token operands (k, q and the decay of its channels) are
+//     contiguous in the token buffer: vector loads instead of gathers through pi;
+//   * the partial sums r~ = S~^T k and p~ = S~^T q of a lane's 16 columns over its NR
+//     channels go through one shared-memory transpose, after which lane L sums column L
+//     over the 16 channel groups; H d = H v - r~ comes back through shared memory.
+// The rank-1 update of token t is applied in the same pass over the registers as the
+// decay of token t+1; o_t is finished during token t+1.
+#pragma once
+
+#include "prefill.cuh"
+
+namespace damp {
+
+// Per-warp shared memory: [transpose buffer: 32 rows of 36 floats][H d][pi^-1][pi]
+// [token buffer 0][token buffer 1][mbarrier][record stage][FP16 rows: K x 32 floats].
+// The token buffers have the layout of prefill_smem; the FP16 rows pass through the last
+// area in row order (lane u holds row u, as in prefill_chunk_kernel), so that their H_32
+// and binary16 conversions run once per row and not on both sides of a divergent branch.
+constexpr int kCgRowBytes = 144;  // 16-byte slots of 8 consecutive lanes hit distinct banks
+struct PrefillCgSmem {
+    int dvec_off, inv_off, perm_off, ops_off, bar_off, stage_off;
+};
+__host__ __device__ constexpr PrefillCgSmem prefill_cg_smem(int dk, bool kda, bool bf16) {
+    const int dvec = 32 * kCgRowBytes, inv = dvec + 128, perm = inv + up16(dk), ops = perm + up16(dk);
+    const int bar = (ops + 2 * prefill_smem(dk, kda, bf16).ops_bytes + 127) & ~127;
+    return PrefillCgSmem{dvec, inv, perm, ops, bar, bar + 128};
+}
+
+__device__ __forceinline__ void sts_u8(uint32_t a, uint32_t v) {
+    asm volatile("st.shared.u8 [%0], %1;" ::"r"(a), "r"(v) : "memory");
+}
+__device__ __forceinline__ uint2 lds64(uint32_t a) {
+    uint2 v;
+    asm volatile("ld.shared.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(a));
+    return v;
+}
+
+// N consecutive operands at shared address a (BF16 or FP32), widened to FP32 (exact).
+template <int N, bool BF16>
+__device__ __forceinline__ void lds_operands(uint32_t a, float (&v)[N]) {
+    static_assert(N % 4 == 0, "operands come in fours");
+    if constexpr (BF16) {
+#pragma unroll
+        for (int c = 0; c < N / 4; ++c) {
+            const uint2 w = lds64(a + 8 * c);
+            v[4 * c + 0] = __uint_as_float(w.x << 16);
+            v[4 * c + 1] = __uint_as_float(w.x & 0xffff0000u);
+            v[4 * c + 2] = __uint_as_float(w.y << 16);
+            v[4 * c + 3] = __uint_as_float(w.y & 0xffff0000u);
+        }
+    } else {
+#pragma unroll
+        for (int c = 0; c < N / 4; ++c) {
+            const uint4 w = lds128(a + 16 * c);
+            v[4 * c + 0] = __uint_as_float(w.x);
+            v[4 * c + 1] = __uint_as_float(w.y);
+            v[4 * c + 2] = __uint_as_float(w.z);
+            v[4 * c + 3] = __uint_as_float(w.w);
+        }
+    }
+}
+
+template <int DK, bool KDA, bool HAD, bool BF16>
+__global__ void __launch_bounds__(256, 1) prefill_cg_kernel(const PrefillParams p) {
+    constexpr int NR = DK / 16;  // key channels per lane
+    constexpr int ESZ = BF16 ? 2 : 4;
+    constexpr PrefillSmem SM = prefill_smem(DK, KDA, BF16);  // offsets inside a token buffer
+    constexpr PrefillCgSmem CG = prefill_cg_smem(DK, KDA, BF16);
+    extern __shared__ __align__(128) uint8_t smem[];
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    const int nw = blockDim.x >> 5;
+    const int hcol = lane & 1;                 // column half: columns 16 hcol .. + 15
+    const int ch0 = (lane >> 1) * NR;          // first key channel of the lane
+    const unsigned pmask = 3u << (lane & ~1);  // the two lanes of a channel group
+    const LaneSigns sg = lane_signs(lane);
+    const uint32_t ws = smem_u32(smem) + (uint32_t)(warp * p.warp_stride);
+    const uint32_t part = ws, dvec = ws + CG.dvec_off, inv_s = ws + CG.inv_off, perm_s = ws + CG.perm_off;
+    const uint32_t ops0 = ws + CG.ops_off, bar = ws + CG.bar_off, st = ws + CG.stage_off;
+    const uint32_t hrow = st + (uint32_t)((p.rec_bytes + 127) & ~127);  // FP16 rows, 128 B each
+    const int K = p.K, lo = DK - K, H = p.H, V = p.V, T = p.T;
+
+    const int64_t gw = (int64_t)blockIdx.x * nw + warp;
+    const int64_t nwt = (int64_t)gridDim.x * nw;
+    const int64_t t0 = p.total_tiles * gw / nwt, t1 = p.total_tiles * (gw + 1) / nwt;
+    if (t0 >= t1) return;
+    bool bad_slot = false, bad_head = false, timed_out = false;
+
+    auto rec_of = [&](int64_t tt, int &b, int &h, int &c, int &mh, int64_t &slot, int &Tb) -> uint8_t * {
+        c = (int)(tt % V);
+        const int64_t bh = tt / V;
+        h = (int)(bh % H);
+        b = (int)(bh / H);
+        mh = p.head_map ? p.head_map[h] : h;
+        slot = p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b;
+        Tb = p.lengths ? min(max(p.lengths[b], 0), T) : T;
+        return p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * p.rec_bytes;
+    };
+    auto issue = [&](int64_t tt) {  // lane 0
+        int b, h, c, mh, Tb;
+        int64_t slot;
+        uint8_t *g = rec_of(tt, b, h, c, mh, slot, Tb);
+        const bool run = slot >= 0 && slot < p.num_slots && mh >= 0 && mh < p.Hm && Tb > 0;
+        mbar_arrive_expect_tx(bar, run ? (uint32_t)p.rec_bytes : 0u);
+        if (run) bulk_g2s(st, g, (uint32_t)p.rec_bytes, bar);
+    };
+    if (lane == 0) {
+        mbar_init(bar, 1);
+        fence_mbar_init();
+        issue(t0);
+    }
+    __syncwarp();
+    uint32_t parity = 0;
+
+    for (int64_t t = t0; t < t1; ++t) {
+        if (!__all_sync(kFull, mbar_wait_bounded(bar, parity))) {
+            timed_out = true;
+            break;
+        }
+        parity ^= 1u;
+        int b, h, c, mh, Tb;
+        int64_t slot;
+        uint8_t *const grec = rec_of(t, b, h, c, mh, slot, Tb);  // written in place
+        const bool slot_ok = slot >= 0 && slot < p.num_slots, head_ok = mh >= 0 && mh < p.Hm;
+        bad_slot |= !slot_ok;
+        bad_head |= !head_ok;
+        if (!slot_ok || !head_ok || Tb == 0) {
+            if (lane == 0 && t + 1 < t1) issue(t + 1);
+            continue;
+        }
+
+        // token 0's operands of this tile and their per-token strides (in bytes)
+        const int Hm = p.Hm;
+        const int hq = (int)(((int64_t)mh * p.Hqk) / Hm);
+        const uint8_t *qt = (const uint8_t *)p.q + ((int64_t)b * T * p.Hqk + hq) * DK * ESZ;
+        const uint8_t *kt = (const uint8_t *)p.k + ((int64_t)b * T * p.Hqk + hq) * DK * ESZ;
+        const uint8_t *gt = (const uint8_t *)(p.g + ((int64_t)b * T * Hm + mh) * (KDA ? DK : 1));
+        const uint8_t *vt = (const uint8_t *)p.v + (((int64_t)b * T * Hm + mh) * p.dv + kG * c) * ESZ;
+        const uint8_t *bt = (const uint8_t *)(p.beta + (int64_t)b * T * Hm + mh);
+        float *ot = p.o + ((int64_t)b * T * Hm + mh) * p.dv + kG * c + lane;
+        const int64_t sqk = (int64_t)p.Hqk * DK * ESZ, sg4 = (int64_t)Hm * (KDA ? DK : 1) * 4,
+                      sv = (int64_t)Hm * p.dv * ESZ, sb = (int64_t)Hm * 4, so = (int64_t)Hm * p.dv;
+        auto load_token = [&](int tok, uint32_t dst) {
+            constexpr int nq = DK * ESZ / 16, ng = KDA ? DK * 4 / 16 : 0, nv = kG * ESZ / 16;
+            const uint8_t *qs = qt + tok * sqk, *ks = kt + tok * sqk, *gs = gt + tok * sg4, *vs = vt + tok * sv;
+#pragma unroll
+            for (int j = lane; j < nq; j += 32) cp_async16(dst + SM.off_q + 16 * j, qs + 16 * j);
+#pragma unroll
+            for (int j = lane; j < nq; j += 32) cp_async16(dst + SM.off_k + 16 * j, ks + 16 * j);
+#pragma unroll
+            for (int j = lane; j < ng; j += 32) cp_async16(dst + SM.off_g + 16 * j, gs + 16 * j);
+#pragma unroll
+            for (int j = lane; j < nv; j += 32) cp_async16(dst + SM.off_v + 16 * j, vs + 16 * j);
+            if (lane == 0) {
+                cp_async4(dst + SM.off_beta, bt + tok * sb);
+                if (!KDA) cp_async4(dst + SM.off_g, gs);
+            }
+            cp_async_commit();
+        };
+
+        // pi of this head and token 0's operands; then pi^-1 (the row of each channel)
+        __syncwarp();  // the previous tile's readers of the shared buffers are done
+        for (int ci = lane; ci < DK / 16; ci += 32) cp_async16(perm_s + 16 * ci, p.perm + (int64_t)h * DK + 16 * ci);
+        load_token(0, ops0);
+        cp_async_wait_all();
+        __syncwarp();
+#pragma unroll
+        for (int u = lane; u < DK; u += 32) sts_u8(inv_s + (lds_u8(perm_s + u) & (DK - 1)), (uint32_t)u);
+        __syncwarp();
+
+        // ---- the lane's channels x its 16 columns, FP32, undecayed, scaled by 2^-39;
+        //      with H_32 in the transformed domain (FP16 rows transformed here) ----
+        // FP16 rows in row order: lane u of each slot of 32 rows, H_32 in registers,
+        // scaled by 2^-39, into the row area
+        for (int u0 = 0; u0 < K; u0 += 32) {
+            const int u = u0 + lane;
+            if (u < K) {
+                float2 y[16];
+                load_hi_row(st, u, y);
+                if (HAD) hadamard_pairs(y);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const float2 a = mul2(y[2 * q], splat2(kDown)), b = mul2(y[2 * q + 1], splat2(kDown));  // exact
+                    sts128(hrow + 128 * u + 16 * q, make_uint4(__float_as_uint(a.x), __float_as_uint(a.y),
+                                                               __float_as_uint(b.x), __float_as_uint(b.y)));
+                }
+            }
+        }
+        __syncwarp();
+        float2 x[NR][8];
+#pragma unroll
+        for (int i = 0; i < NR; ++i) {
+            const int u = (int)(lds_u8(inv_s + ch0 + i) & (DK - 1));  // the same for both lanes of the group
+            if (u < K) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const uint4 w = lds128(hrow + 128 * u + 64 * hcol + 16 * q);
+                    x[i][2 * q] = make_float2(__uint_as_float(w.x), __uint_as_float(w.y));
+                    x[i][2 * q + 1] = make_float2(__uint_as_float(w.z), __uint_as_float(w.w));
+                }
+            } else {
+                const int r = u - K;
+                const uint4 cw = lds128(st + (uint32_t)(p.codes_off + lo_chunk_off(r, hcol, lo)));
+                const uint32_t sz = lds32(st + (uint32_t)(p.meta_off + 4 * r));
+                const float s = __half2float(__ushort_as_half((unsigned short)(sz & 0xffffu)));
+                const float z = __half2float(__ushort_as_half((unsigned short)(sz >> 16)));
+                const float2 nzb = splat2(-(8388608.0f + z)), sa = splat2(s * kDown);
+                const uint32_t w[4] = {cw.x, cw.y, cw.z, cw.w};
+#pragma unroll
+                for (int m = 0; m < 4; ++m) {
+                    x[i][2 * m] = mul2(add2(make_float2(u8_biased(w[m], 0), u8_biased(w[m], 1)), nzb), sa);
+                    x[i][2 * m + 1] = mul2(add2(make_float2(u8_biased(w[m], 2), u8_biased(w[m], 3)), nzb), sa);
+                }
+            }
+        }
+
+        // the stage has been read: the next tile's record comes in during this one
+        __syncwarp();
+        if (lane == 0 && t + 1 < t1) {
+            fence_proxy_async_smem();
+            issue(t + 1);
+        }
+
+        // H d of the pending update waits in dvec, beta k of the lane's channels in bkp;
+        // o_t = H (p~ - beta (k^T q) r~) + beta (k^T q) v is finished during token t+1.
+        float bkp[NR];
+#pragma unroll
+        for (int i = 0; i < NR; ++i) bkp[i] = 0.f;
+        sts32(dvec + 4 * lane, 0u);
+        float o_pend = 0.f, o_add = 0.f;
+        auto finish_o = [&](int tok) { ot[tok * so] = (HAD ? hadamard_lanes(o_pend, sg) : o_pend) + o_add; };
+        auto load_d = [&](float2 (&d)[8]) {  // H d at this lane's 16 columns
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const uint4 w = lds128(dvec + 64 * hcol + 16 * q);
+                d[2 * q] = make_float2(__uint_as_float(w.x), __uint_as_float(w.y));
+                d[2 * q + 1] = make_float2(__uint_as_float(w.z), __uint_as_float(w.w));
+            }
+        };
+        for (int tok = 0; tok < Tb; ++tok) {
+            const uint32_t ob = ops0 + (uint32_t)((tok & 1) * SM.ops_bytes);
+            cp_async_wait_all();
+            __syncwarp();
+            if (tok + 1 < Tb) load_token(tok + 1, ops0 + (uint32_t)(((tok + 1) & 1) * SM.ops_bytes));
+
+            // ---- operands of the lane's channels (contiguous) ----
+            const float beta = ldsf(ob + SM.off_beta);
+            float kv[NR], qv[NR], av[NR];
+            lds_operands<NR, BF16>(ob + SM.off_k + ESZ * ch0, kv);
+            lds_operands<NR, BF16>(ob + SM.off_q + ESZ * ch0, qv);
+            if constexpr (KDA) {
+                lds_operands<NR, false>(ob + SM.off_g + 4 * ch0, av);
+#pragma unroll
+                for (int i = 0; i < NR; ++i) av[i] = expf(av[i]);
+            } else {
+                const float alpha = expf(ldsf(ob + SM.off_g));
+#pragma unroll
+                for (int i = 0; i < NR; ++i) av[i] = alpha;
+            }
+            float kq = 0.f;
+#pragma unroll
+            for (int i = 0; i < NR; ++i) kq = fmaf(kv[i], qv[i], kq);
+#pragma unroll
+            for (int m = 2; m <= 16; m <<= 1) kq += __shfl_xor_sync(kFull, kq, m);  // over the channel groups
+            const float bkq = beta * kq;
+            const float vj = BF16 ? lds_bf16(ob + SM.off_v + 2 * lane) : ldsf(ob + SM.off_v + 4 * lane);
+            const float hv = HAD ? hadamard_lanes(vj, sg) : vj;  // H v: independent of the state
+            if (tok > 0) finish_o(tok - 1);
+
+            // ---- the previous token's update, decay and partial sums ----
+            float2 d[8];
+            load_d(d);
+            float2 ar[8], ap[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) ar[j] = ap[j] = make_float2(0.f, 0.f);
+#pragma unroll
+            for (int i = 0; i < NR; ++i) {
+                const float2 b2 = splat2(bkp[i]), a2 = splat2(av[i]), k2 = splat2(kv[i]), q2 = splat2(qv[i]);
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    x[i][j] = mul2(fma2(b2, d[j], x[i][j]), a2);
+                    ar[j] = fma2(x[i][j], k2, ar[j]);
+                    ap[j] = fma2(x[i][j], q2, ap[j]);
+                }
+            }
+            // ---- column sums: the transpose, then lane L sums column L over the 16 groups ----
+            const uint32_t row = part + (uint32_t)(lane * kCgRowBytes);
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                sts128(row + 16 * j, make_uint4(__float_as_uint(ar[j].x), __float_as_uint(ap[j].x),
+                                                __float_as_uint(ar[j].y), __float_as_uint(ap[j].y)));
+            __syncwarp();
+            const uint32_t col = part + (uint32_t)((lane >> 4) * kCgRowBytes + 8 * (lane & 15));
+            float2 s0 = make_float2(0.f, 0.f), s1 = s0, s2 = s0, s3 = s0;
+#pragma unroll
+            for (int g = 0; g < 16; g += 4) {
+                const uint2 w0 = lds64(col + (uint32_t)(2 * (g + 0) * kCgRowBytes));
+                const uint2 w1 = lds64(col + (uint32_t)(2 * (g + 1) * kCgRowBytes));
+                const uint2 w2 = lds64(col + (uint32_t)(2 * (g + 2) * kCgRowBytes));
+                const uint2 w3 = lds64(col + (uint32_t)(2 * (g + 3) * kCgRowBytes));
+                s0 = add2(s0, make_float2(__uint_as_float(w0.x), __uint_as_float(w0.y)));
+                s1 = add2(s1, make_float2(__uint_as_float(w1.x), __uint_as_float(w1.y)));
+                s2 = add2(s2, make_float2(__uint_as_float(w2.x), __uint_as_float(w2.y)));
+                s3 = add2(s3, make_float2(__uint_as_float(w3.x), __uint_as_float(w3.y)));
+            }
+            const float2 sums = add2(add2(s0, s1), add2(s2, s3));
+            const float rs = sums.x * kUp, ps = sums.y * kUp;
+
+            // ---- the column vector of the update, H d = H v - r~, and o_t's parts ----
+            sts32(dvec + 4 * lane, __float_as_uint(hv - rs));
+            o_pend = fmaf(-bkq, rs, ps);
+            o_add = bkq * vj;
+            const float bsc = beta * kDown;  // exact: kv bsc = fl(beta kv) 2^-39
+#pragma unroll
+            for (int i = 0; i < NR; ++i) bkp[i] = kv[i] * bsc;
+        }
+        finish_o(Tb - 1);
+        {  // the last token's update
+            __syncwarp();
+            float2 d[8];
+            load_d(d);
+#pragma unroll
+            for (int i = 0; i < NR; ++i) {
+#pragma unroll
+                for (int j = 0; j < 8; ++j) x[i][j] = fma2(splat2(bkp[i]), d[j], x[i][j]);
+            }
+        }
+
+        // ---- the chunk-final tile: FP16 rows rounded once, low-tier rows requantized ----
+#pragma unroll
+        for (int i = 0; i < NR; ++i) {
+            const int u = (int)(lds_u8(inv_s + ch0 + i) & (DK - 1));
+            if (u < K) {  // to the row area; written out in row order below
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    sts128(hrow + 128 * u + 64 * hcol + 16 * q,
+                           make_uint4(__float_as_uint(x[i][2 * q].x), __float_as_uint(x[i][2 * q].y),
+                                      __float_as_uint(x[i][2 * q + 1].x), __float_as_uint(x[i][2 * q + 1].y)));
+                continue;
+            }
+            const int r = u - K;
+            float v[16];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                v[2 * j] = x[i][j].x;
+                v[2 * j + 1] = x[i][j].y;
+            }
+            float a[5], bb[5];
+#pragma unroll
+            for (int m = 0; m < 5; ++m) {
+                a[m] = fmin3(v[3 * m], v[3 * m + 1], v[3 * m + 2]);
+                bb[m] = fmax3(v[3 * m], v[3 * m + 1], v[3 * m + 2]);
+            }
+            float mn = fmin3(fmin3(a[0], a[1], a[2]), a[3], fminf(a[4], v[15]));
+            float mx = fmax3(fmax3(bb[0], bb[1], bb[2]), bb[3], fmaxf(bb[4], v[15]));
+            mn = fminf(mn, __shfl_xor_sync(pmask, mn, 1));
+            mx = fmaxf(mx, __shfl_xor_sync(pmask, mx, 1));
+            float inv, zq;
+            const float sc = scale_of(mn, mx);
+            const uint32_t szw = sc == 0.0f ? affine_params_scaled(mn, mx, inv, zq) : affine_finish(sc, mn, inv, zq);
+            const float2 inv2 = splat2(inv * 0x1p-110f), zc2 = splat2(zq * 0x1p-149f);
+            uint32_t w[4];
+#pragma unroll
+            for (int m = 0; m < 4; ++m) w[m] = encode4(x[i][2 * m], x[i][2 * m + 1], inv2, zc2);
+            stg128(grec + p.codes_off + lo_chunk_off(r, hcol, lo), make_uint4(w[0], w[1], w[2], w[3]));
+            if (hcol == 0) stg32(grec + p.meta_off + 4 * r, szw);
+        }
+        // FP16 rows in row order: back to the natural domain, rounded once, in row pairs
+        __syncwarp();
+        for (int u0 = 0; u0 < K; u0 += 32) {  // warp-uniform: store_hi_row shuffles
+            const int u = u0 + lane;
+            float2 y[16];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                const uint4 w = u < K ? lds128(hrow + 128 * u + 16 * q) : make_uint4(0u, 0u, 0u, 0u);
+                y[2 * q] = make_float2(__uint_as_float(w.x), __uint_as_float(w.y));
+                y[2 * q + 1] = make_float2(__uint_as_float(w.z), __uint_as_float(w.w));
+            }
+            if (HAD) hadamard_pairs(y);
+            uint32_t own[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) own[j] = f2_to_h2(y[j].x * kUp, y[j].y * kUp);
+            store_hi_row(grec, u, K, lane, own);
+        }
+    }
+    if (timed_out) mbar_wait_bounded(bar, parity);
+    cp_async_wait_all();
+    if (lane == 0) {
+        const uint32_t bits =
+            (timed_out ? kDevWaitTimeout : 0u) | (bad_slot ? kDevBadSlot : 0u) | (bad_head ? kDevBadHead : 0u);
+        if (bits) atomicOr(p.status, bits);
+    }
+}
+
+}  // namespace damp

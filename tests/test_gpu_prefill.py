@@ -59,7 +59,7 @@ def _oracle_chunk(w, perm_units, tiers, u, lens_units):
     return o, new, lo_rows
 
 
-def _run(w, T, lengths=None, slot_of=None, pool=None, chunks=1):
+def _run(w, T, lengths=None, slot_of=None, pool=None, chunks=1, o_offset=None):
     rows = list(range(w.batch))
     perms, _ = runs.calibrate_layout(w, n_docs=2, n_tokens=16)
     perm_units, tiers = P.initial_tiers(w, rows, perms, prefix=min(w.prefix, 24))
@@ -79,7 +79,11 @@ def _run(w, T, lengths=None, slot_of=None, pool=None, chunks=1):
         u = _unit_chunk(w, inp, T)
         o_ref, tiers, lo_pre = _oracle_chunk(w, perm_units, tiers, u, lens_units)
         d = {key: P.to_dev(val, DEV, dt if key in ("q", "k", "v") else None) for key, val in inp.items()}
-        o = fn(L, state, dperm, d["q"], d["k"], d["v"], d["g"], d["beta"],
+        o_arg = None
+        if o_offset is not None:  # o at an offset of o_offset floats from a 16-byte boundary
+            n = len(rows) * T * w.heads * w.d_v
+            o_arg = torch.zeros(n + 4, device=DEV)[o_offset:o_offset + n].view(len(rows), T, w.heads, w.d_v)
+        o = fn(L, state, dperm, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o_arg,
                lengths=None if lengths is None else P.to_dev(lens, DEV), slot_idx=slot_idx)
         torch.cuda.synchronize()
         o = o.cpu().numpy().transpose(0, 2, 1, 3).reshape(len(rows) * w.heads, T, w.d_v)
@@ -116,6 +120,31 @@ def test_ragged_lengths_and_slot_indirection():
 ], ids=lambda w: w.name)
 def test_layouts(w):
     _run(w, 6)
+
+
+@pytest.mark.parametrize("w", [
+    wl.Workload("gdn_d64_dv96_k5_f1", "gdn", 2, 4, 2, 64, 96, 5, 4, 8, "fp32", 21, 1),
+    wl.Workload("kda_uniform", "kda", 1, 4, 4, 128, 64, 0, 4, 8, "bf16", 22, 0),
+    wl.Workload("kda_d64_all_fp16", "kda", 1, 2, 2, 64, 64, 64, 4, 8, "fp32", 23, 0),
+    wl.Workload("kda_k31_f1", "kda", 2, 2, 1, 128, 32, 31, 4, 8, "bf16", 25, 1),
+    wl.Workload("gdn_k127", "gdn", 1, 2, 2, 128, 64, 127, 4, 8, "fp32", 26, 0),
+], ids=lambda w: w.name)
+def test_layouts_long_chunks(w):
+    """Chunks of 32 and more tokens on the UINT8 tiers (d_k 64 and 128) run the kernel
+    that holds the tile in key-channel order: odd K_hi, all-FP16 and uniform tiers,
+    d_v = 32 and 96."""
+    _run(w, 32)
+
+
+def test_long_chunk_ragged_lengths_and_slot_indirection():
+    """Rows of 33, 17 and 0 tokens in a 33-token chunk, scattered over a larger pool."""
+    w = wl.GDN_B64_GQA.replace(batch=3, heads=4, qk_heads=2)
+    _run(w, 33, lengths=[33, 17, 0], slot_of={0: 4, 1: 1, 2: 0}, pool=5)
+
+
+def test_unaligned_output_runs_the_short_chunk_kernel():
+    """o that is not 16-byte aligned: a long chunk runs the kernel with 4-byte stores."""
+    _run(wl.KDA_B256.replace(batch=2, heads=4, qk_heads=4), 32, o_offset=1)
 
 
 def test_decode_after_prefill_reads_the_chunk_state():
