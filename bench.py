@@ -923,6 +923,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true", help="K_hi sweep (GDN and KDA, B=256) instead of the bench line")
     ap.add_argument("--prefill", action="store_true", help="prefill chunks (64 tokens, B=256) instead of the bench line")
+    ap.add_argument("--chunk-tokens", type=int, default=64, help="tokens per slot of a --prefill chunk")
     ap.add_argument("--multitoken", action="store_true",
                     help="fused multi-token steps (T = 1..16 tokens per launch, B=256) instead of the bench line")
     ap.add_argument("--calibrate", action="store_true", help="GPU calibration run instead of the bench line")
@@ -942,7 +943,7 @@ def main():
         sweep_arm(args.steps, args.warmup)
         return
     if args.prefill:
-        prefill_arm(args.steps, args.warmup)
+        prefill_arm(args.steps, args.warmup, args.chunk_tokens)
         return
     if args.multitoken:
         multitoken_arm(args.steps, args.warmup)
