@@ -150,28 +150,35 @@ __global__ void __launch_bounds__(256, 1) prefill_cg_kernel(const PrefillParams 
         float *ot = p.o + ((int64_t)b * T * Hm + mh) * p.dv + kG * c + lane;
         const int64_t sqk = (int64_t)p.Hqk * DK * ESZ, sg4 = (int64_t)Hm * (KDA ? DK : 1) * 4,
                       sv = (int64_t)Hm * p.dv * ESZ, sb = (int64_t)Hm * 4, so = (int64_t)Hm * p.dv;
-        auto load_token = [&](int tok, uint32_t dst) {
-            constexpr int nq = DK * ESZ / 16, ng = KDA ? DK * 4 / 16 : 0, nv = kG * ESZ / 16;
-            const uint8_t *qs = qt + tok * sqk, *ks = kt + tok * sqk, *gs = gt + tok * sg4, *vs = vt + tok * sv;
-#pragma unroll
-            for (int j = lane; j < nq; j += 32) cp_async16(dst + SM.off_q + 16 * j, qs + 16 * j);
-#pragma unroll
-            for (int j = lane; j < nq; j += 32) cp_async16(dst + SM.off_k + 16 * j, ks + 16 * j);
-#pragma unroll
-            for (int j = lane; j < ng; j += 32) cp_async16(dst + SM.off_g + 16 * j, gs + 16 * j);
-#pragma unroll
-            for (int j = lane; j < nv; j += 32) cp_async16(dst + SM.off_v + 16 * j, vs + 16 * j);
+        // each lane copies at most one 16-byte chunk of each operand vector per token
+        // (d_k <= 128); its source pointers advance by one token per copy
+        constexpr int nq = DK * ESZ / 16, ng = KDA ? DK * 4 / 16 : 0, nv = kG * ESZ / 16;
+        static_assert(nq <= 32 && ng <= 32 && nv <= 32, "one chunk per lane");
+        const uint8_t *sq = qt + 16 * lane, *sk = kt + 16 * lane, *sgl = gt + (KDA ? 16 * lane : 0),
+                      *svl = vt + 16 * lane, *sbl = bt;
+        auto load_next_token = [&](uint32_t dst) {
+            if (lane < nq) {
+                cp_async16(dst + SM.off_q + 16 * lane, sq);
+                cp_async16(dst + SM.off_k + 16 * lane, sk);
+            }
+            if (KDA && lane < ng) cp_async16(dst + SM.off_g + 16 * lane, sgl);
+            if (lane < nv) cp_async16(dst + SM.off_v + 16 * lane, svl);
             if (lane == 0) {
-                cp_async4(dst + SM.off_beta, bt + tok * sb);
-                if (!KDA) cp_async4(dst + SM.off_g, gs);
+                cp_async4(dst + SM.off_beta, sbl);
+                if (!KDA) cp_async4(dst + SM.off_g, sgl);
             }
             cp_async_commit();
+            sq += sqk;
+            sk += sqk;
+            sgl += sg4;
+            svl += sv;
+            sbl += sb;
         };
 
         // pi of this head and token 0's operands; then pi^-1 (the row of each channel)
         __syncwarp();  // the previous tile's readers of the shared buffers are done
         for (int ci = lane; ci < DK / 16; ci += 32) cp_async16(perm_s + 16 * ci, p.perm + (int64_t)h * DK + 16 * ci);
-        load_token(0, ops0);
+        load_next_token(ops0);
         cp_async_wait_all();
         __syncwarp();
 #pragma unroll
@@ -238,7 +245,11 @@ __global__ void __launch_bounds__(256, 1) prefill_cg_kernel(const PrefillParams 
         for (int i = 0; i < NR; ++i) bkp[i] = 0.f;
         sts32(dvec + 4 * lane, 0u);
         float o_pend = 0.f, o_add = 0.f;
-        auto finish_o = [&](int tok) { ot[tok * so] = (HAD ? hadamard_lanes(o_pend, sg) : o_pend) + o_add; };
+        float *op = ot;  // o of the token being finished
+        auto finish_o = [&]() {
+            *op = (HAD ? hadamard_lanes(o_pend, sg) : o_pend) + o_add;
+            op += so;
+        };
         auto load_d = [&](float2 (&d)[8]) {  // H d at this lane's 16 columns
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -251,7 +262,7 @@ __global__ void __launch_bounds__(256, 1) prefill_cg_kernel(const PrefillParams 
             const uint32_t ob = ops0 + (uint32_t)((tok & 1) * SM.ops_bytes);
             cp_async_wait_all();
             __syncwarp();
-            if (tok + 1 < Tb) load_token(tok + 1, ops0 + (uint32_t)(((tok + 1) & 1) * SM.ops_bytes));
+            if (tok + 1 < Tb) load_next_token(ops0 + (uint32_t)(((tok + 1) & 1) * SM.ops_bytes));
 
             // ---- operands of the lane's channels (contiguous) ----
             const float beta = ldsf(ob + SM.off_beta);
@@ -275,7 +286,7 @@ __global__ void __launch_bounds__(256, 1) prefill_cg_kernel(const PrefillParams 
             const float bkq = beta * kq;
             const float vj = BF16 ? lds_bf16(ob + SM.off_v + 2 * lane) : ldsf(ob + SM.off_v + 4 * lane);
             const float hv = HAD ? hadamard_lanes(vj, sg) : vj;  // H v: independent of the state
-            if (tok > 0) finish_o(tok - 1);
+            if (tok > 0) finish_o();  // token tok - 1
 
             // ---- the previous token's update, decay and partial sums ----
             float2 d[8];
@@ -324,7 +335,7 @@ __global__ void __launch_bounds__(256, 1) prefill_cg_kernel(const PrefillParams 
 #pragma unroll
             for (int i = 0; i < NR; ++i) bkp[i] = kv[i] * bsc;
         }
-        finish_o(Tb - 1);
+        finish_o();  // token Tb - 1
         {  // the last token's update
             __syncwarp();
             float2 d[8];

@@ -277,3 +277,40 @@ def run_teacher_forced(w: wl.Workload, steps: int, dev, rows=None, n_docs=2, n_t
         tiers = new_ref
     stats.check_fraction()
     return stats
+
+
+# ---- prefill chunks (App. A.5) ----
+
+def chunk_inputs(w, t0, T, rows):
+    """Per-token draws of the decode stream, stacked on a token axis after the batch axis."""
+    steps = [wl.step_inputs(w, t0 + t, rows=rows) for t in range(T)]
+    return {key: np.stack([s[key] for s in steps], axis=1) for key in steps[0]}
+
+
+def unit_chunk(w, inp, T):
+    """Per-(slot, head) operands [n, T, ...] (GQA expanded) for the oracle."""
+    per_t = [runs.unit_operands(w, {key: val[:, t] for key, val in inp.items()}) for t in range(T)]
+    return {key: np.stack([u[key] for u in per_t], axis=1) for key in per_t[0]}
+
+
+def oracle_chunk(w, perm_units, tiers, u, lens_units):
+    """The oracle's chunk, plus its chunk-final FP32 state for the tie rules."""
+    n = perm_units.shape[0]
+    S = core.unpack_heads(perm_units, *tiers, w.k_hi, w.lo_format, w.d_k, w.d_v)
+    for t in range(u["q"].shape[1]):
+        live = lens_units > t
+        if live.any():
+            sub = np.ascontiguousarray(S[live])
+            core.delta_step_heads(sub, u["q"][live, t], u["k"][live, t], u["v"][live, t], u["g"][live, t],
+                                  u["beta"][live, t], w.kind)
+            S[live] = sub
+    new = tuple(np.ascontiguousarray(t).copy() for t in tiers)
+    o = core.prefill_chunk_heads(perm_units, *new, u["q"], u["k"], u["v"], u["g"], u["beta"], w.k_hi, w.lo_format,
+                                 w.kind, lengths=lens_units)
+    assert np.array_equal(core.unpack_heads(perm_units, *new, w.k_hi, w.lo_format, w.d_k, w.d_v)[lens_units > 0],
+                          core.unpack_heads(perm_units, *core.pack_heads(perm_units, S, w.k_hi, w.lo_format),
+                                            w.k_hi, w.lo_format, w.d_k, w.d_v)[lens_units > 0])
+    lo_rows = np.stack([S[i][perm_units[i][w.k_hi:]] for i in range(n)])
+    if w.lo_format in (core.FMT_U8_H32, core.FMT_U4_H32) and lo_rows.size:
+        lo_rows = core.hadamard32(lo_rows.reshape(-1, 32)).reshape(lo_rows.shape)
+    return o, new, lo_rows

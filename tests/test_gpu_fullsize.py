@@ -59,3 +59,48 @@ def test_gdn_b64_gqa_full_batch_sampled_rows():
 @pytest.mark.parametrize("kind", ["gdn", "kda"])
 def test_sweep_k16_full_batch_sampled_rows(kind):
     _fullsize(wl.sweep(kind, 16), [5, 200], 1)
+
+
+def _fullsize_chunk(w, sample_rows, T):
+    """One prefill chunk of T tokens over the whole batch (the launch the prefill bench
+    times); the oracle runs the chunk for every head of the sampled rows."""
+    perms, _ = runs.calibrate_layout(w, n_docs=4, n_tokens=64)
+    perm_units, tiers = P.initial_tiers(w, sample_rows, perms)
+    L = P.layout_of(w)
+    state = damp.new_state(L, w.batch, DEV)
+    dperm = P.to_dev(perms, DEV)
+    gen = torch.Generator(device=DEV)
+    gen.manual_seed(w.seed)
+    S = 0.3 * torch.randn((w.batch, w.heads, w.d_k, w.d_v), generator=gen, device=DEV)
+    damp.quantize_state(L, S, dperm, state)
+    del S
+    sidx = torch.tensor(sample_rows, dtype=torch.int32, device=DEV)
+    damp.pack_tiers(L, *P.tiers_to_dev(w, tiers, len(sample_rows), DEV), state, slot_idx=sidx)
+    inp = P.chunk_inputs(w, 0, T, list(range(w.batch)))
+    u = P.unit_chunk(w, {k: v[sample_rows] for k, v in inp.items()}, T)
+    lens_units = np.full(len(sample_rows) * w.heads, T, np.int32)
+    o_ref, new_ref, lo_pre = P.oracle_chunk(w, perm_units, tiers, u, lens_units)
+    dt = torch.bfloat16 if w.in_dtype == "bf16" else torch.float32
+    d = {k: P.to_dev(v, DEV, dt if k in ("q", "k", "v") else None) for k, v in inp.items()}
+    del inp
+    fn = damp.kda_prefill_chunk if w.kind == "kda" else damp.gdn_prefill_chunk
+    o = fn(L, state, dperm, d["q"], d["k"], d["v"], d["g"], d["beta"])
+    o = o[sample_rows].cpu().numpy().transpose(0, 2, 1, 3).reshape(len(sample_rows) * w.heads, T, w.d_v)
+    for i in range(o.shape[0]):
+        P.compare_o(o[i], o_ref[i], f"{w.name} chunk unit {i}")
+    got = P.tiers_from_dev(w, damp.unpack_tiers(L, state, batch=len(sample_rows), slot_idx=sidx),
+                           len(sample_rows) * w.heads)
+    stats = P.CodeStats()
+    P.compare_tiers(w, new_ref, got, lo_pre, stats, f"{w.name} chunk")
+    stats.check_fraction()
+    assert damp.device_status() == 0
+
+
+def test_kda_b256_prefill_chunk_sampled_rows():
+    """KDA B=256, H=32, d=128, K_hi=10, BF16, one 64-token chunk: rows 0 and 255."""
+    _fullsize_chunk(wl.KDA_B256, [0, 255], 64)
+
+
+def test_gdn_k16_prefill_chunk_sampled_rows():
+    """GDN B=256, H=32, d=128, K_hi=16, one 64-token chunk: rows 3 and 128."""
+    _fullsize_chunk(wl.sweep("gdn", 16), [3, 128], 64)

@@ -7,7 +7,7 @@ import torch
 
 import paper_2608_27513_gb300 as damp
 import workloads as wl
-from oracle import core, runs
+from oracle import runs
 from tests import parity as P
 
 pytestmark = pytest.mark.gpu
@@ -22,41 +22,6 @@ def _built():
     assert damp.device_status() == 0
     yield
     assert damp.device_status() == 0
-
-
-def _chunk_inputs(w, t0, T, rows):
-    """Per-token draws of the decode stream, stacked on a token axis after the batch axis."""
-    steps = [wl.step_inputs(w, t0 + t, rows=rows) for t in range(T)]
-    return {key: np.stack([s[key] for s in steps], axis=1) for key in steps[0]}
-
-
-def _unit_chunk(w, inp, T):
-    """Per-(slot, head) operands [n, T, ...] (GQA expanded) for the oracle."""
-    per_t = [runs.unit_operands(w, {key: val[:, t] for key, val in inp.items()}) for t in range(T)]
-    return {key: np.stack([u[key] for u in per_t], axis=1) for key in per_t[0]}
-
-
-def _oracle_chunk(w, perm_units, tiers, u, lens_units):
-    """The oracle's chunk, plus its chunk-final FP32 state for the tie rules."""
-    n = perm_units.shape[0]
-    S = core.unpack_heads(perm_units, *tiers, w.k_hi, w.lo_format, w.d_k, w.d_v)
-    for t in range(u["q"].shape[1]):
-        live = lens_units > t
-        if live.any():
-            sub = np.ascontiguousarray(S[live])
-            core.delta_step_heads(sub, u["q"][live, t], u["k"][live, t], u["v"][live, t], u["g"][live, t],
-                                  u["beta"][live, t], w.kind)
-            S[live] = sub
-    new = tuple(np.ascontiguousarray(t).copy() for t in tiers)
-    o = core.prefill_chunk_heads(perm_units, *new, u["q"], u["k"], u["v"], u["g"], u["beta"], w.k_hi, w.lo_format,
-                                 w.kind, lengths=lens_units)
-    assert np.array_equal(core.unpack_heads(perm_units, *new, w.k_hi, w.lo_format, w.d_k, w.d_v)[lens_units > 0],
-                          core.unpack_heads(perm_units, *core.pack_heads(perm_units, S, w.k_hi, w.lo_format),
-                                            w.k_hi, w.lo_format, w.d_k, w.d_v)[lens_units > 0])
-    lo_rows = np.stack([S[i][perm_units[i][w.k_hi:]] for i in range(n)])
-    if w.lo_format in (core.FMT_U8_H32, core.FMT_U4_H32) and lo_rows.size:
-        lo_rows = core.hadamard32(lo_rows.reshape(-1, 32)).reshape(lo_rows.shape)
-    return o, new, lo_rows
 
 
 def _run(w, T, lengths=None, slot_of=None, pool=None, chunks=1, o_offset=None):
@@ -75,9 +40,9 @@ def _run(w, T, lengths=None, slot_of=None, pool=None, chunks=1, o_offset=None):
     for ch in range(chunks):
         # teacher-forced: every chunk starts from the oracle's packed state
         damp.pack_tiers(L, *P.tiers_to_dev(w, tiers, len(rows), DEV), state, slot_idx=slot_idx)
-        inp = _chunk_inputs(w, ch * T, T, rows)
-        u = _unit_chunk(w, inp, T)
-        o_ref, tiers, lo_pre = _oracle_chunk(w, perm_units, tiers, u, lens_units)
+        inp = P.chunk_inputs(w, ch * T, T, rows)
+        u = P.unit_chunk(w, inp, T)
+        o_ref, tiers, lo_pre = P.oracle_chunk(w, perm_units, tiers, u, lens_units)
         d = {key: P.to_dev(val, DEV, dt if key in ("q", "k", "v") else None) for key, val in inp.items()}
         o_arg = None
         if o_offset is not None:  # o at an offset of o_offset floats from a 16-byte boundary
