@@ -62,11 +62,11 @@ def test_decode_steps_replay_from_a_graph(fmt, K):
         assert torch.equal(state, eager)
 
 
-def test_prefill_chunk_replays_from_a_graph():
+@pytest.mark.parametrize("T", [4, 32])
+def test_prefill_chunk_replays_from_a_graph(T):
     w = wl.GDN_B64_GQA.replace(batch=2)
     L, perm, state = _setup(w, 82)
     eager = state.clone()
-    T = 4
     steps = [wl.step_inputs(w, t) for t in range(T)]
     dt = torch.bfloat16
     chunk = {k: P.to_dev(np.stack([s[k] for s in steps], axis=1), DEV, dt if k in ("q", "k", "v") else None)

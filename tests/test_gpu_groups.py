@@ -90,15 +90,16 @@ def test_groups_at_one_k_hi_reproduce_the_layer(kind, fmt, K):
         assert bool((back[:, others] == 0).all())
 
 
-@pytest.mark.parametrize("fmt", [0, 3])
-def test_group_prefill_chunks_reproduce_the_layer(fmt):
+@pytest.mark.parametrize("fmt,T", [(0, 5), (3, 5), (0, 32), (1, 40)])
+def test_group_prefill_chunks_reproduce_the_layer(fmt, T):
+    """Both chunk kernels (5 tokens; 32 and 40 tokens on the UINT8 tiers) with head maps."""
     w = wl.KDA_B256.replace(batch=2, heads=8, qk_heads=8, lo_format=fmt, k_hi=12)
     L = P.layout_of(w)
     S, perm = _layer(w, 92)
     pool = damp.new_state(L, w.batch, DEV)
     damp.quantize_state(L, S, perm, pool)
-    c = _chunk(w, 5)
-    lens = torch.tensor([5, 3], dtype=torch.int32, device=DEV)
+    c = _chunk(w, T)
+    lens = torch.tensor([T, 3], dtype=torch.int32, device=DEV)
     o = damp.kda_prefill_chunk(L, pool, perm, c["q"], c["k"], c["v"], c["g"], c["beta"], lengths=lens)
     og = torch.zeros_like(o)
     for hs in (HEADS_A, HEADS_B):

@@ -79,10 +79,10 @@ def test_decode_step_writes_only_its_slots_and_o(fmt, K):
     assert bool(torch.isfinite(o.t).all())
 
 
-def test_prefill_leaves_rows_past_their_length_and_guards_alone():
+@pytest.mark.parametrize("T", [5, 32])
+def test_prefill_leaves_rows_past_their_length_and_guards_alone(T):
     w = wl.KDA_B256.replace(batch=3, heads=4, qk_heads=4)
     L = P.layout_of(w)
-    T = 5
     pool = _pool(L, 3)
     S = P.to_dev(wl.random_states(72, 12, 128, 128).reshape(3, 4, 128, 128), DEV)
     perm = P.to_dev(np.tile(np.arange(128, dtype=np.uint8), (4, 1)), DEV)
@@ -91,7 +91,7 @@ def test_prefill_leaves_rows_past_their_length_and_guards_alone():
     o = Guarded((3, T, 4, 128), torch.float32)
     o.t.fill_(7.0)
     d = _inputs(w, T)
-    lens = torch.tensor([5, 2, 0], dtype=torch.int32, device=DEV)
+    lens = torch.tensor([T, 2, 0], dtype=torch.int32, device=DEV)
     damp.kda_prefill_chunk(L, pool.t, perm, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o.t, lengths=lens)
     pool.check()
     o.check()
