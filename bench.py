@@ -564,7 +564,7 @@ def sweep_arm(steps: int, warmup: int):
         print(json.dumps(row), flush=True)
 
 
-def prefill_arm(steps: int, warmup: int, T: int = 64):
+def prefill_arm(steps: int, warmup: int, T: int = 64, lo_format: int = 0):
     """Prefill chunks (App. A.5 prefill path) at B = 256, H = 32, d = 128: one launch per
     chunk of T tokens per slot.  The chunk keeps each tile's FP32 state on chip, so it
     is bound by FP32 FMA throughput, not HBM: achieved = algorithmic FLOPs / time against
@@ -578,7 +578,7 @@ def prefill_arm(steps: int, warmup: int, T: int = 64):
     torch.cuda.set_device(dev)
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     out = []
-    for w in (wl.KDA_B256, wl.sweep("gdn", 16)):
+    for w in (wl.KDA_B256.replace(lo_format=lo_format), wl.sweep("gdn", 16, lo_format)):
         L = damp.Layout(w.heads, w.qk_heads, w.d_k, w.d_v, w.k_hi, w.lo_format)
         per_t = wl.torch_step_inputs(w, T, dev)
         chunk = {key: torch.stack([d[key] for d in per_t], dim=1).contiguous() for key in per_t[0]}
@@ -615,7 +615,8 @@ def prefill_arm(steps: int, warmup: int, T: int = 64):
         hbm = (2 * w.batch * w.heads * damp.slot_bytes(L) // w.heads
                + w.batch * T * (2 * w.qk_heads * w.d_k * esz + w.heads * w.d_v * (esz + 4)
                                 + w.heads * 4 * ((w.d_k if w.kind == "kda" else 1) + 1)))
-        out.append({"mode": "prefill_chunk", "kind": w.kind, "workload": w.name, "chunk_tokens": T,
+        out.append({"mode": "prefill_chunk", "kind": w.kind, "workload": w.name, "lo_format": w.lo_format,
+                    "chunk_tokens": T,
                     "us_per_chunk": us, "tokens_per_s": w.batch * T / (us * 1e-6),
                     "roofline": {"bound": "fma", "achieved": flops / (us * 1e-6) / 1e12, "peak": peak / 1e12,
                                  "unit": "TFLOP/s", "frac": flops / (us * 1e-6) / peak,
@@ -924,6 +925,7 @@ def main():
     ap.add_argument("--sweep", action="store_true", help="K_hi sweep (GDN and KDA, B=256) instead of the bench line")
     ap.add_argument("--prefill", action="store_true", help="prefill chunks (64 tokens, B=256) instead of the bench line")
     ap.add_argument("--chunk-tokens", type=int, default=64, help="tokens per slot of a --prefill chunk")
+    ap.add_argument("--lo-format", type=int, default=0, help="low-tier format of the --prefill workloads (0-5)")
     ap.add_argument("--multitoken", action="store_true",
                     help="fused multi-token steps (T = 1..16 tokens per launch, B=256) instead of the bench line")
     ap.add_argument("--calibrate", action="store_true", help="GPU calibration run instead of the bench line")
@@ -943,7 +945,7 @@ def main():
         sweep_arm(args.steps, args.warmup)
         return
     if args.prefill:
-        prefill_arm(args.steps, args.warmup, args.chunk_tokens)
+        prefill_arm(args.steps, args.warmup, args.chunk_tokens, args.lo_format)
         return
     if args.multitoken:
         multitoken_arm(args.steps, args.warmup)

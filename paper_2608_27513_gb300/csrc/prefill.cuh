@@ -339,9 +339,7 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
         for (int i = 0; i < R; ++i) bkp[i] = make_float2(0.f, 0.f);
         sts32(dvec + 4 * lane, 0u);
         float o_pend = 0.f, o_add = 0.f;
-        auto finish_o = [&](int tok) {
-            ot[tok * so] = (HAD ? hadamard_lanes(o_pend, sg) : o_pend) + o_add;
-        };
+        auto finish_o = [&]() { return (HAD ? hadamard_lanes(o_pend, sg) : o_pend) + o_add; };
         for (int tok = 0; tok < Tb; ++tok) {
             const uint32_t ob = ops0 + (uint32_t)((tok & 1) * SM.ops_bytes);
             cp_async_wait_all();
@@ -370,7 +368,9 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
             const float bkq = beta * kq;
             const float vj = BF16 ? lds_bf16(ob + SM.off_v + 2 * lane) : ldsf(ob + SM.off_v + 4 * lane);
             const float hv = HAD ? hadamard_lanes(vj, sg) : vj;  // H v: independent of the state
-            if (tok > 0) finish_o(tok - 1);
+            // o of token tok - 1 (meaningless at tok = 0, not stored): computed here without a
+            // branch, so that its butterfly and that of H v overlap the pass over the registers
+            const float o_prev = finish_o();
 
             // ---- the previous token's update, decay and partial sums ----
             float2 d[16];
@@ -392,12 +392,13 @@ __global__ void __launch_bounds__(256, 1) prefill_chunk_kernel(const PrefillPara
 
             // ---- the column vector of the update, H d = H v - r~, and o_t's parts ----
             sts32(dvec + 4 * lane, __float_as_uint(hv - rs));
+            if (tok > 0) ot[(tok - 1) * so] = o_prev;
             o_pend = fmaf(-bkq, rs, ps);
             o_add = bkq * vj;
 #pragma unroll
             for (int i = 0; i < R; ++i) bkp[i] = bk[i];
         }
-        finish_o(Tb - 1);
+        ot[(Tb - 1) * so] = finish_o();
         {  // the last token's update
             __syncwarp();
             float2 d[16];

@@ -246,10 +246,7 @@ __global__ void __launch_bounds__(256, 1) prefill_cg_kernel(const PrefillParams 
         sts32(dvec + 4 * lane, 0u);
         float o_pend = 0.f, o_add = 0.f;
         float *op = ot;  // o of the token being finished
-        auto finish_o = [&]() {
-            *op = (HAD ? hadamard_lanes(o_pend, sg) : o_pend) + o_add;
-            op += so;
-        };
+        auto finish_o = [&]() { return (HAD ? hadamard_lanes(o_pend, sg) : o_pend) + o_add; };
         auto load_d = [&](float2 (&d)[8]) {  // H d at this lane's 16 columns
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
@@ -286,7 +283,9 @@ __global__ void __launch_bounds__(256, 1) prefill_cg_kernel(const PrefillParams 
             const float bkq = beta * kq;
             const float vj = BF16 ? lds_bf16(ob + SM.off_v + 2 * lane) : ldsf(ob + SM.off_v + 4 * lane);
             const float hv = HAD ? hadamard_lanes(vj, sg) : vj;  // H v: independent of the state
-            if (tok > 0) finish_o();  // token tok - 1
+            // o of token tok - 1 (meaningless at tok = 0, not stored): computed here without a
+            // branch, so that its butterfly and that of H v overlap the pass over the registers
+            const float o_prev = finish_o();
 
             // ---- the previous token's update, decay and partial sums ----
             float2 d[8];
@@ -329,13 +328,17 @@ __global__ void __launch_bounds__(256, 1) prefill_cg_kernel(const PrefillParams 
 
             // ---- the column vector of the update, H d = H v - r~, and o_t's parts ----
             sts32(dvec + 4 * lane, __float_as_uint(hv - rs));
+            if (tok > 0) {
+                *op = o_prev;
+                op += so;
+            }
             o_pend = fmaf(-bkq, rs, ps);
             o_add = bkq * vj;
             const float bsc = beta * kDown;  // exact: kv bsc = fl(beta kv) 2^-39
 #pragma unroll
             for (int i = 0; i < NR; ++i) bkp[i] = kv[i] * bsc;
         }
-        finish_o();  // token Tb - 1
+        *op = finish_o();  // token Tb - 1
         {  // the last token's update
             __syncwarp();
             float2 d[8];
