@@ -60,3 +60,18 @@ def test_prefix_then_quantized_decode_stays_close_to_fp32():
         den += float((o_ref ** 2).sum())
     rrmse = np.sqrt(num / den)  # App. E trajectory RRMSE of the output
     assert 0 < rrmse < 0.05
+
+
+def test_gqa_mapping_is_consecutive_pairs():
+    """Reading of the GQA mapping (not in the paper): value head h reads q/k head
+    floor(h * H_qk / H), so with 32 value heads over 16 q/k heads heads 2j and 2j+1 share
+    q/k head j; without GQA the map is the identity.  unit_operands takes q and k rows
+    through that map and v, beta, g through the value head."""
+    w = wl.GDN_B64_GQA
+    assert (w.heads, w.qk_heads) == (32, 16)
+    assert [wl.qk_head_of(w, h) for h in range(32)] == [h // 2 for h in range(32)]
+    assert [wl.qk_head_of(wl.KDA_B256, h) for h in range(32)] == list(range(32))
+    inp = wl.step_inputs(w, 0, rows=[2])
+    u = runs.unit_operands(w, inp, heads=[5, 6])
+    assert np.array_equal(u["q"][0], inp["q"][0, 2]) and np.array_equal(u["k"][1], inp["k"][0, 3])
+    assert np.array_equal(u["v"][1], inp["v"][0, 6]) and u["beta"][0] == inp["beta"][0, 5]
