@@ -58,3 +58,25 @@ def test_reference_arm_prints_from_rank_zero_only():
     r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1",
                         "--warmup", "3"], env=env, capture_output=True, text=True, timeout=300)
     assert r.returncode == 0 and r.stdout.strip() == ""
+
+
+def test_bench_line_carries_the_contract_keys():
+    """The JSON line of one rank: every key the bench contract names, with its type."""
+    sys.path.insert(0, ROOT)
+    import json
+
+    import bench
+    r = {"w": bench.WORKLOAD, "total_ms": 8.0, "launch_ms": 0.08, "fp32_launch_ms": 0.2, "e2e_ms": 0.085,
+         "h2d": 10, "d2h": 4, "clocks": {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": []}, "bits": 9.5,
+         "dev_name": "cpu", "reps_ms": [0.08] * 5, "graph_ms": 0.079}
+    line = json.loads(json.dumps(bench.make_line(r, 100, 5, 1)))
+    for key, typ in (("metric", str), ("value", float), ("unit", str), ("n_gpus", int), ("steps", int),
+                     ("warmup", int), ("ms_per_step", float), ("higher_is_better", bool), ("scaling", str),
+                     ("dtype", str), ("data", str), ("config", dict), ("clocks", dict), ("e2e", dict),
+                     ("gpu_launches", int), ("roofline", dict)):
+        assert isinstance(line[key], typ), key
+    assert "vs_baseline" in line and line["config"]["workload"] == bench.WORKLOAD.name
+    assert set(line["e2e"]) >= {"value", "unit", "h2d_bytes_per_step", "d2h_bytes_per_step"}
+    assert set(line["roofline"]) >= {"bound", "achieved", "peak", "unit", "frac", "traffic"}
+    assert line["roofline"]["frac"] == pytest.approx(line["roofline"]["achieved"] / line["roofline"]["peak"])
+    assert line["value"] == pytest.approx(bench.algorithmic_bytes(bench.WORKLOAD) / 0.08e-3 / 1e12)
