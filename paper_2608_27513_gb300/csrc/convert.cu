@@ -181,7 +181,7 @@ __global__ void __launch_bounds__(256) convert_kernel(const ConvParams p) {
 template <int OP>
 static cudaError_t launch_convert(const ConvArgs &a, cudaStream_t stream) {
     ConvParams p{};
-    static uint32_t *cache[64];
+    static std::atomic<uint32_t *> cache[64];
     cudaError_t e = symbol_address_cached(&g_status_convert, cache, &p.status);
     if (e != cudaSuccess) return e;
     const RecGeom rg = rec_geom(a.dk, a.K, a.fmt);

@@ -310,16 +310,19 @@ cudaError_t ensure_smem_limit(const void *kernel, int bytes) {
     return e;
 }
 
-cudaError_t symbol_address_cached(const void *symbol, uint32_t **cache, uint32_t **out) {
+cudaError_t symbol_address_cached(const void *symbol, std::atomic<uint32_t *> *cache, uint32_t **out) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    if (dev >= 0 && dev < kMaxDevices && cache[dev]) {
-        *out = cache[dev];
-        return cudaSuccess;
+    if (dev >= 0 && dev < kMaxDevices) {
+        uint32_t *known = cache[dev].load(std::memory_order_acquire);
+        if (known) {
+            *out = known;
+            return cudaSuccess;
+        }
     }
     e = cudaGetSymbolAddress(reinterpret_cast<void **>(out), symbol);
-    if (e == cudaSuccess && dev >= 0 && dev < kMaxDevices) cache[dev] = *out;
+    if (e == cudaSuccess && dev >= 0 && dev < kMaxDevices) cache[dev].store(*out, std::memory_order_release);
     return e;
 }
 int max_smem_per_block() { return device_attr(g_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, 48 * 1024); }

@@ -5,6 +5,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 namespace damp {
 
 struct StepArgs {
@@ -101,6 +103,9 @@ int max_smem_per_block();
 cudaError_t ensure_smem_limit(const void *kernel, int bytes);
 
 // Device address of a __device__ status word, looked up once per device.
-cudaError_t symbol_address_cached(const void *symbol, uint32_t **cache_per_device, uint32_t **out);
+// The device address of a status-word symbol, looked up once per device (the cache is
+// an array of 64 per-device slots, written atomically: concurrent first calls store the
+// same address).
+cudaError_t symbol_address_cached(const void *symbol, std::atomic<uint32_t *> *cache_per_device, uint32_t **out);
 
 }  // namespace damp

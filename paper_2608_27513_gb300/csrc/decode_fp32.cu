@@ -126,7 +126,7 @@ __global__ void __launch_bounds__(256, 1) fp32_step_kernel(const Fp32Params p) {
 
 cudaError_t launch_fp32_step(const StepArgs &a, cudaStream_t stream) {
     Fp32Params p{};
-    static uint32_t *cache[64];
+    static std::atomic<uint32_t *> cache[64];
     cudaError_t e = symbol_address_cached(&g_status_fp32, cache, &p.status);
     if (e != cudaSuccess) return e;
     p.state = static_cast<float *>(a.state);

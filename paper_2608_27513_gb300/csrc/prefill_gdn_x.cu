@@ -7,7 +7,7 @@ namespace damp {
 static __device__ uint32_t g_status_prefill_gdn_x;
 
 cudaError_t launch_prefill_gdn_x(const StepArgs &a, cudaStream_t s) {
-    static uint32_t *cache[64];
+    static std::atomic<uint32_t *> cache[64];
     uint32_t *status = nullptr;
     cudaError_t e = symbol_address_cached(&g_status_prefill_gdn_x, cache, &status);
     if (e != cudaSuccess) return e;

@@ -9,7 +9,7 @@ static __device__ uint32_t g_status_prefill_kda;
 
 cudaError_t launch_prefill_kda(const StepArgs &a, cudaStream_t s) {
     if (a.fmt != kFmtU8H32 && a.fmt != kFmtU8) return launch_prefill_kda_x(a, s);
-    static uint32_t *cache[64];
+    static std::atomic<uint32_t *> cache[64];
     uint32_t *status = nullptr;
     cudaError_t e = symbol_address_cached(&g_status_prefill_kda, cache, &status);
     if (e != cudaSuccess) return e;

@@ -319,7 +319,7 @@ __global__ void __launch_bounds__(256) rowabs_convert_kernel(const RowAbsConv p)
 }
 
 uint32_t *status_word(cudaError_t *e) {
-    static uint32_t *cache[64];
+    static std::atomic<uint32_t *> cache[64];
     uint32_t *p = nullptr;
     *e = symbol_address_cached(&g_status_rowabs, cache, &p);
     return p;
