@@ -26,11 +26,11 @@ namespace damp {
 
 namespace {
 
-// One CTA per (head, 32 key channels); warp w takes batch rows w, w + 8, ...; lane u
-// accumulates its row's error over those rows and the value blocks; the eight warp
+// One CTA per (head, 32 key channels); warp w takes batch rows w, w + 16, ...; lane u
+// accumulates its row's error over those rows and the value blocks; the sixteen warp
 // partials are added in warp order (a fixed order: the result does not depend on
 // scheduling).
-constexpr int kEeWarps = 8;
+constexpr int kEeWarps = 16;
 
 __device__ uint32_t g_status_calib;
 
