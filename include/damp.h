@@ -252,6 +252,9 @@ DAMP_API damp_status damp_fp32_kda_decode_step(const damp_layout *layout, float 
  *   beta       float [B][T][H_m], 4-B aligned
  *   o          float [B][T][H_m][d_v]: o_t from the FP32 state after token t; rows past
  *              a row's length are not written.  Must not overlap the pool or inputs.
+ *              4-B aligned; when it is 16-B aligned, chunks of T >= 32 tokens on the
+ *              UINT8 tiers (formats 0, 1; d_k 64 or 128) run a kernel with less work per
+ *              token (the results differ only in FP32 rounding order).
  * Other arguments as in damp_gdn_decode_step.  Any lo_format; the row-absmax format
  * (2) needs d_v <= 128 (DAMP_ERR_SHAPE otherwise): its row scale spans the value blocks
  * of a head, which four warps then share.
