@@ -29,7 +29,8 @@
  *
  * Conventions for every call:
  *   - Every array pointer is a CUDA device pointer owned by the caller.  libdamp
- *     never allocates, frees or synchronizes.  Work is enqueued on `stream`
+ *     never allocates or frees, and never synchronizes except in
+ *     damp_device_status (below).  Work is enqueued on `stream`
  *     (a cudaStream_t passed as void*; NULL means the legacy default stream)
  *     and is ordered with the caller's other work on that stream.
  *   - Every argument check runs on the host before anything is enqueued.  A
@@ -349,8 +350,28 @@ DAMP_API damp_status damp_calib_select(const damp_layout *layout, const float *E
                                        const float *G_acc, int64_t n_tokens, float tau, float *C_out,
                                        uint8_t *perm_out, void *stream);
 
+/*
+ * Test hook for the bounded waits (no counterpart in the paper; not part of the decode
+ * path).  Runs the KDA packed step's kernel in a variant whose stage barriers expect 16
+ * bytes more than each record copy delivers, with the wait limit cut to ~1 ms: every
+ * warp's first wait runs out, the kernel settles the missing bytes itself, waits for
+ * its copies in flight to land and returns.  No record and no row of o is written;
+ * DAMP_DEV_WAIT_TIMEOUT is set in the device status word.  It lets a test check the
+ * timeout path without a fault or a hang.  Arguments as damp_kda_decode_step; only the
+ * layout d_k = 128, K_hi = 10, DAMP_LO_U8_AFFINE_G32_H32, BF16 inputs and no head map
+ * (DAMP_ERR_SHAPE otherwise).
+ */
+DAMP_API damp_status damp_test_kda_wait_timeout(const damp_layout *layout, void *state, int64_t num_slots,
+                                                const int32_t *slot_idx, int32_t batch, const uint8_t *perm,
+                                                const void *q, const void *k, const void *v, const float *g,
+                                                const float *beta, float *o, int32_t in_dtype, void *stream);
+
 /* Reads and clears the device status word of the current device (DAMP_DEV_* bits).
- * Synchronous with respect to the device.  DAMP_ERR_NULL if status is NULL. */
+ * It first waits for all work on the current device (cudaDeviceSynchronize: the one
+ * call of libdamp that synchronizes), so every kernel enqueued before the call, on
+ * any stream, has reported before the word is read; a bit is never cleared without
+ * being returned.  DAMP_ERR_NULL if status is NULL; DAMP_ERR_CUDA if the wait or a
+ * copy fails. */
 DAMP_API damp_status damp_device_status(uint32_t *status);
 
 /* Human-readable name of a status code (static string). */

@@ -29,7 +29,7 @@ __all__ = [
     "gdn_decode_step", "kda_decode_step", "gdn_prefill_chunk", "kda_prefill_chunk", "calib_error_energy", "calib_log_decay", "calib_select", "u8_gdn_decode_step", "u8_kda_decode_step",
     "fp32_gdn_decode_step", "fp32_kda_decode_step", "quantize_state", "dequantize_state",
     "pack_tiers", "unpack_tiers", "device_status", "version", "DEV_WAIT_TIMEOUT", "DEV_BAD_SLOT", "DEV_BAD_HEAD",
-    "head_groups",
+    "head_groups", "test_kda_wait_timeout",
 ]
 
 LO_U8_AFFINE_G32_H32 = 0
@@ -134,6 +134,62 @@ def _cuda_contig(name, t):
         raise ValueError(f"{name} must be a contiguous CUDA tensor")
 
 
+def _want(name, t, shape, *, dtype=None, esize=None):
+    """Raise ValueError unless tensor t (if given) has exactly `shape` (and dtype or
+    element size).  The C ABI sees only pointers, so a mis-sized tensor would make a
+    kernel read or write outside it: every size is checked here, before any call."""
+    if t is None:
+        return
+    if tuple(t.shape) != tuple(int(x) for x in shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(int(x) for x in shape)}")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} has dtype {t.dtype}, expected {dtype}")
+    if esize is not None and t.element_size() not in ((esize,) if isinstance(esize, int) else esize):
+        raise ValueError(f"{name} has {t.element_size()}-byte elements, expected {esize}")
+
+
+def _want_pool(layout, state, num_slots, fp32=False):
+    """The packed pool (uint8 [slots, slot_bytes]) or FP32 state (float32 [slots, H, d_k,
+    d_v]) must hold num_slots slots; returns num_slots (default: all of them)."""
+    import torch
+    if state is None:
+        raise ValueError("state is required")
+    if fp32:
+        _want("state", state, (state.shape[0], layout.num_heads, layout.d_k, layout.d_v), dtype=torch.float32)
+    else:
+        if state.dim() != 2:
+            raise ValueError(f"state has shape {tuple(state.shape)}, expected [slots, {slot_bytes(layout)}]")
+        _want("state", state, (state.shape[0], slot_bytes(layout)), dtype=torch.uint8)
+    n = state.shape[0] if num_slots is None else int(num_slots)
+    if n < 0 or n > state.shape[0]:
+        raise ValueError(f"num_slots {n} exceeds the {state.shape[0]} slots of state")
+    return n
+
+
+def _want_batch(slot_idx, B, num_slots):
+    import torch
+    _want("slot_idx", slot_idx, (B,), dtype=torch.int32)
+    if slot_idx is None and B > num_slots:
+        raise ValueError(f"batch {B} exceeds num_slots {num_slots} without slot_idx")
+
+
+def _want_operands(layout, kind, q, k, v, g, beta, o, lead):
+    """q, k [*lead, H_qk, d_k]; v [*lead, H_m, d_v]; g [*lead, H_m] (GDN) or [*lead, H_m,
+    d_k] (KDA); beta [*lead, H_m]; o float32 [*lead, H_m, d_v]."""
+    import torch
+    Hm = layout.heads_of_operands
+    for n, t in (("q", q), ("k", k), ("v", v), ("g", g), ("beta", beta)):
+        if t is None:
+            raise ValueError(f"{n} is required")
+    lead = tuple(lead)
+    _want("q", q, lead + (layout.num_qk_heads, layout.d_k))
+    _want("k", k, lead + (layout.num_qk_heads, layout.d_k))
+    _want("v", v, lead + (Hm, layout.d_v))
+    _want("g", g, lead + ((Hm, layout.d_k) if kind == "kda" else (Hm,)), dtype=torch.float32)
+    _want("beta", beta, lead + (Hm,), dtype=torch.float32)
+    _want("o", o, lead + (Hm, layout.d_v), dtype=torch.float32)
+
+
 def version() -> int:
     return int(lib().damp_version())
 
@@ -169,16 +225,22 @@ def new_fp32_state(layout: Layout, num_slots: int, device="cuda"):
 
 def _step(fn_name, layout, state, perm, q, k, v, g, beta, o, slot_idx, num_slots, stream):
     import torch
+    fp32 = fn_name.startswith("damp_fp32")
+    if v is None or v.dim() < 1:
+        raise ValueError("v must be a [B, H, d_v] tensor")
+    B = v.shape[0]
+    num_slots = _want_pool(layout, state, num_slots, fp32=fp32)
+    _want_batch(slot_idx, B, num_slots)
+    if not fp32:
+        _want("perm", perm, (layout.num_heads, layout.d_k), dtype=torch.uint8)
+    _want_operands(layout, "kda" if "_kda_" in fn_name else "gdn", q, k, v, g, beta, o, (B,))
     for n, t in (("state", state), ("perm", perm), ("q", q), ("k", k), ("v", v), ("g", g), ("beta", beta),
                  ("o", o), ("slot_idx", slot_idx)):
         _cuda_contig(n, t)
-    B = v.shape[0]
     if o is None:
         # a head group writes only its heads' rows: the others start at zero
         alloc = torch.empty if layout.head_map is None else torch.zeros
         o = alloc((B, layout.heads_of_operands, layout.d_v), dtype=torch.float32, device=v.device)
-    if num_slots is None:
-        num_slots = state.shape[0]
     c = layout.c()
     args = [ctypes.byref(c), _ptr(state), num_slots, _ptr(slot_idx), B]
     if perm is not None or not fn_name.startswith("damp_fp32"):
@@ -196,6 +258,15 @@ def gdn_decode_step(layout, state, perm, q, k, v, g, beta, o=None, slot_idx=None
 def kda_decode_step(layout, state, perm, q, k, v, g, beta, o=None, slot_idx=None, num_slots=None, stream=None):
     """One KDA decode step on the packed state (in place); returns o [B, H, d_v] float32."""
     return _step("damp_kda_decode_step", layout, state, perm, q, k, v, g, beta, o, slot_idx, num_slots, stream)
+
+
+def test_kda_wait_timeout(layout, state, perm, q, k, v, g, beta, o=None, slot_idx=None, num_slots=None,
+                          stream=None):
+    """The bounded-wait test hook (damp_test_kda_wait_timeout): every wait of the KDA step's
+    kernel runs out after ~1 ms; nothing is written and the status word reports
+    DEV_WAIT_TIMEOUT.  For tests of the timeout path only."""
+    return _step("damp_test_kda_wait_timeout", layout, state, perm, q, k, v, g, beta, o, slot_idx, num_slots,
+                 stream)
 
 
 def u8_gdn_decode_step(layout, state, perm, q, k, v, g, beta, o=None, slot_idx=None, num_slots=None, stream=None):
@@ -217,14 +288,19 @@ def fp32_kda_decode_step(layout, state, q, k, v, g, beta, o=None, slot_idx=None,
 
 def _prefill(fn_name, layout, state, perm, q, k, v, g, beta, o, lengths, slot_idx, num_slots, stream):
     import torch
+    if v is None or v.dim() < 2:
+        raise ValueError("v must be a [B, T, H, d_v] tensor")
+    B, T = v.shape[0], v.shape[1]
+    num_slots = _want_pool(layout, state, num_slots)
+    _want_batch(slot_idx, B, num_slots)
+    _want("lengths", lengths, (B,), dtype=torch.int32)
+    _want("perm", perm, (layout.num_heads, layout.d_k), dtype=torch.uint8)
+    _want_operands(layout, "kda" if "_kda_" in fn_name else "gdn", q, k, v, g, beta, o, (B, T))
     for n, t in (("state", state), ("perm", perm), ("q", q), ("k", k), ("v", v), ("g", g), ("beta", beta),
                  ("o", o), ("lengths", lengths), ("slot_idx", slot_idx)):
         _cuda_contig(n, t)
-    B, T = v.shape[0], v.shape[1]
     if o is None:
         o = torch.zeros((B, T, layout.heads_of_operands, layout.d_v), dtype=torch.float32, device=v.device)
-    if num_slots is None:
-        num_slots = state.shape[0]
     c = layout.c()
     _check(getattr(lib(), fn_name)(ctypes.byref(c), _ptr(state), num_slots, _ptr(slot_idx), B, T, _ptr(lengths),
                                    _ptr(perm), _ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(beta), _ptr(o),
@@ -249,6 +325,12 @@ def kda_prefill_chunk(layout, state, perm, q, k, v, g, beta, o=None, lengths=Non
 
 def calib_error_energy(layout, S, E_acc, stream=None):
     """E_acc [H, d_k] += per-channel squared low-tier round-trip error of S [B, H, d_k, d_v]."""
+    import torch
+    Hm = layout.heads_of_operands
+    if S is None or S.dim() != 4:
+        raise ValueError("S must be a [B, H, d_k, d_v] tensor")
+    _want("S", S, (S.shape[0], Hm, layout.d_k, layout.d_v), dtype=torch.float32)
+    _want("E_acc", E_acc, (Hm, layout.d_k), dtype=torch.float32)
     _cuda_contig("S", S)
     _cuda_contig("E_acc", E_acc)
     _check(lib().damp_calib_error_energy(ctypes.byref(layout.c()), _ptr(S), S.shape[0], _ptr(E_acc), _stream(stream)),
@@ -258,6 +340,12 @@ def calib_error_energy(layout, S, E_acc, stream=None):
 
 def calib_log_decay(layout, g, G_acc, stream=None):
     """G_acc [H, d_k] += log-decay g summed over the batch (g [B, H] GDN or [B, H, d_k] KDA)."""
+    import torch
+    Hm = layout.heads_of_operands
+    if g is None or g.dim() not in (2, 3):
+        raise ValueError("g must be a [B, H] or [B, H, d_k] tensor")
+    _want("g", g, (g.shape[0], Hm) + ((layout.d_k,) if g.dim() == 3 else ()), dtype=torch.float32)
+    _want("G_acc", G_acc, (Hm, layout.d_k), dtype=torch.float32)
     _cuda_contig("g", g)
     _cuda_contig("G_acc", G_acc)
     _check(lib().damp_calib_log_decay(ctypes.byref(layout.c()), _ptr(g), g.shape[0], 1 if g.dim() == 3 else 0,
@@ -268,6 +356,9 @@ def calib_log_decay(layout, g, G_acc, stream=None):
 def calib_select(layout, E_acc, n_samples, G_acc, n_tokens, tau=1e-4, stream=None):
     """Scores C [H, d_k] float32 and permutations pi [H, d_k] uint8 (Algorithm 1)."""
     import torch
+    Hm = layout.heads_of_operands
+    _want("E_acc", E_acc, (Hm, layout.d_k), dtype=torch.float32)
+    _want("G_acc", G_acc, (Hm, layout.d_k), dtype=torch.float32)
     _cuda_contig("E_acc", E_acc)
     _cuda_contig("G_acc", G_acc)
     C = torch.empty((layout.num_heads, layout.d_k), dtype=torch.float32, device=E_acc.device)
@@ -279,41 +370,69 @@ def calib_select(layout, E_acc, n_samples, G_acc, n_tokens, tau=1e-4, stream=Non
 
 def quantize_state(layout, S, perm, state, slot_idx=None, num_slots=None, stream=None):
     """Write natural-order FP32 states S [B, H, d_k, d_v] into packed slots."""
+    import torch
+    if S is None or S.dim() != 4:
+        raise ValueError("S must be a [B, H, d_k, d_v] tensor")
+    n_slots = _want_pool(layout, state, num_slots)
+    _want_batch(slot_idx, S.shape[0], n_slots)
+    _want("S", S, (S.shape[0], layout.heads_of_operands, layout.d_k, layout.d_v), dtype=torch.float32)
+    _want("perm", perm, (layout.num_heads, layout.d_k), dtype=torch.uint8)
     for n, t in (("S", S), ("perm", perm), ("state", state), ("slot_idx", slot_idx)):
         _cuda_contig(n, t)
     c = layout.c()
-    _check(lib().damp_quantize_state(ctypes.byref(c), _ptr(S), _ptr(perm), _ptr(state),
-                                     state.shape[0] if num_slots is None else num_slots, _ptr(slot_idx),
+    _check(lib().damp_quantize_state(ctypes.byref(c), _ptr(S), _ptr(perm), _ptr(state), n_slots, _ptr(slot_idx),
                                      S.shape[0], _stream(stream)), "damp_quantize_state")
 
 
 def dequantize_state(layout, state, perm, batch=None, S=None, slot_idx=None, num_slots=None, stream=None):
     """Reconstruct natural-order FP32 states [B, H, d_k, d_v] from packed slots."""
     import torch
+    n_slots = _want_pool(layout, state, num_slots)
+    B = (slot_idx.shape[0] if slot_idx is not None else n_slots) if batch is None else int(batch)
+    _want_batch(slot_idx, B, n_slots)
+    _want("S", S, (B, layout.heads_of_operands, layout.d_k, layout.d_v), dtype=torch.float32)
+    _want("perm", perm, (layout.num_heads, layout.d_k), dtype=torch.uint8)
     for n, t in (("S", S), ("perm", perm), ("state", state), ("slot_idx", slot_idx)):
         _cuda_contig(n, t)
-    B = (slot_idx.shape[0] if slot_idx is not None else state.shape[0]) if batch is None else batch
     if S is None:
         S = torch.zeros((B, layout.heads_of_operands, layout.d_k, layout.d_v), dtype=torch.float32, device=state.device)
     c = layout.c()
-    _check(lib().damp_dequantize_state(ctypes.byref(c), _ptr(state),
-                                       state.shape[0] if num_slots is None else num_slots, _ptr(slot_idx), B,
+    _check(lib().damp_dequantize_state(ctypes.byref(c), _ptr(state), n_slots, _ptr(slot_idx), B,
                                        _ptr(perm), _ptr(S), _stream(stream)), "damp_dequantize_state")
     return S
+
+
+def _tier_shapes(layout, B, hi, codes, meta):
+    """(name, tensor, shape, element bytes) of the logical tiers of B slots (damp_pack_tiers)."""
+    H, dk, dv, K, f = layout.num_heads, layout.d_k, layout.d_v, layout.k_hi, layout.lo_format
+    lo = dk - K
+    codes_cols = dv // 2 if f in (LO_U4_AFFINE_G32_H32, LO_U4_AFFINE_G32) else dv
+    if f == LO_S8_ABSMAX_ROW:
+        meta_shape, meta_es = (B, H, lo), 4
+    elif f == LO_FP8_E4M3_G32:
+        meta_shape, meta_es = (B, H, lo, dv // 32), 4
+    else:
+        meta_shape, meta_es = (B, H, lo, dv // 32, 2), 2
+    return [("hi", hi, (B, H, K, dv), 2), ("codes", codes, (B, H, lo, codes_cols), 1),
+            ("meta", meta, meta_shape, meta_es)]
 
 
 def pack_tiers(layout, hi, codes, meta, state, slot_idx=None, num_slots=None, stream=None):
     """Copy logical tiers (hi uint16/fp16 [B,H,K,d_v], codes uint8 [B,H,d_k-K,d_v],
     meta uint16/fp16 [B,H,d_k-K,d_v/32,2]; row-absmax format: codes int8, meta float32
     [B,H,d_k-K]) into packed slots, bit for bit."""
+    B = codes.shape[0] if codes is not None else (hi.shape[0] if hi is not None else 0)
+    n_slots = _want_pool(layout, state, num_slots)
+    _want_batch(slot_idx, B, n_slots)
+    for n, t, shape, es in _tier_shapes(layout, B, hi, codes, meta):
+        _want(n, t, shape, esize=es)
     for n, t in (("hi", hi), ("codes", codes), ("meta", meta), ("state", state), ("slot_idx", slot_idx)):
         _cuda_contig(n, t)
-    B = codes.shape[0] if codes is not None else hi.shape[0]
     c = layout.c()
     _check(lib().damp_pack_tiers(ctypes.byref(c), _ptr(hi if hi is not None and hi.numel() else None),
                                  _ptr(codes if codes is not None and codes.numel() else None),
                                  _ptr(meta if meta is not None and meta.numel() else None), _ptr(state),
-                                 state.shape[0] if num_slots is None else num_slots, _ptr(slot_idx), B,
+                                 n_slots, _ptr(slot_idx), B,
                                  _stream(stream)), "damp_pack_tiers")
 
 
@@ -321,9 +440,11 @@ def unpack_tiers(layout, state, batch=None, slot_idx=None, num_slots=None, strea
     """Logical tiers (hi int16 bits, codes uint8, meta int16 bits; row-absmax format: codes
     int8, meta float32 [B,H,d_k-K]) of `batch` packed slots."""
     import torch
+    n_slots = _want_pool(layout, state, num_slots)
+    B = (slot_idx.shape[0] if slot_idx is not None else n_slots) if batch is None else int(batch)
+    _want_batch(slot_idx, B, n_slots)
     _cuda_contig("state", state)
     _cuda_contig("slot_idx", slot_idx)
-    B = (slot_idx.shape[0] if slot_idx is not None else state.shape[0]) if batch is None else batch
     H, dk, dv, K = layout.num_heads, layout.d_k, layout.d_v, layout.k_hi
     dev = state.device
     hi = torch.empty((B, H, K, dv), dtype=torch.int16, device=dev)
@@ -340,7 +461,7 @@ def unpack_tiers(layout, state, batch=None, slot_idx=None, num_slots=None, strea
         codes = torch.empty((B, H, dk - K, dv), dtype=torch.uint8, device=dev)
         meta = torch.empty((B, H, dk - K, dv // 32, 2), dtype=torch.int16, device=dev)
     c = layout.c()
-    _check(lib().damp_unpack_tiers(ctypes.byref(c), _ptr(state), state.shape[0] if num_slots is None else num_slots,
+    _check(lib().damp_unpack_tiers(ctypes.byref(c), _ptr(state), n_slots,
                                    _ptr(slot_idx), B, _ptr(hi if hi.numel() else None),
                                    _ptr(codes if codes.numel() else None), _ptr(meta if meta.numel() else None),
                                    _stream(stream)), "damp_unpack_tiers")

@@ -37,6 +37,7 @@ SIGNATURES = {
     "damp_bits_per_value": (ctypes.c_double, [_L]),
     "damp_gdn_decode_step": (_status, _STEP),
     "damp_kda_decode_step": (_status, _STEP),
+    "damp_test_kda_wait_timeout": (_status, _STEP),
     "damp_u8_gdn_decode_step": (_status, _STEP),
     "damp_u8_kda_decode_step": (_status, _STEP),
     "damp_fp32_gdn_decode_step": (_status, _FP32_STEP),

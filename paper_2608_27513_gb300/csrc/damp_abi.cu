@@ -72,7 +72,8 @@ damp_status check_pool(const void *state, int64_t num_slots, const int32_t *slot
     return DAMP_OK;
 }
 
-cudaError_t launch_step(const StepArgs &a, bool packed, cudaStream_t s) {
+cudaError_t launch_step(const StepArgs &a, bool packed, cudaStream_t s, bool waittest = false) {
+    if (waittest) return launch_packed_kda_waittest(a, s);
     if (!packed) return launch_fp32_step(a, s);
     if (a.fmt == DAMP_LO_S8_ABSMAX_ROW) {
         if (a.dv > 4 * 32) return launch_rowabs_step(a, s);  // the two-sweep step for d_v > 128
@@ -90,7 +91,7 @@ cudaError_t launch_step(const StepArgs &a, bool packed, cudaStream_t s) {
 damp_status step(const damp_layout *L, void *state, int64_t num_slots, const int32_t *slot_idx, int32_t batch,
                  const uint8_t *perm, const void *q, const void *k, const void *v, const float *g,
                  const float *beta, float *o, int32_t in_dtype, void *stream, bool kda, bool packed,
-                 bool uniform) {
+                 bool uniform, bool waittest = false) {
     damp_status st = check_layout(L);
     if (st != DAMP_OK && packed) return st;
     if (!packed) {  // the FP32 state ignores k_hi and lo_format and holds every model head
@@ -103,6 +104,9 @@ damp_status step(const damp_layout *L, void *state, int64_t num_slots, const int
     }
     if (uniform && L->k_hi != 0) return DAMP_ERR_SHAPE;
     if (in_dtype != DAMP_IN_BF16 && in_dtype != DAMP_IN_FP32) return DAMP_ERR_FORMAT;
+    if (waittest && (L->d_k != 128 || L->k_hi != 10 || L->lo_format != DAMP_LO_U8_AFFINE_G32_H32 ||
+                     in_dtype != DAMP_IN_BF16 || L->head_map))
+        return DAMP_ERR_SHAPE;
     if (batch < 0) return DAMP_ERR_SHAPE;
     if (batch == 0) return DAMP_OK;
     const int64_t sb = packed ? slot_bytes_of(L) : (int64_t)L->num_heads * L->d_k * L->d_v * 4;
@@ -146,7 +150,8 @@ damp_status step(const damp_layout *L, void *state, int64_t num_slots, const int
     a.o = o;
     a.in_bf16 = in_dtype == DAMP_IN_BF16;
     a.kda = kda;
-    return launch_step(a, packed, static_cast<cudaStream_t>(stream)) == cudaSuccess ? DAMP_OK : DAMP_ERR_CUDA;
+    return launch_step(a, packed, static_cast<cudaStream_t>(stream), waittest) == cudaSuccess ? DAMP_OK
+                                                                                           : DAMP_ERR_CUDA;
 }
 
 damp_status prefill(const damp_layout *L, void *state, int64_t num_slots, const int32_t *slot_idx, int32_t batch,
@@ -369,6 +374,14 @@ damp_status damp_kda_decode_step(const damp_layout *layout, void *state, int64_t
                 false);
 }
 
+damp_status damp_test_kda_wait_timeout(const damp_layout *layout, void *state, int64_t num_slots,
+                                       const int32_t *slot_idx, int32_t batch, const uint8_t *perm, const void *q,
+                                       const void *k, const void *v, const float *g, const float *beta, float *o,
+                                       int32_t in_dtype, void *stream) {
+    return step(layout, state, num_slots, slot_idx, batch, perm, q, k, v, g, beta, o, in_dtype, stream, true, true,
+                false, true);
+}
+
 damp_status damp_u8_gdn_decode_step(const damp_layout *layout, void *state, int64_t num_slots,
                                     const int32_t *slot_idx, int32_t batch, const uint8_t *perm, const void *q,
                                     const void *k, const void *v, const float *g, const float *beta, float *o,
@@ -500,6 +513,9 @@ damp_status damp_calib_select(const damp_layout *layout, const float *E_acc, int
 
 damp_status damp_device_status(uint32_t *status) {
     if (!status) return DAMP_ERR_NULL;
+    // Kernels on non-blocking streams do not order with the copies below: wait for
+    // all of them first, so a bit set by a kernel in flight is not cleared unread.
+    if (cudaDeviceSynchronize() != cudaSuccess) return DAMP_ERR_CUDA;
     uint32_t all = 0, bits = 0;
     if (take_status_packed_gdn(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;

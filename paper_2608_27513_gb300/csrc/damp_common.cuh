@@ -88,16 +88,25 @@ __device__ __forceinline__ uint64_t global_timer_ns() {
     return t;
 }
 
-// Bounded wait on an mbarrier phase: gives up after ~2 s (or 2^26 polls) and
-// returns false, so a lost copy ends the kernel with an error flag, not a hang.
-__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
+// Bounded wait on an mbarrier phase: gives up after limit_ns (~2 s by default) or
+// 2^26 polls and returns false, so a lost copy ends the kernel with an error flag,
+// not a hang.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
+                                                  uint64_t limit_ns = 2000000000ull) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = global_timer_ns();
     for (uint32_t it = 0; it < (1u << 26); ++it) {
         if (mbar_try_wait(bar, parity)) return true;
-        if ((it & 255u) == 255u && global_timer_ns() - t0 > 2000000000ull) break;
+        if ((it & 255u) == 255u && global_timer_ns() - t0 > limit_ns) break;
     }
     return false;
+}
+
+// Counts `bytes` of expected transaction bytes of the barrier's current phase as done
+// (without a copy): used only to settle a phase that was armed for more bytes than
+// its copy delivers.
+__device__ __forceinline__ void mbar_complete_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.complete_tx.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
 
 // 1-D bulk copy global -> shared (TMA engine), completion on an mbarrier.

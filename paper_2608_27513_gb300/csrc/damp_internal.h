@@ -50,6 +50,7 @@ struct ConvArgs {
 // Launchers (return the CUDA error of the launch; they perform no host-side argument checks).
 cudaError_t launch_packed_gdn(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_packed_kda(const StepArgs &a, cudaStream_t s);
+cudaError_t launch_packed_kda_waittest(const StepArgs &a, cudaStream_t s);
 // the UINT4 low tiers (formats 3, 4)
 cudaError_t launch_packed_gdn_u4(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_packed_kda_u4(const StepArgs &a, cudaStream_t s);

@@ -100,8 +100,15 @@ __device__ __forceinline__ void advance(Cursor &k, int H, int V) {
 // LT: the low tier's code type -- kLtU8 (formats 0, 1), kLtU4 (formats 3, 4: 32 nibbles
 // in one 16-byte chunk per row, levels 15) or kLtE4M3 (format 5: FP8 codes in the natural
 // domain, one FP32 scale per group).
+// WAITTEST: a test instance, outside the decode dispatch, that exercises the bounded
+// wait: every stage barrier expects kWaitTestExtra bytes more than its copy delivers,
+// so the first wait runs out after kWaitTestNs; the kernel then settles those bytes
+// itself, waits for the copies in flight to land, reports DAMP_DEV_WAIT_TIMEOUT and
+// returns without touching a record or o.
 enum : int { kLtU8 = 0, kLtU4 = 1, kLtE4M3 = 2 };
-template <int RL, int DKC, int KC, bool KDA, bool HAD, bool BF16, bool HMAP, int LT = kLtU8>
+constexpr uint32_t kWaitTestExtra = 16;
+constexpr uint64_t kWaitTestNs = 1000000;  // 1 ms
+template <int RL, int DKC, int KC, bool KDA, bool HAD, bool BF16, bool HMAP, int LT = kLtU8, bool WAITTEST = false>
 __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams p) {
     constexpr int R = RL > 0 ? RL : 1;
     extern __shared__ __align__(128) uint8_t smem[];
@@ -156,7 +163,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
         const bool ok = slot >= 0 && slot < p.num_slots && (!HMAP || model_head(k.h) >= 0);
         const uint32_t st = stage0 + (uint32_t)(s * p.stage_bytes);
         const uint32_t bar = bar0 + 8 * s;
-        mbar_arrive_expect_tx(bar, ok ? (uint32_t)rec_bytes : 0u);
+        mbar_arrive_expect_tx(bar, ok ? (uint32_t)rec_bytes + (WAITTEST ? kWaitTestExtra : 0u) : 0u);
         if (ok) bulk_g2s(st, p.state + slot * p.slot_bytes + (int64_t)(k.h * V + k.c) * rec_bytes, rec_bytes, bar);
     };
 
@@ -214,7 +221,8 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
 
     for (int64_t t = t0; t < t1; ++t, advance(cur, H, V)) {
         const uint32_t st = stage0 + (uint32_t)(s * p.stage_bytes);
-        if (!__all_sync(kFull, mbar_wait_bounded(bar0 + 8 * s, parity))) {
+        if (!__all_sync(kFull, WAITTEST ? mbar_wait_bounded(bar0 + 8 * s, parity, kWaitTestNs)
+                                        : mbar_wait_bounded(bar0 + 8 * s, parity))) {
             timed_out = true;
             t_fail = t;
             break;
@@ -539,6 +547,19 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
         // let the loads already in flight land (each wait bounded) before the CTA's
         // shared memory goes away
         const int64_t last = min(t1 - 1, t_fail + p.nstage - 1);
+        if constexpr (WAITTEST) {
+            // settle the extra bytes of every armed stage, so its phase completes
+            // exactly when its copy has landed
+            if (lane == 0) {
+                for (int64_t tt = t_fail; tt <= last; ++tt) {
+                    const Cursor k = cursor_at(tt, H, V);
+                    const int64_t slot = slot_of(k.b);
+                    if (slot >= 0 && slot < p.num_slots && (!HMAP || model_head(k.h) >= 0))
+                        mbar_complete_tx(bar0 + 8 * (int)((tt - t0) % p.nstage), kWaitTestExtra);
+                }
+            }
+            __syncwarp();
+        }
         for (int64_t tt = t_fail; tt <= last; ++tt) {
             const int64_t idx = tt - t0;
             mbar_wait_bounded(bar0 + 8 * (int)(idx % p.nstage), (uint32_t)((idx / p.nstage) & 1));

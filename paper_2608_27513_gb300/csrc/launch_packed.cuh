@@ -17,7 +17,9 @@ constexpr int kPackedWarps = 8;
 constexpr int kPackedStages = 3;
 
 // LT: the low tier's code type (kLtU8: formats 0, 1; kLtU4: formats 3, 4; kLtE4M3: format 5).
-template <bool KDA, int LT>
+// WAITTEST launches the bounded-wait test instance instead of the decode step (layout
+// d_k = 128, K_hi = 10, format 0, BF16 inputs, no head map only).
+template <bool KDA, int LT, bool WAITTEST = false>
 static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, uint32_t *status) {
     const int V = a.dv / kG;
     const RecGeom rg = rec_geom(a.dk, a.K, a.fmt);
@@ -109,7 +111,11 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
                                    : packed_step_kernel<RL_, 0, -1, KDA, false, false, true, LT>; \
     }
     const int rl = (a.dk - a.K + 31) / 32;
-    if (hmap) {
+    if constexpr (WAITTEST) {
+        if (a.dk != 128 || a.K != 10 || a.fmt != 0 || !a.in_bf16 || hmap) return cudaErrorInvalidValue;
+        kern = packed_step_kernel<4, 128, 10, KDA, true, true, false, kLtU8, true>;
+    }
+    if (!kern && hmap) {
         switch (rl) {
             case 0: DAMP_PICK4_HMAP(0) break;
             case 1: DAMP_PICK4_HMAP(1) break;

@@ -11,7 +11,8 @@ Tolerances (the decode-step contract):
         s32 = (x_max - x_min)/255 lies within TIE_REL of a binary16 rounding
         midpoint or -x_min/s within TIE of a half-integer; then s is within
         one binary16 ulp, z within 1, and every reconstructed level s (q - z)
-        within one quantization step (raw codes shift with z).
+        within one quantization step; where only z moved, the raw codes shift
+        with z and each code's level q - z is within 1 LSB.
 """
 from __future__ import annotations
 
@@ -157,6 +158,13 @@ def compare_tiers(w: wl.Workload, ref, gpu, lo_pre, stats: CodeStats, what=""):
         tie = (frac_s * sp < TIE_REL * np.abs(s32) + 1e-30) | (frac_z < TIE)
         bad = meta_diff & ~tie
         assert not bad.any(), f"{what}: (s, z) differ away from a rounding tie at {np.argwhere(bad)[:5].tolist()}"
+        # A code means the level q - z of its group.  Where only z moved (a tie of
+        # -x_min/s), every raw code of the group shifts with z, and the 1-LSB bound
+        # holds for the level: |(q_gpu - z_gpu) - (q_ref - z_ref)| <= 1.
+        z_only = meta_diff & (s_g == s_r)
+        lvl = np.abs((cg - z_g[..., None]) - (cr - z_r[..., None]))
+        assert np.all(lvl[np.broadcast_to(z_only[..., None], lvl.shape)] <= 1), \
+            f"{what}: a code level differs by more than 1 LSB in a group whose zero point moved"
         # in such a group the reconstructed level s (q - z) moves by at most one step
         rec_r = s_r[..., None] * (cr - z_r[..., None])
         rec_g = s_g[..., None] * (cg - z_g[..., None])

@@ -232,3 +232,18 @@ def test_conversions_reject_bad_arguments(L):
 def test_status_strings(L):
     for s in range(7):
         assert L.damp_status_string(s).decode().startswith("DAMP_")
+
+
+def test_wait_test_hook_accepts_only_its_layout(L):
+    """The bounded-wait test hook runs one kernel instance: any other layout or input
+    type is rejected on the host, before a launch."""
+    fb = FakeBuffers()
+    for kw in (dict(k_hi=16), dict(d_k=64, k_hi=10), dict(lo_format=1, k_hi=10)):
+        c = _layout(**kw).c()
+        assert L.damp_test_kda_wait_timeout(ctypes.byref(c), fb[0], 4, None, 4, fb[1], fb[2], fb[3], fb[4], fb[5],
+                                            fb[6], fb[7], 0, None) == 2
+    c = _layout(k_hi=10).c()
+    assert L.damp_test_kda_wait_timeout(ctypes.byref(c), fb[0], 4, None, 4, fb[1], fb[2], fb[3], fb[4], fb[5],
+                                        fb[6], fb[7], 1, None) == 2  # FP32 inputs
+    assert L.damp_test_kda_wait_timeout(ctypes.byref(c), fb[0], 4, None, 0, fb[1], fb[2], fb[3], fb[4], fb[5],
+                                        fb[6], fb[7], 0, None) == 0  # empty batch: nothing enqueued

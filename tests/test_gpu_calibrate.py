@@ -97,8 +97,8 @@ def test_calibration_run_matches_oracle(kind):
         inputs.append({key: P.to_dev(val, DEV, dt if key in ("q", "k", "v") else None) for key, val in inp.items()})
     L = P.layout_of(w)
     C, perm = calibration.calibrate(L, kind, inputs)
-    E, mean_log_a = runs.calibration_stats(w, n_docs, n_tokens)
-    Cref = E * calibrate.persistence(np.exp(mean_log_a))
+    E, a_eff = runs.calibration_stats(w, n_docs, n_tokens)
+    Cref = E * calibrate.persistence(a_eff)
     C = C.cpu().numpy().astype(np.float64)
     assert np.all(np.abs(C - Cref) <= 2e-2 * Cref + 1e-12), np.max(np.abs(C - Cref) / Cref)
     perm = perm.cpu().numpy()

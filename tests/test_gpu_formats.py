@@ -78,9 +78,20 @@ def test_quantize_and_dequantize_match_oracle(fmt):
 
 @pytest.mark.parametrize("fmt", NEW)
 @pytest.mark.parametrize("kind", ["gdn", "kda"])
-def test_decode_steps_match_oracle(kind, fmt):
-    w = wl.sweep(kind, 10, fmt).replace(batch=2, heads=4, qk_heads=4)
+@pytest.mark.parametrize("K", [10, 16])
+def test_decode_steps_match_oracle(kind, fmt, K):
+    """d_k = 128: K_hi = 10 runs the general instance of the format's step, K_hi = 16
+    its compile-time layout (the instance the K_hi sweep times)."""
+    w = wl.sweep(kind, K, fmt).replace(batch=2, heads=4, qk_heads=4)
     P.run_teacher_forced(w, 3, DEV)
+
+
+@pytest.mark.parametrize("fmt", NEW)
+def test_decode_k16_full_batch_sampled_rows(fmt):
+    """KDA B=256, H=32, d=128, K_hi=16 in the 4-bit and FP8 formats, the whole batch in
+    one launch (compile-time instances), rows 9 and 250 against the oracle."""
+    from tests.test_gpu_fullsize import _fullsize
+    _fullsize(wl.sweep("kda", 16, fmt), [9, 250], 1)
 
 
 @pytest.mark.parametrize("fmt", NEW)

@@ -194,6 +194,26 @@ def test_bad_slot_index_is_skipped_and_reported():
     assert damp.device_status() == 0
 
 
+def test_status_of_a_side_stream_step_is_read_without_a_sync():
+    """device_status() waits for kernels on every stream, including PyTorch's
+    non-blocking side streams: a bad slot reported by a step still in flight there is
+    returned, not cleared unread."""
+    w = wl.KDA_B256.replace(batch=2, heads=2, qk_heads=2)
+    L = P.layout_of(w)
+    state = damp.new_state(L, 2, DEV)
+    perms = P.to_dev(np.tile(np.arange(128, dtype=np.uint8), (2, 1)), DEV)
+    d = P.inputs_to_dev(w, wl.step_inputs(w, 0), DEV)
+    slot_idx = torch.tensor([0, 5], dtype=torch.int32, device=DEV)
+    side = torch.cuda.Stream(device=DEV)
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for _ in range(3):
+            damp.kda_decode_step(L, state, perms, d["q"], d["k"], d["v"], d["g"], d["beta"], slot_idx=slot_idx,
+                                 stream=side)
+    assert damp.device_status() == damp.DEV_BAD_SLOT  # no synchronize before the read
+    assert damp.device_status() == 0
+
+
 def test_empty_batch_is_a_no_op():
     w = wl.KDA_B256.replace(batch=1, heads=2, qk_heads=2)
     L = P.layout_of(w)

@@ -42,14 +42,20 @@ def test_quantizer_invariants(x):
     q, sz, s, z = _params(x)
     # s > 0 always (degenerate blocks widen to 0, an all-zero block takes s = 1), z an integer
     assert s > 0 and np.isfinite(s) and z == np.round(z)
-    # s is the binary16 value nearest (x_max - x_min)/255, or of the widened range
-    for lo, hi in ((mn, mx), (min(mn, 0.0), max(mx, 0.0))):
-        r = (hi - lo) / 255.0
-        if float(np.float16(r)) != 0.0:
-            assert s == float(np.float16(np.float32(r))) or abs(s - r) <= float(np.spacing(np.float16(r)))
-            break
-    else:
+    # s is binary16 round-to-nearest-even of the FP32 range / 255 (Sec. 3.2, App. A.1),
+    # taken over [min, max], or over the range widened to contain 0 only when that
+    # rounds to 0; z is binary16 of rint(-min / s) over the same range
+    f32 = np.float32
+    lo, hi = f32(mn), f32(mx)
+    s_ref = float(np.float16((hi - lo) / f32(255)))
+    if s_ref == 0.0:
+        lo, hi = min(lo, f32(0)), max(hi, f32(0))
+        s_ref = float(np.float16((hi - lo) / f32(255)))
+    if s_ref == 0.0:
         assert s == 1.0 and z == 0.0
+    else:
+        assert s == s_ref, (s, s_ref)
+        assert z == float(np.float16(np.rint(-lo / f32(s)))), z
     # codes: the nearest integer to x/s + z (clamped), except at ties of float64 rounding
     y = x.astype(np.float64) / s + z
     near_tie = np.abs(np.abs(y - np.floor(y)) - 0.5) < 1e-4
