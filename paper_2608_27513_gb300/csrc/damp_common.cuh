@@ -359,6 +359,33 @@ __device__ __forceinline__ void dequantize_group(const uint32_t (&w)[8], uint32_
     }
 }
 
+// Byte b of the word as the binary32 denormal byte * 2^-133 (the byte in bits 16..23,
+// every other bit zero): an exact float that an FMA multiplies without rounding.
+__device__ __forceinline__ float u8_denormal(uint32_t word, int b) {
+    return __uint_as_float(prmt(word, 0u, 0x4044u | ((uint32_t)b << 8)));
+}
+
+// Dequantize 8 code words with one FMA per pair: x_j = q_j (s scale) - z (s scale),
+// with scale94 = scale * 2^133 (the row's decay times 2^94 on the decode path, whose
+// working scale is 2^-39).  The code enters as q_j 2^-133 (u8_denormal) and is
+// multiplied by m = s * scale94 = (s scale) 2^133, so the product q_j (s scale) is
+// exact inside the FMA; the constant c = (-z 2^-133) m = -z (s scale) is rounded once
+// and so is the sum (within one unit in the last place of max(|x_j|, |z s scale|)).
+// Needs m < 2^128: s * scale < 2^-5 (for the decode path, decays below 2^18).
+__device__ __forceinline__ void dequantize_group_fma(const uint32_t (&w)[8], uint32_t sz, float scale94,
+                                                     float2 (&x)[16]) {
+    const float s = __half2float(__ushort_as_half((unsigned short)(sz & 0xffffu)));
+    const float z = __half2float(__ushort_as_half((unsigned short)(sz >> 16)));
+    const float m = s * scale94;
+    const float2 m2 = splat2(m);
+    const float2 c2 = splat2((z * -0x1p-133f) * m);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        x[2 * i] = fma2(make_float2(u8_denormal(w[i], 0), u8_denormal(w[i], 1)), m2, c2);
+        x[2 * i + 1] = fma2(make_float2(u8_denormal(w[i], 2), u8_denormal(w[i], 3)), m2, c2);
+    }
+}
+
 // In-thread H_32 on 16 pairs (component j of the group is y[j/2].x or .y).
 __device__ __forceinline__ void hadamard_pairs(float2 (&y)[16]) {
     float x[32];

@@ -272,7 +272,9 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
                 kk[i] = splat2(kv);
                 qq[i] = splat2(qv);
                 bk[i] = splat2(beta * kv * kDown);  // working scale of the low tier
-                aa[i] = av_at(ch) * kDown;
+                // the decay times the working scale 2^-39; UINT8 rows keep it times 2^133
+                // for dequantize_group_fma
+                aa[i] = av_at(ch) * (LT == kLtU8 ? 0x1p94f : kDown);
                 kq = fmaf(kv, qv, kq);
             }
             // FP16 rows in pairs: {a_u, a_u+1, bk_u, bk_u+1} {k_u, k_u+1, q_u, q_u+1};
@@ -325,7 +327,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
                     const uint4 c1 = lds128(st + codes_off + lo_chunk_off(r, 1, lo));
                     const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
                     if constexpr (F8) dequantize_group_e4m3(w, __uint_as_float(sz), aa[i], x[i]);
-                    else dequantize_group(w, sz, aa[i], x[i]);
+                    else dequantize_group_fma(w, sz, aa[i], x[i]);
                 }
 #pragma unroll
                 for (int j = 0; j < 16; ++j) {

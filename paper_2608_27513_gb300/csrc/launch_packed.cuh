@@ -16,11 +16,14 @@ namespace damp {
 constexpr int kPackedWarps = 8;
 constexpr int kPackedStages = 3;
 
-// LT: the low tier's code type (kLtU8: formats 0, 1; kLtU4: formats 3, 4; kLtE4M3: format 5).
-// WAITTEST launches the bounded-wait test instance instead of the decode step (layout
-// d_k = 128, K_hi = 10, format 0, BF16 inputs, no head map only).
-template <bool KDA, int LT, bool WAITTEST = false>
-static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, uint32_t *status) {
+// Parameters and launch shape of one packed step (no launch).
+struct PackedLaunch {
+    PackedParams p;
+    int warps, grid, smem;
+};
+
+template <bool KDA>
+static cudaError_t packed_launch_shape(const StepArgs &a, uint32_t *status, PackedLaunch *out) {
     const int V = a.dv / kG;
     const RecGeom rg = rec_geom(a.dk, a.K, a.fmt);
     const int esz = a.in_bf16 ? 2 : 4;
@@ -72,7 +75,6 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
     p.warp_smem = p.stage0_off + p.nstage * p.stage_bytes;
     p.total_tiles = (int64_t)a.batch * a.H * V;
     p.status = status;
-    if (p.total_tiles == 0) return cudaSuccess;
 
     // shrink the warp count (then the ring) until the per-CTA shared memory fits
     const int smem_cap = max_smem_per_block();
@@ -84,8 +86,24 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
     }
     if (warps * p.warp_smem > smem_cap) return cudaErrorInvalidConfiguration;
     const int64_t want = (p.total_tiles + warps - 1) / warps;
-    const int grid = (int)std::min<int64_t>(want, (int64_t)sm_count());
-    const int smem = p.warp_smem * warps;
+    out->p = p;
+    out->warps = warps;
+    out->grid = (int)std::min<int64_t>(std::max<int64_t>(want, 1), (int64_t)sm_count());
+    out->smem = p.warp_smem * warps;
+    return cudaSuccess;
+}
+
+// LT: the low tier's code type (kLtU8: formats 0, 1; kLtU4: formats 3, 4; kLtE4M3: format 5).
+// WAITTEST launches the bounded-wait test instance instead of the decode step (layout
+// d_k = 128, K_hi = 10, format 0, BF16 inputs, no head map only).
+template <bool KDA, int LT, bool WAITTEST = false>
+static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, uint32_t *status) {
+    PackedLaunch sh;
+    cudaError_t e0 = packed_launch_shape<KDA>(a, status, &sh);
+    if (e0 != cudaSuccess) return e0;
+    const PackedParams &p = sh.p;
+    if (p.total_tiles == 0) return cudaSuccess;
+    const int warps = sh.warps, grid = sh.grid, smem = sh.smem;
 
     void (*kern)(PackedParams) = nullptr;
     const bool had = fmt_had(a.fmt);
