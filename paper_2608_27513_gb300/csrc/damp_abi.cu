@@ -77,6 +77,9 @@ cudaError_t launch_step(const StepArgs &a, bool packed, cudaStream_t s, bool wai
     if (!packed) return launch_fp32_step(a, s);
     if (a.fmt == DAMP_LO_S8_ABSMAX_ROW) {
         if (a.dv > 4 * 32) return launch_rowabs_step(a, s);  // the two-sweep step for d_v > 128
+        // d_k = d_v = 128: the full-row quad step (four warps share each row's maximum)
+        const cudaError_t eq = a.kda ? launch_quad_rowabs_kda(a, s) : launch_quad_rowabs_gdn(a, s);
+        if (eq != cudaErrorNotSupported) return eq;
         StepArgs one = a;  // otherwise a one-token chunk: four warps share each row's maximum
         one.T = 1;
         one.lengths = nullptr;
@@ -528,6 +531,10 @@ damp_status damp_device_status(uint32_t *status) {
     if (take_status_packed_gdn_f8(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     if (take_status_packed_kda_f8(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_quad_gdn(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_quad_kda(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     if (take_status_fp32(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;

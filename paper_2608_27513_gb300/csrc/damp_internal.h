@@ -57,6 +57,10 @@ cudaError_t launch_packed_kda_u4(const StepArgs &a, cudaStream_t s);
 // the FP8 E4M3 low tier (format 5)
 cudaError_t launch_packed_gdn_f8(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_packed_kda_f8(const StepArgs &a, cudaStream_t s);
+// the row-absmax format (2) at d_k = d_v = 128 with BF16 operands and a compile-time
+// K_hi: the full-row quad step (cudaErrorNotSupported, nothing launched, otherwise)
+cudaError_t launch_quad_rowabs_gdn(const StepArgs &a, cudaStream_t s);
+cudaError_t launch_quad_rowabs_kda(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_fp32_step(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_quantize(const ConvArgs &a, cudaStream_t s);
 cudaError_t launch_dequantize(const ConvArgs &a, cudaStream_t s);
@@ -87,6 +91,8 @@ cudaError_t take_status_packed_gdn_u4(uint32_t *bits);
 cudaError_t take_status_packed_kda_u4(uint32_t *bits);
 cudaError_t take_status_packed_gdn_f8(uint32_t *bits);
 cudaError_t take_status_packed_kda_f8(uint32_t *bits);
+cudaError_t take_status_quad_gdn(uint32_t *bits);
+cudaError_t take_status_quad_kda(uint32_t *bits);
 cudaError_t take_status_fp32(uint32_t *bits);
 cudaError_t take_status_convert(uint32_t *bits);
 cudaError_t take_status_rowabs(uint32_t *bits);

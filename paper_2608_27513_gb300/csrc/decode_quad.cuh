@@ -1,0 +1,497 @@
+// decode_quad.cuh -- fused DAMP decode step with four warps per (slot, head), for
+// d_k = d_v = 128 (qfr_step_kernel).
+//
+// Same update and requantization as packed_step_kernel (Sec. 3.1, Eq. delta_update;
+// Sec. 3.3, Eq. quantized_recurrence; record layout of Sec. 5.2 / App. A.5), but the
+// four value-block records of a (slot, head) unit are updated at the same time by the
+// four warps of a quad (warp c takes value block c):
+//   * the unit's operands (k, q, decay and beta gathered into record row order, v,
+//     k^T q) are copied in by the quad's 128 threads and prepared once per unit into
+//     quad-shared shared memory -- warp c gathers record rows 32c .. 32c+31 -- one unit
+//     ahead, with one named barrier per unit;
+//   * a warp keeps the full-row layout of packed_step_kernel: lane l owns low-tier rows
+//     l, l+32, ... with all 32 columns in registers across the column sums, and three
+//     record copies (one 1-D bulk copy each) in flight;
+//   * the row-absmax format (2), whose row scale spans the head's four value blocks,
+//     combines each row's maximum across the quad through shared memory at a second
+//     barrier, so a step is one pass over the records.
+// Units are split evenly between the quads of the grid (two quads per CTA, one CTA per
+// SM).
+#pragma once
+
+#include "damp_common.cuh"
+
+namespace damp {
+
+struct QuadParams {
+    uint8_t *state;
+    int64_t num_slots;
+    const int32_t *slot_idx;
+    const uint8_t *perm;
+    const void *q, *k, *v;
+    const float *g, *beta;
+    float *o;
+    int32_t batch, H, Hqk;
+    int32_t Hm;                // heads of the operands: held head h is model head head_map[h] (or h)
+    const int32_t *head_map;
+    int64_t slot_bytes;
+    int64_t total_tiles;
+    uint32_t *status;
+};
+
+// Compile-time geometry of the four-warp step (d_k = d_v = 128, V = 4 value blocks).
+template <int KC, bool KDA, bool BF16>
+struct QuadGeom {
+    static constexpr int DK = 128, DV = 128, V = 4;
+    static constexpr int LO = DK - KC;              // low-tier rows
+    static constexpr int KP = (KC + 1) / 2;         // FP16 row pairs
+    static constexpr int CODES = 128 * KP;          // record: FP16 pairs, codes, (s, z)
+    static constexpr int META = CODES + 32 * LO;
+    static constexpr int REC = (META + 4 * LO + 15) & ~15;
+    static constexpr int ESZ = BF16 ? 2 : 4;
+    // raw operands of a unit (cp.async from global): v | q | k | g | beta | perm
+    static constexpr int R_V = 0;
+    static constexpr int R_Q = R_V + DV * ESZ;
+    static constexpr int R_K = R_Q + DK * ESZ;
+    static constexpr int R_G = R_K + DK * ESZ;
+    static constexpr int R_B = R_G + (KDA ? DK * 4 : 16);
+    static constexpr int R_P = R_B + 16;
+    static constexpr int RAW = R_P + DK;
+    static constexpr int N16 = (DV + 2 * DK) * ESZ / 16 + (KDA ? DK * 4 / 16 : 0) + DK / 16;  // 16-B chunks
+    // prepared operands of a unit: low rows {a 2^94, beta k 2^-39, k, q}, FP16 pairs
+    // {a_u, a_u+1, bk_u, bk_u+1, k_u, k_u+1, q_u, q_u+1}, v (FP32), k^T q partials and beta
+    static constexpr int P_ROW = 0;
+    static constexpr int P_HOP = P_ROW + 16 * LO;
+    static constexpr int P_V = P_HOP + 32 * KP;
+    static constexpr int P_MISC = P_V + 4 * DV;
+    static constexpr int PREP = P_MISC + 32;
+    // quad region: two raw buffers, two prepared buffers
+    static constexpr int Q_RAW0 = 0;
+    static constexpr int Q_PREP0 = 2 * RAW;
+    static constexpr int QUAD = (Q_PREP0 + 2 * PREP + 127) & ~127;
+};
+
+__device__ __forceinline__ void quad_sync(int quad) {
+    asm volatile("bar.sync %0, 128;" ::"r"(1 + quad) : "memory");
+}
+
+// model head of held head h: head_map[h] (-1 when out of range), or h
+__device__ __forceinline__ int quad_model_head(const QuadParams &p, int h) {
+    if (!p.head_map) return h;
+    const int m = p.head_map[h];
+    return (m >= 0 && m < p.Hm) ? m : -1;
+}
+
+// ---- per-unit operands of unit u (batch row u / H, head u % H): 16-byte copies by the
+//      quad's 128 threads (qt = thread index in the quad) into the raw buffer dst ----
+template <int KC, bool KDA, bool BF16>
+__device__ __forceinline__ void quad_load_raw(const QuadParams &p, int u, uint32_t dst, int qt) {
+    using G = QuadGeom<KC, KDA, BF16>;
+    constexpr int DK = G::DK, DV = G::DV;
+    const int H = p.H;
+    const int b = u / H, h = u - b * H;
+    const int mh = quad_model_head(p, h);
+    const int m = mh >= 0 ? mh : 0;  // an invalid map entry's unit is skipped; its loads stay in bounds
+    const int64_t bh = (int64_t)b * p.Hm + m;
+    const int hq = (m * p.Hqk) / p.Hm;
+    const uint8_t *vrow = (const uint8_t *)p.v + bh * DV * G::ESZ;
+    const uint8_t *qrow = (const uint8_t *)p.q + ((int64_t)b * p.Hqk + hq) * DK * G::ESZ;
+    const uint8_t *krow = (const uint8_t *)p.k + ((int64_t)b * p.Hqk + hq) * DK * G::ESZ;
+    constexpr int nv = DV * G::ESZ / 16, nqk = DK * G::ESZ / 16, ng = KDA ? DK * 4 / 16 : 0, np = DK / 16;
+    for (int ci = qt; ci < G::N16 + 2; ci += 128) {
+        int j = ci;
+        if (j < nv) {
+            cp_async16(dst + G::R_V + 16 * j, vrow + 16 * j);
+        } else if ((j -= nv) < nqk) {
+            cp_async16(dst + G::R_Q + 16 * j, qrow + 16 * j);
+        } else if ((j -= nqk) < nqk) {
+            cp_async16(dst + G::R_K + 16 * j, krow + 16 * j);
+        } else if ((j -= nqk) < ng) {
+            cp_async16(dst + G::R_G + 16 * j, (const uint8_t *)(p.g + bh * DK) + 16 * j);
+        } else if ((j -= ng) < np) {
+            cp_async16(dst + G::R_P + 16 * j, p.perm + (int64_t)h * DK + 16 * j);
+        } else if ((j -= np) == 0) {
+            cp_async4(dst + G::R_B, p.beta + bh);
+        } else if (!KDA) {
+            cp_async4(dst + G::R_G, p.g + bh);
+        }
+    }
+    cp_async_commit();
+}
+
+// ---- preparation of a unit from its raw buffer rb into the prepared buffer pb:
+//      warp c of the quad gathers record rows 32c .. 32c+31 (row r holds channel perm[r]) ----
+template <int KC, bool KDA, bool BF16>
+__device__ __forceinline__ void quad_prep(uint32_t rb, uint32_t pb, int c, int lane) {
+    using G = QuadGeom<KC, KDA, BF16>;
+    constexpr int DK = G::DK;
+    const int r = 32 * c + lane;
+    const int ch = (int)((lds32(rb + G::R_P + (r & ~3)) >> (8 * (r & 3))) & (DK - 1));
+    const float kv = BF16 ? bf16_at(rb + G::R_K, ch) : ldsf(rb + G::R_K + 4 * ch);
+    const float qv = BF16 ? bf16_at(rb + G::R_Q, ch) : ldsf(rb + G::R_Q + 4 * ch);
+    const float av = expf(ldsf(rb + G::R_G + (KDA ? 4 * ch : 0)));
+    const float beta = ldsf(rb + G::R_B);
+    const float vv = BF16 ? bf16_at(rb + G::R_V, r) : ldsf(rb + G::R_V + 4 * r);
+    sts32(pb + G::P_V + 4 * r, __float_as_uint(vv));
+    if (r < KC) {
+        const uint32_t e = pb + G::P_HOP + 32 * (r >> 1) + 4 * (r & 1);
+        sts32(e, __float_as_uint(av));
+        sts32(e + 8, __float_as_uint(beta * kv));
+        sts32(e + 16, __float_as_uint(kv));
+        sts32(e + 24, __float_as_uint(qv));
+    } else {
+        // the decay times 2^94 (the FMA dequantization at the working scale 2^-39)
+        sts128(pb + G::P_ROW + 16 * (r - KC), make_uint4(__float_as_uint(av * 0x1p94f),
+                                                         __float_as_uint(beta * kv * kDown),
+                                                         __float_as_uint(kv), __float_as_uint(qv)));
+    }
+    float kq = kv * qv;
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) kq += __shfl_xor_sync(kFull, kq, m);
+    if (lane == 0) {
+        sts32(pb + G::P_MISC + 4 * c, __float_as_uint(kq));
+        if (c == 0) sts32(pb + G::P_MISC + 16, __float_as_uint(beta));
+    }
+}
+
+// ===========================================================================
+// Full-row quad step (8 warps, two quads per CTA).  Same quad machinery as
+// quad_step_kernel (units split between quads, operands prepared once per unit
+// and shared, one named barrier per unit), but every warp keeps the full-row layout
+// of packed_step_kernel: lane l owns low-tier rows l, l+32, ... with all 32 columns,
+// holds them in registers across the column sums (no second dequantization), and
+// keeps three record copies in flight.  The row-absmax format (2) uses it because a
+// row's scale spans the head's four value blocks: the quad's warps meet once per unit
+// to combine each row's maximum through shared memory.
+// ===========================================================================
+constexpr int kQfrWarps = 8;
+constexpr int kQfrStages = 3;
+
+template <int KC, bool KDA, bool BF16>
+struct QfrGeom {
+    using Q = QuadGeom<KC, KDA, BF16>;
+    static constexpr int LO = Q::LO, RL = (LO + 31) / 32, KP = Q::KP, REC = Q::REC;
+    static constexpr int STAGE = (REC + 127) & ~127;
+    // quad region: two raw buffers, two prepared buffers, one row-maximum buffer [row][block]
+    static constexpr int Q_AMAX = Q::Q_PREP0 + 2 * Q::PREP;
+    static constexpr int QUAD = (Q_AMAX + 128 * 4 * 4 + 127) & ~127;
+    // warp region: mbarriers, H d vector, column partial sums (column_sum2), record stages
+    static constexpr int W_BAR = 0;
+    static constexpr int W_D = 64;
+    static constexpr int W_PART = 256;
+    static constexpr int W_STAGE = (W_PART + 32 * kPartStride * 4 + 127) & ~127;
+    static constexpr int WARP = W_STAGE + kQfrStages * STAGE;
+    static constexpr int SMEM = (kQfrWarps / 4) * (QUAD + 4 * WARP);
+};
+
+// x_j = u_j m + c for 8 words of codes (u_j: byte j as a denormal, see u8_denormal)
+__device__ __forceinline__ void dequant32_fma(const uint32_t (&w)[8], float m, float c, float2 (&x)[16]) {
+    const float2 m2 = splat2(m), c2 = splat2(c);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        x[2 * i] = fma2(make_float2(u8_denormal(w[i], 0), u8_denormal(w[i], 1)), m2, c2);
+        x[2 * i + 1] = fma2(make_float2(u8_denormal(w[i], 2), u8_denormal(w[i], 3)), m2, c2);
+    }
+}
+
+// max |y_j| over 32 values (three-input max with absolute operands)
+__device__ __forceinline__ float absmax32(const float2 (&y)[16]) {
+    float a[11];
+#pragma unroll
+    for (int i = 0; i < 10; ++i) {
+        const int j0 = 3 * i, j1 = 3 * i + 1, j2 = 3 * i + 2;
+        const float v0 = (j0 & 1) ? y[j0 >> 1].y : y[j0 >> 1].x;
+        const float v1 = (j1 & 1) ? y[j1 >> 1].y : y[j1 >> 1].x;
+        const float v2 = (j2 & 1) ? y[j2 >> 1].y : y[j2 >> 1].x;
+        a[i] = fmax3(fabsf(v0), fabsf(v1), fabsf(v2));
+    }
+    a[10] = fmaxf(fabsf(y[15].x), fabsf(y[15].y));
+    return fmax3(fmax3(fmax3(a[0], a[1], a[2]), fmax3(a[3], a[4], a[5]), fmax3(a[6], a[7], a[8])), a[9], a[10]);
+}
+
+// ROWABS: the row-absmax INT8 low tier (format 2: int8 codes, one FP32 scale per row
+// over all d_v values, stored in every value block's metadata slot; no H_32).
+// Otherwise the UINT8 affine G32 tier (formats 0 with HAD, 1 without).
+template <int KC, bool KDA, bool HAD, bool BF16, bool ROWABS>
+__global__ void __launch_bounds__(32 * kQfrWarps, 1) qfr_step_kernel(const QuadParams p) {
+    using Q = QuadGeom<KC, KDA, BF16>;
+    using G = QfrGeom<KC, KDA, BF16>;
+    constexpr int LO = G::LO, RL = G::RL, KP = G::KP, DK = Q::DK, DV = Q::DV, V = Q::V, NST = kQfrStages;
+    constexpr int NQ = kQfrWarps / 4;
+    static_assert(!(ROWABS && HAD), "the row-absmax format has no block transform");
+    extern __shared__ __align__(128) uint8_t smem[];
+    const int lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5;
+    const int quad = warp >> 2;
+    const int c = warp & 3;
+    const int qt = threadIdx.x & 127;
+    const LaneSigns sg = lane_signs(lane);
+    const uint32_t base = smem_u32(smem) + (uint32_t)(quad * (G::QUAD + 4 * G::WARP));
+    const uint32_t raw0 = base + Q::Q_RAW0;
+    const uint32_t prep0 = base + Q::Q_PREP0;
+    const uint32_t amax = base + G::Q_AMAX;
+    const uint32_t ws = base + G::QUAD + c * G::WARP;
+    const uint32_t bar0 = ws + G::W_BAR;
+    const uint32_t dvec = ws + G::W_D;
+    const uint32_t part = ws + G::W_PART;
+    const uint32_t stage0 = ws + G::W_STAGE;
+
+    // units [u0, u1) of this quad; warp c updates value block c of each
+    const int64_t nq = (int64_t)gridDim.x * NQ;
+    const int64_t qi = (int64_t)blockIdx.x * NQ + quad;
+    const int64_t units = p.total_tiles / V;
+    const int u0 = (int)(units * qi / nq), u1 = (int)(units * (qi + 1) / nq);
+    if (u0 >= u1) return;  // the whole quad
+    const int H = p.H;
+
+    if (lane == 0) {
+#pragma unroll
+        for (int s = 0; s < NST; ++s) mbar_init(bar0 + 8 * s, 1);
+        fence_mbar_init();
+    }
+    if constexpr (KP > 0) {
+        for (int i = qt; i < 4 * KP; i += 128)
+            sts128(prep0 + (uint32_t)((i / (2 * KP)) * Q::PREP + Q::P_HOP + 16 * (i % (2 * KP))), make_uint4(0u, 0u, 0u, 0u));
+    }
+    __syncwarp();
+
+    auto load_raw = [&](int u, uint32_t dst) { quad_load_raw<KC, KDA, BF16>(p, u, dst, qt); };
+    auto prep = [&](uint32_t rb, uint32_t pb) { quad_prep<KC, KDA, BF16>(rb, pb, c, lane); };
+    auto slot_of = [&](int u) -> int64_t {
+        const int b = u / H;
+        return p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b;
+    };
+    // lane 0: the record of (unit u, block c) into stage s
+    auto issue = [&](int u, int s) {
+        const int64_t slot = slot_of(u);
+        const int h = u - (u / H) * H;
+        const bool ok = slot >= 0 && slot < p.num_slots && quad_model_head(p, h) >= 0;
+        const uint32_t bar = bar0 + 8 * s;
+        mbar_arrive_expect_tx(bar, ok ? (uint32_t)Q::REC : 0u);
+        if (ok) bulk_g2s(stage0 + s * G::STAGE, p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * Q::REC, Q::REC, bar);
+    };
+
+    load_raw(u0, raw0);
+    if (u0 + 1 < u1) load_raw(u0 + 1, raw0 + Q::RAW);
+    if (lane == 0) {
+        for (int s = 0; s < NST && u0 + s < u1; ++s) issue(u0 + s, s);
+    }
+    bool dead = false, bad_slot = false, bad_head = false;
+    int k_fail = 0;
+    cp_async_wait_all();
+    quad_sync(quad);
+    prep(raw0, prep0);
+
+    int s = 0;
+    uint32_t parity = 0;
+    for (int u = u0; u < u1; ++u) {
+        const int k = u - u0;
+        const int j = k & 1;
+        const uint32_t pb = prep0 + (uint32_t)(j * Q::PREP);
+        cp_async_wait_all();
+        quad_sync(quad);
+        if (u + 2 < u1) load_raw(u + 2, raw0 + (uint32_t)(j * Q::RAW));
+        const uint32_t st = stage0 + (uint32_t)(s * G::STAGE);
+        if (!dead && !__all_sync(kFull, mbar_wait_bounded(bar0 + 8 * s, parity))) {
+            dead = true;
+            k_fail = k;
+        }
+        const int b = u / H, h = u - b * H;
+        const int64_t slot = p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b;
+        const int mh = quad_model_head(p, h);
+        const bool slot_ok = slot >= 0 && slot < p.num_slots;
+        const bool ok = slot_ok && mh >= 0;  // the same for the quad's four warps
+        bad_slot |= !slot_ok;
+        bad_head |= mh < 0;
+        if (ok) {
+            uint8_t *const grec = p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * Q::REC;
+            float2 x[RL > 0 ? RL : 1][16];
+            float2 bk[RL > 0 ? RL : 1];
+            float dj = 0.f;
+            if (!dead) {
+                const float vj = ldsf(pb + Q::P_V + 4 * (32 * c + lane));
+                const float vt = HAD ? hadamard_lanes(vj, sg) : vj;  // H v
+                // ---- phase 1, low tier: reconstruct and decay (scaled by 2^-39), partial
+                //      r~ = S~_bar^T k and p~ = S~_bar^T q over this lane's rows ----
+                float2 acc[16], accp[16];
+#pragma unroll
+                for (int i = 0; i < RL; ++i) {
+                    const int r = lane + 32 * i;
+                    const bool live = (i < RL - 1) || (r < LO);
+                    const int rc = min(r, LO - 1);
+                    const uint4 op = lds128(pb + Q::P_ROW + 16 * rc);
+                    const float2 kk = splat2(live ? __uint_as_float(op.z) : 0.f);
+                    const float2 qq = splat2(live ? __uint_as_float(op.w) : 0.f);
+                    bk[i] = splat2(__uint_as_float(op.y));
+                    const uint4 c0 = lds128(st + Q::CODES + 16 * rc);
+                    const uint4 c1 = lds128(st + Q::CODES + 16 * (LO + rc));
+                    const uint32_t mw = lds32(st + Q::META + 4 * rc);
+                    if constexpr (ROWABS) {
+                        // int8 codes q: u = q + 128 (bit 7 flipped); x = (u - 128) s a, exact
+                        // constant 128 m (a power of two times m)
+                        const uint32_t w[8] = {c0.x ^ 0x80808080u, c0.y ^ 0x80808080u, c0.z ^ 0x80808080u,
+                                               c0.w ^ 0x80808080u, c1.x ^ 0x80808080u, c1.y ^ 0x80808080u,
+                                               c1.z ^ 0x80808080u, c1.w ^ 0x80808080u};
+                        const float m = __uint_as_float(mw) * __uint_as_float(op.x);
+                        dequant32_fma(w, m, m * -0x1p-126f, x[i]);
+                    } else {
+                        const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+                        dequantize_group_fma(w, mw, __uint_as_float(op.x), x[i]);
+                    }
+#pragma unroll
+                    for (int m = 0; m < 16; ++m) {
+                        acc[m] = (i == 0) ? mul2(x[i][m], kk) : fma2(x[i][m], kk, acc[m]);
+                        accp[m] = (i == 0) ? mul2(x[i][m], qq) : fma2(x[i][m], qq, accp[m]);
+                    }
+                }
+                if (RL == 0) {
+#pragma unroll
+                    for (int m = 0; m < 16; ++m) acc[m] = accp[m] = make_float2(0.f, 0.f);
+                }
+                // ---- phase 1, FP16 tier (lane = column) ----
+                float2 rh[4], ph[4];
+#pragma unroll
+                for (int m = 0; m < 4; ++m) rh[m] = ph[m] = make_float2(0.f, 0.f);
+#pragma unroll
+                for (int pi = 0; pi < KP; ++pi) {
+                    const uint4 oa = lds128(pb + Q::P_HOP + 32 * pi);
+                    const uint4 okq = lds128(pb + Q::P_HOP + 32 * pi + 16);
+                    const float2 xa = mul2(h2_to_f2(lds32(st + 128 * pi + 4 * lane)),
+                                           make_float2(__uint_as_float(oa.x), __uint_as_float(oa.y)));
+                    rh[pi & 3] = fma2(xa, make_float2(__uint_as_float(okq.x), __uint_as_float(okq.y)), rh[pi & 3]);
+                    ph[pi & 3] = fma2(xa, make_float2(__uint_as_float(okq.z), __uint_as_float(okq.w)), ph[pi & 3]);
+                }
+                rh[0] = add2(add2(rh[0], rh[1]), add2(rh[2], rh[3]));
+                ph[0] = add2(add2(ph[0], ph[1]), add2(ph[2], ph[3]));
+                const float rhi = rh[0].x + rh[0].y, phi = ph[0].x + ph[0].y;
+                const float hr_hi = (HAD && KC > 0) ? hadamard_lanes(rhi, sg) : 0.f;
+                const float2 lo_sums = column_sum2(acc, accp, part, lane);
+                const float rlo = lo_sums.x * kUp, plo = lo_sums.y * kUp;  // back from the working scale
+                const uint4 mk = lds128(pb + Q::P_MISC);
+                const float kq = (__uint_as_float(mk.x) + __uint_as_float(mk.y)) +
+                                 (__uint_as_float(mk.z) + __uint_as_float(mk.w));
+                const float bkq = ldsf(pb + Q::P_MISC + 16) * kq;  // beta k^T q
+                // H d = H v - r~_lo - H r_hi out first; d and o in the natural domain
+                const float dt = HAD ? vt - (rlo + hr_hi) : vj - (rlo + rhi);
+                sts32(dvec + 4 * lane, __float_as_uint(dt));
+                __syncwarp();
+                float2 d[16];
+#pragma unroll
+                for (int m = 0; m < 8; ++m) {
+                    const uint4 w = lds128(dvec + 16 * m);
+                    d[2 * m] = make_float2(__uint_as_float(w.x), __uint_as_float(w.y));
+                    d[2 * m + 1] = make_float2(__uint_as_float(w.z), __uint_as_float(w.w));
+                }
+#pragma unroll
+                for (int i = 0; i < RL; ++i) {
+#pragma unroll
+                    for (int m = 0; m < 16; ++m) x[i][m] = fma2(bk[i], d[m], x[i][m]);
+                }
+                float pj;
+                if (HAD) {
+                    dj = vj - (hadamard_lanes(rlo, sg) + rhi);
+                    pj = hadamard_lanes(plo, sg) + phi;
+                } else {
+                    dj = vj - (rlo + rhi);
+                    pj = plo + phi;
+                }
+                p.o[((int64_t)b * p.Hm + mh) * DV + c * kG + lane] = fmaf(bkq, dj, pj);
+            }
+
+            // ---- phase 2, low tier: requantize in place ----
+            if constexpr (ROWABS) {
+                // each row's maximum over the head's four value blocks ([row][block] floats)
+                if (!dead) {
+#pragma unroll
+                    for (int i = 0; i < RL; ++i)
+                        sts32(amax + (uint32_t)(16 * (lane + 32 * i) + 4 * c), __float_as_uint(absmax32(x[i])));
+                }
+                quad_sync(quad);
+                if (!dead) {
+#pragma unroll
+                    for (int i = 0; i < RL; ++i) {
+                        const int r = lane + 32 * i;
+                        const uint4 a4 = lds128(amax + (uint32_t)(16 * r));
+                        const float am = fmaxf(fmaxf(__uint_as_float(a4.x), __uint_as_float(a4.y)),
+                                               fmaxf(__uint_as_float(a4.z), __uint_as_float(a4.w)));
+                        // s = max|x| / 127 over the whole row (IEEE division); codes sat(rne(x / s))
+                        // taken as x (1/s) + 128 on the denormal grid, moved back to int8
+                        const float sc = __fdiv_rn(am * kUp, 127.0f);
+                        const float inv = sc > 0.0f ? __frcp_rn(sc) : 0.0f;
+                        const float2 inv2 = splat2(inv * 0x1p-110f), zc2 = splat2(128.0f * 0x1p-149f);
+                        uint32_t w[8];
+#pragma unroll
+                        for (int m = 0; m < 8; ++m) w[m] = encode4(x[i][2 * m], x[i][2 * m + 1], inv2, zc2) ^ 0x80808080u;
+                        if ((i < RL - 1) || (r < LO)) {
+                            stg128(grec + Q::CODES + 16 * r, make_uint4(w[0], w[1], w[2], w[3]));
+                            stg128(grec + Q::CODES + 16 * (LO + r), make_uint4(w[4], w[5], w[6], w[7]));
+                            stg32(grec + Q::META + 4 * r, __float_as_uint(sc));
+                        }
+                    }
+                }
+            } else if (!dead) {
+                float mn[RL > 0 ? RL : 1], mx[RL > 0 ? RL : 1], sc[RL > 0 ? RL : 1];
+                bool any_zero = false;
+#pragma unroll
+                for (int i = 0; i < RL; ++i) {
+                    minmax32(x[i], mn[i], mx[i]);
+                    sc[i] = scale_of(mn[i], mx[i]);
+                    any_zero |= sc[i] == 0.0f;
+                }
+                const bool fix = __any_sync(kFull, any_zero);  // a block whose scale rounds to 0 (rare)
+#pragma unroll
+                for (int i = 0; i < RL; ++i) {
+                    const int r = lane + 32 * i;
+                    float inv, zq;
+                    const uint32_t szw = fix ? affine_params_scaled(mn[i], mx[i], inv, zq)
+                                             : affine_finish(sc[i], mn[i], inv, zq);
+                    const float2 inv2 = splat2(inv * 0x1p-110f), zc2 = splat2(zq * 0x1p-149f);
+                    uint32_t w[8];
+#pragma unroll
+                    for (int m = 0; m < 8; ++m) w[m] = encode4(x[i][2 * m], x[i][2 * m + 1], inv2, zc2);
+                    if ((i < RL - 1) || (r < LO)) {
+                        stg128(grec + Q::CODES + 16 * r, make_uint4(w[0], w[1], w[2], w[3]));
+                        stg128(grec + Q::CODES + 16 * (LO + r), make_uint4(w[4], w[5], w[6], w[7]));
+                        stg32(grec + Q::META + 4 * r, szw);
+                    }
+                }
+            }
+            // ---- phase 2, FP16 tier: S = S_bar + beta k d, FP16 store (two rows per word) ----
+            if (!dead) {
+                const float2 dj2 = splat2(dj);
+#pragma unroll
+                for (int pi = 0; pi < KP; ++pi) {
+                    const uint4 oa = lds128(pb + Q::P_HOP + 32 * pi);
+                    const float2 xa = mul2(h2_to_f2(lds32(st + 128 * pi + 4 * lane)),
+                                           make_float2(__uint_as_float(oa.x), __uint_as_float(oa.y)));
+                    const float2 y = fma2(make_float2(__uint_as_float(oa.z), __uint_as_float(oa.w)), dj2, xa);
+                    stg32(grec + 128 * pi + 4 * lane, f2_to_h2(y.x, y.y));
+                }
+            }
+        }
+        // the stage has been read: refill it with this warp's tile NST units ahead
+        if (!dead) {
+            __syncwarp();
+            if (lane == 0 && u + NST < u1) {
+                fence_proxy_async_smem();
+                issue(u + NST, s);
+            }
+            if (++s == NST) {
+                s = 0;
+                parity ^= 1u;
+            }
+        }
+        if (u + 1 < u1) prep(raw0 + (uint32_t)((j ^ 1) * Q::RAW), prep0 + (uint32_t)((j ^ 1) * Q::PREP));
+    }
+    if (dead) {
+        // copies that may still land (tiles k_fail .. k_fail + NST - 1), each wait bounded
+        for (int kt = k_fail; kt < min(k_fail + NST, u1 - u0); ++kt)
+            mbar_wait_bounded(bar0 + 8 * (kt % NST), (uint32_t)((kt / NST) & 1));
+    }
+    cp_async_wait_all();
+    if (lane == 0) {
+        const uint32_t bits = (dead ? kDevWaitTimeout : 0u) | (bad_slot ? kDevBadSlot : 0u) | (bad_head ? kDevBadHead : 0u);
+        if (bits) atomicOr(p.status, bits);
+    }
+}
+}  // namespace damp

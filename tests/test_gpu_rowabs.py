@@ -128,3 +128,12 @@ def test_row_absmax_small_heads(dk, dv, K):
     """One or two value blocks per head: three or two warps of each group only meet."""
     w = wl.Workload("t", "gdn", 3, 4, 4, dk, dv, K, 1, 1, "fp32", 18, S8)
     P.run_teacher_forced(w, 2, DEV)
+
+
+@pytest.mark.parametrize("kind,K", [("kda", 10), ("gdn", 16)])
+def test_row_absmax_full_batch_sampled_rows(kind, K):
+    """B=256, H=32, d=128, BF16 (the four-warp row-absmax step at a compile-time K_hi):
+    rows 0, 77, 255 against the oracle over two steps."""
+    from tests.test_gpu_fullsize import _fullsize
+    w = (wl.KDA_B256 if kind == "kda" else wl.sweep("gdn", K)).replace(lo_format=S8)
+    _fullsize(w, [0, 77, 255], 2)
