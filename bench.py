@@ -197,7 +197,22 @@ def make_line(r: dict, steps: int, warmup: int, world: int) -> dict:
                               "bytes_per_step": bytes_fp32,
                               "speedup_of_packed": r["fp32_launch_ms"] / r["launch_ms"]},
         "device": r.get("dev_name"),
+        "other_kernels": _side_lines(r.get("side"), peak_gbs, peak_note),
     }
+
+
+def _side_lines(side, peak_gbs, peak_note):
+    """The GDN and row-absmax figures of the same run, each against the same peak."""
+    if not side:
+        return None
+    out = {}
+    for k, v in side.items():
+        v = dict(v)
+        v["frac"] = v["achieved_gbs"] / peak_gbs
+        v["frac_of_8TBs"] = v["achieved_gbs"] / 8000.0
+        v["peak_source"] = f"{peak_note} copy bandwidth"
+        out[k] = v
+    return out
 
 
 def workload_config(w: wl.Workload, bits=None) -> dict:
@@ -395,11 +410,61 @@ def gpu_arm(args, rank: int, world: int):
     if world > 1:
         dist.barrier()
     e2e_total = max_over_ranks_(e0.elapsed_time(e1))
+
+    # ---- the other kernels the target names, timed the same way on this GPU: GDN B=256
+    # K_hi=16 (packed and FP32-state steps) and the row-absmax format on the KDA workload ----
+    def side_kernel(ws: wl.Workload, with_fp32: bool):
+        Lw = damp.Layout(ws.heads, ws.qk_heads, ws.d_k, ws.d_v, ws.k_hi, ws.lo_format)
+        pin = wl.torch_step_inputs(ws, 16, dev, seed_offset=2000 + rank)
+        Sw = damp.new_fp32_state(Lw, ws.batch, dev)
+        fstep = damp.fp32_kda_decode_step if ws.kind == "kda" else damp.fp32_gdn_decode_step
+        pstep = damp.kda_decode_step if ws.kind == "kda" else damp.gdn_decode_step
+        for t in range(ws.prefix):
+            d = pin[t % len(pin)]
+            fstep(Lw, Sw, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o)
+        pw = torch.from_numpy(wl.random_perm(ws)).to(dev)
+        wpools = [damp.new_state(Lw, ws.batch, dev) for _ in range(POOLS)]
+        for p_ in wpools:
+            damp.quantize_state(Lw, Sw, pw, p_)
+        win = wl.torch_step_inputs(ws, N_INPUT_SETS, dev, seed_offset=3000 + rank)
+        wfp = [Sw] + [Sw.clone() for _ in range(POOLS - 1)] if with_fp32 else None
+        torch.cuda.synchronize()
+
+        def run_p(i, o_buf):
+            d = win[i % N_INPUT_SETS]
+            pstep(Lw, wpools[i % POOLS], pw, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o_buf)
+
+        def run_f(i, o_buf):
+            d = win[i % N_INPUT_SETS]
+            fstep(Lw, wfp[i % POOLS], d["q"], d["k"], d["v"], d["g"], d["beta"], o=o_buf)
+
+        res = {"workload": ws.name, "lo_format": ws.lo_format, "bits_per_value": damp.bits_per_value(Lw)}
+        with ClockSampler(dev.index) as clk2:
+            _, lp = timed(run_p, args.steps, max(args.warmup, 3))
+            lp = max_over_ranks_(lp)
+            bytes_w = algorithmic_bytes(ws)
+            res.update({"us_per_step": lp * 1e3, "bytes_per_step": bytes_w,
+                        "achieved_gbs": bytes_w / (lp * 1e-3) / 1e9})
+            if with_fp32:
+                _, lf = timed(run_f, max(args.steps // 4, 10), max(args.warmup, 3))
+                lf = max_over_ranks_(lf)
+                bf = algorithmic_bytes(ws, packed=False)
+                res["fp32_state_kernel"] = {"us_per_step": lf * 1e3, "bytes_per_step": bf,
+                                            "achieved_gbs": bf / (lf * 1e-3) / 1e9, "speedup_of_packed": lf / lp}
+        res["clocks"] = clk2.summary()
+        if damp.device_status() != 0:
+            raise RuntimeError(f"device status word set during the {ws.name} run")
+        del wpools, wfp, Sw
+        torch.cuda.empty_cache()
+        return res
+
+    side = {"gdn_b256_k16": side_kernel(wl.sweep("gdn", 16), True),
+            "kda_b256_k10_row_absmax": side_kernel(w.replace(lo_format=2, name=w.name + "_f2"), False)}
     return {
         "w": w, "total_ms": total_ms, "launch_ms": launch_ms, "fp32_launch_ms": fp_launch, "graph_ms": graph_ms,
         "reps_ms": reps,
         "e2e_ms": e2e_total / e2e_steps, "h2d": h2d, "d2h": d2h, "clocks": clk.summary(),
-        "bits": damp.bits_per_value(L), "dev_name": torch.cuda.get_device_name(dev),
+        "bits": damp.bits_per_value(L), "dev_name": torch.cuda.get_device_name(dev), "side": side,
     }
 
 
