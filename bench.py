@@ -961,8 +961,19 @@ def tiered_arm(steps: int = 512, every: int = 64, batch: int = 64, timing_steps:
         for (L, hs, pi), pl in zip(tiered, pt[i % 2]):
             damp.gdn_decode_step(L, pl, pi, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o2)
 
+    def one_launch(setup):
+        pools2 = [[damp.new_state(L, 256, dev) for L, _, _ in setup] for _ in range(2)]
+
+        def run(i):
+            d = inputs[i % 4]
+            damp.gdn_decode_step_groups([(L, pl, pi) for (L, _, pi), pl in zip(setup, pools2[i % 2])],
+                                        d["q"], d["k"], d["v"], d["g"], d["beta"], o=o2)
+        return run
+
     timing = {}
-    for name, fn in (("common_k16_one_launch", common), ("tiered_4_28_two_launches", groups)):
+    for name, fn in (("common_k16_one_launch", common), ("tiered_4_28_two_launches", groups),
+                     ("tiered_12_20_one_launch", one_launch(setups[1])), ("tiered_8_24_one_launch", one_launch(setups[2])),
+                     ("tiered_4_28_one_launch", one_launch(setups[3]))):
         for i in range(20):
             fn(i)
         torch.cuda.synchronize()

@@ -121,8 +121,9 @@ typedef enum { DAMP_IN_BF16 = 0, DAMP_IN_FP32 = 1 } damp_in_dtype;
  * Head groups.  A layer whose heads protect different numbers of key channels (the
  * decay-tiered allocation of App. E: fast- and slow-decay heads with different K_hi)
  * is a set of layouts, one per K_hi, whose head maps partition 0 .. H_m-1; each group
- * has its own pool and permutation table, and one call per group updates the layer
- * (the groups write disjoint rows of o).  A head_map entry outside 0 .. H_m-1 sets
+ * has its own pool and permutation table, and one call per group -- or one
+ * damp_*_decode_step_groups call for all groups -- updates the layer (the groups write
+ * disjoint rows of o).  A head_map entry outside 0 .. H_m-1 sets
  * DAMP_DEV_BAD_HEAD in the device status word and that head is skipped.
  */
 typedef struct {
@@ -206,6 +207,38 @@ DAMP_API damp_status damp_kda_decode_step(const damp_layout *layout, void *state
                                  const int32_t *slot_idx, int32_t batch, const uint8_t *perm,
                                  const void *q, const void *k, const void *v, const float *g,
                                  const float *beta, float *o, int32_t in_dtype, void *stream);
+
+/*
+ * One decode step of a layer stored as head groups (App. E, "Common Per-Head Budget for
+ * GDN": per-head protected-channel counts as budget-specific kernel groups; the
+ * decay-tiered allocations of Tab. gdn_head_budget give half the heads K_fast and half
+ * K_slow channels).  Group i is layouts[i] with its own pool states[i] (num_slots[i]
+ * slots) and permutation table perms[i] (uint8 [layouts[i].num_heads][d_k]); every
+ * group has a head map, and the head maps must partition 0 .. model_heads - 1 (not
+ * checked on the device).  The operands q, k, v, g, beta, o, slot_idx, batch and
+ * in_dtype are shared by the groups, with the shapes and alignment of
+ * damp_gdn_decode_step (indexed by model head).
+ *   n_groups   1 .. 8; all groups have the same model_heads, num_qk_heads, d_k, d_v
+ *              (DAMP_ERR_SHAPE otherwise) and lo_format (DAMP_ERR_FORMAT otherwise);
+ *              pools must not overlap each other, the operands or o (DAMP_ERR_ALIAS).
+ * Two groups with d_k = 128, BF16 operands, lo_format 0 or 1 and K_hi pairs 12/20,
+ * 8/24 or 4/28 run as one launch whose CTAs are split between the groups in proportion
+ * to their records; other groups run one launch per group.  Results are the same as
+ * one damp_gdn_decode_step call per group.  Every argument check runs before anything
+ * is enqueued.
+ */
+DAMP_API damp_status damp_gdn_decode_step_groups(const damp_layout *layouts, int32_t n_groups, void *const *states,
+                                                 const int64_t *num_slots, const uint8_t *const *perms,
+                                                 const int32_t *slot_idx, int32_t batch, const void *q,
+                                                 const void *k, const void *v, const float *g, const float *beta,
+                                                 float *o, int32_t in_dtype, void *stream);
+/* The KDA step of a layer stored as head groups: as damp_gdn_decode_step_groups, with the
+ * KDA operands of damp_kda_decode_step. */
+DAMP_API damp_status damp_kda_decode_step_groups(const damp_layout *layouts, int32_t n_groups, void *const *states,
+                                                 const int64_t *num_slots, const uint8_t *const *perms,
+                                                 const int32_t *slot_idx, int32_t batch, const void *q,
+                                                 const void *k, const void *v, const float *g, const float *beta,
+                                                 float *o, int32_t in_dtype, void *stream);
 
 /*
  * Uniform-INT8 baselines (the paper's INT8 / INT8+Hadamard rows of Tab. main):

@@ -29,7 +29,7 @@ __all__ = [
     "gdn_decode_step", "kda_decode_step", "gdn_prefill_chunk", "kda_prefill_chunk", "calib_error_energy", "calib_log_decay", "calib_select", "u8_gdn_decode_step", "u8_kda_decode_step",
     "fp32_gdn_decode_step", "fp32_kda_decode_step", "quantize_state", "dequantize_state",
     "pack_tiers", "unpack_tiers", "device_status", "version", "DEV_WAIT_TIMEOUT", "DEV_BAD_SLOT", "DEV_BAD_HEAD",
-    "head_groups", "test_kda_wait_timeout",
+    "head_groups", "test_kda_wait_timeout", "gdn_decode_step_groups", "kda_decode_step_groups",
 ]
 
 LO_U8_AFFINE_G32_H32 = 0
@@ -258,6 +258,53 @@ def gdn_decode_step(layout, state, perm, q, k, v, g, beta, o=None, slot_idx=None
 def kda_decode_step(layout, state, perm, q, k, v, g, beta, o=None, slot_idx=None, num_slots=None, stream=None):
     """One KDA decode step on the packed state (in place); returns o [B, H, d_v] float32."""
     return _step("damp_kda_decode_step", layout, state, perm, q, k, v, g, beta, o, slot_idx, num_slots, stream)
+
+
+def _step_groups(fn_name, groups, q, k, v, g, beta, o, slot_idx, stream):
+    """groups: [(layout, state, perm)] of one layer (head_groups layouts)."""
+    import torch
+    n = len(groups)
+    if n < 1:
+        raise ValueError("at least one head group is required")
+    if v is None or v.dim() < 1:
+        raise ValueError("v must be a [B, H_m, d_v] tensor")
+    B = v.shape[0]
+    kind = "kda" if "_kda_" in fn_name else "gdn"
+    layouts = (DampLayout * n)()
+    states = (ctypes.c_void_p * n)()
+    perms = (ctypes.c_void_p * n)()
+    slots = (ctypes.c_int64 * n)()
+    for i, (layout, state, perm) in enumerate(groups):
+        if layout.head_map is None:
+            raise ValueError(f"group {i} has no head map (build the groups with head_groups)")
+        ns = _want_pool(layout, state, None)
+        _want_batch(slot_idx, B, ns)
+        _want("perm", perm, (layout.num_heads, layout.d_k), dtype=torch.uint8)
+        _want_operands(layout, kind, q, k, v, g, beta, o, (B,))
+        _cuda_contig("state", state)
+        _cuda_contig("perm", perm)
+        layouts[i] = layout.c()
+        states[i] = state.data_ptr()
+        perms[i] = perm.data_ptr()
+        slots[i] = ns
+    for nm, t in (("q", q), ("k", k), ("v", v), ("g", g), ("beta", beta), ("o", o), ("slot_idx", slot_idx)):
+        _cuda_contig(nm, t)
+    if o is None:
+        o = torch.empty((B, groups[0][0].heads_of_operands, groups[0][0].d_v), dtype=torch.float32, device=v.device)
+    _check(getattr(lib(), fn_name)(layouts, n, states, slots, perms, _ptr(slot_idx), B, _ptr(q), _ptr(k), _ptr(v),
+                                   _ptr(g), _ptr(beta), _ptr(o), _in_dtype(q, k, v), _stream(stream)), fn_name)
+    return o
+
+
+def gdn_decode_step_groups(groups, q, k, v, g, beta, o=None, slot_idx=None, stream=None):
+    """One GDN decode step of a layer stored as head groups, groups = [(layout, state, perm)]
+    (one launch for two groups with a compile-time K_hi pair); returns o [B, H_m, d_v]."""
+    return _step_groups("damp_gdn_decode_step_groups", groups, q, k, v, g, beta, o, slot_idx, stream)
+
+
+def kda_decode_step_groups(groups, q, k, v, g, beta, o=None, slot_idx=None, stream=None):
+    """One KDA decode step of a layer stored as head groups (see gdn_decode_step_groups)."""
+    return _step_groups("damp_kda_decode_step_groups", groups, q, k, v, g, beta, o, slot_idx, stream)
 
 
 def test_kda_wait_timeout(layout, state, perm, q, k, v, g, beta, o=None, slot_idx=None, num_slots=None,

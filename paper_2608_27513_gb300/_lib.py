@@ -29,6 +29,7 @@ _status = ctypes.c_int
 
 _STEP = [_L, _P, _i64, _P, _i32, _P, _P, _P, _P, _P, _P, _P, _i32, _P]
 _FP32_STEP = [_L, _P, _i64, _P, _i32, _P, _P, _P, _P, _P, _P, _i32, _P]
+_GROUP_STEP = [_L, _i32, _P, _P, _P, _P, _i32, _P, _P, _P, _P, _P, _P, _i32, _P]
 
 SIGNATURES = {
     "damp_validate_layout": (_status, [_L]),
@@ -37,6 +38,8 @@ SIGNATURES = {
     "damp_bits_per_value": (ctypes.c_double, [_L]),
     "damp_gdn_decode_step": (_status, _STEP),
     "damp_kda_decode_step": (_status, _STEP),
+    "damp_gdn_decode_step_groups": (_status, _GROUP_STEP),
+    "damp_kda_decode_step_groups": (_status, _GROUP_STEP),
     "damp_test_kda_wait_timeout": (_status, _STEP),
     "damp_u8_gdn_decode_step": (_status, _STEP),
     "damp_u8_kda_decode_step": (_status, _STEP),

@@ -94,7 +94,7 @@ cudaError_t launch_step(const StepArgs &a, bool packed, cudaStream_t s, bool wai
 damp_status step(const damp_layout *L, void *state, int64_t num_slots, const int32_t *slot_idx, int32_t batch,
                  const uint8_t *perm, const void *q, const void *k, const void *v, const float *g,
                  const float *beta, float *o, int32_t in_dtype, void *stream, bool kda, bool packed,
-                 bool uniform, bool waittest = false) {
+                 bool uniform, bool waittest = false, StepArgs *prepared = nullptr) {
     damp_status st = check_layout(L);
     if (st != DAMP_OK && packed) return st;
     if (!packed) {  // the FP32 state ignores k_hi and lo_format and holds every model head
@@ -153,8 +153,55 @@ damp_status step(const damp_layout *L, void *state, int64_t num_slots, const int
     a.o = o;
     a.in_bf16 = in_dtype == DAMP_IN_BF16;
     a.kda = kda;
+    if (prepared) {  // checked, not launched (the head-group step launches)
+        *prepared = a;
+        return DAMP_OK;
+    }
     return launch_step(a, packed, static_cast<cudaStream_t>(stream), waittest) == cudaSuccess ? DAMP_OK
                                                                                            : DAMP_ERR_CUDA;
+}
+
+// The head groups of one layer (App. E): each group checked as a one-group step, the
+// groups against each other (same operand shapes and format, pools disjoint from each
+// other); two groups with a compile-time pair of K_hi run in one launch, other groups
+// one launch each.
+damp_status step_groups(const damp_layout *layouts, int32_t n_groups, void *const *states, const int64_t *num_slots,
+                        const uint8_t *const *perms, const int32_t *slot_idx, int32_t batch, const void *q,
+                        const void *k, const void *v, const float *g, const float *beta, float *o, int32_t in_dtype,
+                        void *stream, bool kda) {
+    constexpr int kMaxGroups = 8;
+    if (!layouts || !states || !num_slots || !perms) return DAMP_ERR_NULL;
+    if (n_groups < 1 || n_groups > kMaxGroups) return DAMP_ERR_SHAPE;
+    if (batch < 0) return DAMP_ERR_SHAPE;
+    StepArgs a[kMaxGroups];
+    Range pools[kMaxGroups];
+    for (int i = 0; i < n_groups; ++i) {
+        const damp_layout &L = layouts[i];
+        damp_status st = check_layout(&L);
+        if (st != DAMP_OK) return st;
+        if (!L.head_map) return DAMP_ERR_SHAPE;  // a group is a head subset
+        const damp_layout &L0 = layouts[0];
+        if (L.model_heads != L0.model_heads || L.num_qk_heads != L0.num_qk_heads || L.d_k != L0.d_k ||
+            L.d_v != L0.d_v)
+            return DAMP_ERR_SHAPE;
+        if (L.lo_format != L0.lo_format) return DAMP_ERR_FORMAT;
+        if (batch == 0) continue;
+        st = step(&L, states[i], num_slots[i], slot_idx, batch, perms[i], q, k, v, g, beta, o, in_dtype, stream, kda,
+                  true, false, false, &a[i]);
+        if (st != DAMP_OK) return st;
+        pools[i] = range_of(states[i], num_slots[i] * slot_bytes_of(&L));
+        for (int j = 0; j < i; ++j)
+            if (overlap(pools[i], pools[j])) return DAMP_ERR_ALIAS;
+    }
+    if (batch == 0) return DAMP_OK;
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (n_groups == 2) {
+        const cudaError_t e = kda ? launch_packed2_kda(a[0], a[1], s) : launch_packed2_gdn(a[0], a[1], s);
+        if (e != cudaErrorNotSupported) return e == cudaSuccess ? DAMP_OK : DAMP_ERR_CUDA;
+    }
+    for (int i = 0; i < n_groups; ++i)
+        if (launch_step(a[i], true, s) != cudaSuccess) return DAMP_ERR_CUDA;
+    return DAMP_OK;
 }
 
 damp_status prefill(const damp_layout *L, void *state, int64_t num_slots, const int32_t *slot_idx, int32_t batch,
@@ -377,6 +424,24 @@ damp_status damp_kda_decode_step(const damp_layout *layout, void *state, int64_t
                 false);
 }
 
+damp_status damp_gdn_decode_step_groups(const damp_layout *layouts, int32_t n_groups, void *const *states,
+                                        const int64_t *num_slots, const uint8_t *const *perms,
+                                        const int32_t *slot_idx, int32_t batch, const void *q, const void *k,
+                                        const void *v, const float *g, const float *beta, float *o,
+                                        int32_t in_dtype, void *stream) {
+    return step_groups(layouts, n_groups, states, num_slots, perms, slot_idx, batch, q, k, v, g, beta, o, in_dtype,
+                       stream, false);
+}
+
+damp_status damp_kda_decode_step_groups(const damp_layout *layouts, int32_t n_groups, void *const *states,
+                                        const int64_t *num_slots, const uint8_t *const *perms,
+                                        const int32_t *slot_idx, int32_t batch, const void *q, const void *k,
+                                        const void *v, const float *g, const float *beta, float *o,
+                                        int32_t in_dtype, void *stream) {
+    return step_groups(layouts, n_groups, states, num_slots, perms, slot_idx, batch, q, k, v, g, beta, o, in_dtype,
+                       stream, true);
+}
+
 damp_status damp_test_kda_wait_timeout(const damp_layout *layout, void *state, int64_t num_slots,
                                        const int32_t *slot_idx, int32_t batch, const uint8_t *perm, const void *q,
                                        const void *k, const void *v, const float *g, const float *beta, float *o,
@@ -531,6 +596,10 @@ damp_status damp_device_status(uint32_t *status) {
     if (take_status_packed_gdn_f8(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     if (take_status_packed_kda_f8(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_groups_gdn(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
+    all |= bits;
+    if (take_status_groups_kda(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;
     if (take_status_quad_gdn(&bits) != cudaSuccess) return DAMP_ERR_CUDA;
     all |= bits;

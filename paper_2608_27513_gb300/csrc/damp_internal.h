@@ -51,6 +51,10 @@ struct ConvArgs {
 cudaError_t launch_packed_gdn(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_packed_kda(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_packed_kda_waittest(const StepArgs &a, cudaStream_t s);
+// two head groups of a layer in one launch (cudaErrorNotSupported, nothing launched, for
+// a pair of layouts without a compile-time instance)
+cudaError_t launch_packed2_gdn(const StepArgs &a1, const StepArgs &a2, cudaStream_t s);
+cudaError_t launch_packed2_kda(const StepArgs &a1, const StepArgs &a2, cudaStream_t s);
 // the UINT4 low tiers (formats 3, 4)
 cudaError_t launch_packed_gdn_u4(const StepArgs &a, cudaStream_t s);
 cudaError_t launch_packed_kda_u4(const StepArgs &a, cudaStream_t s);
@@ -91,6 +95,8 @@ cudaError_t take_status_packed_gdn_u4(uint32_t *bits);
 cudaError_t take_status_packed_kda_u4(uint32_t *bits);
 cudaError_t take_status_packed_gdn_f8(uint32_t *bits);
 cudaError_t take_status_packed_kda_f8(uint32_t *bits);
+cudaError_t take_status_groups_gdn(uint32_t *bits);
+cudaError_t take_status_groups_kda(uint32_t *bits);
 cudaError_t take_status_quad_gdn(uint32_t *bits);
 cudaError_t take_status_quad_kda(uint32_t *bits);
 cudaError_t take_status_fp32(uint32_t *bits);

@@ -108,8 +108,10 @@ __device__ __forceinline__ void advance(Cursor &k, int H, int V) {
 enum : int { kLtU8 = 0, kLtU4 = 1, kLtE4M3 = 2 };
 constexpr uint32_t kWaitTestExtra = 16;
 constexpr uint64_t kWaitTestNs = 1000000;  // 1 ms
+// The body runs as CTA `blk` of a grid of `nblk` CTAs; it returns true when one of the
+// warp's copy waits ran out (its stage barriers are then left as they are).
 template <int RL, int DKC, int KC, bool KDA, bool HAD, bool BF16, bool HMAP, int LT = kLtU8, bool WAITTEST = false>
-__global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams p) {
+__device__ __forceinline__ bool packed_step_body(const PackedParams p, const int blk, const int nblk) {
     constexpr int R = RL > 0 ? RL : 1;
     extern __shared__ __align__(128) uint8_t smem[];
     const int lane = threadIdx.x & 31;
@@ -136,11 +138,11 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
         (KFIX && DFIX) ? (128 * ((KC + 1) / 2) + (kCodeRow + 4) * (DKC - KC) + 15) & ~15 : p.rec_bytes;
     const int H = p.H, V = p.V;
 
-    const int64_t gw = (int64_t)blockIdx.x * nw + warp;
-    const int64_t nwt = (int64_t)gridDim.x * nw;
+    const int64_t gw = (int64_t)blk * nw + warp;
+    const int64_t nwt = (int64_t)nblk * nw;
     const int64_t t0 = p.total_tiles * gw / nwt;
     const int64_t t1 = p.total_tiles * (gw + 1) / nwt;
-    if (t0 >= t1) return;
+    if (t0 >= t1) return false;
 
     if (lane == 0) {
         for (int s = 0; s < p.nstage; ++s) mbar_init(bar0 + 8 * s, 1);
@@ -201,6 +203,7 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
     Cursor pre = cur;  // next tile to load (lane 0)
     int64_t t_pre = t0;
     if (lane == 0) {
+        fence_proxy_async_smem();  // shared memory this warp used before (a previous body) ahead of the copies
         for (int j = 0; j < p.nstage && t_pre < t1; ++j) {
             issue(t_pre, pre, j);
             ++t_pre;
@@ -572,7 +575,30 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
         const uint32_t bits =
             (timed_out ? kDevWaitTimeout : 0u) | (bad_slot ? kDevBadSlot : 0u) | (bad_head ? kDevBadHead : 0u);
         if (bits) atomicOr(p.status, bits);
+        // every phase has completed: the barriers' memory may be reused by a following body
+        if (!timed_out)
+            for (int s2 = 0; s2 < p.nstage; ++s2) mbar_inval(bar0 + 8 * s2);
     }
+    __syncwarp();
+    return timed_out;
+}
+
+template <int RL, int DKC, int KC, bool KDA, bool HAD, bool BF16, bool HMAP, int LT = kLtU8, bool WAITTEST = false>
+__global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams p) {
+    packed_step_body<RL, DKC, KC, KDA, HAD, BF16, HMAP, LT, WAITTEST>(p, blockIdx.x, gridDim.x);
+}
+
+// Two head groups of one layer in one launch (App. E: per-head budgets as budget-specific
+// kernel groups).  Every warp first takes its share of group 1's tiles (K_hi = KC1), then
+// its share of group 2's (K_hi = KC2), so each SM carries the same mix of both and no
+// split of the grid needs tuning; each group keeps its compile-time record layout, pool,
+// permutation table and head map.  Both parameter blocks give the warps the same
+// shared-memory stride, so a warp's region is the same in both bodies.  d_k = 128.
+template <int KC1, int KC2, bool KDA, bool HAD, bool BF16>
+__global__ void __launch_bounds__(256, 1) packed_step2_kernel(const PackedParams p1, const PackedParams p2) {
+    if (packed_step_body<(128 - KC1 + 31) / 32, 128, KC1, KDA, HAD, BF16, true>(p1, blockIdx.x, gridDim.x))
+        return;  // a copy of group 1 was lost (status set): its barriers cannot be reused
+    packed_step_body<(128 - KC2 + 31) / 32, 128, KC2, KDA, HAD, BF16, true>(p2, blockIdx.x, gridDim.x);
 }
 
 }  // namespace damp

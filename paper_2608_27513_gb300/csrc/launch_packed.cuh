@@ -4,6 +4,8 @@
 #pragma once
 
 #include <algorithm>
+#include <initializer_list>
+#include <utility>
 
 #include "damp_internal.h"
 #include "decode_packed.cuh"
@@ -181,6 +183,46 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
     cudaError_t e = ensure_smem_limit(reinterpret_cast<const void *>(kern), smem);
     if (e != cudaSuccess) return e;
     kern<<<grid, 32 * warps, smem, stream>>>(p);
+    return cudaGetLastError();
+}
+
+// Two head groups of a layer in one launch (packed_step2_kernel): the K_hi pairs of the
+// paper's head-budget table (12/20, 8/24, 4/28 of 128 key channels) with BF16 operands and
+// the UINT8 tiers.  Returns cudaErrorNotSupported (nothing launched) for other pairs.
+template <bool KDA>
+static cudaError_t launch_packed2_impl(const StepArgs &a1, const StepArgs &a2, cudaStream_t stream,
+                                       uint32_t *status) {
+    const StepArgs *g1 = &a1, *g2 = &a2;
+    if (g1->K > g2->K) std::swap(g1, g2);
+    for (const StepArgs *g : {g1, g2})
+        if (g->dk != 128 || !g->in_bf16 || (g->fmt != 0 && g->fmt != 1) || !g->head_map) return cudaErrorNotSupported;
+    if (g1->fmt != g2->fmt || g1->dv != g2->dv) return cudaErrorNotSupported;
+    PackedLaunch s1, s2;
+    cudaError_t e = packed_launch_shape<KDA>(*g1, status, &s1);
+    if (e != cudaSuccess) return e;
+    if ((e = packed_launch_shape<KDA>(*g2, status, &s2)) != cudaSuccess) return e;
+    if (s1.warps != kPackedWarps || s2.warps != kPackedWarps) return cudaErrorNotSupported;
+    const int64_t t1 = s1.p.total_tiles, t2 = s2.p.total_tiles;
+    if (t1 == 0 || t2 == 0) return cudaErrorNotSupported;  // one group alone: the one-group launch
+    const bool had = fmt_had(g1->fmt);
+    void (*kern)(PackedParams, PackedParams) = nullptr;
+#define DAMP_PAIR2(A_, B_)                                                                         \
+    if (g1->K == A_ && g2->K == B_)                                                                \
+        kern = had ? packed_step2_kernel<A_, B_, KDA, true, true> : packed_step2_kernel<A_, B_, KDA, false, true>;
+    DAMP_PAIR2(12, 20)
+    DAMP_PAIR2(8, 24)
+    DAMP_PAIR2(4, 28)
+#undef DAMP_PAIR2
+    if (!kern) return cudaErrorNotSupported;
+    // one warp stride for both bodies (each group's stages and operand buffers fit in it)
+    const int ws = std::max(s1.p.warp_smem, s2.p.warp_smem);
+    s1.p.warp_smem = s2.p.warp_smem = ws;
+    const int smem = ws * kPackedWarps;
+    if (smem > max_smem_per_block()) return cudaErrorNotSupported;
+    if ((e = ensure_smem_limit(reinterpret_cast<const void *>(kern), smem)) != cudaSuccess) return e;
+    const int grid = (int)std::min<int64_t>(std::max<int64_t>((std::max(t1, t2) + kPackedWarps - 1) / kPackedWarps, 1),
+                                            (int64_t)sm_count());
+    kern<<<grid, 32 * kPackedWarps, smem, stream>>>(s1.p, s2.p);
     return cudaGetLastError();
 }
 

@@ -247,3 +247,43 @@ def test_wait_test_hook_accepts_only_its_layout(L):
                                         fb[6], fb[7], 1, None) == 2  # FP32 inputs
     assert L.damp_test_kda_wait_timeout(ctypes.byref(c), fb[0], 4, None, 0, fb[1], fb[2], fb[3], fb[4], fb[5],
                                         fb[6], fb[7], 0, None) == 0  # empty batch: nothing enqueued
+
+
+def test_group_step_rejects_bad_arguments_before_launch(L):
+    """damp_*_decode_step_groups checks every group and the groups against each other
+    before anything is enqueued (fake host pointers: nothing is dereferenced)."""
+    fb = FakeBuffers()
+
+    def grp(k_hi, map_buf, **kw):
+        base = dict(num_heads=4, num_qk_heads=4, d_k=128, d_v=128, k_hi=k_hi, lo_format=0, model_heads=8)
+        base.update(kw)
+        c = _lib.DampLayout(base["num_heads"], base["num_qk_heads"], base["d_k"], base["d_v"], base["k_hi"],
+                            base["lo_format"], base["model_heads"], map_buf)
+        return c
+
+    def call(cs, states=None, perms=(10, 11), n=None, batch=4, slots=(4, 4), **kw):
+        n = len(cs) if n is None else n
+        arr = (_lib.DampLayout * max(len(cs), 1))(*cs)
+        st = (ctypes.c_void_p * 2)(*(states or (fb.ptrs[8], fb.ptrs[9])))
+        pm = (ctypes.c_void_p * 2)(*[fb.ptrs[i] for i in perms])
+        ns = (ctypes.c_int64 * 2)(*slots)
+        args = dict(slot_idx=None, q=fb[2], k=fb[3], v=fb[4], g=fb[5], beta=fb[6], o=fb[7], in_dtype=0, stream=None)
+        args.update(kw)
+        return L.damp_kda_decode_step_groups(arr, n, st, ns, pm, args["slot_idx"], batch, args["q"], args["k"],
+                                             args["v"], args["g"], args["beta"], args["o"], args["in_dtype"],
+                                             args["stream"])
+
+    a, b = grp(8, fb.ptrs[12]), grp(24, fb.ptrs[13])
+    assert call([a, b], batch=0) == 0                                         # empty batch: nothing enqueued
+    assert call([a, b], n=0) == 2
+    assert call([a, b], n=9) == 2
+    assert call([a, grp(24, None, model_heads=0)]) == 2                       # a group without a head map
+    assert call([a, grp(24, fb.ptrs[13], d_v=64)]) == 2                       # operand shapes differ
+    assert call([a, grp(24, fb.ptrs[13], model_heads=16)]) == 2
+    assert call([a, grp(24, fb.ptrs[13], lo_format=1)]) == 5                  # formats differ
+    assert call([a, b], states=(fb.ptrs[8], fb.ptrs[8] + 4096)) == 4         # overlapping pools
+    assert call([a, b], o=ctypes.c_void_p(fb.ptrs[9] + 64)) == 4              # o inside a pool
+    assert call([a, b], in_dtype=7) == 5
+    assert call([a, b], states=(fb.ptrs[8], fb.ptrs[9] + 8)) == 3            # a misaligned pool
+    assert L.damp_kda_decode_step_groups(None, 2, None, None, None, None, 4, fb[2], fb[3], fb[4], fb[5], fb[6],
+                                         fb[7], 0, None) == 1

@@ -195,3 +195,91 @@ def test_group_layout_checkpoint_round_trip(tmp_path):
     G2, p2 = checkpoint.load_layout(path, device=DEV)
     assert G2 == G and G2.heads_of_operands == 8
     assert G2.head_map.cpu().tolist() == HEADS_B and np.array_equal(p2, perms)
+
+
+def _same_up_to_ties(G, a, b, what):
+    """Two pools of one group layout that hold the same updated states up to the rounding
+    of float-ordering ties: the one-launch group step runs compile-time layouts, one call
+    per group the general instance, and their instruction streams may round one value of
+    a rare tie differently.  FP16 rows equal; codes within 1 LSB on at most 1e-5 of the
+    entries; every reconstructed value within one quantization step of its group."""
+    ha, ca, ma = damp.unpack_tiers(G, a)
+    hb, cb, mb = damp.unpack_tiers(G, b)
+    assert torch.equal(ha, hb), f"{what}: FP16 rows differ"
+    dc = (ca.int() - cb.int()).abs()
+    assert float((dc > 0).float().mean()) <= 1e-5, f"{what}: {int((dc > 0).sum())} codes differ"
+    same_meta = (ma == mb).all(dim=-1)
+    if bool(same_meta.all()):
+        assert int(dc.max()) <= 1, f"{what}: a code moved by {int(dc.max())}"
+    assert float((~same_meta).float().mean()) <= 1e-5, f"{what}: {int((~same_meta).sum())} group scales differ"
+    perm = torch.stack([torch.arange(G.d_k, dtype=torch.uint8, device=DEV)] * G.num_heads)
+    Sa = damp.dequantize_state(G, a, perm)
+    Sb = damp.dequantize_state(G, b, perm)
+    s = ma[..., 0].view(torch.float16).float().abs().amax()
+    assert float((Sa - Sb).abs().max()) <= float(s) * 1.0001, f"{what}: reconstruction moved by more than a step"
+
+
+@pytest.mark.parametrize("kind", ["gdn", "kda"])
+@pytest.mark.parametrize("fmt,ka,kb", [(0, 12, 20), (0, 8, 24), (1, 4, 28), (0, 28, 4), (0, 10, 6)])
+def test_group_step_reproduces_the_group_calls(kind, fmt, ka, kb):
+    """damp_*_decode_step_groups: the K_hi pairs of the paper's head-budget table run as one
+    launch (either order of the groups), other pairs as one launch per group; o equals one
+    decode-step call per group bit for bit, the records up to float-ordering ties."""
+    w = wl.sweep(kind, ka, fmt).replace(batch=3, heads=8, qk_heads=4)
+    L = P.layout_of(w)
+    S, perm = _layer(w, 93)
+    groups = [(_group(L, HEADS_A, ka), HEADS_A), (_group(L, HEADS_B, kb), HEADS_B)]
+    pools = {}
+    for tag in ("one", "each"):
+        pools[tag] = []
+        for G, hs in groups:
+            pg = damp.new_state(G, w.batch, DEV)
+            damp.quantize_state(G, S, perm[hs].contiguous(), pg)
+            pools[tag].append(pg)
+    perms = [perm[hs].contiguous() for _, hs in groups]
+    step = damp.kda_decode_step if kind == "kda" else damp.gdn_decode_step
+    gstep = damp.kda_decode_step_groups if kind == "kda" else damp.gdn_decode_step_groups
+    for t in range(3):
+        d = P.inputs_to_dev(w, wl.step_inputs(w, t), DEV)
+        o_each = torch.full((w.batch, w.heads, w.d_v), float("nan"), device=DEV)
+        for (G, hs), pg, pm in zip(groups, pools["each"], perms):
+            step(G, pg, pm, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o_each)
+        o_one = gstep([(G, pg, pm) for (G, _), pg, pm in zip(groups, pools["one"], perms)],
+                      d["q"], d["k"], d["v"], d["g"], d["beta"])
+        assert torch.equal(o_one, o_each), f"step {t}: o differs"
+        for (G, _), a, b in zip(groups, pools["one"], pools["each"]):
+            _same_up_to_ties(G, a, b, f"step {t}")
+
+
+@pytest.mark.parametrize("kind", ["gdn", "kda"])
+def test_group_step_full_batch_4_28(kind):
+    """B=256, H=32, d=128, half the heads at K_hi = 4 and half at 28 (the tiered bench's
+    split), with slot indirection: the one-launch step equals the per-group calls (o bit
+    for bit, records up to float-ordering ties)."""
+    w = wl.sweep(kind, 4).replace(batch=256)
+    L = P.layout_of(w)
+    S, perm = _layer(w.replace(batch=4), 94)
+    S = S.repeat(64, 1, 1, 1)
+    heads_fast = list(range(0, 32, 2))
+    heads_slow = list(range(1, 32, 2))
+    groups = [(_group(L, heads_fast, 4), heads_fast), (_group(L, heads_slow, 28), heads_slow)]
+    perms = [perm[hs].contiguous() for _, hs in groups]
+    slot_idx = torch.randperm(300, device=DEV)[:256].to(torch.int32)
+    pools = {}
+    for tag in ("one", "each"):
+        pools[tag] = []
+        for (G, hs), pm in zip(groups, perms):
+            pg = damp.new_state(G, 300, DEV)
+            damp.quantize_state(G, S, pm, pg, slot_idx=slot_idx)
+            pools[tag].append(pg)
+    step = damp.kda_decode_step if kind == "kda" else damp.gdn_decode_step
+    gstep = damp.kda_decode_step_groups if kind == "kda" else damp.gdn_decode_step_groups
+    d = P.inputs_to_dev(w, wl.step_inputs(w, 0), DEV)
+    o_each = torch.zeros((w.batch, w.heads, w.d_v), device=DEV)
+    for (G, _), pg, pm in zip(groups, pools["each"], perms):
+        step(G, pg, pm, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o_each, slot_idx=slot_idx)
+    o_one = gstep([(G, pg, pm) for (G, _), pg, pm in zip(groups, pools["one"], perms)],
+                  d["q"], d["k"], d["v"], d["g"], d["beta"], slot_idx=slot_idx)
+    assert torch.equal(o_one, o_each)
+    for (G, _), a, b in zip(groups, pools["one"], pools["each"]):
+        _same_up_to_ties(G, a, b, "full batch")
