@@ -24,11 +24,23 @@ def accumulate(layout, kind: str, token_inputs, every: int = 8, stream=None):
     n_samples = 0
     for t, d in enumerate(inputs):
         step(layout, S, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o, stream=stream)
-        damp.calib_log_decay(layout, d["g"], G_acc, stream=stream)
         if (t + 1) % every == 0:
             damp.calib_error_energy(layout, S, E_acc, stream=stream)
             n_samples += n_docs
+    # the log-decay sums of every token and document in one call (the tokens' gates stacked
+    # as one batch of n_tokens * n_docs rows)
+    with torch.cuda.stream(stream) if stream is not None else _nullcontext():
+        g_all = torch.stack([d["g"] for d in inputs]).flatten(0, 1)
+    damp.calib_log_decay(layout, g_all, G_acc, stream=stream)
     return E_acc, max(n_samples, 1), G_acc, n_docs * len(inputs)
+
+
+class _nullcontext:
+    def __enter__(self):
+        return None
+
+    def __exit__(self, *exc):
+        return False
 
 
 def calibrate(layout, kind: str, token_inputs, every: int = 8, tau: float = 1e-4, stream=None):
