@@ -391,7 +391,7 @@ DAMP_API damp_status damp_calib_select(const damp_layout *layout, const float *E
  * its copies in flight to land and returns.  No record and no row of o is written;
  * DAMP_DEV_WAIT_TIMEOUT is set in the device status word.  It lets a test check the
  * timeout path without a fault or a hang.  Arguments as damp_kda_decode_step; only the
- * layout d_k = 128, K_hi = 10, DAMP_LO_U8_AFFINE_G32_H32, BF16 inputs and no head map
+ * layout d_k = d_v = 128, K_hi = 10, DAMP_LO_U8_AFFINE_G32_H32, BF16 inputs and no head map
  * (DAMP_ERR_SHAPE otherwise).
  */
 DAMP_API damp_status damp_test_kda_wait_timeout(const damp_layout *layout, void *state, int64_t num_slots,

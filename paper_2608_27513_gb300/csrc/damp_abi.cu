@@ -107,7 +107,7 @@ damp_status step(const damp_layout *L, void *state, int64_t num_slots, const int
     }
     if (uniform && L->k_hi != 0) return DAMP_ERR_SHAPE;
     if (in_dtype != DAMP_IN_BF16 && in_dtype != DAMP_IN_FP32) return DAMP_ERR_FORMAT;
-    if (waittest && (L->d_k != 128 || L->k_hi != 10 || L->lo_format != DAMP_LO_U8_AFFINE_G32_H32 ||
+    if (waittest && (L->d_k != 128 || L->d_v != 128 || L->k_hi != 10 || L->lo_format != DAMP_LO_U8_AFFINE_G32_H32 ||
                      in_dtype != DAMP_IN_BF16 || L->head_map))
         return DAMP_ERR_SHAPE;
     if (batch < 0) return DAMP_ERR_SHAPE;

@@ -136,7 +136,22 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
     const int meta_off = (KFIX && DFIX) ? 128 * ((KC + 1) / 2) + kCodeRow * (DKC - KC) : p.meta_off;
     const int rec_bytes =
         (KFIX && DFIX) ? (128 * ((KC + 1) / 2) + (kCodeRow + 4) * (DKC - KC) + 15) & ~15 : p.rec_bytes;
-    const int H = p.H, V = p.V;
+    // Compile-time layouts (K_hi and d_k fixed) are launched for d_v = 128 only, with three
+    // record stages (the launcher checks both): the stage size, the operand buffer's layout
+    // and the value-block count are then constants too.
+    constexpr bool FX = KFIX && DFIX;
+    constexpr int FX_ESZ = BF16 ? 2 : 4;
+    constexpr int FX_OFF_Q = 128 * FX_ESZ, FX_OFF_K = 256 * FX_ESZ, FX_OFF_G = 384 * FX_ESZ;
+    constexpr int FX_OFF_P = FX_OFF_G + (KDA ? 512 : 0), FX_OPS = FX_OFF_P + 128;
+    constexpr int FX_REC = FX ? (128 * ((KC + 1) / 2) + (kCodeRow + 4) * (DKC - KC) + 15) & ~15 : 16;
+    constexpr int FX_STAGE = (FX_REC + 127) & ~127;
+    const int nstage = FX ? 3 : p.nstage;
+    const int stage_bytes = FX ? FX_STAGE : p.stage_bytes;
+    const int ops_bytes = FX ? FX_OPS : p.ops_bytes;
+    const int off_v = FX ? 0 : p.off_v, off_q = FX ? FX_OFF_Q : p.off_q, off_k = FX ? FX_OFF_K : p.off_k;
+    const int off_g = FX ? FX_OFF_G : p.off_g, off_perm = FX ? FX_OFF_P : p.off_perm;
+    const int dvv = FX ? 128 : p.dv;
+    const int H = p.H, V = FX ? 4 : p.V;
 
     const int64_t gw = (int64_t)blk * nw + warp;
     const int64_t nwt = (int64_t)nblk * nw;
@@ -145,7 +160,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
     if (t0 >= t1) return false;
 
     if (lane == 0) {
-        for (int s = 0; s < p.nstage; ++s) mbar_init(bar0 + 8 * s, 1);
+        for (int s = 0; s < nstage; ++s) mbar_init(bar0 + 8 * s, 1);
         fence_mbar_init();
     }
     __syncwarp();
@@ -163,7 +178,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
     auto issue = [&](int64_t t, const Cursor &k, int s) {
         const int64_t slot = slot_of(k.b);
         const bool ok = slot >= 0 && slot < p.num_slots && (!HMAP || model_head(k.h) >= 0);
-        const uint32_t st = stage0 + (uint32_t)(s * p.stage_bytes);
+        const uint32_t st = stage0 + (uint32_t)(s * stage_bytes);
         const uint32_t bar = bar0 + 8 * s;
         mbar_arrive_expect_tx(bar, ok ? (uint32_t)rec_bytes + (WAITTEST ? kWaitTestExtra : 0u) : 0u);
         if (ok) bulk_g2s(st, p.state + slot * p.slot_bytes + (int64_t)(k.h * V + k.c) * rec_bytes, rec_bytes, bar);
@@ -175,7 +190,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
         const int mh = HMAP ? max(model_head(uh), 0) : uh;  // an invalid head's tiles are skipped
         const int64_t bh = (int64_t)ub * Hm + mh;
         const int hq = (mh * p.Hqk) / Hm;
-        const int nv = p.bytes_v >> 4, nq = p.bytes_qk >> 4, ng = p.bytes_g >> 4, np = p.bytes_perm >> 4;
+        const int nv = FX ? 8 * FX_ESZ : p.bytes_v >> 4, nq = FX ? 8 * FX_ESZ : p.bytes_qk >> 4, ng = FX ? (KDA ? 32 : 0) : p.bytes_g >> 4, np = FX ? 8 : p.bytes_perm >> 4;
         const int total = nv + 2 * nq + ng + np;
         const uint8_t *qrow = (const uint8_t *)p.q + ((int64_t)ub * p.Hqk + hq) * dk * esz;
         const uint8_t *krow = (const uint8_t *)p.k + ((int64_t)ub * p.Hqk + hq) * dk * esz;
@@ -183,7 +198,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
             int j = ci;
             const uint8_t *src;
             if (j < nv) {
-                src = (const uint8_t *)p.v + bh * p.dv * esz + 16 * j;
+                src = (const uint8_t *)p.v + bh * dvv * esz + 16 * j;
             } else if ((j -= nv) < nq) {
                 src = qrow + 16 * j;
             } else if ((j -= nq) < nq) {
@@ -204,7 +219,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
     int64_t t_pre = t0;
     if (lane == 0) {
         fence_proxy_async_smem();  // shared memory this warp used before (a previous body) ahead of the copies
-        for (int j = 0; j < p.nstage && t_pre < t1; ++j) {
+        for (int j = 0; j < nstage && t_pre < t1; ++j) {
             issue(t_pre, pre, j);
             ++t_pre;
             advance(pre, H, V);
@@ -223,7 +238,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
     int64_t t_fail = t1;
 
     for (int64_t t = t0; t < t1; ++t, advance(cur, H, V)) {
-        const uint32_t st = stage0 + (uint32_t)(s * p.stage_bytes);
+        const uint32_t st = stage0 + (uint32_t)(s * stage_bytes);
         if (!__all_sync(kFull, WAITTEST ? mbar_wait_bounded(bar0 + 8 * s, parity, kWaitTestNs)
                                         : mbar_wait_bounded(bar0 + 8 * s, parity))) {
             timed_out = true;
@@ -240,7 +255,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
 
         // ---- per-(slot, head) operands, gathered into calibrated key order ----
         if (t == t0 || c == 0) {
-            ob = ops0 + (uint32_t)((unit & 1) * p.ops_bytes);
+            ob = ops0 + (uint32_t)((unit & 1) * ops_bytes);
             cp_async_wait_all();
             __syncwarp();
             // beta (and the GDN log-decay) of the next 32 (slot, head) units are
@@ -260,10 +275,10 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
             const float alpha = KDA ? 0.f : expf(__shfl_sync(kFull, unit_g, unit & 31));
             ++unit;
             // d_k is a power of two: masking keeps a malformed permutation in bounds
-            auto chan = [&](int u) { return (int)(lds32(ob + p.off_perm + (u & ~3)) >> (8 * (u & 3))) & (dk - 1); };
-            auto kv_at = [&](int ch) { return BF16 ? bf16_at(ob + p.off_k, ch) : ldsf(ob + p.off_k + 4 * ch); };
-            auto qv_at = [&](int ch) { return BF16 ? bf16_at(ob + p.off_q, ch) : ldsf(ob + p.off_q + 4 * ch); };
-            auto av_at = [&](int ch) { return KDA ? expf(ldsf(ob + p.off_g + 4 * ch)) : alpha; };
+            auto chan = [&](int u) { return (int)(lds32(ob + off_perm + (u & ~3)) >> (8 * (u & 3))) & (dk - 1); };
+            auto kv_at = [&](int ch) { return BF16 ? bf16_at(ob + off_k, ch) : ldsf(ob + off_k + 4 * ch); };
+            auto qv_at = [&](int ch) { return BF16 ? bf16_at(ob + off_q, ch) : ldsf(ob + off_q + 4 * ch); };
+            auto av_at = [&](int ch) { return KDA ? expf(ldsf(ob + off_g + 4 * ch)) : alpha; };
             float kq = 0.f;  // this lane's share of k^T q (all d_k channels)
 #pragma unroll
             for (int i = 0; i < R; ++i) {
@@ -306,11 +321,11 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
             // operands of the next (slot, head) go into the other buffer
             if (t + (V - c) < t1) {
                 const int nb = h + 1 == H ? b + 1 : b, nh = h + 1 == H ? 0 : h + 1;
-                load_ops(nb, nh, ops0 + (uint32_t)((unit & 1) * p.ops_bytes));  // unit was incremented above
+                load_ops(nb, nh, ops0 + (uint32_t)((unit & 1) * ops_bytes));  // unit was incremented above
             }
         }
 
-        const float vj = BF16 ? bf16_at(ob + p.off_v + c * kG * 2, lane) : ldsf(ob + p.off_v + c * kG * 4 + 4 * lane);
+        const float vj = BF16 ? bf16_at(ob + off_v + c * kG * 2, lane) : ldsf(ob + off_v + c * kG * 4 + 4 * lane);
 
         if (ok) {
             const float vt = HAD ? hadamard_lanes(vj, sg) : vj;  // H v
@@ -399,7 +414,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
                     dj = vj - (rlo + rhi);
                     pj = plo + phi;
                 }
-                p.o[((int64_t)b * Hm + mh) * p.dv + c * kG + lane] = fmaf(bkq, dj, pj);
+                p.o[((int64_t)b * Hm + mh) * dvv + c * kG + lane] = fmaf(bkq, dj, pj);
             };
             if constexpr (kLateD) {
                 dt = HAD ? vt - (rlo + hr_hi_early) : vj - (rlo + rhi);
@@ -543,7 +558,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
             ++t_pre;
             advance(pre, H, V);
         }
-        if (++s == p.nstage) {
+        if (++s == nstage) {
             s = 0;
             parity ^= 1u;
         }
@@ -551,7 +566,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
     if (timed_out) {
         // let the loads already in flight land (each wait bounded) before the CTA's
         // shared memory goes away
-        const int64_t last = min(t1 - 1, t_fail + p.nstage - 1);
+        const int64_t last = min(t1 - 1, t_fail + nstage - 1);
         if constexpr (WAITTEST) {
             // settle the extra bytes of every armed stage, so its phase completes
             // exactly when its copy has landed
@@ -560,14 +575,14 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
                     const Cursor k = cursor_at(tt, H, V);
                     const int64_t slot = slot_of(k.b);
                     if (slot >= 0 && slot < p.num_slots && (!HMAP || model_head(k.h) >= 0))
-                        mbar_complete_tx(bar0 + 8 * (int)((tt - t0) % p.nstage), kWaitTestExtra);
+                        mbar_complete_tx(bar0 + 8 * (int)((tt - t0) % nstage), kWaitTestExtra);
                 }
             }
             __syncwarp();
         }
         for (int64_t tt = t_fail; tt <= last; ++tt) {
             const int64_t idx = tt - t0;
-            mbar_wait_bounded(bar0 + 8 * (int)(idx % p.nstage), (uint32_t)((idx / p.nstage) & 1));
+            mbar_wait_bounded(bar0 + 8 * (int)(idx % nstage), (uint32_t)((idx / nstage) & 1));
         }
     }
     cp_async_wait_all();  // operand copies of a (slot, head) that will not run
@@ -577,7 +592,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
         if (bits) atomicOr(p.status, bits);
         // every phase has completed: the barriers' memory may be reused by a following body
         if (!timed_out)
-            for (int s2 = 0; s2 < p.nstage; ++s2) mbar_inval(bar0 + 8 * s2);
+            for (int s2 = 0; s2 < nstage; ++s2) mbar_inval(bar0 + 8 * s2);
     }
     __syncwarp();
     return timed_out;

@@ -97,7 +97,7 @@ static cudaError_t packed_launch_shape(const StepArgs &a, uint32_t *status, Pack
 
 // LT: the low tier's code type (kLtU8: formats 0, 1; kLtU4: formats 3, 4; kLtE4M3: format 5).
 // WAITTEST launches the bounded-wait test instance instead of the decode step (layout
-// d_k = 128, K_hi = 10, format 0, BF16 inputs, no head map only).
+// d_k = d_v = 128, K_hi = 10, format 0, BF16 inputs, no head map only).
 template <bool KDA, int LT, bool WAITTEST = false>
 static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, uint32_t *status) {
     PackedLaunch sh;
@@ -132,7 +132,8 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
     }
     const int rl = (a.dk - a.K + 31) / 32;
     if constexpr (WAITTEST) {
-        if (a.dk != 128 || a.K != 10 || a.fmt != 0 || !a.in_bf16 || hmap) return cudaErrorInvalidValue;
+        if (a.dk != 128 || a.dv != 128 || p.nstage != 3 || a.K != 10 || a.fmt != 0 || !a.in_bf16 || hmap)
+            return cudaErrorInvalidValue;
         kern = packed_step_kernel<4, 128, 10, KDA, true, true, false, kLtU8, true>;
     }
     if (!kern && hmap) {
@@ -146,9 +147,11 @@ static cudaError_t launch_packed_impl(const StepArgs &a, cudaStream_t stream, ui
         }
         if (!kern) return cudaErrorInvalidValue;
     }
-    // compile-time layouts: d_k = 128 with the K_hi values below
+    // compile-time layouts: d_k = d_v = 128 with the K_hi values below, three record stages
+    // (the kernel takes the stage size and the operand buffer's layout as constants)
+    const bool fixed_ok = a.dk == 128 && a.dv == 128 && p.nstage == 3;
 #define DAMP_FIXED(KC_)                                                                           \
-    if (!kern && a.dk == 128 && a.K == KC_) {                                                     \
+    if (!kern && fixed_ok && a.K == KC_) {                                                        \
         DAMP_PICK4((128 - KC_ + 31) / 32, 128, KC_)                                               \
     }
     // (the 4-bit and FP8 tiers: uniform and FP16 + low tier at K_hi = 16)
@@ -196,12 +199,13 @@ static cudaError_t launch_packed2_impl(const StepArgs &a1, const StepArgs &a2, c
     if (g1->K > g2->K) std::swap(g1, g2);
     for (const StepArgs *g : {g1, g2})
         if (g->dk != 128 || !g->in_bf16 || (g->fmt != 0 && g->fmt != 1) || !g->head_map) return cudaErrorNotSupported;
-    if (g1->fmt != g2->fmt || g1->dv != g2->dv) return cudaErrorNotSupported;
+    if (g1->fmt != g2->fmt || g1->dv != 128 || g2->dv != 128) return cudaErrorNotSupported;
     PackedLaunch s1, s2;
     cudaError_t e = packed_launch_shape<KDA>(*g1, status, &s1);
     if (e != cudaSuccess) return e;
     if ((e = packed_launch_shape<KDA>(*g2, status, &s2)) != cudaSuccess) return e;
-    if (s1.warps != kPackedWarps || s2.warps != kPackedWarps) return cudaErrorNotSupported;
+    if (s1.warps != kPackedWarps || s2.warps != kPackedWarps || s1.p.nstage != 3 || s2.p.nstage != 3)
+        return cudaErrorNotSupported;
     const int64_t t1 = s1.p.total_tiles, t2 = s2.p.total_tiles;
     if (t1 == 0 || t2 == 0) return cudaErrorNotSupported;  // one group alone: the one-group launch
     const bool had = fmt_had(g1->fmt);
