@@ -224,8 +224,10 @@ DAMP_API damp_status damp_kda_decode_step(const damp_layout *layout, void *state
  * Two groups with d_k = 128, BF16 operands, lo_format 0 or 1 and K_hi pairs 12/20,
  * 8/24 or 4/28 run as one launch whose CTAs are split between the groups in proportion
  * to their records; other groups run one launch per group.  Results are the same as
- * one damp_gdn_decode_step call per group.  Every argument check runs before anything
- * is enqueued.
+ * one damp_gdn_decode_step call per group (the records up to the rounding of a rare
+ * float-ordering tie: the one-launch form runs compile-time record layouts), except that in the one-launch form a lost record copy of the first
+ * group also leaves the second group's records unwritten (DAMP_DEV_WAIT_TIMEOUT is set).
+ * Every argument check runs before anything is enqueued.
  */
 DAMP_API damp_status damp_gdn_decode_step_groups(const damp_layout *layouts, int32_t n_groups, void *const *states,
                                                  const int64_t *num_slots, const uint8_t *const *perms,

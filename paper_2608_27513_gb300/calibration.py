@@ -1,9 +1,11 @@
 """Calibration run on the GPU (Algorithm 1, App. A.2): FP32 trajectories of the
 calibration documents, error energy of the states sampled every `every` tokens,
 mean log-decay over every token, then the selection of K_hi protected channels and
-the permutation pi per head.  Every step is a libdamp call; this module only orders
-them."""
+the permutation pi per head.  Every arithmetic step is a libdamp call; this module
+orders them (and stacks the tokens' gates into one batch for the log-decay sums)."""
 from __future__ import annotations
+
+import contextlib
 
 import paper_2608_27513_gb300 as damp
 
@@ -29,18 +31,11 @@ def accumulate(layout, kind: str, token_inputs, every: int = 8, stream=None):
             n_samples += n_docs
     # the log-decay sums of every token and document in one call (the tokens' gates stacked
     # as one batch of n_tokens * n_docs rows)
-    with torch.cuda.stream(stream) if stream is not None else _nullcontext():
+    with torch.cuda.stream(stream) if stream is not None else contextlib.nullcontext():
         g_all = torch.stack([d["g"] for d in inputs]).flatten(0, 1)
     damp.calib_log_decay(layout, g_all, G_acc, stream=stream)
     return E_acc, max(n_samples, 1), G_acc, n_docs * len(inputs)
 
-
-class _nullcontext:
-    def __enter__(self):
-        return None
-
-    def __exit__(self, *exc):
-        return False
 
 
 def calibrate(layout, kind: str, token_inputs, every: int = 8, tau: float = 1e-4, stream=None):
