@@ -781,6 +781,8 @@ def calibrate_arm(steps: int, warmup: int, n_docs: int = 32, n_tokens: int = 256
         L = damp.Layout(w.heads, w.qk_heads, w.d_k, w.d_v, w.k_hi, w.lo_format)
         inputs = wl.torch_step_inputs(w, n_tokens, dev)
         calibration.calibrate(L, w.kind, inputs[:16])  # warm-up
+        # the documents' tokens as stacked [T, B, ...] tensors, as a calibration set is stored
+        inputs = {n: torch.stack([d[n] for d in inputs]) for n in ("q", "k", "v", "g", "beta")}
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record()
@@ -788,6 +790,22 @@ def calibrate_arm(steps: int, warmup: int, n_docs: int = 32, n_tokens: int = 256
         e1.record()
         torch.cuda.synchronize()
         run_ms = e0.elapsed_time(e1)
+        # the same run captured in one CUDA graph and replayed: the GPU time of the run's
+        # launches without the host issuing them one by one
+        gs = torch.cuda.Stream(dev)
+        gs.wait_stream(torch.cuda.current_stream())
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=gs):
+            calibration.calibrate(L, w.kind, inputs, stream=gs)
+        torch.cuda.current_stream().wait_stream(gs)
+        graph.replay()
+        torch.cuda.synchronize()
+        e0.record()
+        graph.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        graph_ms = e0.elapsed_time(e1)
+        del graph
         S = 0.3 * torch.randn((n_docs, w.heads, w.d_k, w.d_v), device=dev)
         E = torch.zeros((w.heads, w.d_k), device=dev)
         for _ in range(max(warmup, 3)):
@@ -802,7 +820,8 @@ def calibrate_arm(steps: int, warmup: int, n_docs: int = 32, n_tokens: int = 256
         ee_us = e0.elapsed_time(e1) / n * 1e3
         gbs = S.numel() * 4 / (ee_us * 1e-6) / 1e9
         out.append({"mode": "calibration", "kind": w.kind, "docs": n_docs, "tokens": n_tokens, "heads": w.heads,
-                    "d": w.d_k, "k_hi": w.k_hi, "run_ms": run_ms, "error_energy_us_per_call": ee_us,
+                    "d": w.d_k, "k_hi": w.k_hi, "run_ms": run_ms, "run_ms_cuda_graph_replay": graph_ms,
+                    "error_energy_us_per_call": ee_us,
                     "error_energy_roofline": {"bound": "hbm", "achieved": gbs, "peak": peak, "unit": "GB/s",
                                               "frac": gbs / peak, "bytes_per_call": S.numel() * 4}})
         del inputs, S

@@ -381,6 +381,32 @@ DAMP_API damp_status damp_calib_error_energy(const damp_layout *layout, const fl
                                              void *stream);
 DAMP_API damp_status damp_calib_log_decay(const damp_layout *layout, const float *g, int32_t batch, int32_t kda,
                                           float *G_acc, void *stream);
+/*
+ * The accumulation of a calibration run in one call (App. A.2, Calibration Protocol;
+ * Algorithm 1's statistics): the FP32 trajectories of n_docs calibration documents over
+ * n_tokens tokens (one FP32-state step per token, Sec. 3.1, outputs not written), the
+ * error energy of the states after tokens every, 2 every, ... (damp_calib_error_energy)
+ * and the log-decay sums of every token (damp_calib_log_decay), enqueued by the library
+ * instead of one call per token.
+ *   layout     holds every head of the layer (no head map: DAMP_ERR_SHAPE); lo_format
+ *              chooses the round trip of the error energy
+ *   S          float [n_docs][H][d_k][d_v]: the trajectories' FP32 states (the initial
+ *              states on entry, the final ones on return), 16-B aligned
+ *   q, k       [n_tokens][n_docs][H_qk][d_k] of in_dtype, 16-B aligned
+ *   v          [n_tokens][n_docs][H][d_v] of in_dtype, 16-B aligned
+ *   g          float [n_tokens][n_docs][H][d_k] (kda != 0, 16-B aligned) or
+ *              [n_tokens][n_docs][H] (GDN, 4-B aligned)
+ *   beta       float [n_tokens][n_docs][H], 4-B aligned
+ *   every      sampling period of the error energy, >= 1
+ *   E_acc, G_acc  float [H][d_k], accumulated (the caller zeroes them first), 4-B aligned
+ * Afterwards n_samples = n_docs * (n_tokens / every) and n_tokens * n_docs log-decay rows
+ * go to damp_calib_select.  The results equal the per-token calls in the same order, bit for
+ * bit.  Inputs, S and the accumulators must not overlap (DAMP_ERR_ALIAS).
+ */
+DAMP_API damp_status damp_calib_accumulate(const damp_layout *layout, float *S, int32_t n_docs, int32_t n_tokens,
+                                           const void *q, const void *k, const void *v, const float *g,
+                                           const float *beta, int32_t in_dtype, int32_t kda, int32_t every,
+                                           float *E_acc, float *G_acc, void *stream);
 DAMP_API damp_status damp_calib_select(const damp_layout *layout, const float *E_acc, int64_t n_samples,
                                        const float *G_acc, int64_t n_tokens, float tau, float *C_out,
                                        uint8_t *perm_out, void *stream);

@@ -30,6 +30,7 @@ __all__ = [
     "fp32_gdn_decode_step", "fp32_kda_decode_step", "quantize_state", "dequantize_state",
     "pack_tiers", "unpack_tiers", "device_status", "version", "DEV_WAIT_TIMEOUT", "DEV_BAD_SLOT", "DEV_BAD_HEAD",
     "head_groups", "test_kda_wait_timeout", "gdn_decode_step_groups", "kda_decode_step_groups",
+    "calib_accumulate",
 ]
 
 LO_U8_AFFINE_G32_H32 = 0
@@ -398,6 +399,31 @@ def calib_log_decay(layout, g, G_acc, stream=None):
     _check(lib().damp_calib_log_decay(ctypes.byref(layout.c()), _ptr(g), g.shape[0], 1 if g.dim() == 3 else 0,
                                       _ptr(G_acc), _stream(stream)), "damp_calib_log_decay")
     return G_acc
+
+
+def calib_accumulate(layout, kind, S, q, k, v, g, beta, E_acc, G_acc, every=8, stream=None):
+    """One calibration run's statistics in one call (damp_calib_accumulate): q, k [T, B, H_qk,
+    d_k]; v [T, B, H, d_v]; g [T, B, H, d_k] (KDA) or [T, B, H] (GDN); beta [T, B, H]; S the
+    FP32 states [B, H, d_k, d_v] (updated); E_acc, G_acc [H, d_k] accumulated.  Returns
+    (n_samples, n_token_rows) for calib_select."""
+    import torch
+    if layout.head_map is not None:
+        raise ValueError("the calibration trajectories hold every head: use a layout without a head map")
+    if v is None or v.dim() != 4:
+        raise ValueError("v must be a [T, B, H, d_v] tensor")
+    T, B = v.shape[0], v.shape[1]
+    H = layout.num_heads
+    _want("S", S, (B, H, layout.d_k, layout.d_v), dtype=torch.float32)
+    _want_operands(layout, kind, q, k, v, g, beta, None, (T, B))
+    _want("E_acc", E_acc, (H, layout.d_k), dtype=torch.float32)
+    _want("G_acc", G_acc, (H, layout.d_k), dtype=torch.float32)
+    for n, t in (("S", S), ("q", q), ("k", k), ("v", v), ("g", g), ("beta", beta), ("E_acc", E_acc),
+                 ("G_acc", G_acc)):
+        _cuda_contig(n, t)
+    _check(lib().damp_calib_accumulate(ctypes.byref(layout.c()), _ptr(S), B, T, _ptr(q), _ptr(k), _ptr(v), _ptr(g),
+                                       _ptr(beta), _in_dtype(q, k, v), 1 if kind == "kda" else 0, int(every),
+                                       _ptr(E_acc), _ptr(G_acc), _stream(stream)), "damp_calib_accumulate")
+    return max(B * (T // int(every)), 1), B * T
 
 
 def calib_select(layout, E_acc, n_samples, G_acc, n_tokens, tau=1e-4, stream=None):

@@ -50,6 +50,7 @@ SIGNATURES = {
     "damp_calib_error_energy": (_status, [_L, _P, _i32, _P, _P]),
     "damp_calib_log_decay": (_status, [_L, _P, _i32, _i32, _P, _P]),
     "damp_calib_select": (_status, [_L, _P, _i64, _P, _i64, ctypes.c_float, _P, _P, _P]),
+    "damp_calib_accumulate": (_status, [_L, _P, _i32, _i32, _P, _P, _P, _P, _P, _i32, _i32, _i32, _P, _P, _P]),
     "damp_quantize_state": (_status, [_L, _P, _P, _P, _i64, _P, _i32, _P]),
     "damp_dequantize_state": (_status, [_L, _P, _i64, _P, _i32, _P, _P, _P]),
     "damp_pack_tiers": (_status, [_L, _P, _P, _P, _P, _i64, _P, _i32, _P]),

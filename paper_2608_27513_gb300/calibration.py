@@ -2,7 +2,7 @@
 calibration documents, error energy of the states sampled every `every` tokens,
 mean log-decay over every token, then the selection of K_hi protected channels and
 the permutation pi per head.  Every arithmetic step is a libdamp call; this module
-orders them (and stacks the tokens' gates into one batch for the log-decay sums)."""
+stacks the per-token inputs and orders the calls."""
 from __future__ import annotations
 
 import contextlib
@@ -13,35 +13,32 @@ import paper_2608_27513_gb300 as damp
 def accumulate(layout, kind: str, token_inputs, every: int = 8, stream=None):
     """The FP32 trajectories of the calibration documents under a layout holding every
     head of the layer (no head map): returns (E_acc, n_samples, G_acc, n_tokens), the
-    error-energy and log-decay sums over the layer's heads [H, d_k]."""
+    error-energy and log-decay sums over the layer's heads [H, d_k].  token_inputs is a
+    sequence of per-token dicts (rows = documents) or one dict of tensors stacked over
+    the tokens ([T, B, ...]); the whole run is one damp_calib_accumulate call."""
     import torch
-    inputs = list(token_inputs)
-    n_docs = inputs[0]["v"].shape[0]
-    dev = inputs[0]["v"].device
-    S = damp.new_fp32_state(layout, n_docs, dev)
-    o = torch.empty((n_docs, layout.num_heads, layout.d_v), dtype=torch.float32, device=dev)
-    E_acc = torch.zeros((layout.num_heads, layout.d_k), dtype=torch.float32, device=dev)
-    G_acc = torch.zeros_like(E_acc)
-    step = damp.fp32_kda_decode_step if kind == "kda" else damp.fp32_gdn_decode_step
-    n_samples = 0
-    for t, d in enumerate(inputs):
-        step(layout, S, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o, stream=stream)
-        if (t + 1) % every == 0:
-            damp.calib_error_energy(layout, S, E_acc, stream=stream)
-            n_samples += n_docs
-    # the log-decay sums of every token and document in one call (the tokens' gates stacked
-    # as one batch of n_tokens * n_docs rows)
+    if isinstance(token_inputs, dict):
+        stacked = token_inputs
+    else:
+        inputs = list(token_inputs)
+        with torch.cuda.stream(stream) if stream is not None else contextlib.nullcontext():
+            stacked = {n: torch.stack([d[n] for d in inputs]) for n in ("q", "k", "v", "g", "beta")}
+    n_docs = stacked["v"].shape[1]
+    dev = stacked["v"].device
     with torch.cuda.stream(stream) if stream is not None else contextlib.nullcontext():
-        g_all = torch.stack([d["g"] for d in inputs]).flatten(0, 1)
-    damp.calib_log_decay(layout, g_all, G_acc, stream=stream)
-    return E_acc, max(n_samples, 1), G_acc, n_docs * len(inputs)
-
+        S = damp.new_fp32_state(layout, n_docs, dev)
+        E_acc = torch.zeros((layout.num_heads, layout.d_k), dtype=torch.float32, device=dev)
+        G_acc = torch.zeros_like(E_acc)
+    n_samples, n_tokens = damp.calib_accumulate(layout, kind, S, stacked["q"], stacked["k"], stacked["v"],
+                                                stacked["g"], stacked["beta"], E_acc, G_acc, every, stream)
+    return E_acc, n_samples, G_acc, n_tokens
 
 
 def calibrate(layout, kind: str, token_inputs, every: int = 8, tau: float = 1e-4, stream=None):
     """token_inputs: sequence of per-token dicts of device tensors (q, k, v, g, beta) for
-    the calibration documents (rows = documents), in token order.  Returns (C, perm):
-    float32 [H, d_k] scores and uint8 [H, d_k] permutations."""
+    the calibration documents (rows = documents), in token order, or one dict of those
+    tensors stacked over the tokens.  Returns (C, perm): float32 [H, d_k] scores and uint8
+    [H, d_k] permutations."""
     E_acc, n_samples, G_acc, n_tokens = accumulate(layout, kind, token_inputs, every, stream)
     return damp.calib_select(layout, E_acc, n_samples, G_acc, n_tokens, tau, stream=stream)
 

@@ -559,6 +559,64 @@ damp_status damp_calib_log_decay(const damp_layout *layout, const float *g, int3
                : DAMP_ERR_CUDA;
 }
 
+damp_status damp_calib_accumulate(const damp_layout *layout, float *S, int32_t n_docs, int32_t n_tokens,
+                                  const void *q, const void *k, const void *v, const float *g, const float *beta,
+                                  int32_t in_dtype, int32_t kda, int32_t every, float *E_acc, float *G_acc,
+                                  void *stream) {
+    damp_status st = check_layout(layout);
+    if (st != DAMP_OK) return st;
+    if (layout->head_map) return DAMP_ERR_SHAPE;  // the trajectories hold every head of the layer
+    if (in_dtype != DAMP_IN_BF16 && in_dtype != DAMP_IN_FP32) return DAMP_ERR_FORMAT;
+    if (n_docs < 0 || n_tokens < 0 || every < 1) return DAMP_ERR_SHAPE;
+    if (!E_acc || !G_acc) return DAMP_ERR_NULL;
+    if (n_docs == 0 || n_tokens == 0) return DAMP_OK;
+    if (!S || !q || !k || !v || !g || !beta) return DAMP_ERR_NULL;
+    if (!aligned(S, 16) || !aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(g, kda ? 16 : 4) ||
+        !aligned(beta, 4) || !aligned(E_acc, 4) || !aligned(G_acc, 4))
+        return DAMP_ERR_ALIGN;
+    const int64_t B = n_docs, T = n_tokens, H = layout->num_heads, Hq = layout->num_qk_heads, dk = layout->d_k,
+                  dv = layout->d_v;
+    if (B * T > INT32_MAX) return DAMP_ERR_SHAPE;  // the log-decay call takes the (token, document) rows
+    const int64_t esz = in_dtype == DAMP_IN_BF16 ? 2 : 4;
+    const int64_t sq = B * Hq * dk * esz, sv = B * H * dv * esz, sg = B * H * (kda ? dk : 1) * 4, sb = B * H * 4;
+    const Range rs = range_of(S, B * H * dk * dv * 4), re = range_of(E_acc, H * dk * 4), rg = range_of(G_acc, H * dk * 4);
+    const Range inputs[] = {range_of(q, T * sq), range_of(k, T * sq), range_of(v, T * sv), range_of(g, T * sg),
+                            range_of(beta, T * sb)};
+    if (overlap(rs, re) || overlap(rs, rg) || overlap(re, rg)) return DAMP_ERR_ALIAS;
+    for (const Range &r : inputs)
+        if (overlap(rs, r) || overlap(re, r) || overlap(rg, r)) return DAMP_ERR_ALIAS;
+    const cudaStream_t s = static_cast<cudaStream_t>(stream);
+    StepArgs a{};
+    a.H = (int32_t)H;
+    a.Hqk = (int32_t)Hq;
+    a.Hm = (int32_t)H;
+    a.dk = (int32_t)dk;
+    a.dv = (int32_t)dv;
+    a.state = S;
+    a.num_slots = B;
+    a.batch = n_docs;
+    a.o = nullptr;  // the trajectories' outputs are not needed
+    a.in_bf16 = in_dtype == DAMP_IN_BF16;
+    a.kda = kda ? 1 : 0;
+    for (int64_t t = 0; t < T; ++t) {
+        a.q = static_cast<const uint8_t *>(q) + t * sq;
+        a.k = static_cast<const uint8_t *>(k) + t * sq;
+        a.v = static_cast<const uint8_t *>(v) + t * sv;
+        a.g = reinterpret_cast<const float *>(reinterpret_cast<const uint8_t *>(g) + t * sg);
+        a.beta = reinterpret_cast<const float *>(reinterpret_cast<const uint8_t *>(beta) + t * sb);
+        if (launch_fp32_step(a, s) != cudaSuccess) return DAMP_ERR_CUDA;
+        if ((t + 1) % every == 0 &&
+            launch_calib_error_energy(S, n_docs, (int32_t)H, (int32_t)H, nullptr, (int32_t)dk, (int32_t)dv,
+                                      layout->lo_format, E_acc, s) != cudaSuccess)
+            return DAMP_ERR_CUDA;
+    }
+    // the log-decay sums of every (token, document) row: the stacked gates as one batch
+    return launch_calib_log_decay(g, (int32_t)(B * T), (int32_t)H, (int32_t)H, nullptr, (int32_t)dk, kda ? 1 : 0,
+                                  G_acc, s) == cudaSuccess
+               ? DAMP_OK
+               : DAMP_ERR_CUDA;
+}
+
 damp_status damp_calib_select(const damp_layout *layout, const float *E_acc, int64_t n_samples, const float *G_acc,
                               int64_t n_tokens, float tau, float *C_out, uint8_t *perm_out, void *stream) {
     damp_status st = check_layout(layout);

@@ -119,7 +119,7 @@ __global__ void __launch_bounds__(256, 1) fp32_step_kernel(const Fp32Params p) {
         // d_k load addresses live until the stores
 #pragma unroll
         for (int u = 0; u < DK; ++u) __stcs(base + u * ld, x[u]);
-        p.o[((int64_t)b * p.H + h) * p.dv + c * kG + lane] = (o0 + o1) + (o2 + o3);
+        if (p.o) p.o[((int64_t)b * p.H + h) * p.dv + c * kG + lane] = (o0 + o1) + (o2 + o3);  // no o: calibration runs
     }
     if (bad_slot && lane == 0) atomicOr(p.status, (uint32_t)kDevBadSlot);
 }

@@ -287,3 +287,28 @@ def test_group_step_rejects_bad_arguments_before_launch(L):
     assert call([a, b], states=(fb.ptrs[8], fb.ptrs[9] + 8)) == 3            # a misaligned pool
     assert L.damp_kda_decode_step_groups(None, 2, None, None, None, None, 4, fb[2], fb[3], fb[4], fb[5], fb[6],
                                          fb[7], 0, None) == 1
+
+
+def test_calib_accumulate_rejects_bad_arguments_before_launch(L):
+    fb = FakeBuffers()
+    off = lambda i, d: ctypes.c_void_p(fb.ptrs[i] + d)
+
+    def call(lay=None, **over):
+        c = (lay or _layout(k_hi=0)).c()
+        args = dict(S=fb[0], n_docs=4, n_tokens=8, q=fb[1], k=fb[2], v=fb[3], g=fb[4], beta=fb[5], in_dtype=0,
+                    kda=1, every=8, E=fb[6], G=fb[7], stream=None)
+        args.update(over)
+        return L.damp_calib_accumulate(ctypes.byref(c), *args.values())
+
+    assert call(n_docs=0) == 0 and call(n_tokens=0) == 0            # nothing to do: nothing enqueued
+    assert call(every=0) == 2 and call(n_docs=-1) == 2
+    assert call(in_dtype=9) == 5
+    assert call(S=None) == 1 and call(E=None) == 1 and call(beta=None) == 1
+    assert call(S=off(0, 8)) == 3 and call(g=off(4, 4)) == 3          # KDA gates: 16-B aligned
+    assert call(E=fb[7]) == 4                                          # E_acc over G_acc
+    assert call(q=off(0, 4096)) == 4                                   # an input inside the states
+    lay = damp.Layout(4, 4, 128, 128, 0, 0, model_heads=8, head_map=None)
+    c = lay.c()
+    c.head_map = fb.ptrs[8]
+    assert L.damp_calib_accumulate(ctypes.byref(c), fb[0], 4, 8, fb[1], fb[2], fb[3], fb[4], fb[5], 0, 1, 8, fb[6],
+                                   fb[7], None) == 2                   # a head group: not a whole layer

@@ -108,3 +108,35 @@ def test_calibration_run_matches_oracle(kind):
         kth = np.sort(Cref[h])[::-1][w.k_hi - 1]
         for u in ref_prot ^ got_prot:
             assert abs(Cref[h][u] - kth) <= 1e-2 * kth, (h, u)
+
+
+@pytest.mark.parametrize("kind,fmt", [("kda", 0), ("gdn", 2), ("kda", 3)])
+def test_accumulate_in_one_call_equals_the_per_token_calls(kind, fmt):
+    """damp_calib_accumulate enqueues the same kernels in the same order as one FP32 step
+    per token, an error-energy pass every 8 tokens and one log-decay call over all rows:
+    the FP32 states and both accumulators are identical, bit for bit."""
+    w = (wl.stack_layer(1, 16) if kind == "kda" else wl.stack_layer(0, 16)).replace(batch=4, lo_format=fmt)
+    L = damp.Layout(w.heads, w.qk_heads, w.d_k, w.d_v, w.k_hi, w.lo_format)
+    T, every = 20, 8
+    inputs = wl.torch_step_inputs(w, T, DEV)
+    stacked = {n: torch.stack([d[n] for d in inputs]) for n in ("q", "k", "v", "g", "beta")}
+    S1 = damp.new_fp32_state(L, w.batch, DEV)
+    E1 = torch.zeros((w.heads, w.d_k), device=DEV)
+    G1 = torch.zeros_like(E1)
+    n_samples, n_rows = damp.calib_accumulate(L, kind, S1, stacked["q"], stacked["k"], stacked["v"], stacked["g"],
+                                              stacked["beta"], E1, G1, every)
+    assert (n_samples, n_rows) == (w.batch * (T // every), w.batch * T)
+    S2 = damp.new_fp32_state(L, w.batch, DEV)
+    E2 = torch.zeros_like(E1)
+    G2 = torch.zeros_like(E1)
+    step = damp.fp32_kda_decode_step if kind == "kda" else damp.fp32_gdn_decode_step
+    for t, d in enumerate(inputs):
+        step(L, S2, d["q"], d["k"], d["v"], d["g"], d["beta"])
+        if (t + 1) % every == 0:
+            damp.calib_error_energy(L, S2, E2)
+    damp.calib_log_decay(L, stacked["g"].flatten(0, 1), G2)
+    torch.cuda.synchronize()
+    assert torch.equal(S1, S2)
+    assert torch.equal(E1, E2)
+    assert torch.equal(G1, G2)
+    assert damp.device_status() == 0
