@@ -82,14 +82,25 @@ __device__ __forceinline__ int quad_model_head(const QuadParams &p, int h) {
     return (m >= 0 && m < p.Hm) ? m : -1;
 }
 
-// ---- per-unit operands of unit u (batch row u / H, head u % H): 16-byte copies by the
-//      quad's 128 threads (qt = thread index in the quad) into the raw buffer dst ----
+// (batch row, held head) of a unit, advanced without divisions
+struct UnitPos {
+    int b, h;
+};
+__device__ __forceinline__ UnitPos unit_pos(int u, int H) { return UnitPos{u / H, u - (u / H) * H}; }
+__device__ __forceinline__ void advance_unit(UnitPos &x, int H) {
+    if (++x.h == H) {
+        x.h = 0;
+        ++x.b;
+    }
+}
+
+// ---- per-unit operands of unit (b, h): 16-byte copies by the quad's 128 threads
+//      (qt = thread index in the quad) into the raw buffer dst ----
 template <int KC, bool KDA, bool BF16>
-__device__ __forceinline__ void quad_load_raw(const QuadParams &p, int u, uint32_t dst, int qt) {
+__device__ __forceinline__ void quad_load_raw(const QuadParams &p, const UnitPos x, uint32_t dst, int qt) {
     using G = QuadGeom<KC, KDA, BF16>;
     constexpr int DK = G::DK, DV = G::DV;
-    const int H = p.H;
-    const int b = u / H, h = u - b * H;
+    const int b = x.b, h = x.h;
     const int mh = quad_model_head(p, h);
     const int m = mh >= 0 ? mh : 0;  // an invalid map entry's unit is skipped; its loads stay in bounds
     const int64_t bh = (int64_t)b * p.Hm + m;
@@ -255,26 +266,29 @@ __global__ void __launch_bounds__(32 * kQfrWarps, 1) qfr_step_kernel(const QuadP
     }
     __syncwarp();
 
-    auto load_raw = [&](int u, uint32_t dst) { quad_load_raw<KC, KDA, BF16>(p, u, dst, qt); };
+    auto load_raw = [&](const UnitPos x, uint32_t dst) { quad_load_raw<KC, KDA, BF16>(p, x, dst, qt); };
     auto prep = [&](uint32_t rb, uint32_t pb) { quad_prep<KC, KDA, BF16>(rb, pb, c, lane); };
-    auto slot_of = [&](int u) -> int64_t {
-        const int b = u / H;
-        return p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b;
-    };
-    // lane 0: the record of (unit u, block c) into stage s
-    auto issue = [&](int u, int s) {
-        const int64_t slot = slot_of(u);
-        const int h = u - (u / H) * H;
-        const bool ok = slot >= 0 && slot < p.num_slots && quad_model_head(p, h) >= 0;
+    // lane 0: the record of (unit x, block c) into stage s
+    auto issue = [&](const UnitPos x, int s) {
+        const int64_t slot = p.slot_idx ? (int64_t)p.slot_idx[x.b] : (int64_t)x.b;
+        const bool ok = slot >= 0 && slot < p.num_slots && quad_model_head(p, x.h) >= 0;
         const uint32_t bar = bar0 + 8 * s;
         mbar_arrive_expect_tx(bar, ok ? (uint32_t)Q::REC : 0u);
-        if (ok) bulk_g2s(stage0 + s * G::STAGE, p.state + slot * p.slot_bytes + (int64_t)(h * V + c) * Q::REC, Q::REC, bar);
+        if (ok) bulk_g2s(stage0 + s * G::STAGE, p.state + slot * p.slot_bytes + (int64_t)(x.h * V + c) * Q::REC, Q::REC, bar);
     };
 
-    load_raw(u0, raw0);
-    if (u0 + 1 < u1) load_raw(u0 + 1, raw0 + Q::RAW);
+    UnitPos cur = unit_pos(u0, H);   // unit u of the loop
+    UnitPos rawp = cur;              // the next unit whose operands are copied in
+    load_raw(rawp, raw0);
+    advance_unit(rawp, H);
+    if (u0 + 1 < u1) load_raw(rawp, raw0 + Q::RAW);
+    advance_unit(rawp, H);           // now unit u0 + 2
+    UnitPos issp = cur;              // the next unit whose record is copied in (lane 0)
     if (lane == 0) {
-        for (int s = 0; s < NST && u0 + s < u1; ++s) issue(u0 + s, s);
+        for (int s = 0; s < NST && u0 + s < u1; ++s) {
+            issue(issp, s);
+            advance_unit(issp, H);
+        }
     }
     bool dead = false, bad_slot = false, bad_head = false;
     int k_fail = 0;
@@ -290,13 +304,15 @@ __global__ void __launch_bounds__(32 * kQfrWarps, 1) qfr_step_kernel(const QuadP
         const uint32_t pb = prep0 + (uint32_t)(j * Q::PREP);
         cp_async_wait_all();
         quad_sync(quad);
-        if (u + 2 < u1) load_raw(u + 2, raw0 + (uint32_t)(j * Q::RAW));
+        if (u + 2 < u1) load_raw(rawp, raw0 + (uint32_t)(j * Q::RAW));
+        advance_unit(rawp, H);
         const uint32_t st = stage0 + (uint32_t)(s * G::STAGE);
         if (!dead && !__all_sync(kFull, mbar_wait_bounded(bar0 + 8 * s, parity))) {
             dead = true;
             k_fail = k;
         }
-        const int b = u / H, h = u - b * H;
+        const int b = cur.b, h = cur.h;
+        advance_unit(cur, H);
         const int64_t slot = p.slot_idx ? (int64_t)p.slot_idx[b] : (int64_t)b;
         const int mh = quad_model_head(p, h);
         const bool slot_ok = slot >= 0 && slot < p.num_slots;
@@ -474,7 +490,8 @@ __global__ void __launch_bounds__(32 * kQfrWarps, 1) qfr_step_kernel(const QuadP
             __syncwarp();
             if (lane == 0 && u + NST < u1) {
                 fence_proxy_async_smem();
-                issue(u + NST, s);
+                issue(issp, s);
+                advance_unit(issp, H);
             }
             if (++s == NST) {
                 s = 0;
