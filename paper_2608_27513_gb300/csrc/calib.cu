@@ -31,6 +31,10 @@ namespace {
 // partials are added in warp order (a fixed order: the result does not depend on
 // scheduling).
 constexpr int kEeWarps = 16;
+constexpr int kEeRow = 36;  // floats per row of a warp's staging tile (32 + 4 of padding)
+constexpr int kEeTile = 32 * kEeRow / 4;  // float4 per staging tile
+constexpr int kEeStages = 3;
+constexpr int kEeSmem = kEeWarps * kEeStages * kEeTile * 16;
 
 __device__ uint32_t g_status_calib;
 
@@ -56,9 +60,9 @@ __global__ void __launch_bounds__(32 * kEeWarps) calib_error_energy_kernel(const
     const int m = calib_model_head(head_map, h, Hm);  // the same for the whole CTA
     if (m < 0) return;
     float err = 0.f;
-    for (int b = warp; b < batch; b += kEeWarps) {
-        const float *row = S + (((int64_t)b * Hm + m) * dk + u) * dv;
-        if (FMT == 2) {
+    if constexpr (FMT == 2) {
+        for (int b = warp; b < batch; b += kEeWarps) {
+            const float *row = S + (((int64_t)b * Hm + m) * dk + u) * dv;
             // per-row symmetric absmax INT8: s = max|x| / 127, q = sat(rne(x / s)), x^ = s q
             float amax = 0.f;
             for (int j = 0; j < dv; ++j) amax = fmaxf(amax, fabsf(row[j]));
@@ -69,26 +73,59 @@ __global__ void __launch_bounds__(32 * kEeWarps) calib_error_energy_kernel(const
                 const float dlt = __fmul_rn(s, t) - row[j];
                 err = fmaf(dlt, dlt, err);
             }
-            continue;
         }
-        for (int c = 0; c < dv / kG; ++c) {
+    } else {
+        // items (row b, value block c) of this warp in the order b = warp, warp + 16, ...,
+        // c = 0 .. V-1.  An item is the 32 x 32 tile S[b, m, u0 .. u0+31, 32c .. 32c+31]:
+        // the warp copies it with 16-byte cp.async (each instruction covers four whole
+        // 128-B rows) into one of its kEeStages shared-memory tiles (rows padded to 36
+        // floats: the row-wise copies and each lane's reads of its own row are free of bank
+        // conflicts); two items are in flight while the current one is quantized.
+        extern __shared__ float4 ee_tiles[];
+        float4 *tiles = ee_tiles + warp * (kEeStages * kEeTile);
+        const int Vb = dv / kG;
+        const int nb = warp < batch ? (batch - warp + kEeWarps - 1) / kEeWarps : 0;
+        const int n_items = nb * Vb;
+        const int u0 = u - lane, lr = lane >> 3, lc = lane & 7;
+        auto issue_item = [&](int i) {
+            if (i < n_items) {
+                const int bi = i / Vb, c = i - bi * Vb;
+                const float *base =
+                    S + (((int64_t)(warp + kEeWarps * bi) * Hm + m) * dk + u0 + lr) * dv + kG * c + 4 * lc;
+                const uint32_t dst = smem_u32(tiles + (i % kEeStages) * kEeTile + lr * (kEeRow / 4) + lc);
+#pragma unroll
+                for (int q = 0; q < 8; ++q) cp_async16(dst + 16 * q * kEeRow, base + (int64_t)(4 * q) * dv);
+            }
+            cp_async_commit();  // one group per item index, empty past the end
+        };
+#pragma unroll
+        for (int i = 0; i < kEeStages - 1; ++i) issue_item(i);
+        for (int i = 0; i < n_items; ++i) {
+            __syncwarp();  // every lane is done reading the tile item i + 2 overwrites
+            issue_item(i + kEeStages - 1);
+            cp_async_wait<kEeStages - 1>();  // this lane's copies of item i have landed
+            __syncwarp();                    // ... and every other lane's
+            const float4 *tile = tiles + (i % kEeStages) * kEeTile;
             float2 x[16], y[16];
 #pragma unroll
-            for (int m = 0; m < 8; ++m) {
-                const float4 f = reinterpret_cast<const float4 *>(row + kG * c)[m];
-                x[2 * m] = make_float2(f.x, f.y);
-                x[2 * m + 1] = make_float2(f.z, f.w);
+            for (int q = 0; q < 8; ++q) {
+                const float4 t = tile[lane * (kEeRow / 4) + q];
+                x[2 * q] = make_float2(t.x, t.y);
+                x[2 * q + 1] = make_float2(t.z, t.w);
             }
+            // x becomes the group in the quantizer's domain (H_32 x for the Hadamard formats):
+            // H_32 / sqrt(32) is orthonormal, so ||H^T y - H^T x||^2 = ||y - x||^2 and the
+            // error energy is taken there, without the inverse transform
+            if (fmt_had(FMT)) hadamard_pairs(x);
 #pragma unroll
-            for (int m = 0; m < 16; ++m) y[m] = x[m];
-            if (fmt_had(FMT)) hadamard_pairs(y);
+            for (int q = 0; q < 16; ++q) y[q] = x[q];
             if (FMT == kFmtE4M3) {  // natural domain, one FP32 scale per group
                 uint32_t w[8];
                 const float sc = quantize_group_e4m3(y, w);
                 dequantize_group_e4m3(w, sc, 1.0f, y);
             } else {
 #pragma unroll
-                for (int m = 0; m < 16; ++m) y[m] = mul2(y[m], splat2(kDown));  // working scale of the quantizer
+                for (int q = 0; q < 16; ++q) y[q] = mul2(y[q], splat2(kDown));  // working scale of the quantizer
                 if (fmt_u4(FMT)) {
                     uint32_t w[4];
                     const uint32_t sz = quantize_group_u4(y, w);
@@ -99,10 +136,9 @@ __global__ void __launch_bounds__(32 * kEeWarps) calib_error_energy_kernel(const
                     dequantize_group(w, sz, 1.0f, y);
                 }
             }
-            if (fmt_had(FMT)) hadamard_pairs(y);
 #pragma unroll
-            for (int m = 0; m < 16; ++m) {
-                const float d0 = y[m].x - x[m].x, d1 = y[m].y - x[m].y;
+            for (int q = 0; q < 16; ++q) {
+                const float d0 = y[q].x - x[q].x, d1 = y[q].y - x[q].y;
                 err = fmaf(d0, d0, fmaf(d1, d1, err));
             }
         }
@@ -196,7 +232,11 @@ cudaError_t launch_calib_error_energy(const float *S, int32_t batch, int32_t H, 
         case kFmtE4M3: kern = calib_error_energy_kernel<kFmtE4M3>; break;
         default: return cudaErrorInvalidValue;
     }
-    kern<<<(unsigned)grid, 32 * kEeWarps, 0, stream>>>(S, batch, H, Hm, head_map, dk, dv, E_acc);
+    if (fmt != kFmtS8Row) {
+        const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kEeSmem);
+        if (e != cudaSuccess) return e;
+    }
+    kern<<<(unsigned)grid, 32 * kEeWarps, fmt == kFmtS8Row ? 0 : kEeSmem, stream>>>(S, batch, H, Hm, head_map, dk, dv, E_acc);
     return cudaGetLastError();
 }
 

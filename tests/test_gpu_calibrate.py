@@ -24,7 +24,7 @@ def _built():
     assert damp.device_status() == 0
 
 
-@pytest.mark.parametrize("fmt", [0, 1, 2])
+@pytest.mark.parametrize("fmt", [0, 1, 2, 3, 4, 5])
 def test_error_energy_matches_oracle(fmt):
     B, H, dk, dv = 6, 3, 64, 96
     L = damp.Layout(H, H, dk, dv, 8, fmt)
