@@ -108,6 +108,7 @@ __device__ __forceinline__ void advance(Cursor &k, int H, int V) {
 enum : int { kLtU8 = 0, kLtU4 = 1, kLtE4M3 = 2 };
 constexpr uint32_t kWaitTestExtra = 16;
 constexpr uint64_t kWaitTestNs = 1000000;  // 1 ms
+constexpr int kHiUnroll = 16;             // largest fixed K_hi whose FP16 sums follow the low tier
 // The body runs as CTA `blk` of a grid of `nblk` CTAs; it returns true when one of the
 // warp's copy waits ran out (its stage barriers are then left as they are).
 template <int RL, int DKC, int KC, bool KDA, bool HAD, bool BF16, bool HMAP, int LT = kLtU8, bool WAITTEST = false>
@@ -140,6 +141,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
     // record stages (the launcher checks both): the stage size, the operand buffer's layout
     // and the value-block count are then constants too.
     constexpr bool FX = KFIX && DFIX;
+    constexpr bool kHiFirst = KFIX && KC > kHiUnroll;
     constexpr int FX_ESZ = BF16 ? 2 : 4;
     constexpr int FX_OFF_Q = 128 * FX_ESZ, FX_OFF_K = 256 * FX_ESZ, FX_OFF_G = 384 * FX_ESZ;
     constexpr int FX_OFF_P = FX_OFF_G + (KDA ? 512 : 0), FX_OPS = FX_OFF_P + 128;
@@ -329,6 +331,48 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
 
         if (ok) {
             const float vt = HAD ? hadamard_lanes(vj, sg) : vj;  // H v
+            // ---- phase 1, FP16 tier (lane = column): one 32-bit load per row pair ----
+            const uint32_t col = st + 4 * lane;  // this lane's word in FP16 row pair 0
+            const int KP = (K + 1) >> 1;         // row pairs in the record
+            // pair pi accumulates into rh[pi & 3], ph[pi & 3] (four independent chains)
+            float2 rh[4], ph[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) rh[q] = ph[q] = make_float2(0.f, 0.f);
+            auto hi_pair1 = [&](int pi, uint32_t wv, const uint4 &oa, const uint4 &ok) {
+                const float2 xa = mul2(h2_to_f2(wv), make_float2(__uint_as_float(oa.x), __uint_as_float(oa.y)));
+                rh[pi & 3] = fma2(xa, make_float2(__uint_as_float(ok.x), __uint_as_float(ok.y)), rh[pi & 3]);
+                ph[pi & 3] = fma2(xa, make_float2(__uint_as_float(ok.z), __uint_as_float(ok.w)), ph[pi & 3]);
+            };
+            // K_hi above kHiUnroll: the FP16 rows' sums run before the low tier's rows are
+            // reconstructed, so their loads do not compete with x for registers
+            auto hi_phase1 = [&]() {
+                if constexpr (KFIX) {
+#pragma unroll
+                    for (int pi = 0; pi < (KC + 1) / 2; ++pi)
+                        hi_pair1(pi, lds32(col + 128 * pi), lds128(hops + 32 * pi), lds128(hops + 32 * pi + 16));
+                } else {
+                    // chunks of 4 pairs, loads first; pairs past the last carry zero
+                    // weights and read a zero word
+                    for (int p0 = 0; p0 < KP; p0 += 4) {
+                        uint32_t wv[4];
+                        uint4 oa[4], ok[4];
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            wv[q] = p0 + q < KP ? lds32(col + 128 * (p0 + q)) : 0u;
+                            oa[q] = lds128(hops + 32 * (p0 + q));
+                            ok[q] = lds128(hops + 32 * (p0 + q) + 16);
+                        }
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) hi_pair1(q, wv[q], oa[q], ok[q]);
+                    }
+                }
+            };
+            if constexpr (kHiFirst) {
+                hi_phase1();
+                // K_hi >= 24: a warp barrier keeps the low tier's loads from being scheduled
+                // into the FP16 rows' sums (fewer spilled registers)
+                if constexpr (KC >= 24) __syncwarp();
+            }
             float2 x[R][16];
             float2 acc[16], accp[16];
             // ---- phase 1, low tier: reconstruct and decay (scaled by 2^-39), partial
@@ -358,38 +402,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
                 for (int j = 0; j < 16; ++j) acc[j] = accp[j] = make_float2(0.f, 0.f);
             }
 
-            // ---- phase 1, FP16 tier (lane = column): one 32-bit load per row pair ----
-            const uint32_t col = st + 4 * lane;  // this lane's word in FP16 row pair 0
-            const int KP = (K + 1) >> 1;         // row pairs in the record
-            // pair pi accumulates into rh[pi & 3], ph[pi & 3] (four independent chains)
-            float2 rh[4], ph[4];
-#pragma unroll
-            for (int q = 0; q < 4; ++q) rh[q] = ph[q] = make_float2(0.f, 0.f);
-            auto hi_pair1 = [&](int pi, uint32_t wv, const uint4 &oa, const uint4 &ok) {
-                const float2 xa = mul2(h2_to_f2(wv), make_float2(__uint_as_float(oa.x), __uint_as_float(oa.y)));
-                rh[pi & 3] = fma2(xa, make_float2(__uint_as_float(ok.x), __uint_as_float(ok.y)), rh[pi & 3]);
-                ph[pi & 3] = fma2(xa, make_float2(__uint_as_float(ok.z), __uint_as_float(ok.w)), ph[pi & 3]);
-            };
-            if constexpr (KFIX) {
-#pragma unroll
-                for (int pi = 0; pi < (KC + 1) / 2; ++pi)
-                    hi_pair1(pi, lds32(col + 128 * pi), lds128(hops + 32 * pi), lds128(hops + 32 * pi + 16));
-            } else {
-                // chunks of 4 pairs, loads first; pairs past the last carry zero
-                // weights and read a zero word
-                for (int p0 = 0; p0 < KP; p0 += 4) {
-                    uint32_t wv[4];
-                    uint4 oa[4], ok[4];
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        wv[q] = p0 + q < KP ? lds32(col + 128 * (p0 + q)) : 0u;
-                        oa[q] = lds128(hops + 32 * (p0 + q));
-                        ok[q] = lds128(hops + 32 * (p0 + q) + 16);
-                    }
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) hi_pair1(q, wv[q], oa[q], ok[q]);
-                }
-            }
+            if constexpr (!kHiFirst) hi_phase1();
             rh[0] = add2(add2(rh[0], rh[1]), add2(rh[2], rh[3]));
             ph[0] = add2(add2(ph[0], ph[1]), add2(ph[2], ph[3]));
             const float rhi = rh[0].x + rh[0].y, phi = ph[0].x + ph[0].y;
