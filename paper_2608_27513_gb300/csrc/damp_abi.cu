@@ -14,6 +14,7 @@ namespace {
 constexpr int kMaxDevices = 64;
 std::atomic<int> g_sm_count[kMaxDevices];
 std::atomic<int> g_smem_optin[kMaxDevices];
+std::atomic<int> g_smem_sm[kMaxDevices];
 
 int device_attr(std::atomic<int> *cache, cudaDeviceAttr attr, int fallback) {
     int dev = 0;
@@ -381,6 +382,7 @@ cudaError_t symbol_address_cached(const void *symbol, std::atomic<uint32_t *> *c
     return e;
 }
 int max_smem_per_block() { return device_attr(g_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, 48 * 1024); }
+int max_smem_per_sm() { return device_attr(g_smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, 0); }
 
 }  // namespace damp
 

@@ -110,6 +110,7 @@ cudaError_t take_status_prefill_kda_x(uint32_t *bits);
 // Streaming multiprocessors / opt-in shared memory per block of the current device (cached per device).
 int sm_count();
 int max_smem_per_block();
+int max_smem_per_sm();  // shared memory of one SM (0 if unknown)
 
 // Raises a kernel's dynamic shared-memory limit to at least `bytes` on the current
 // device (the attribute call is made once per kernel, device and larger size).
