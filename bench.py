@@ -629,11 +629,12 @@ def sweep_arm(steps: int, warmup: int):
         print(json.dumps(row), flush=True)
 
 
-def prefill_arm(steps: int, warmup: int, T: int = 64, lo_format: int = 0):
-    """Prefill chunks (App. A.5 prefill path) at B = 256, H = 32, d = 128: one launch per
-    chunk of T tokens per slot.  The chunk keeps each tile's FP32 state on chip, so it
-    is bound by FP32 FMA throughput, not HBM: achieved = algorithmic FLOPs / time against
-    the FP32 FMA peak (SMs x 4 sub-partitions x 32 lanes x 2 flops x SM clock)."""
+def prefill_arm(steps: int, warmup: int, T: int = 64, lo_format: int = 0, kinds=("kda", "gdn"), batch: int = 256):
+    """Prefill chunks (App. A.5 prefill path) at B = 256 (or `batch`), H = 32, d = 128: one
+    launch per chunk of T tokens per slot.  KDA chunks run the per-token FP32 recurrence
+    with each tile's state on chip; GDN chunks of 32+ tokens on the UINT8 tiers run the
+    chunkwise closed form on the tensor cores.  Reported against the FP32 FMA peak (SMs x 4
+    sub-partitions x 32 lanes x 2 flops x SM clock) with the per-token form's FLOPs."""
     import torch
 
     import paper_2608_27513_gb300 as damp
@@ -643,7 +644,8 @@ def prefill_arm(steps: int, warmup: int, T: int = 64, lo_format: int = 0):
     torch.cuda.set_device(dev)
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     out = []
-    for w in (wl.KDA_B256.replace(lo_format=lo_format), wl.sweep("gdn", 16, lo_format)):
+    ws = {"kda": wl.KDA_B256.replace(lo_format=lo_format), "gdn": wl.sweep("gdn", 16, lo_format)}
+    for w in (ws[k].replace(batch=batch) for k in kinds):
         L = damp.Layout(w.heads, w.qk_heads, w.d_k, w.d_v, w.k_hi, w.lo_format)
         per_t = wl.torch_step_inputs(w, T, dev)
         chunk = {key: torch.stack([d[key] for d in per_t], dim=1).contiguous() for key in per_t[0]}
@@ -680,12 +682,20 @@ def prefill_arm(steps: int, warmup: int, T: int = 64, lo_format: int = 0):
         hbm = (2 * w.batch * w.heads * damp.slot_bytes(L) // w.heads
                + w.batch * T * (2 * w.qk_heads * w.d_k * esz + w.heads * w.d_v * (esz + 4)
                                 + w.heads * 4 * ((w.d_k if w.kind == "kda" else 1) + 1)))
+        # which chunk kernel the library runs for this call (the dispatch rule of launch_prefill.cuh)
+        tc = w.kind == "gdn" and w.lo_format in (0, 1) and T >= 32 and w.d_k == w.d_v == 128 and w.in_dtype == "bf16"
+        kernel = ("prefill_tc_gdn_kernel (chunkwise closed form on the tensor cores)" if tc else
+                  "prefill_cg_kernel (per-token FP32 recurrence)" if w.lo_format in (0, 1) and T >= 32 else
+                  "prefill_chunk_kernel (per-token FP32 recurrence)")
         out.append({"mode": "prefill_chunk", "kind": w.kind, "workload": w.name, "lo_format": w.lo_format,
-                    "chunk_tokens": T,
+                    "chunk_tokens": T, "kernel": kernel,
                     "us_per_chunk": us, "tokens_per_s": w.batch * T / (us * 1e-6),
+                    # the per-token form's FLOPs against the FP32 FMA peak: for the tensor-core
+                    # kernel an equivalent rate (its work is tensor-core products plus the solve)
                     "roofline": {"bound": "fma", "achieved": flops / (us * 1e-6) / 1e12, "peak": peak / 1e12,
                                  "unit": "TFLOP/s", "frac": flops / (us * 1e-6) / peak,
-                                 "peak_source": f"FP32 FMA: {sms} SMs x 128 lanes x 2 flops x {mhz:.0f} MHz"},
+                                 "peak_source": f"FP32 FMA: {sms} SMs x 128 lanes x 2 flops x {mhz:.0f} MHz",
+                                 "flops": "7 per state element per token (per-token form)"},
                     "hbm_gbs": hbm / (us * 1e-6) / 1e9, "clocks": clocks})
         del pools, chunk, o
     if damp.device_status() != 0:
@@ -1024,6 +1034,8 @@ def main():
     ap.add_argument("--prefill", action="store_true", help="prefill chunks (64 tokens, B=256) instead of the bench line")
     ap.add_argument("--chunk-tokens", type=int, default=64, help="tokens per slot of a --prefill chunk")
     ap.add_argument("--lo-format", type=int, default=0, help="low-tier format of the --prefill workloads (0-5)")
+    ap.add_argument("--prefill-kind", choices=["kda", "gdn", "both"], default="both", help="--prefill workloads")
+    ap.add_argument("--prefill-batch", type=int, default=256, help="slots of the --prefill workloads (a smaller case for ncu)")
     ap.add_argument("--multitoken", action="store_true",
                     help="fused multi-token steps (T = 1..16 tokens per launch, B=256) instead of the bench line")
     ap.add_argument("--calibrate", action="store_true", help="GPU calibration run instead of the bench line")
@@ -1043,7 +1055,8 @@ def main():
         sweep_arm(args.steps, args.warmup)
         return
     if args.prefill:
-        prefill_arm(args.steps, args.warmup, args.chunk_tokens, args.lo_format)
+        kinds = ("kda", "gdn") if args.prefill_kind == "both" else (args.prefill_kind,)
+        prefill_arm(args.steps, args.warmup, args.chunk_tokens, args.lo_format, kinds, args.prefill_batch)
         return
     if args.multitoken:
         multitoken_arm(args.steps, args.warmup)

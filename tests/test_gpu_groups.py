@@ -113,6 +113,29 @@ def test_group_prefill_chunks_reproduce_the_layer(fmt, T):
     assert torch.equal(og, o)
 
 
+@pytest.mark.parametrize("fmt,T", [(0, 64), (1, 40)])
+def test_group_gdn_prefill_on_the_tensor_cores_reproduces_the_layer(fmt, T):
+    """The GDN tensor-core chunk (d = 128, bf16, 32+ tokens) with head maps and GQA."""
+    w = wl.sweep("gdn", 12, fmt).replace(batch=2, heads=8, qk_heads=4)
+    L = P.layout_of(w)
+    S, perm = _layer(w, 93)
+    pool = damp.new_state(L, w.batch, DEV)
+    damp.quantize_state(L, S, perm, pool)
+    c = _chunk(w, T)
+    lens = torch.tensor([T, 17], dtype=torch.int32, device=DEV)
+    o = damp.gdn_prefill_chunk(L, pool, perm, c["q"], c["k"], c["v"], c["g"], c["beta"], lengths=lens)
+    og = torch.zeros_like(o)
+    for hs in (HEADS_A, HEADS_B):
+        G = _group(L, hs)
+        pg = damp.new_state(G, w.batch, DEV)
+        damp.quantize_state(G, S, perm[hs].contiguous(), pg)
+        damp.gdn_prefill_chunk(G, pg, perm[hs].contiguous(), c["q"], c["k"], c["v"], c["g"], c["beta"], o=og,
+                               lengths=lens)
+        for a, b in zip(damp.unpack_tiers(G, pg), damp.unpack_tiers(L, pool)):
+            assert torch.equal(a, b[:, hs])
+    assert torch.equal(og, o)
+
+
 @pytest.mark.parametrize("kind", ["gdn", "kda"])
 def test_decay_tiered_groups_match_oracle(kind):
     """Fast-decay heads with K_hi = 4, slow-decay heads with K_hi = 28 (mean 16, App. E):
