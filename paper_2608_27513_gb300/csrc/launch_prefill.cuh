@@ -16,10 +16,12 @@ constexpr int kPrefillWarps = 8;
 // aligned) run prefill_cg_kernel, whose per-token work is lower and per-tile work higher;
 // shorter chunks and the other tiers run prefill_chunk_kernel.
 constexpr int kPrefillCgMinT = 32;
-// GDN chunks of at least this many tokens on the UINT8 tiers with d_k = d_v = 128, bf16
-// inputs and a 16-byte aligned o run the tensor-core kernel (prefill_tc_gdn.cu).
+// GDN chunks of at least this many tokens with d_k = d_v = 128, bf16 inputs, a 16-byte
+// aligned o and any low tier but the row-absmax one run the tensor-core kernel
+// (prefill_tc_gdn.cu: formats 0, 1; prefill_tc_gdn_x.cu: formats 3-5).
 constexpr int kPrefillTcMinT = 32;
-cudaError_t launch_prefill_tc_gdn(const PrefillParams &p, bool had, cudaStream_t stream);
+cudaError_t launch_prefill_tc_gdn(const PrefillParams &p, int fmt, cudaStream_t stream);
+cudaError_t launch_prefill_tc_gdn_x(const PrefillParams &p, int fmt, cudaStream_t stream);
 
 template <bool KDA, bool HAD>
 static cudaError_t launch_prefill_cg(const PrefillParams &p0, const StepArgs &a, int rec_bytes, cudaStream_t stream) {
@@ -77,10 +79,11 @@ static cudaError_t launch_prefill_impl(const StepArgs &a, cudaStream_t stream, u
     const int warp_smem = prefill_smem(a.dk, KDA, a.in_bf16).warp_bytes + 128 + ((rg.bytes + 127) & ~127);
     p.warp_stride = warp_smem;
     if (p.total_tiles == 0 || a.T == 0) return cudaSuccess;
-    if constexpr (!KDA && (FMT == kFmtU8H32 || FMT == kFmtU8)) {
+    if constexpr (!KDA && FMT != kFmtS8Row) {
         if (a.T >= kPrefillTcMinT && a.dk == 128 && a.dv == 128 && a.in_bf16 &&
             (reinterpret_cast<uintptr_t>(a.o) & 15) == 0) {
-            const cudaError_t e = launch_prefill_tc_gdn(p, FMT == kFmtU8H32, stream);
+            const cudaError_t e = (FMT == kFmtU8H32 || FMT == kFmtU8) ? launch_prefill_tc_gdn(p, FMT, stream)
+                                                                      : launch_prefill_tc_gdn_x(p, FMT, stream);
             if (e != cudaErrorNotSupported) return e;
         }
     }

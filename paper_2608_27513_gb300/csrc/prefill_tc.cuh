@@ -179,11 +179,14 @@ __device__ __forceinline__ uint32_t tc_k64_off(int row, int k) {
 }
 
 // One CTA of kTcThreads threads per (slot, head) unit at a time (persistent over units);
-// d_k = d_v = 128, bf16 q/k/v, UINT8 low tier (HAD: with H_32).  Thread (row, half):
+// d_k = d_v = 128, bf16 q/k/v, low tier FMT (UINT8 or UINT4 affine with or without H_32,
+// FP8 E4M3; not the row-absmax format).  Thread (row, half):
 // row = tensor-memory lane (warps w and w + 4 reach the same lanes), half = 0 / 1 splits
 // a row's value blocks (0-1 / 2-3) or a phase's tasks between the two.
-template <bool HAD>
+template <int FMT>
 __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_gdn_kernel(const PrefillParams p) {
+    static_assert(FMT != kFmtS8Row, "the row-absmax format shares a row scale over the value blocks");
+    constexpr bool HAD = fmt_had(FMT);
     extern __shared__ __align__(128) uint8_t smem[];  // descriptors need 16-byte alignment (no swizzle)
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int row = tid & 127, half = tid >> 7;
@@ -321,10 +324,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_gdn_kernel(const Pre
                 } else {
                     const int r = u - K;
                     const uint4 c0 = lds128(rec + (uint32_t)(p.codes_off + lo_chunk_off(r, 0, lo)));
-                    const uint4 c1 = lds128(rec + (uint32_t)(p.codes_off + lo_chunk_off(r, 1, lo)));
                     const uint32_t sz = lds32(rec + (uint32_t)(p.meta_off + 4 * r));
-                    const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-                    dequantize_group(w, sz, 1.0f, y);
+                    if constexpr (fmt_u4(FMT)) {
+                        const uint32_t w[4] = {c0.x, c0.y, c0.z, c0.w};
+                        dequantize_group_u4(w, sz, 1.0f, y);
+                    } else {
+                        const uint4 c1 = lds128(rec + (uint32_t)(p.codes_off + lo_chunk_off(r, 1, lo)));
+                        const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+                        if constexpr (FMT == kFmtE4M3) dequantize_group_e4m3(w, __uint_as_float(sz), 1.0f, y);
+                        else dequantize_group(w, sz, 1.0f, y);
+                    }
                 }
                 float v[32];
 #pragma unroll
@@ -657,7 +666,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_gdn_kernel(const Pre
         if (timed_out) break;
         // ---- the chunk-final state (tensor-memory lane u = record row u, this half's value
         //      blocks) into the record in place: FP16 rows back to the natural domain and
-        //      rounded once, low-tier rows requantized at the working scale 2^-39 ----
+        //      rounded once, low-tier rows requantized (the affine formats at the working
+        //      scale 2^-39, FP8 in the natural domain) ----
         {
             const int u = row;
 #pragma unroll 1
@@ -679,19 +689,35 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_gdn_kernel(const Pre
                 }
                 if (u >= K) {
                     const int r = u - K;
+                    if constexpr (FMT == kFmtE4M3) {  // natural domain, one FP32 scale per group
+                        uint32_t w[8];
+                        const float sc = quantize_group_e4m3(y, w);
+                        stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                        stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
+                        stg32(grec + p.meta_off + 4 * r, __float_as_uint(sc));
+                    } else {
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) y[i] = mul2(y[i], splat2(kDown));  // exact
-                    float mn, mx, inv, zq;
-                    minmax32(y, mn, mx);
-                    const float sc = scale_of(mn, mx);
-                    const uint32_t szw = sc == 0.0f ? affine_params_scaled(mn, mx, inv, zq) : affine_finish(sc, mn, inv, zq);
-                    const float2 inv2 = splat2(inv * 0x1p-110f), zc2 = splat2(zq * 0x1p-149f);
-                    uint32_t w[8];
+                        for (int i = 0; i < 16; ++i) y[i] = mul2(y[i], splat2(kDown));  // exact
+                        if constexpr (fmt_u4(FMT)) {
+                            uint32_t w[4];
+                            const uint32_t szw = quantize_group_u4(y, w);
+                            stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                            stg32(grec + p.meta_off + 4 * r, szw);
+                        } else {
+                            float mn, mx, inv, zq;
+                            minmax32(y, mn, mx);
+                            const float sc = scale_of(mn, mx);
+                            const uint32_t szw =
+                                sc == 0.0f ? affine_params_scaled(mn, mx, inv, zq) : affine_finish(sc, mn, inv, zq);
+                            const float2 inv2 = splat2(inv * 0x1p-110f), zc2 = splat2(zq * 0x1p-149f);
+                            uint32_t w[8];
 #pragma unroll
-                    for (int m = 0; m < 8; ++m) w[m] = encode4(y[2 * m], y[2 * m + 1], inv2, zc2);
-                    stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
-                    stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
-                    stg32(grec + p.meta_off + 4 * r, szw);
+                            for (int m = 0; m < 8; ++m) w[m] = encode4(y[2 * m], y[2 * m + 1], inv2, zc2);
+                            stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                            stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
+                            stg32(grec + p.meta_off + 4 * r, szw);
+                        }
+                    }
                 }
             }
         }

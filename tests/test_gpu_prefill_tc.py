@@ -1,7 +1,7 @@
 """GPU parity of the GDN prefill chunk on the tensor cores (chunkwise closed form of
 Sec. 3.1 Eq. delta_update, App. A.5 "Prefill path") against the oracle's per-token
-chunk: GDN, d_k = d_v = 128, bf16 q/k/v, UINT8 tiers with and without H_32, chunks of
-at least 32 tokens (one or more pieces of 64 tokens, ragged rows masked)."""
+chunk: GDN, d_k = d_v = 128, bf16 q/k/v, chunks of at least 32 tokens (one or more
+pieces of 64 tokens, ragged rows masked); the UINT8, UINT4 and FP8 low tiers."""
 import pytest
 
 import workloads as wl
@@ -30,10 +30,10 @@ def test_ragged_rows_and_slot_indirection():
     _run(_gdn("tc_ragged", 3, 2, 2, 6, seed=33), 40, lengths=[40, 17, 0], slot_of={0: 4, 1: 1, 2: 0}, pool=5)
 
 
-@pytest.mark.parametrize("k_hi,fmt", [(0, 0), (16, 1), (40, 0), (127, 1)])
+@pytest.mark.parametrize("k_hi,fmt", [(0, 0), (16, 1), (40, 0), (127, 1), (10, 3), (16, 4), (10, 5), (0, 3)])
 def test_tiers(k_hi, fmt):
-    """No FP16 rows, FP16 rows in one warp or over two, all but one row FP16; the UINT8
-    tier with and without H_32."""
+    """No FP16 rows, FP16 rows in one warp or over two, all but one row FP16; the UINT8 and
+    UINT4 tiers with and without H_32, FP8 E4M3."""
     _run(_gdn(f"tc_k{k_hi}_f{fmt}", 1, 2, 1, k_hi, fmt, seed=34 + k_hi), 64)
 
 
