@@ -631,9 +631,9 @@ def sweep_arm(steps: int, warmup: int):
 
 def prefill_arm(steps: int, warmup: int, T: int = 64, lo_format: int = 0, kinds=("kda", "gdn"), batch: int = 256):
     """Prefill chunks (App. A.5 prefill path) at B = 256 (or `batch`), H = 32, d = 128: one
-    launch per chunk of T tokens per slot.  KDA chunks run the per-token FP32 recurrence
-    with each tile's state on chip; GDN chunks of 32+ tokens (all low tiers but row-absmax)
-    run the chunkwise closed form on the tensor cores.  Reported against the FP32 FMA peak (SMs x 4
+    launch per chunk of T tokens per slot.  Chunks of 32+ tokens on the affine tiers run
+    the chunkwise closed form on the tensor cores; others the per-token FP32 recurrence
+    with each tile's state on chip.  Reported against the FP32 FMA peak (SMs x 4
     sub-partitions x 32 lanes x 2 flops x SM clock) with the per-token form's FLOPs."""
     import torch
 
@@ -683,8 +683,8 @@ def prefill_arm(steps: int, warmup: int, T: int = 64, lo_format: int = 0, kinds=
                + w.batch * T * (2 * w.qk_heads * w.d_k * esz + w.heads * w.d_v * (esz + 4)
                                 + w.heads * 4 * ((w.d_k if w.kind == "kda" else 1) + 1)))
         # which chunk kernel the library runs for this call (the dispatch rule of launch_prefill.cuh)
-        tc = w.kind == "gdn" and w.lo_format != 2 and T >= 32 and w.d_k == w.d_v == 128 and w.in_dtype == "bf16"
-        kernel = ("prefill_tc_gdn_kernel (chunkwise closed form on the tensor cores)" if tc else
+        tc = w.lo_format in (0, 1, 3, 4) and T >= 32 and w.d_k == w.d_v == 128 and w.in_dtype == "bf16"
+        kernel = (f"prefill_tc_{w.kind}_kernel (chunkwise closed form on the tensor cores)" if tc else
                   "prefill_cg_kernel (per-token FP32 recurrence)" if w.lo_format in (0, 1) and T >= 32 else
                   "prefill_chunk_kernel (per-token FP32 recurrence)")
         out.append({"mode": "prefill_chunk", "kind": w.kind, "workload": w.name, "lo_format": w.lo_format,

@@ -18,7 +18,7 @@ INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
               "--expt-relaxed-constexpr", "-I", CSRC, "-I", INCLUDE]
-SOURCES = ["damp_abi.cu", "decode_packed_gdn.cu", "decode_packed_kda.cu", "decode_packed_gdn_u4.cu", "decode_packed_kda_u4.cu", "decode_packed_gdn_f8.cu", "decode_packed_kda_f8.cu", "decode_quad_gdn.cu", "decode_quad_kda.cu", "decode_groups_gdn.cu", "decode_groups_kda.cu", "decode_fp32.cu", "convert.cu", "rowabs.cu", "prefill_gdn.cu", "prefill_kda.cu", "prefill_gdn_x.cu", "prefill_kda_x.cu", "prefill_tc_gdn.cu", "prefill_tc_gdn_x.cu", "calib.cu"]
+SOURCES = ["damp_abi.cu", "decode_packed_gdn.cu", "decode_packed_kda.cu", "decode_packed_gdn_u4.cu", "decode_packed_kda_u4.cu", "decode_packed_gdn_f8.cu", "decode_packed_kda_f8.cu", "decode_quad_gdn.cu", "decode_quad_kda.cu", "decode_groups_gdn.cu", "decode_groups_kda.cu", "decode_fp32.cu", "convert.cu", "rowabs.cu", "prefill_gdn.cu", "prefill_kda.cu", "prefill_gdn_x.cu", "prefill_kda_x.cu", "prefill_tc_gdn.cu", "prefill_tc_gdn_x.cu", "prefill_tc_kda.cu", "prefill_tc_kda_x.cu", "calib.cu"]
 
 
 def nvcc() -> str:

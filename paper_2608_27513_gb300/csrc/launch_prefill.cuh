@@ -16,12 +16,17 @@ constexpr int kPrefillWarps = 8;
 // aligned) run prefill_cg_kernel, whose per-token work is lower and per-tile work higher;
 // shorter chunks and the other tiers run prefill_chunk_kernel.
 constexpr int kPrefillCgMinT = 32;
-// GDN chunks of at least this many tokens with d_k = d_v = 128, bf16 inputs, a 16-byte
-// aligned o and any low tier but the row-absmax one run the tensor-core kernel
-// (prefill_tc_gdn.cu: formats 0, 1; prefill_tc_gdn_x.cu: formats 3-5).
+// GDN and KDA chunks of at least this many tokens with d_k = d_v = 128, bf16 inputs, a
+// 16-byte aligned o and an affine low tier (UINT8 or UINT4, with or without H_32) run the
+// tensor-core kernels (prefill_tc_gdn.cu / prefill_tc_kda.cu: formats 0, 1; the _x units:
+// formats 3, 4).  FP8 E4M3 keeps the per-token kernels: its code spacing is relative, so a
+// value far below its group's maximum has a spacing finer than the closed form's rounding
+// error (absolute, about 2^-24 of the largest terms of its sums).
 constexpr int kPrefillTcMinT = 32;
 cudaError_t launch_prefill_tc_gdn(const PrefillParams &p, int fmt, cudaStream_t stream);
 cudaError_t launch_prefill_tc_gdn_x(const PrefillParams &p, int fmt, cudaStream_t stream);
+cudaError_t launch_prefill_tc_kda(const PrefillParams &p, int fmt, cudaStream_t stream);
+cudaError_t launch_prefill_tc_kda_x(const PrefillParams &p, int fmt, cudaStream_t stream);
 
 template <bool KDA, bool HAD>
 static cudaError_t launch_prefill_cg(const PrefillParams &p0, const StepArgs &a, int rec_bytes, cudaStream_t stream) {
@@ -79,11 +84,12 @@ static cudaError_t launch_prefill_impl(const StepArgs &a, cudaStream_t stream, u
     const int warp_smem = prefill_smem(a.dk, KDA, a.in_bf16).warp_bytes + 128 + ((rg.bytes + 127) & ~127);
     p.warp_stride = warp_smem;
     if (p.total_tiles == 0 || a.T == 0) return cudaSuccess;
-    if constexpr (!KDA && FMT != kFmtS8Row) {
+    if constexpr (FMT != kFmtS8Row && FMT != kFmtE4M3) {
         if (a.T >= kPrefillTcMinT && a.dk == 128 && a.dv == 128 && a.in_bf16 &&
             (reinterpret_cast<uintptr_t>(a.o) & 15) == 0) {
-            const cudaError_t e = (FMT == kFmtU8H32 || FMT == kFmtU8) ? launch_prefill_tc_gdn(p, FMT, stream)
-                                                                      : launch_prefill_tc_gdn_x(p, FMT, stream);
+            constexpr bool u8 = FMT == kFmtU8H32 || FMT == kFmtU8;
+            const cudaError_t e = KDA ? (u8 ? launch_prefill_tc_kda(p, FMT, stream) : launch_prefill_tc_kda_x(p, FMT, stream))
+                                      : (u8 ? launch_prefill_tc_gdn(p, FMT, stream) : launch_prefill_tc_gdn_x(p, FMT, stream));
             if (e != cudaErrorNotSupported) return e;
         }
     }

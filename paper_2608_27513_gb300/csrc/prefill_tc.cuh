@@ -178,9 +178,171 @@ __device__ __forceinline__ uint32_t tc_k64_off(int row, int k) {
     return (uint32_t)(row >> 3) * 1024u + (uint32_t)(k >> 3) * 128u + (uint32_t)(row & 7) * 16u + (uint32_t)(k & 7) * 2u;
 }
 
+// The record rows of a (slot, head) (four value-block records at `recs`, `rstride` apart
+// in shared memory) reconstructed into tensor-memory lane u = record row, value blocks
+// 2 half and 2 half + 1: FP32 at the natural scale, FP16 rows taken into the H_32 domain
+// with the H_32 formats (where the low tier's codes already are).
+template <int FMT>
+__device__ __forceinline__ void tc_reconstruct(const PrefillParams &p, uint32_t recs, int rstride, int u, int half,
+                                               uint32_t tS) {
+    constexpr bool HAD = fmt_had(FMT);
+    const int K = p.K, lo = 128 - K;
+#pragma unroll 1
+    for (int c = 2 * half; c < 2 * half + 2; ++c) {
+        const uint32_t rec = recs + (uint32_t)(c * rstride);
+        float2 y[16];
+        if (u < K) {
+            load_hi_row(rec, u, y);
+            if (HAD) hadamard_pairs(y);
+        } else {
+            const int r = u - K;
+            const uint4 c0 = lds128(rec + (uint32_t)(p.codes_off + lo_chunk_off(r, 0, lo)));
+            const uint32_t sz = lds32(rec + (uint32_t)(p.meta_off + 4 * r));
+            if constexpr (fmt_u4(FMT)) {
+                const uint32_t w[4] = {c0.x, c0.y, c0.z, c0.w};
+                dequantize_group_u4(w, sz, 1.0f, y);
+            } else {
+                const uint4 c1 = lds128(rec + (uint32_t)(p.codes_off + lo_chunk_off(r, 1, lo)));
+                const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+                if constexpr (FMT == kFmtE4M3) dequantize_group_e4m3(w, __uint_as_float(sz), 1.0f, y);
+                else dequantize_group(w, sz, 1.0f, y);
+            }
+        }
+        float v[32];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            v[2 * i] = y[i].x;
+            v[2 * i + 1] = y[i].y;
+        }
+        tc_st32(tS + 32 * c, v);
+    }
+}
+
+// U = L^-1 Y by forward substitution for one value column, in place: col addresses row 0 of
+// the column (rows kTcRowY floats apart), lt the rows of L'^T (L' = L - I, kTcRowL floats
+// apart).  Blocks of 16 rows, 8 per half of the thread pair that owns the column: the rows
+// of a block take the solved rows of the earlier blocks (each loaded once for 8
+// independent sums), then half 0 solves its 8 rows and half 1 takes them out of its own
+// and solves those.  Every thread of the CTA calls it (two barriers per block).
+__device__ __forceinline__ void tc_solve(uint32_t col, uint32_t lt, int half) {
+    auto lt8 = [&](int srow, int t0, float (&lv)[8]) {
+        const uint32_t lrow = lt + (uint32_t)(srow * kTcRowL * 4 + 4 * t0);
+        const uint4 la = lds128(lrow), lb = lds128(lrow + 16);
+        lv[0] = __uint_as_float(la.x);
+        lv[1] = __uint_as_float(la.y);
+        lv[2] = __uint_as_float(la.z);
+        lv[3] = __uint_as_float(la.w);
+        lv[4] = __uint_as_float(lb.x);
+        lv[5] = __uint_as_float(lb.y);
+        lv[6] = __uint_as_float(lb.z);
+        lv[7] = __uint_as_float(lb.w);
+    };
+    auto triangle = [&](int r0, float (&acc)[8]) {  // rows r0 .. r0 + 7 among themselves
+#pragma unroll
+        for (int q = 0; q < 7; ++q) {
+            float lv[8];
+            lt8(r0 + q, r0, lv);
+#pragma unroll
+            for (int r = q + 1; r < 8; ++r) acc[r] = fmaf(-lv[r], acc[q], acc[r]);
+        }
+#pragma unroll
+        for (int r = 0; r < 8; ++r) sts32(col + (uint32_t)((r0 + r) * kTcRowY * 4), __float_as_uint(acc[r]));
+    };
+#pragma unroll 1
+    for (int t0 = 0; t0 < kTcC; t0 += 16) {
+        const int r0 = t0 + 8 * half;
+        float acc[8];
+#pragma unroll
+        for (int r = 0; r < 8; ++r) acc[r] = ldsf(col + (uint32_t)((r0 + r) * kTcRowY * 4));
+#pragma unroll 4
+        for (int s2 = 0; s2 < t0; ++s2) {
+            const float us = ldsf(col + (uint32_t)(s2 * kTcRowY * 4));
+            float lv[8];
+            lt8(s2, r0, lv);
+#pragma unroll
+            for (int r = 0; r < 8; ++r) acc[r] = fmaf(-lv[r], us, acc[r]);
+        }
+        if (half == 0) triangle(r0, acc);
+        __syncthreads();
+        if (half == 1) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {  // the rows half 0 just solved
+                const float us = ldsf(col + (uint32_t)((t0 + q) * kTcRowY * 4));
+                float lv[8];
+                lt8(t0 + q, r0, lv);
+#pragma unroll
+                for (int r = 0; r < 8; ++r) acc[r] = fmaf(-lv[r], us, acc[r]);
+            }
+            triangle(r0, acc);
+        }
+        __syncthreads();
+    }
+}
+
+// The chunk-final state (tensor-memory lane u = record row u, value blocks 2 half and
+// 2 half + 1) into the records at grec0 in place: FP16 rows back to the natural domain and
+// rounded once, low-tier rows requantized (the affine formats at the working scale 2^-39,
+// FP8 in the natural domain).  Warps holding FP16 rows store them warp-collectively.
+template <int FMT>
+__device__ __forceinline__ void tc_requantize(const PrefillParams &p, uint8_t *grec0, int u, int half, int lane,
+                                              uint32_t tS) {
+    constexpr bool HAD = fmt_had(FMT);
+    const int K = p.K, lo = 128 - K;
+#pragma unroll 1
+    for (int c = 2 * half; c < 2 * half + 2; ++c) {
+        float v[32];
+        tc_ld32(tS + 32 * c, v);
+        uint8_t *const grec = grec0 + (int64_t)c * p.rec_bytes;
+        float2 y[16];
+        tc_pairs(v, y);
+        if ((u & ~31) < K) {  // the warp holds FP16 rows: the row-pair store is warp-collective
+            float2 z[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) z[i] = y[i];
+            if (HAD) hadamard_pairs(z);
+            uint32_t own[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) own[i] = f2_to_h2(z[i].x, z[i].y);
+            store_hi_row(grec, u, K, lane, own);
+        }
+        if (u >= K) {
+            const int r = u - K;
+            if constexpr (FMT == kFmtE4M3) {  // natural domain, one FP32 scale per group
+                uint32_t w[8];
+                const float sc = quantize_group_e4m3(y, w);
+                stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
+                stg32(grec + p.meta_off + 4 * r, __float_as_uint(sc));
+            } else {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) y[i] = mul2(y[i], splat2(kDown));  // exact
+                if constexpr (fmt_u4(FMT)) {
+                    uint32_t w[4];
+                    const uint32_t szw = quantize_group_u4(y, w);
+                    stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                    stg32(grec + p.meta_off + 4 * r, szw);
+                } else {
+                    float mn, mx, inv, zq;
+                    minmax32(y, mn, mx);
+                    const float sc = scale_of(mn, mx);
+                    const uint32_t szw =
+                        sc == 0.0f ? affine_params_scaled(mn, mx, inv, zq) : affine_finish(sc, mn, inv, zq);
+                    const float2 inv2 = splat2(inv * 0x1p-110f), zc2 = splat2(zq * 0x1p-149f);
+                    uint32_t w[8];
+#pragma unroll
+                    for (int m = 0; m < 8; ++m) w[m] = encode4(y[2 * m], y[2 * m + 1], inv2, zc2);
+                    stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
+                    stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
+                    stg32(grec + p.meta_off + 4 * r, szw);
+                }
+            }
+        }
+    }
+}
+
 // One CTA of kTcThreads threads per (slot, head) unit at a time (persistent over units);
-// d_k = d_v = 128, bf16 q/k/v, low tier FMT (UINT8 or UINT4 affine with or without H_32,
-// FP8 E4M3; not the row-absmax format).  Thread (row, half):
+// d_k = d_v = 128, bf16 q/k/v, low tier FMT (UINT8 or UINT4 affine, with or without H_32;
+// the launchers also instantiate no FP8 or row-absmax kernel).  Thread (row, half):
 // row = tensor-memory lane (warps w and w + 4 reach the same lanes), half = 0 / 1 splits
 // a row's value blocks (0-1 / 2-3) or a phase's tasks between the two.
 template <int FMT>
@@ -191,7 +353,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_gdn_kernel(const Pre
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int row = tid & 127, half = tid >> 7;
     const uint32_t sb = smem_u32(smem);
-    const int K = p.K, lo = 128 - K, H = p.H, T = p.T, Hm = p.Hm;
+    const int H = p.H, T = p.T, Hm = p.Hm;
     const int rec_bytes = p.rec_bytes, rstride = tc_rec_stride(rec_bytes);
     const uint32_t scal = sb + (uint32_t)kSmScal;
     const uint32_t s_a = scal, s_beta = scal + 256, s_gam = scal + 512, s_rev = scal + 768, s_perm = scal + 1024;
@@ -312,38 +474,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_gdn_kernel(const Pre
 
         // ---- S_0: record row u = row, reconstructed (FP32, natural scale, transformed domain
         //      with H_32) into tensor-memory lane u; this half's two value blocks ----
-        {
-            const int u = row;
-#pragma unroll 1
-            for (int c = 2 * half; c < 2 * half + 2; ++c) {
-                const uint32_t rec = sb + (uint32_t)(kSmRec + c * rstride);
-                float2 y[16];
-                if (u < K) {
-                    load_hi_row(rec, u, y);
-                    if (HAD) hadamard_pairs(y);
-                } else {
-                    const int r = u - K;
-                    const uint4 c0 = lds128(rec + (uint32_t)(p.codes_off + lo_chunk_off(r, 0, lo)));
-                    const uint32_t sz = lds32(rec + (uint32_t)(p.meta_off + 4 * r));
-                    if constexpr (fmt_u4(FMT)) {
-                        const uint32_t w[4] = {c0.x, c0.y, c0.z, c0.w};
-                        dequantize_group_u4(w, sz, 1.0f, y);
-                    } else {
-                        const uint4 c1 = lds128(rec + (uint32_t)(p.codes_off + lo_chunk_off(r, 1, lo)));
-                        const uint32_t w[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-                        if constexpr (FMT == kFmtE4M3) dequantize_group_e4m3(w, __uint_as_float(sz), 1.0f, y);
-                        else dequantize_group(w, sz, 1.0f, y);
-                    }
-                }
-                float v[32];
-#pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    v[2 * i] = y[i].x;
-                    v[2 * i + 1] = y[i].y;
-                }
-                tc_st32(tS + 32 * c, v);
-            }
-        }
+        tc_reconstruct<FMT>(p, sb + (uint32_t)kSmRec, rstride, row, half, tS);
 
 #pragma unroll 1
         for (int p0 = 0; p0 < Tb; p0 += kTcC) {
@@ -536,66 +667,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_gdn_kernel(const Pre
                 }
             }
             __syncthreads();
-            // ---- U = L^-1 Y by forward substitution, value column n = row, in place, in blocks
-            //      of 16 rows (8 per half): the rows of a block take the solved rows of the
-            //      earlier blocks (each loaded once for 8 independent sums), then half 0 solves
-            //      its 8 rows, half 1 takes them out of its own and solves those ----
-            {
-                const uint32_t col = sb + (uint32_t)(kSmYU + 4 * row);
-                const uint32_t lt = sb + (uint32_t)kSmLP;  // L'^T: row s, column t
-                auto lt8 = [&](int srow, int t0, float (&lv)[8]) {
-                    const uint32_t lrow = lt + (uint32_t)(srow * kTcRowL * 4 + 4 * t0);
-                    const uint4 la = lds128(lrow), lb = lds128(lrow + 16);
-                    lv[0] = __uint_as_float(la.x);
-                    lv[1] = __uint_as_float(la.y);
-                    lv[2] = __uint_as_float(la.z);
-                    lv[3] = __uint_as_float(la.w);
-                    lv[4] = __uint_as_float(lb.x);
-                    lv[5] = __uint_as_float(lb.y);
-                    lv[6] = __uint_as_float(lb.z);
-                    lv[7] = __uint_as_float(lb.w);
-                };
-                auto triangle = [&](int r0, float (&acc)[8]) {  // rows r0 .. r0 + 7 among themselves
-#pragma unroll
-                    for (int q = 0; q < 7; ++q) {
-                        float lv[8];
-                        lt8(r0 + q, r0, lv);
-#pragma unroll
-                        for (int r = q + 1; r < 8; ++r) acc[r] = fmaf(-lv[r], acc[q], acc[r]);
-                    }
-#pragma unroll
-                    for (int r = 0; r < 8; ++r) sts32(col + (uint32_t)((r0 + r) * kTcRowY * 4), __float_as_uint(acc[r]));
-                };
-#pragma unroll 1
-                for (int t0 = 0; t0 < kTcC; t0 += 16) {
-                    const int r0 = t0 + 8 * half;
-                    float acc[8];
-#pragma unroll
-                    for (int r = 0; r < 8; ++r) acc[r] = ldsf(col + (uint32_t)((r0 + r) * kTcRowY * 4));
-#pragma unroll 4
-                    for (int s2 = 0; s2 < t0; ++s2) {
-                        const float us = ldsf(col + (uint32_t)(s2 * kTcRowY * 4));
-                        float lv[8];
-                        lt8(s2, r0, lv);
-#pragma unroll
-                        for (int r = 0; r < 8; ++r) acc[r] = fmaf(-lv[r], us, acc[r]);
-                    }
-                    if (half == 0) triangle(r0, acc);
-                    __syncthreads();
-                    if (half == 1) {
-#pragma unroll
-                        for (int q = 0; q < 8; ++q) {  // the rows half 0 just solved
-                            const float us = ldsf(col + (uint32_t)((t0 + q) * kTcRowY * 4));
-                            float lv[8];
-                            lt8(t0 + q, r0, lv);
-#pragma unroll
-                            for (int r = 0; r < 8; ++r) acc[r] = fmaf(-lv[r], us, acc[r]);
-                        }
-                        triangle(r0, acc);
-                    }
-                    __syncthreads();
-                }
-            }
+            // ---- U = L^-1 Y by forward substitution (value column n = row, in place) ----
+            tc_solve(sb + (uint32_t)(kSmYU + 4 * row), sb + (uint32_t)kSmLP, half);
             // ---- U (half 0) and f_C. U (half 1) as three bf16 parts, K-major (value columns n x
             //      tokens s) ----
             {
@@ -665,62 +738,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_gdn_kernel(const Pre
         }
         if (timed_out) break;
         // ---- the chunk-final state (tensor-memory lane u = record row u, this half's value
-        //      blocks) into the record in place: FP16 rows back to the natural domain and
-        //      rounded once, low-tier rows requantized (the affine formats at the working
-        //      scale 2^-39, FP8 in the natural domain) ----
-        {
-            const int u = row;
-#pragma unroll 1
-            for (int c = 2 * half; c < 2 * half + 2; ++c) {
-                float v[32];
-                tc_ld32(tS + 32 * c, v);
-                uint8_t *const grec = grec0 + (int64_t)c * rec_bytes;
-                float2 y[16];
-                tc_pairs(v, y);
-                if (32 * (warp & 3) < K) {  // the warp holds FP16 rows: the row-pair store is warp-collective
-                    float2 z[16];
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) z[i] = y[i];
-                    if (HAD) hadamard_pairs(z);
-                    uint32_t own[16];
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) own[i] = f2_to_h2(z[i].x, z[i].y);
-                    store_hi_row(grec, u, K, lane, own);
-                }
-                if (u >= K) {
-                    const int r = u - K;
-                    if constexpr (FMT == kFmtE4M3) {  // natural domain, one FP32 scale per group
-                        uint32_t w[8];
-                        const float sc = quantize_group_e4m3(y, w);
-                        stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
-                        stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
-                        stg32(grec + p.meta_off + 4 * r, __float_as_uint(sc));
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) y[i] = mul2(y[i], splat2(kDown));  // exact
-                        if constexpr (fmt_u4(FMT)) {
-                            uint32_t w[4];
-                            const uint32_t szw = quantize_group_u4(y, w);
-                            stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
-                            stg32(grec + p.meta_off + 4 * r, szw);
-                        } else {
-                            float mn, mx, inv, zq;
-                            minmax32(y, mn, mx);
-                            const float sc = scale_of(mn, mx);
-                            const uint32_t szw =
-                                sc == 0.0f ? affine_params_scaled(mn, mx, inv, zq) : affine_finish(sc, mn, inv, zq);
-                            const float2 inv2 = splat2(inv * 0x1p-110f), zc2 = splat2(zq * 0x1p-149f);
-                            uint32_t w[8];
-#pragma unroll
-                            for (int m = 0; m < 8; ++m) w[m] = encode4(y[2 * m], y[2 * m + 1], inv2, zc2);
-                            stg128(grec + p.codes_off + lo_chunk_off(r, 0, lo), make_uint4(w[0], w[1], w[2], w[3]));
-                            stg128(grec + p.codes_off + lo_chunk_off(r, 1, lo), make_uint4(w[4], w[5], w[6], w[7]));
-                            stg32(grec + p.meta_off + 4 * r, szw);
-                        }
-                    }
-                }
-            }
-        }
+        //      blocks) into the record in place ----
+        tc_requantize<FMT>(p, grec0, row, half, lane, tS);
         cur = nxt;
     }
     // a copy or a product that did not complete in time gets one more bounded wait before

@@ -1,5 +1,6 @@
 // prefill_tc_gdn_x.cu -- launcher of the GDN prefill chunk on the tensor cores
-// (prefill_tc.cuh), d_k = d_v = 128, bf16 q/k/v: the UINT4 (with and without H_32) and FP8 E4M3 tiers (formats 3-5).
+// (prefill_tc.cuh), d_k = d_v = 128, bf16 q/k/v: the UINT4 tiers with and without H_32
+// (formats 3, 4; FP8 E4M3 chunks keep the per-token kernel).
 #include <algorithm>
 
 #include "damp_internal.h"
@@ -11,7 +12,6 @@ cudaError_t launch_prefill_tc_gdn_x(const PrefillParams &p, int fmt, cudaStream_
     void (*kern)(PrefillParams) = nullptr;
     if (fmt == kFmtU4H32) kern = prefill_tc_gdn_kernel<kFmtU4H32>;
     if (fmt == kFmtU4) kern = prefill_tc_gdn_kernel<kFmtU4>;
-    if (fmt == kFmtE4M3) kern = prefill_tc_gdn_kernel<kFmtE4M3>;
     if (!kern) return cudaErrorNotSupported;
     const int smem = kTcSmem;
     if (p.rec_bytes > kTcMaxRec || smem > max_smem_per_block()) return cudaErrorNotSupported;

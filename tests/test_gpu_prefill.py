@@ -24,7 +24,7 @@ def _built():
     assert damp.device_status() == 0
 
 
-def _run(w, T, lengths=None, slot_of=None, pool=None, chunks=1, o_offset=None):
+def _run(w, T, lengths=None, slot_of=None, pool=None, chunks=1, o_offset=None, g_scale=1.0):
     rows = list(range(w.batch))
     perms, _ = runs.calibrate_layout(w, n_docs=2, n_tokens=16)
     perm_units, tiers = P.initial_tiers(w, rows, perms, prefix=min(w.prefix, 24))
@@ -41,6 +41,8 @@ def _run(w, T, lengths=None, slot_of=None, pool=None, chunks=1, o_offset=None):
         # teacher-forced: every chunk starts from the oracle's packed state
         damp.pack_tiers(L, *P.tiers_to_dev(w, tiers, len(rows), DEV), state, slot_idx=slot_idx)
         inp = P.chunk_inputs(w, ch * T, T, rows)
+        if g_scale != 1.0:  # stronger decay (the same log-decays on both sides)
+            inp["g"] = (inp["g"] * np.float32(g_scale)).astype(np.float32)
         u = P.unit_chunk(w, inp, T)
         o_ref, tiers, lo_pre = P.oracle_chunk(w, perm_units, tiers, u, lens_units)
         d = {key: P.to_dev(val, DEV, dt if key in ("q", "k", "v") else None) for key, val in inp.items()}
