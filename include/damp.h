@@ -290,7 +290,11 @@ DAMP_API damp_status damp_fp32_kda_decode_step(const damp_layout *layout, float 
  *              a row's length are not written.  Must not overlap the pool or inputs.
  *              4-B aligned; when it is 16-B aligned, chunks of T >= 32 tokens on the
  *              UINT8 tiers (formats 0, 1; d_k 64 or 128) run a kernel with less work per
- *              token (the results differ only in FP32 rounding order).
+ *              token, and chunks of T >= 32 tokens with d_k = d_v = 128, bf16 inputs and
+ *              a UINT8 or UINT4 tier (formats 0, 1, 3, 4) run the chunkwise closed form of
+ *              the delta rule on the tensor cores (pieces of up to 64 tokens; KDA pieces
+ *              are cut shorter where a channel's decay within a piece would leave FP32).
+ *              The results differ only in FP32 rounding order.
  * Other arguments as in damp_gdn_decode_step.  Any lo_format; the row-absmax format
  * (2) needs d_v <= 128 (DAMP_ERR_SHAPE otherwise): its row scale spans the value blocks
  * of a head, which four warps then share.
