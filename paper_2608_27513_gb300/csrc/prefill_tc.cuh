@@ -60,7 +60,7 @@ constexpr int kTcRowL = 68;     // floats per row of L'^T
 constexpr int kTcRowY = 132;    // floats per row of Y / U
 constexpr int kTcRowV = 272;    // bytes per row of v
 constexpr int kTcSmem = kSmScal + 1472;
-constexpr int kTcMaxRec = 8192; // largest record (d_k = 128): four fit below kSmB4 + 48K
+constexpr int kTcMaxRec = 8192; // largest record (d_k = 128): four fit in [kSmRec, kSmV)
 __host__ __device__ constexpr int tc_rec_stride(int rec_bytes) { return (rec_bytes + 127) & ~127; }
 
 // ---- tcgen05 / tensor-memory primitives (inline PTX) ----
@@ -151,11 +151,6 @@ __device__ __forceinline__ uint32_t tc_mn_off(int mn, int k, uint32_t kstride) {
 __device__ __forceinline__ uint32_t lds_u16(uint32_t a) {
     uint32_t v;
     asm volatile("ld.shared.u16 %0, [%1];" : "=r"(v) : "r"(a));
-    return v;
-}
-__device__ __forceinline__ uint4 ldg128_nc(const void *p) {
-    uint4 v;
-    asm volatile("ld.global.nc.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
     return v;
 }
 // all threads of the CTA wait for the phase (bounded) and agree on the outcome

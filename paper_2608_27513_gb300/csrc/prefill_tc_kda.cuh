@@ -47,7 +47,7 @@ constexpr int kKdYU = 0;            // Y, then U: 64 rows of kTcRowY FP32
 constexpr int kKdBU = 0;            // U: three bf16 parts, K-major (value columns x tokens)
 constexpr int kKdScal = 208896;     // beta, pi, gamma_m, xi_C, mbarriers, TMEM address
 constexpr int kKdSmem = kKdScal + 2048;
-constexpr int kKdMaxRec = 8192;     // four records fit below kKdX + 48K
+constexpr int kKdMaxRec = 8192;     // four records fit in [kKdRec, kKdZ)
 constexpr float kKdMaxLog = 85.0f;  // largest log-range of xi on either side of the reference token
 
 // One CTA of kTcThreads threads per (slot, head) unit at a time (persistent over units);
