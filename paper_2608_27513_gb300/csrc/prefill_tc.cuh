@@ -174,16 +174,16 @@ __device__ __forceinline__ uint32_t tc_k64_off(int row, int k) {
 }
 
 // The record rows of a (slot, head) (four value-block records at `recs`, `rstride` apart
-// in shared memory) reconstructed into tensor-memory lane u = record row, value blocks
-// 2 half and 2 half + 1: FP32 at the natural scale, FP16 rows taken into the H_32 domain
-// with the H_32 formats (where the low tier's codes already are).
-template <int FMT>
-__device__ __forceinline__ void tc_reconstruct(const PrefillParams &p, uint32_t recs, int rstride, int u, int half,
+// in shared memory) reconstructed into tensor-memory lane u = record row, the value blocks
+// of part `part` of NQ (4 / NQ blocks each): FP32 at the natural scale, FP16 rows taken
+// into the H_32 domain with the H_32 formats (where the low tier's codes already are).
+template <int FMT, int NQ>
+__device__ __forceinline__ void tc_reconstruct(const PrefillParams &p, uint32_t recs, int rstride, int u, int part,
                                                uint32_t tS) {
     constexpr bool HAD = fmt_had(FMT);
     const int K = p.K, lo = 128 - K;
 #pragma unroll 1
-    for (int c = 2 * half; c < 2 * half + 2; ++c) {
+    for (int c = part * (4 / NQ); c < (part + 1) * (4 / NQ); ++c) {
         const uint32_t rec = recs + (uint32_t)(c * rstride);
         float2 y[16];
         if (u < K) {
@@ -215,76 +215,78 @@ __device__ __forceinline__ void tc_reconstruct(const PrefillParams &p, uint32_t 
 
 // U = L^-1 Y by forward substitution for one value column, in place: col addresses row 0 of
 // the column (rows kTcRowY floats apart), lt the rows of L'^T (L' = L - I, kTcRowL floats
-// apart).  Blocks of 16 rows, 8 per half of the thread pair that owns the column: the rows
-// of a block take the solved rows of the earlier blocks (each loaded once for 8
-// independent sums), then half 0 solves its 8 rows and half 1 takes them out of its own
-// and solves those.  Every thread of the CTA calls it (two barriers per block).
-__device__ __forceinline__ void tc_solve(uint32_t col, uint32_t lt, int half) {
-    auto lt8 = [&](int srow, int t0, float (&lv)[8]) {
+// apart).  Blocks of 16 rows, 16 / NQ per part of the NQ threads that own the column: the
+// rows of a block take the solved rows of the earlier blocks (each loaded once for 16 / NQ
+// independent sums), then the parts solve their rows in turn, each first taking the rows
+// solved before it out of its own.  Every thread of the CTA calls it (NQ barriers per block).
+template <int NQ>
+__device__ __forceinline__ void tc_solve(uint32_t col, uint32_t lt, int part) {
+    constexpr int RB = 16 / NQ;  // rows per part and block (4 or 8)
+    auto ltr = [&](int srow, int t0, float (&lv)[RB]) {
         const uint32_t lrow = lt + (uint32_t)(srow * kTcRowL * 4 + 4 * t0);
-        const uint4 la = lds128(lrow), lb = lds128(lrow + 16);
-        lv[0] = __uint_as_float(la.x);
-        lv[1] = __uint_as_float(la.y);
-        lv[2] = __uint_as_float(la.z);
-        lv[3] = __uint_as_float(la.w);
-        lv[4] = __uint_as_float(lb.x);
-        lv[5] = __uint_as_float(lb.y);
-        lv[6] = __uint_as_float(lb.z);
-        lv[7] = __uint_as_float(lb.w);
-    };
-    auto triangle = [&](int r0, float (&acc)[8]) {  // rows r0 .. r0 + 7 among themselves
 #pragma unroll
-        for (int q = 0; q < 7; ++q) {
-            float lv[8];
-            lt8(r0 + q, r0, lv);
-#pragma unroll
-            for (int r = q + 1; r < 8; ++r) acc[r] = fmaf(-lv[r], acc[q], acc[r]);
+        for (int i = 0; i < RB / 4; ++i) {
+            const uint4 l4 = lds128(lrow + 16 * i);
+            lv[4 * i] = __uint_as_float(l4.x);
+            lv[4 * i + 1] = __uint_as_float(l4.y);
+            lv[4 * i + 2] = __uint_as_float(l4.z);
+            lv[4 * i + 3] = __uint_as_float(l4.w);
         }
-#pragma unroll
-        for (int r = 0; r < 8; ++r) sts32(col + (uint32_t)((r0 + r) * kTcRowY * 4), __float_as_uint(acc[r]));
     };
 #pragma unroll 1
     for (int t0 = 0; t0 < kTcC; t0 += 16) {
-        const int r0 = t0 + 8 * half;
-        float acc[8];
+        const int r0 = t0 + RB * part;
+        float acc[RB];
 #pragma unroll
-        for (int r = 0; r < 8; ++r) acc[r] = ldsf(col + (uint32_t)((r0 + r) * kTcRowY * 4));
+        for (int r = 0; r < RB; ++r) acc[r] = ldsf(col + (uint32_t)((r0 + r) * kTcRowY * 4));
 #pragma unroll 4
         for (int s2 = 0; s2 < t0; ++s2) {
             const float us = ldsf(col + (uint32_t)(s2 * kTcRowY * 4));
-            float lv[8];
-            lt8(s2, r0, lv);
+            float lv[RB];
+            ltr(s2, r0, lv);
 #pragma unroll
-            for (int r = 0; r < 8; ++r) acc[r] = fmaf(-lv[r], us, acc[r]);
+            for (int r = 0; r < RB; ++r) acc[r] = fmaf(-lv[r], us, acc[r]);
         }
-        if (half == 0) triangle(r0, acc);
-        __syncthreads();
-        if (half == 1) {
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {  // the rows half 0 just solved
-                const float us = ldsf(col + (uint32_t)((t0 + q) * kTcRowY * 4));
-                float lv[8];
-                lt8(t0 + q, r0, lv);
+        for (int q = 0; q < NQ; ++q) {
+            if (part == q) {  // own rows among themselves, then stored
 #pragma unroll
-                for (int r = 0; r < 8; ++r) acc[r] = fmaf(-lv[r], us, acc[r]);
+                for (int a = 0; a < RB - 1; ++a) {
+                    float lv[RB];
+                    ltr(r0 + a, r0, lv);
+#pragma unroll
+                    for (int r = a + 1; r < RB; ++r) acc[r] = fmaf(-lv[r], acc[a], acc[r]);
+                }
+#pragma unroll
+                for (int r = 0; r < RB; ++r) sts32(col + (uint32_t)((r0 + r) * kTcRowY * 4), __float_as_uint(acc[r]));
             }
-            triangle(r0, acc);
+            __syncthreads();
+            if (part > q) {  // the rows part q just solved
+#pragma unroll
+                for (int a = 0; a < RB; ++a) {
+                    const int sr = t0 + RB * q + a;
+                    const float us = ldsf(col + (uint32_t)(sr * kTcRowY * 4));
+                    float lv[RB];
+                    ltr(sr, r0, lv);
+#pragma unroll
+                    for (int r = 0; r < RB; ++r) acc[r] = fmaf(-lv[r], us, acc[r]);
+                }
+            }
         }
-        __syncthreads();
     }
 }
 
-// The chunk-final state (tensor-memory lane u = record row u, value blocks 2 half and
-// 2 half + 1) into the records at grec0 in place: FP16 rows back to the natural domain and
-// rounded once, low-tier rows requantized (the affine formats at the working scale 2^-39,
-// FP8 in the natural domain).  Warps holding FP16 rows store them warp-collectively.
-template <int FMT>
-__device__ __forceinline__ void tc_requantize(const PrefillParams &p, uint8_t *grec0, int u, int half, int lane,
+// The chunk-final state (tensor-memory lane u = record row u, the value blocks of part
+// `part` of NQ) into the records at grec0 in place: FP16 rows back to the natural domain
+// and rounded once, low-tier rows requantized (the affine formats at the working scale
+// 2^-39, FP8 in the natural domain).  Warps holding FP16 rows store them warp-collectively.
+template <int FMT, int NQ>
+__device__ __forceinline__ void tc_requantize(const PrefillParams &p, uint8_t *grec0, int u, int part, int lane,
                                               uint32_t tS) {
     constexpr bool HAD = fmt_had(FMT);
     const int K = p.K, lo = 128 - K;
 #pragma unroll 1
-    for (int c = 2 * half; c < 2 * half + 2; ++c) {
+    for (int c = part * (4 / NQ); c < (part + 1) * (4 / NQ); ++c) {
         float v[32];
         tc_ld32(tS + 32 * c, v);
         uint8_t *const grec = grec0 + (int64_t)c * p.rec_bytes;
@@ -469,7 +471,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_gdn_kernel(const Pre
 
         // ---- S_0: record row u = row, reconstructed (FP32, natural scale, transformed domain
         //      with H_32) into tensor-memory lane u; this half's two value blocks ----
-        tc_reconstruct<FMT>(p, sb + (uint32_t)kSmRec, rstride, row, half, tS);
+        tc_reconstruct<FMT, 2>(p, sb + (uint32_t)kSmRec, rstride, row, half, tS);
 
 #pragma unroll 1
         for (int p0 = 0; p0 < Tb; p0 += kTcC) {
@@ -663,7 +665,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_gdn_kernel(const Pre
             }
             __syncthreads();
             // ---- U = L^-1 Y by forward substitution (value column n = row, in place) ----
-            tc_solve(sb + (uint32_t)(kSmYU + 4 * row), sb + (uint32_t)kSmLP, half);
+            tc_solve<2>(sb + (uint32_t)(kSmYU + 4 * row), sb + (uint32_t)kSmLP, half);
             // ---- U (half 0) and f_C. U (half 1) as three bf16 parts, K-major (value columns n x
             //      tokens s) ----
             {
@@ -734,7 +736,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_gdn_kernel(const Pre
         if (timed_out) break;
         // ---- the chunk-final state (tensor-memory lane u = record row u, this half's value
         //      blocks) into the record in place ----
-        tc_requantize<FMT>(p, grec0, row, half, lane, tS);
+        tc_requantize<FMT, 2>(p, grec0, row, half, lane, tS);
         cur = nxt;
     }
     // a copy or a product that did not complete in time gets one more bounded wait before

@@ -22,7 +22,7 @@ cudaError_t launch_prefill_tc_kda(const PrefillParams &p, int fmt, cudaStream_t 
     if (e != cudaSuccess) return e;
     const int64_t units = (int64_t)p.batch * p.H;
     const int grid = (int)std::min<int64_t>(units, (int64_t)sm_count());
-    kern<<<grid, kTcThreads, smem, stream>>>(p);
+    kern<<<grid, kKdThreads, smem, stream>>>(p);
     return cudaGetLastError();
 }
 

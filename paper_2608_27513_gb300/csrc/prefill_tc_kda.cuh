@@ -49,17 +49,19 @@ constexpr int kKdScal = 208896;     // beta, pi, gamma_m, xi_C, mbarriers, TMEM 
 constexpr int kKdSmem = kKdScal + 2048;
 constexpr int kKdMaxRec = 8192;     // four records fit in [kKdRec, kKdZ)
 constexpr float kKdMaxLog = 85.0f;  // largest log-range of xi on either side of the reference token
+constexpr int kKdThreads = 512;     // four threads per tensor-memory lane (warps w, w + 4, w + 8, w + 12)
 
-// One CTA of kTcThreads threads per (slot, head) unit at a time (persistent over units);
+// One CTA of kKdThreads threads per (slot, head) unit at a time (persistent over units);
 // d_k = d_v = 128, bf16 q/k/v, low tier FMT (UINT8 or UINT4 affine, with or without H_32).
-// Thread (row, half) as in prefill_tc_gdn_kernel.
+// Thread (row, quarter qq): row = tensor-memory lane (warps w, w + 4, w + 8 and w + 12
+// reach the same lanes); the quarters split a row's value blocks (one each) or a phase's tasks.
 template <int FMT>
-__global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const PrefillParams p) {
+__global__ void __launch_bounds__(kKdThreads, 1) prefill_tc_kda_kernel(const PrefillParams p) {
     static_assert(FMT != kFmtS8Row, "the row-absmax format shares a row scale over the value blocks");
     constexpr bool HAD = fmt_had(FMT);
     extern __shared__ __align__(128) uint8_t smem[];  // descriptors need 16-byte alignment (no swizzle)
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int row = tid & 127, half = tid >> 7;
+    const int row = tid & 127, qq = tid >> 7;
     const uint32_t sb = smem_u32(smem);
     const int H = p.H, T = p.T, Hm = p.Hm;
     const int rec_bytes = p.rec_bytes, rstride = tc_rec_stride(rec_bytes);
@@ -117,7 +119,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
     auto load_piece = [&](const Unit &n, int p0) {
         const int nl = min(kTcC, n.Tb - p0);
 #pragma unroll 1
-        for (int i = tid; i < 2048; i += kTcThreads) {  // k rows 0..63, q rows 64..127: 16 chunks each
+        for (int i = tid; i < 2048; i += kKdThreads) {  // k rows 0..63, q rows 64..127: 16 chunks each
             const int m = i >> 4, j = i & 15, t = m & 63;
             const uint32_t dst = kq + (uint32_t)(m * kKdRowKQ + 16 * j);
             if (t < nl)
@@ -127,7 +129,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
                 sts128(dst, make_uint4(0u, 0u, 0u, 0u));
         }
 #pragma unroll 1
-        for (int i = tid; i < 2048; i += kTcThreads) {  // g: 64 rows of 32 chunks
+        for (int i = tid; i < 2048; i += kKdThreads) {  // g: 64 rows of 32 chunks
             const int t = i >> 5, j = i & 31;
             const uint32_t dst = xi + (uint32_t)(t * kKdRowXI * 4 + 16 * j);
             if (t < nl)
@@ -137,7 +139,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
                 sts128(dst, make_uint4(0u, 0u, 0u, 0u));
         }
 #pragma unroll 1
-        for (int i = tid; i < 1024; i += kTcThreads) {
+        for (int i = tid; i < 1024; i += kKdThreads) {
             const int t = i >> 4, j = i & 15;
             const uint32_t dst = sb + (uint32_t)(kKdV + t * kTcRowV + 16 * j);
             if (t < nl)
@@ -178,8 +180,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
         }
         ph_rec ^= 1u;
         rec_pending = false;
-        // ---- S_0: record row u = row into tensor-memory lane u (this half's value blocks) ----
-        tc_reconstruct<FMT>(p, sb + (uint32_t)kKdRec, rstride, row, half, tS);
+        // ---- S_0: record row u = row into tensor-memory lane u (this quarter's value block) ----
+        tc_reconstruct<FMT, 4>(p, sb + (uint32_t)kKdRec, rstride, row, qq, tS);
         __syncthreads();  // the records are read: the first piece's operands go over them
 
         int p0 = 0;
@@ -192,9 +194,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
             __syncthreads();
             // ---- the piece's length: the largest of 64, 32, ..., 1 tokens over which every
             //      channel decays by at most e^kKdMaxLog on either side of the reference
-            //      token m = L / 2 - 1 (thread c = row of half 0 owns channel c) ----
+            //      token m = L / 2 - 1 (thread c = row of quarter 0 owns channel c) ----
             float lam[7] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};  // Lambda_t = sum_{i<=t} g_i at t = 0, 1, 3, ..., 63
-            if (half == 0) {
+            if (qq == 0) {
                 float acc = 0.f;
 #pragma unroll
                 for (int t = 0; t < kTcC; ++t) {  // unrolled: the indices of lam are constants
@@ -211,18 +213,18 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
             int L = 1;
 #pragma unroll
             for (int j = 6; j >= 1; --j) {  // L = 2^j, m = 2^(j-1) - 1
-                const bool ok_c = half == 1 || ((lam[0] - lam[j - 1] <= kKdMaxLog) && (lam[j - 1] - lam[j] <= kKdMaxLog));
+                const bool ok_c = qq != 0 || ((lam[0] - lam[j - 1] <= kKdMaxLog) && (lam[j - 1] - lam[j] <= kKdMaxLog));
                 if (L == 1 && __syncthreads_and(ok_c)) L = 1 << j;
             }
             const int nt = min(L, Tb - p0);   // tokens of this piece; the rest are masked
             const int m = L > 1 ? L / 2 - 1 : 0;
             // ---- xi_t = gamma_t / gamma_m in place of g (0 for masked tokens), as running
-            //      products from m (half 0: downward, xi_{t-1} = xi_t e^{-g_t}, and gamma_m;
-            //      half 1: upward, xi_t = xi_{t-1} e^{g_t}); xi_C at C = nt - 1 ----
+            //      products from m (quarter 0: downward, xi_{t-1} = xi_t e^{-g_t}, and gamma_m;
+            //      quarter 1: upward, xi_t = xi_{t-1} e^{g_t}); xi_C at C = nt - 1 ----
             {
                 const uint32_t colc = xi + (uint32_t)(4 * row);
                 float x = 1.f;
-                if (half == 0) {
+                if (qq == 0) {
                     float gm = 1.f;
 #pragma unroll 1
                     for (int t = m; t >= 0; --t) {
@@ -234,7 +236,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
                         x *= expf(-g);
                     }
                     sts32(s_gm + 4 * row, __float_as_uint(gm));
-                } else {
+                } else if (qq == 1) {
 #pragma unroll 1
                     for (int t = m + 1; t < kTcC; ++t) {
                         const uint32_t a = colc + (uint32_t)(t * kKdRowXI * 4);
@@ -252,11 +254,11 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
 #pragma unroll 1
             for (int hh = 0; hh < 2; ++hh) {
                 const int c0 = 64 * hh;
-                {  // X: row m = row, channels c0 + 32 half .. + 31
+                {  // X: row m = row, channels c0 + 16 qq .. + 15
                     const uint32_t kqrow = kq + (uint32_t)(row * kKdRowKQ), xrow = xi + (uint32_t)((row & 63) * kKdRowXI * 4);
 #pragma unroll
-                    for (int jj = 0; jj < 4; ++jj) {
-                        const int cl = 32 * half + 8 * jj;
+                    for (int jj = 0; jj < 2; ++jj) {
+                        const int cl = 16 * qq + 8 * jj;
                         const uint4 kw = lds128(kqrow + (uint32_t)(2 * (c0 + cl)));
                         const uint4 xa = lds128(xrow + (uint32_t)(4 * (c0 + cl))), xb = lds128(xrow + (uint32_t)(4 * (c0 + cl) + 16));
                         const uint32_t kk[4] = {kw.x, kw.y, kw.z, kw.w};
@@ -272,7 +274,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
                     }
                 }
 #pragma unroll 1
-                for (int i = tid; i < 512; i += kTcThreads) {  // Z: token s, 8 channels per task
+                for (int i = tid; i < 512; i += kKdThreads) {  // Z: token s, 8 channels per task
                     const int s2 = i >> 3, cl = 8 * (i & 7);
                     const uint4 kw = lds128(kq + (uint32_t)(s2 * kKdRowKQ + 2 * (c0 + cl)));
                     const uint32_t xrow = xi + (uint32_t)(s2 * kKdRowXI * 4 + 4 * (c0 + cl));
@@ -293,8 +295,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
                     const int ch = (int)(lds_u8(s_perm + row) & 127u);
                     const bool mine = (ch >> 6) == hh;
                     const float gmc = ldsf(s_gm + 4 * ch);
-#pragma unroll 1
-                    for (int c = 2 * half; c < 2 * half + 2; ++c) {
+                    {
+                        const int c = qq;
                         float v[32];
                         tc_ld32(tS + 32 * c, v);  // every lane: warp-collective
                         if (mine) {
@@ -334,60 +336,58 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
                 tc_fence_after();
             }
             if (timed_out) break;
-            // ---- half 0: rows of L' = beta_t G_ts (s < t) and M = G_ts (s <= t) from the
-            //      Gram rows (the decay is in G); half 1: the zero rows of [0; M]; all:
+            // ---- quarter 0: rows of L' = beta_t G_ts (s < t) and M = G_ts (s <= t) from the
+            //      Gram rows (the decay is in G); quarter 1: the zero rows of [0; M]; all:
             //      (K (.) Xi_C / Xi)^T in record-row order and gamma_C S_0 in tensor memory ----
-            if (half == 0) {
+            if (qq == 0) {
                 const int t = row & 63;
                 const bool qside = row >= 64;
-                float gr[64];
-                {
-                    float g0[32], g1[32];
-                    tc_ld32(tG, g0);
-                    tc_ld32(tG + 32, g1);
+                const float bt = qside ? 1.f : ldsf(s_beta + 4 * t);
+#pragma unroll 1
+                for (int h2 = 0; h2 < 2; ++h2) {  // columns s of 32 h2 .. 32 h2 + 31
+                    float gr[32];
+                    tc_ld32(tG + 32 * h2, gr);
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        gr[i] = g0[i];
-                        gr[32 + i] = g1[i];
+                    for (int s2 = 0; s2 < 32; ++s2) {
+                        const int sc = 32 * h2 + s2;
+                        gr[s2] = sc < t ? bt * gr[s2] : (sc == t && qside ? gr[s2] : 0.f);
+                    }
+                    if (!qside) {  // column t of L'^T
+                        const uint32_t colt = sb + (uint32_t)(kKdLP + 4 * t + 32 * h2 * kTcRowL * 4);
+#pragma unroll
+                        for (int s2 = 0; s2 < 32; ++s2) sts32(colt + (uint32_t)(s2 * kTcRowL * 4), __float_as_uint(gr[s2]));
+                    } else {
+#pragma unroll
+                        for (int g = 0; g < 4; ++g)
+                            split3_store8(sb + kKdAO + tc_k64_off(64 + t, 32 * h2 + 8 * g), 16384, gr + 8 * g);
                     }
                 }
-                const float bt = qside ? 1.f : ldsf(s_beta + 4 * t);
-#pragma unroll
-                for (int s2 = 0; s2 < 64; ++s2) gr[s2] = s2 < t ? bt * gr[s2] : (s2 == t && qside ? gr[s2] : 0.f);
-                if (!qside) {  // column t of L'^T
-                    const uint32_t colt = sb + (uint32_t)(kKdLP + 4 * t);
-#pragma unroll
-                    for (int s2 = 0; s2 < 64; ++s2) sts32(colt + (uint32_t)(s2 * kTcRowL * 4), __float_as_uint(gr[s2]));
-                } else {
-#pragma unroll
-                    for (int g = 0; g < 8; ++g) split3_store8(sb + kKdAO + tc_k64_off(64 + t, 8 * g), 16384, gr + 8 * g);
-                }
-            } else {
+            } else if (qq == 1) {
 #pragma unroll 1
                 for (int i = row; i < 1536; i += 128)
                     sts128(sb + (uint32_t)(kKdAO + (i >> 9) * 16384 + (i & 511) * 16), make_uint4(0u, 0u, 0u, 0u));
             }
-            {  // (K (.) Xi_C / Xi)^T, K-major: record row u = row (channel pi(u)), tokens 32 half .. + 31
+            {  // (K (.) Xi_C / Xi)^T, K-major: record row u = row (channel pi(u)), tokens 16 qq .. + 15
                 const uint32_t ch = lds_u8(s_perm + row) & 127u;
                 const float xic = ldsf(s_xiC + 4u * ch);
 #pragma unroll
-                for (int g8 = 0; g8 < 4; ++g8) {
+                for (int g8 = 0; g8 < 2; ++g8) {
                     float v[8];
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
-                        const int t = 32 * half + 8 * g8 + e;
+                        const int t = 16 * qq + 8 * g8 + e;
                         const float kv = __uint_as_float(lds_u16(kq + (uint32_t)(t * kKdRowKQ) + 2u * ch) << 16);
                         const float xs = ldsf(xi + (uint32_t)(t * kKdRowXI * 4) + 4u * ch);
                         v[e] = xs != 0.f ? kv * (xic * __frcp_rn(xs)) : 0.f;  // masked tokens: 0
                     }
-                    split3_store8(sb + kKdA3 + tc_k64_off(row, 32 * half + 8 * g8), 16384, v);
+                    split3_store8(sb + kKdA3 + tc_k64_off(row, 16 * qq + 8 * g8), 16384, v);
                 }
             }
             {  // gamma_C S_0 = gamma_m xi_C S_0 (per channel; the state product accumulates onto it)
                 const uint32_t ch = lds_u8(s_perm + row) & 127u;
                 const float gc = ldsf(s_gm + 4u * ch) * ldsf(s_xiC + 4u * ch);
-#pragma unroll 1
-                for (int c = 2 * half; c < 2 * half + 2; ++c) {
+                {
+                    const int c = qq;
                     float v[32];
                     tc_ld32(tS + 32 * c, v);
 #pragma unroll
@@ -396,13 +396,13 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
                 }
             }
             __syncthreads();  // K and Xi are read: Y goes over them
-            // ---- Y = diag(beta) (v~ - W), FP32 rows (this half's value blocks) ----
+            // ---- Y = diag(beta) (v~ - W), FP32 rows (this quarter's value block) ----
             if (row < 64) {
                 const int t = row;
                 const float bt = ldsf(s_beta + 4 * t);
                 const uint32_t vrow = sb + (uint32_t)(kKdV + t * kTcRowV), yrow = sb + (uint32_t)(kKdYU + t * kTcRowY * 4);
-#pragma unroll 1
-                for (int c = 2 * half; c < 2 * half + 2; ++c) {
+                {
+                    const int c = qq;
                     float w[32];
                     tc_ld32(tWP + 32 * c, w);
                     float2 y[16];
@@ -426,16 +426,16 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
             }
             __syncthreads();
             // ---- U = L^-1 Y (value column n = row, in place) ----
-            tc_solve(sb + (uint32_t)(kKdYU + 4 * row), sb + (uint32_t)kKdLP, half);
-            // ---- U as three bf16 parts, K-major (value columns n x tokens s): tokens 32 half .. + 31 ----
+            tc_solve<4>(sb + (uint32_t)(kKdYU + 4 * row), sb + (uint32_t)kKdLP, qq);
+            // ---- U as three bf16 parts, K-major (value columns n x tokens s): tokens 16 qq .. + 15 ----
             {
                 const uint32_t col = sb + (uint32_t)(kKdYU + 4 * row);
-                float uc[32];
+                float uc[16];
 #pragma unroll
-                for (int t = 0; t < 32; ++t) uc[t] = ldsf(col + (uint32_t)((32 * half + t) * kTcRowY * 4));
+                for (int t = 0; t < 16; ++t) uc[t] = ldsf(col + (uint32_t)((16 * qq + t) * kTcRowY * 4));
                 __syncthreads();  // every column is read: the parts go over Y / U
 #pragma unroll
-                for (int g = 0; g < 4; ++g) split3_store8(sb + kKdBU + tc_k64_off(row, 32 * half + 8 * g), 16384, uc + 8 * g);
+                for (int g = 0; g < 2; ++g) split3_store8(sb + kKdBU + tc_k64_off(row, 16 * qq + 8 * g), 16384, uc + 8 * g);
             }
             fence_proxy_async_smem();
             tc_fence_before();
@@ -465,12 +465,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
             ph_mma ^= 1u;
             tc_fence_after();
             if (p0 + nt >= Tb && nxt.unit < units) prefetch(nxt);  // the next unit's loads overlap this one's tail
-            // ---- o_t = H (P_t + (M U)_t) (lanes 64 + t, this half's value blocks) ----
+            // ---- o_t = H (P_t + (M U)_t) (lanes 64 + t, this quarter's value block) ----
             if (row >= 64) {
                 const int t = row - 64;
                 float *orow = p.o + (((int64_t)b * T + p0 + min(t, nt - 1)) * Hm + mh) * 128;
-#pragma unroll 1
-                for (int c = 2 * half; c < 2 * half + 2; ++c) {
+                {
+                    const int c = qq;
                     float ov[32];
                     tc_ld32(tWP + 32 * c, ov);
                     float2 y[16];
@@ -489,7 +489,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) prefill_tc_kda_kernel(const Pre
         }
         if (timed_out) break;
         // ---- the chunk-final state into the record in place ----
-        tc_requantize<FMT>(p, grec0, row, half, lane, tS);
+        tc_requantize<FMT, 4>(p, grec0, row, qq, lane, tS);
         cur = nxt;
     }
     if (rec_pending) mbar_wait_bounded(bar_rec, ph_rec);
