@@ -687,8 +687,8 @@ def prefill_arm(steps: int, warmup: int, T: int = 64, lo_format: int = 0, kinds=
         kernel = (f"prefill_tc_{w.kind}_kernel (chunkwise closed form on the tensor cores)" if tc else
                   "prefill_cg_kernel (per-token FP32 recurrence)" if w.lo_format in (0, 1) and T >= 32 else
                   "prefill_chunk_kernel (per-token FP32 recurrence)")
-        out.append({"mode": "prefill_chunk", "kind": w.kind, "workload": w.name, "lo_format": w.lo_format,
-                    "chunk_tokens": T, "kernel": kernel,
+        out.append({"mode": "prefill_chunk", "kind": w.kind, "workload": w.name, "batch": w.batch,
+                    "lo_format": w.lo_format, "chunk_tokens": T, "kernel": kernel,
                     "us_per_chunk": us, "tokens_per_s": w.batch * T / (us * 1e-6),
                     # the per-token form's FLOPs against the FP32 FMA peak: for the tensor-core
                     # kernel an equivalent rate (its work is tensor-core products plus the solve)
