@@ -306,3 +306,52 @@ def test_group_step_full_batch_4_28(kind):
     assert torch.equal(o_one, o_each)
     for (G, _), a, b in zip(groups, pools["one"], pools["each"]):
         _same_up_to_ties(G, a, b, "full batch")
+
+
+@pytest.mark.parametrize("kind", ["gdn", "kda"])
+def test_group_step_skips_a_bad_slot_and_head_in_the_second_group(kind):
+    """One-launch group step (K_hi 8/24) whose second group maps a head outside the layer
+    and whose slot list names a slot outside the pool (every warp meets the skipped tiles
+    in its second body, after a first body that ran whole).  Both flags are raised, the
+    bad slot's and head's records and output rows stay as they were, and the rest equals
+    the per-group calls."""
+    w = wl.sweep(kind, 8, 0).replace(batch=3, heads=8, qk_heads=4)
+    L = P.layout_of(w)
+    S, perm = _layer(w, 95)
+    heads_b = [1, 2, 11, 7]  # 11 is outside the layer's 8 heads
+    ga = _group(L, HEADS_A, 8)
+    gb = damp.Layout(4, L.num_qk_heads, L.d_k, L.d_v, 24, L.lo_format, model_heads=L.num_heads,
+                     head_map=torch.tensor(heads_b, dtype=torch.int32, device=DEV))
+    good_b = _group(L, [1, 2, 4, 7], 24)
+    perms = [perm[HEADS_A].contiguous(), perm[[1, 2, 4, 7]].contiguous()]
+    setup = torch.tensor([2, 1, 0], dtype=torch.int32, device=DEV)
+    slot_idx = torch.tensor([2, 7, 0], dtype=torch.int32, device=DEV)  # a pool of 3 slots: 7 is outside
+    pools = {}
+    for tag in ("one", "each"):
+        pools[tag] = []
+        for G, pm in ((ga, perms[0]), (good_b, perms[1])):
+            pg = damp.new_state(G, 3, DEV)
+            damp.quantize_state(G, S, pm, pg, slot_idx=setup)
+            pools[tag].append(pg)
+    assert damp.device_status() == 0
+    before = [damp.unpack_tiers(G, pg) for G, pg in zip((ga, good_b), pools["one"])]
+    step = damp.kda_decode_step if kind == "kda" else damp.gdn_decode_step
+    gstep = damp.kda_decode_step_groups if kind == "kda" else damp.gdn_decode_step_groups
+    d = P.inputs_to_dev(w, wl.step_inputs(w, 0), DEV)
+    o_each = torch.zeros((w.batch, w.heads, w.d_v), device=DEV)
+    for G, pg, pm in zip((ga, gb), pools["each"], perms):
+        step(G, pg, pm, d["q"], d["k"], d["v"], d["g"], d["beta"], o=o_each, slot_idx=slot_idx)
+    assert damp.device_status() == damp.DEV_BAD_SLOT | damp.DEV_BAD_HEAD
+    o_one = torch.zeros_like(o_each)
+    gstep([(G, pg, pm) for G, pg, pm in zip((ga, gb), pools["one"], perms)],
+          d["q"], d["k"], d["v"], d["g"], d["beta"], o=o_one, slot_idx=slot_idx)
+    assert damp.device_status() == damp.DEV_BAD_SLOT | damp.DEV_BAD_HEAD
+    assert torch.equal(o_one, o_each)
+    assert bool((o_one[1] == 0).all()) and bool((o_one[:, 4] == 0).all())  # the bad slot's row, head 4 (unmapped)
+    after = [damp.unpack_tiers(G, pg) for G, pg in zip((ga, good_b), pools["one"])]
+    for a, b in zip(after[1], before[1]):
+        assert torch.equal(a[1], b[1])        # slot 1 was not named by the step
+        assert torch.equal(a[2, 2], b[2, 2])  # the unmapped held head (slot 2 = batch row 0)
+        assert not torch.equal(a[2, 0], b[2, 0])
+    for (G, a, b) in zip((ga, good_b), pools["one"], pools["each"]):
+        _same_up_to_ties(G, a, b, "bad slot and head")
