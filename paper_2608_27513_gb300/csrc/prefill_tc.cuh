@@ -221,55 +221,60 @@ __device__ __forceinline__ void tc_reconstruct(const PrefillParams &p, uint32_t 
 // solved before it out of its own.  Every thread of the CTA calls it (NQ barriers per block).
 template <int NQ>
 __device__ __forceinline__ void tc_solve(uint32_t col, uint32_t lt, int part) {
-    constexpr int RB = 16 / NQ;  // rows per part and block (4 or 8)
-    auto ltr = [&](int srow, int t0, float (&lv)[RB]) {
+    constexpr int RB = 16 / NQ;  // rows per part and block (4 or 8), held as RB / 2 pairs
+    constexpr int RP = RB / 2;
+    auto ltr = [&](int srow, int t0, float2 (&lv)[RP]) {
         const uint32_t lrow = lt + (uint32_t)(srow * kTcRowL * 4 + 4 * t0);
 #pragma unroll
         for (int i = 0; i < RB / 4; ++i) {
             const uint4 l4 = lds128(lrow + 16 * i);
-            lv[4 * i] = __uint_as_float(l4.x);
-            lv[4 * i + 1] = __uint_as_float(l4.y);
-            lv[4 * i + 2] = __uint_as_float(l4.z);
-            lv[4 * i + 3] = __uint_as_float(l4.w);
+            lv[2 * i] = make_float2(__uint_as_float(l4.x), __uint_as_float(l4.y));
+            lv[2 * i + 1] = make_float2(__uint_as_float(l4.z), __uint_as_float(l4.w));
         }
     };
+    auto row_at = [&](int r) { return col + (uint32_t)(r * kTcRowY * 4); };
 #pragma unroll 1
     for (int t0 = 0; t0 < kTcC; t0 += 16) {
         const int r0 = t0 + RB * part;
-        float acc[RB];
+        float2 acc[RP];
 #pragma unroll
-        for (int r = 0; r < RB; ++r) acc[r] = ldsf(col + (uint32_t)((r0 + r) * kTcRowY * 4));
+        for (int i = 0; i < RP; ++i) acc[i] = make_float2(ldsf(row_at(r0 + 2 * i)), ldsf(row_at(r0 + 2 * i + 1)));
 #pragma unroll 4
         for (int s2 = 0; s2 < t0; ++s2) {
-            const float us = ldsf(col + (uint32_t)(s2 * kTcRowY * 4));
-            float lv[RB];
+            const float us = ldsf(row_at(s2));
+            float2 lv[RP];
             ltr(s2, r0, lv);
 #pragma unroll
-            for (int r = 0; r < RB; ++r) acc[r] = fmaf(-lv[r], us, acc[r]);
+            for (int i = 0; i < RP; ++i) acc[i] = fma2(lv[i], make_float2(-us, -us), acc[i]);
         }
 #pragma unroll
         for (int q = 0; q < NQ; ++q) {
-            if (part == q) {  // own rows among themselves, then stored
+            if (part == q) {  // own rows among themselves (the pair holding the solved row takes
+                              // zero entries of L'^T, which leave it as it is), then stored
 #pragma unroll
                 for (int a = 0; a < RB - 1; ++a) {
-                    float lv[RB];
+                    const float ua = (a & 1) ? acc[a >> 1].y : acc[a >> 1].x;
+                    float2 lv[RP];
                     ltr(r0 + a, r0, lv);
 #pragma unroll
-                    for (int r = a + 1; r < RB; ++r) acc[r] = fmaf(-lv[r], acc[a], acc[r]);
+                    for (int i = a >> 1; i < RP; ++i) acc[i] = fma2(lv[i], make_float2(-ua, -ua), acc[i]);
                 }
 #pragma unroll
-                for (int r = 0; r < RB; ++r) sts32(col + (uint32_t)((r0 + r) * kTcRowY * 4), __float_as_uint(acc[r]));
+                for (int i = 0; i < RP; ++i) {
+                    sts32(row_at(r0 + 2 * i), __float_as_uint(acc[i].x));
+                    sts32(row_at(r0 + 2 * i + 1), __float_as_uint(acc[i].y));
+                }
             }
             __syncthreads();
             if (part > q) {  // the rows part q just solved
 #pragma unroll
                 for (int a = 0; a < RB; ++a) {
                     const int sr = t0 + RB * q + a;
-                    const float us = ldsf(col + (uint32_t)(sr * kTcRowY * 4));
-                    float lv[RB];
+                    const float us = ldsf(row_at(sr));
+                    float2 lv[RP];
                     ltr(sr, r0, lv);
 #pragma unroll
-                    for (int r = 0; r < RB; ++r) acc[r] = fmaf(-lv[r], us, acc[r]);
+                    for (int i = 0; i < RP; ++i) acc[i] = fma2(lv[i], make_float2(-us, -us), acc[i]);
                 }
             }
         }
