@@ -111,7 +111,10 @@ constexpr uint64_t kWaitTestNs = 1000000;  // 1 ms
 constexpr int kHiUnroll = 16;             // largest fixed K_hi whose FP16 sums follow the low tier
 // The body runs as CTA `blk` of a grid of `nblk` CTAs; it returns true when one of the
 // warp's copy waits ran out (its stage barriers are then left as they are).
-template <int RL, int DKC, int KC, bool KDA, bool HAD, bool BF16, bool HMAP, int LT = kLtU8, bool WAITTEST = false>
+// UMH (head groups): look the model head up once per (slot, head) unit and keep it in a
+// register, instead of once per tile (set where the extra register costs no spills).
+template <int RL, int DKC, int KC, bool KDA, bool HAD, bool BF16, bool HMAP, int LT = kLtU8, bool WAITTEST = false,
+          bool UMH = false>
 __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int blk, const int nblk) {
     constexpr int R = RL > 0 ? RL : 1;
     extern __shared__ __align__(128) uint8_t smem[];
@@ -177,9 +180,11 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
     const int Hm = HMAP ? p.Hm : H;  // heads of the operand tensors
 
     // ---- producer (lane 0): one bulk copy of the record of tile t (cursor k) into stage s ----
+    // (a held head whose map entry is out of range still has its records in the slot: they
+    // are copied and the consumer skips the tile, so no head-map load sits on this path)
     auto issue = [&](int64_t t, const Cursor &k, int s) {
         const int64_t slot = slot_of(k.b);
-        const bool ok = slot >= 0 && slot < p.num_slots && (!HMAP || model_head(k.h) >= 0);
+        const bool ok = slot >= 0 && slot < p.num_slots;
         const uint32_t st = stage0 + (uint32_t)(s * stage_bytes);
         const uint32_t bar = bar0 + 8 * s;
         mbar_arrive_expect_tx(bar, ok ? (uint32_t)rec_bytes + (WAITTEST ? kWaitTestExtra : 0u) : 0u);
@@ -233,6 +238,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
     float aa[R];
     float unit_beta = 0.f, unit_g = 0.f, bkq = 0.f;
     int unit = 0;
+    int unit_mh = 0;     // model head of the current (slot, head) (head groups)
     uint32_t ob = ops0;  // operand buffer of the current (slot, head)
     int s = 0;
     uint32_t parity = 0;
@@ -249,7 +255,8 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
         }
         const int b = cur.b, h = cur.h, c = cur.c;
         const int64_t slot = slot_of(b);
-        const int mh = model_head(h);
+        if (UMH && (t == t0 || c == 0)) unit_mh = model_head(h);
+        const int mh = UMH ? unit_mh : model_head(h);
         const bool slot_ok = slot >= 0 && slot < p.num_slots, ok = slot_ok && (!HMAP || mh >= 0);
         bad_slot |= !slot_ok;
         if (HMAP) bad_head |= mh < 0;
@@ -587,7 +594,7 @@ __device__ __forceinline__ bool packed_step_body(const PackedParams p, const int
                 for (int64_t tt = t_fail; tt <= last; ++tt) {
                     const Cursor k = cursor_at(tt, H, V);
                     const int64_t slot = slot_of(k.b);
-                    if (slot >= 0 && slot < p.num_slots && (!HMAP || model_head(k.h) >= 0))
+                    if (slot >= 0 && slot < p.num_slots)
                         mbar_complete_tx(bar0 + 8 * (int)((tt - t0) % nstage), kWaitTestExtra);
                 }
             }
@@ -624,9 +631,14 @@ __global__ void __launch_bounds__(256, 1) packed_step_kernel(const PackedParams 
 // shared-memory stride, so a warp's region is the same in both bodies.  d_k = 128.
 template <int KC1, int KC2, bool KDA, bool HAD, bool BF16>
 __global__ void __launch_bounds__(256, 1) packed_step2_kernel(const PackedParams p1, const PackedParams p2) {
-    if (packed_step_body<(128 - KC1 + 31) / 32, 128, KC1, KDA, HAD, BF16, true>(p1, blockIdx.x, gridDim.x))
+    // the per-unit model head where both groups keep at most 20 FP16 rows (measured: with a
+    // group of 24 or 28 rows the register goes to spills)
+    constexpr bool UMH = (KC1 > KC2 ? KC1 : KC2) <= 20;
+    if (packed_step_body<(128 - KC1 + 31) / 32, 128, KC1, KDA, HAD, BF16, true, kLtU8, false, UMH>(p1, blockIdx.x,
+                                                                                                  gridDim.x))
         return;  // a copy of group 1 was lost (status set): its barriers cannot be reused
-    packed_step_body<(128 - KC2 + 31) / 32, 128, KC2, KDA, HAD, BF16, true>(p2, blockIdx.x, gridDim.x);
+    packed_step_body<(128 - KC2 + 31) / 32, 128, KC2, KDA, HAD, BF16, true, kLtU8, false, UMH>(p2, blockIdx.x,
+                                                                                              gridDim.x);
 }
 
 }  // namespace damp
